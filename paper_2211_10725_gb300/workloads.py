@@ -1,0 +1,192 @@
+"""Seeded synthetic workloads for the spiking-neuron scan.
+
+This module only draws random inputs and describes workload shapes: it holds
+none of the neuron arithmetic, so both the CUDA path and the CPU oracle can be
+fed from it.  Every tensor is drawn on the CPU with ``torch.Generator`` so that
+the same seed gives the same values on any machine.
+
+Workloads (all synthetic; MNIST/CIFAR-10 shapes from the paper's Tab. I stand
+in for the datasets, which are not used):
+
+* ``leaky_T25_B128_N1000``      Leaky LIF layer (Eq. 4), fp32.
+* ``synaptic_T100_B128_N4096``  current-based LIF layer (Eqs. 5-6), fp32.
+* ``dsnn_784_1000_1000_10``     3-layer dense SNN, bf16 GEMMs, T=25, B=128.
+* ``conv_lif_T25_B128``         LIF on the conv-SNN activation shapes
+                                [12,24,24] and [64,8,8], per-channel beta.
+* ``leaky_bf16_T500_B64_N8192`` large Leaky layer, bf16 storage, per-neuron
+                                beta/threshold.
+"""
+from __future__ import annotations
+
+import dataclasses
+from typing import Optional
+
+import torch
+
+SEED_BASE = 2211_10725
+
+F32, BF16, F16 = "f32", "bf16", "f16"
+TORCH_DTYPE = {F32: torch.float32, BF16: torch.bfloat16, F16: torch.float16}
+
+
+@dataclasses.dataclass(frozen=True)
+class ScanWorkload:
+    """Shape and distribution of one scan layer's synthetic inputs."""
+
+    name: str
+    neuron: str                 # "leaky" (Eq. 4) or "synaptic" (Eqs. 5-6)
+    T: int
+    B: int
+    N: int                      # flattened neurons per sample (C*H*W for conv maps)
+    C: int = 1                  # channels (per-channel parameters)
+    HW: int = 1                 # spatial size per channel
+    in_dtype: str = F32         # dtype of the input current I
+    io_dtype: str = F32         # dtype of spk, mem, grad_spk, grad_I
+    i_mean: float = 0.3
+    i_std: float = 0.5          # second argument of N(mu, s) is the std deviation
+    beta: tuple = ("const", 0.9)        # ("const", v) | ("uniform", lo, hi)
+    thr: tuple = ("const", 1.0)
+    alpha: tuple = ("const", 0.8)
+    beta_mode: str = "scalar"   # scalar | per_neuron | per_channel
+    thr_mode: str = "scalar"
+    alpha_mode: str = "scalar"
+    reset: str = "subtract"     # subtract | zero | none
+    surrogate: str = "fast_sigmoid"     # fast_sigmoid | atan
+    sg_param: float = 25.0
+    detach_reset: bool = True
+    save: str = "mem"           # mem | recompute
+    ckpt_every: int = 8
+    want_mem: bool = True       # the layer's mem output is requested
+    seed_index: int = 0
+
+    def scaled(self, **kw) -> "ScanWorkload":
+        return dataclasses.replace(self, **kw)
+
+    @property
+    def lanes(self) -> int:
+        return self.B * self.N
+
+    @property
+    def neuron_steps(self) -> int:
+        return self.T * self.B * self.N
+
+
+LEAKY_C1 = ScanWorkload(
+    name="leaky_T25_B128_N1000", neuron="leaky", T=25, B=128, N=1000,
+    i_mean=0.3, i_std=0.5, surrogate="fast_sigmoid", sg_param=25.0, seed_index=0)
+
+SYNAPTIC_C2 = ScanWorkload(
+    name="synaptic_T100_B128_N4096", neuron="synaptic", T=100, B=128, N=4096,
+    i_mean=0.2, i_std=0.4, alpha=("const", 0.8), surrogate="atan", sg_param=2.0,
+    seed_index=1)
+
+CONV_C4A = ScanWorkload(
+    name="conv_lif_T25_B128_C12x24x24", neuron="leaky", T=25, B=128, N=12 * 24 * 24,
+    C=12, HW=24 * 24, i_mean=0.25, i_std=0.5, beta=("const", 0.95),
+    beta_mode="per_channel", reset="zero", surrogate="fast_sigmoid", sg_param=25.0,
+    want_mem=False, seed_index=3)
+
+CONV_C4B = CONV_C4A.scaled(name="conv_lif_T25_B128_C64x8x8", N=64 * 8 * 8, C=64, HW=64)
+
+BIG_C5 = ScanWorkload(
+    name="leaky_bf16_T500_B64_N8192", neuron="leaky", T=500, B=64, N=8192,
+    in_dtype=BF16, io_dtype=BF16, i_mean=0.1, i_std=0.3,
+    beta=("uniform", 0.85, 0.99), thr=("uniform", 0.8, 1.2),
+    beta_mode="per_neuron", thr_mode="per_neuron", surrogate="atan", sg_param=2.0,
+    save="recompute", ckpt_every=8, want_mem=False, seed_index=4)
+
+SCAN_WORKLOADS = {w.name: w for w in (LEAKY_C1, SYNAPTIC_C2, CONV_C4A, CONV_C4B, BIG_C5)}
+
+
+def _gen(seed: int) -> torch.Generator:
+    g = torch.Generator(device="cpu")
+    g.manual_seed(seed)
+    return g
+
+
+def _param(spec: tuple, mode: str, w: ScanWorkload, g: torch.Generator) -> torch.Tensor:
+    n = {"scalar": 1, "per_neuron": w.N, "per_channel": w.C}[mode]
+    if spec[0] == "const":
+        return torch.full((n,), float(spec[1]), dtype=torch.float32)
+    if spec[0] == "uniform":
+        lo, hi = spec[1], spec[2]
+        return (lo + (hi - lo) * torch.rand(n, generator=g, dtype=torch.float32))
+    raise ValueError(spec)
+
+
+def make_scan_inputs(w: ScanWorkload, seed: Optional[int] = None,
+                     with_mem0: bool = False, with_grad_mem: bool = False,
+                     with_grad_final: bool = False) -> dict:
+    """Draw the layer's inputs on the CPU.
+
+    Returns a dict of CPU tensors: ``I`` [T,B,N] in_dtype, ``grad_spk`` [T,B,N]
+    io_dtype ~ N(0,1), ``beta``/``thr``/``alpha`` fp32 of length 1, N or C, and
+    optionally ``mem0``/``syn0`` [B,N] fp32, ``grad_mem`` [T,B,N] io_dtype and
+    ``grad_mem_final``/``grad_syn_final`` [B,N] fp32.
+    """
+    seed = SEED_BASE + w.seed_index if seed is None else seed
+    g = _gen(seed)
+    shape = (w.T, w.B, w.N)
+    I = (w.i_mean + w.i_std * torch.randn(shape, generator=g, dtype=torch.float32))
+    out = {"I": I.to(TORCH_DTYPE[w.in_dtype])}
+    out["beta"] = _param(w.beta, w.beta_mode, w, g)
+    out["thr"] = _param(w.thr, w.thr_mode, w, g)
+    if w.neuron == "synaptic":
+        out["alpha"] = _param(w.alpha, w.alpha_mode, w, g)
+    out["grad_spk"] = torch.randn(shape, generator=g, dtype=torch.float32).to(
+        TORCH_DTYPE[w.io_dtype])
+    if with_mem0:
+        out["mem0"] = 0.5 * torch.randn((w.B, w.N), generator=g, dtype=torch.float32) + 0.5
+        if w.neuron == "synaptic":
+            out["syn0"] = 0.3 * torch.randn((w.B, w.N), generator=g, dtype=torch.float32)
+    if with_grad_mem:
+        out["grad_mem"] = (0.1 * torch.randn(shape, generator=g, dtype=torch.float32)).to(
+            TORCH_DTYPE[w.io_dtype])
+    if with_grad_final:
+        out["grad_mem_final"] = torch.randn((w.B, w.N), generator=g, dtype=torch.float32)
+        if w.neuron == "synaptic":
+            out["grad_syn_final"] = torch.randn((w.B, w.N), generator=g, dtype=torch.float32)
+    return out
+
+
+# ---------------------------------------------------------------------------
+# 3-layer dense SNN (784-1000-1000-10, T=25, B=128)
+# ---------------------------------------------------------------------------
+
+@dataclasses.dataclass(frozen=True)
+class DenseWorkload:
+    name: str = "dsnn_784_1000_1000_10_T25_B128"
+    T: int = 25
+    B: int = 128
+    sizes: tuple = (784, 1000, 1000, 10)
+    rate_max: float = 0.3
+    beta: float = 0.9
+    thr: float = 1.0
+    sg_param: float = 25.0      # fast-sigmoid slope
+    n_classes: int = 10
+    seed_index: int = 2
+
+    def scaled(self, **kw) -> "DenseWorkload":
+        return dataclasses.replace(self, **kw)
+
+
+DSNN_C3 = DenseWorkload()
+
+
+def make_dense_inputs(w: DenseWorkload, seed: Optional[int] = None) -> dict:
+    """Bernoulli input spikes with a per-(sample, pixel) rate ~ U(0, rate_max)
+    drawn once and independent over t; He-uniform bf16 weights without bias;
+    uniform labels in 0..n_classes-1."""
+    seed = SEED_BASE + w.seed_index if seed is None else seed
+    g = _gen(seed)
+    k0 = w.sizes[0]
+    rate = w.rate_max * torch.rand((w.B, k0), generator=g, dtype=torch.float32)
+    u = torch.rand((w.T, w.B, k0), generator=g, dtype=torch.float32)
+    X = (u < rate.unsqueeze(0)).to(torch.bfloat16)
+    Ws = []
+    for fan_in, fan_out in zip(w.sizes[:-1], w.sizes[1:]):
+        bound = (6.0 / fan_in) ** 0.5
+        Wl = (2.0 * torch.rand((fan_out, fan_in), generator=g, dtype=torch.float32) - 1.0) * bound
+        Ws.append(Wl.to(torch.bfloat16))
+    labels = torch.randint(0, w.n_classes, (w.B,), generator=g, dtype=torch.int64).to(torch.int32)
+    return {"X": X, "W": Ws, "labels": labels}
