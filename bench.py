@@ -1,0 +1,459 @@
+"""Throughput of the fused LIF scan, forward + BPTT, on GB300.
+
+One step = the whole hot path over one batch: the Leaky forward scan (Eqs.
+3-4) and its BPTT reverse scan with the arctan surrogate, per-neuron beta and
+threshold gradients reduced over the batch.  Default workload: I[T=500,
+B=64, N=8192] bf16 storage with fp32 state, recompute-from-checkpoint BPTT.
+
+Prints one JSON line (rank 0).  `--impl reference` times the CPU oracle (the
+only other implementation of this path) on a bounded sample of the same
+workload instead.
+"""
+from __future__ import annotations
+
+import argparse
+import glob
+import hashlib
+import json
+import os
+import subprocess
+import sys
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "neuron-steps/sec (fwd+BPTT) on 1 GB300; achieved HBM GB/s vs roofline"
+UNIT = "neuron-steps/s"
+DEFAULT_WORKLOAD = "leaky_bf16_T500_B64_N8192"
+FALLBACK_HBM_GBS = 6800.0
+
+
+def parse():
+    p = argparse.ArgumentParser()
+    p.add_argument("--gpus", type=int, default=1)
+    p.add_argument("--steps", type=int, default=1000)
+    p.add_argument("--warmup", type=int, default=10)
+    p.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    p.add_argument("--workload", default=DEFAULT_WORKLOAD)
+    p.add_argument("--save", default=None, choices=[None, "mem", "recompute"])
+    p.add_argument("--no-e2e", action="store_true")
+    p.add_argument("--no-cpu-baseline", action="store_true")
+    p.add_argument("--cpu-seconds", type=float, default=15.0)
+    return p.parse_args()
+
+
+def workload(args):
+    from paper_2211_10725_gb300 import workloads as W
+    w = W.SCAN_WORKLOADS[args.workload]
+    if args.save:
+        w = w.scaled(save=args.save)
+    return w
+
+
+# ---------------------------------------------------------------------------
+# Bytes and peaks
+# ---------------------------------------------------------------------------
+
+def esize(dt):
+    return 4 if dt == "f32" else 2
+
+
+def algorithmic_bytes(w):
+    """Bytes per neuron-step the contract must touch (fwd, bwd).
+
+    Forward: read I, write spk (+ mem if requested).  Backward: read
+    grad_spk, read the cheaper saved state (I for recompute, mem (+spk for
+    half storage) for store), write grad_I.  Checkpoints, parameters and
+    reductions are excluded (they are overhead, not contract)."""
+    ei, eo = esize(w.in_dtype), esize(w.io_dtype)
+    fwd = ei + eo + (eo if (w.want_mem or w.save == "mem") else 0)
+    if w.neuron == "synaptic" and w.save == "mem":
+        fwd += 0
+    if w.save == "recompute":
+        bwd = eo + ei + eo
+    else:
+        bwd = eo + eo + eo + (eo if eo != 4 else 0)
+    return fwd, bwd
+
+
+def hbm_peak():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            v = float(json.load(f)["hbm_gbs"])
+        return v, "measured"
+    except Exception:
+        return FALLBACK_HBM_GBS, "fallback"
+
+
+def kernel_source_hash():
+    h = hashlib.sha256()
+    for f in sorted(glob.glob(os.path.join(ROOT, "paper_2211_10725_gb300", "csrc", "*"))):
+        with open(f, "rb") as fh:
+            h.update(os.path.basename(f).encode())
+            h.update(fh.read())
+    return h.hexdigest()[:16]
+
+
+def profiled_traffic(kernel_key, workload_name):
+    """DRAM bytes per launch from a committed ncu summary, valid only if the
+    kernel sources are unchanged since it was taken."""
+    path = os.path.join(ROOT, "profiles", "traffic.json")
+    try:
+        with open(path) as f:
+            data = json.load(f)
+        ent = data[workload_name][kernel_key]
+        if ent.get("source_hash") != kernel_source_hash():
+            return None
+        return float(ent["dram_bytes_per_launch"])
+    except Exception:
+        return None
+
+
+# ---------------------------------------------------------------------------
+# Clock sampling during the timed region
+# ---------------------------------------------------------------------------
+
+class ClockSampler:
+    QUERY = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+             "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+             "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index):
+        self.gpu = gpu_index
+        self.samples = []
+        self.proc = None
+        self.window = None
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.gpu), f"--query-gpu={self.QUERY}",
+                 "--format=csv,noheader,nounits", "-lms", "50"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            self.thread = threading.Thread(target=self._read, daemon=True)
+            self.thread.start()
+        except Exception:
+            self.proc = None
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.samples.append((time.time(), line.strip()))
+
+    def stop(self):
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except Exception:
+                self.proc.kill()
+
+    def summary(self, t0, t1):
+        rows = []
+        for ts, line in self.samples:
+            parts = [p.strip() for p in line.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                rows.append((ts, float(parts[1]), float(parts[2]), parts))
+            except ValueError:
+                continue
+        inside = [r for r in rows if t0 <= r[0] <= t1]
+        note = "sampled during the timed region"
+        if not inside and rows:
+            mid = 0.5 * (t0 + t1)
+            inside = sorted(rows, key=lambda r: abs(r[0] - mid))[:3]
+            note = "timed region shorter than the sampling period: nearest samples (warm-up)"
+        if not inside:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": [], "note": "no samples"}
+        sm = sorted(r[1] for r in inside)
+        reasons = set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for r in inside:
+            for name, val in zip(names, r[3][5:9]):
+                if val.strip().lower() == "active":
+                    reasons.add(name)
+        return {"sm_mhz": sm[len(sm) // 2], "sm_max_mhz": max(r[2] for r in inside),
+                "reasons": sorted(reasons), "samples": len(inside), "note": note}
+
+
+# ---------------------------------------------------------------------------
+# CPU oracle leg
+# ---------------------------------------------------------------------------
+
+def oracle_inputs(w, inp):
+    """Host arrays the oracle reads (converted once, outside any timing)."""
+    from oracle import snn_oracle as O
+    T, B, N = w.T, w.B, w.N
+    host = {"I": inp["I"].float().numpy().reshape(T, B * N),
+            "gs": inp["grad_spk"].float().numpy().reshape(T, B * N)}
+    for name, mode in (("beta", w.beta_mode), ("thr", w.thr_mode), ("alpha", w.alpha_mode)):
+        if name in inp:
+            host[name] = O.lane_param(inp[name].numpy(), B, N, mode, w.C, w.HW)
+    return host
+
+
+def oracle_step(w, host, lanes):
+    """One oracle fwd+bwd pass (float64, as it stands) over a lane sample."""
+    from oracle import snn_oracle as O
+    import numpy as np
+    I = host["I"][:, lanes].astype(np.float64)
+    gs = host["gs"][:, lanes].astype(np.float64)
+    beta, thr = host["beta"][lanes], host["thr"][lanes]
+    if w.neuron == "synaptic":
+        alpha = host["alpha"][lanes]
+        spk, mem, syn = O.synaptic_forward(I, alpha, beta, thr, w.reset)
+        O.synaptic_backward(mem, spk, syn, gs, alpha, beta, thr, w.reset, w.detach_reset,
+                            w.surrogate, w.sg_param)
+    else:
+        spk, mem = O.leaky_forward(I, beta, thr, w.reset)
+        O.leaky_backward(mem, spk, gs, beta, thr, w.reset, w.detach_reset, w.surrogate,
+                         w.sg_param)
+
+
+def time_oracle(w, inp, seconds):
+    """Time the oracle on a bounded lane sample sized for about `seconds`."""
+    import numpy as np
+    L = w.B * w.N
+    inp = oracle_inputs(w, inp)
+    n = min(L, 4096)
+    t0 = time.perf_counter()
+    oracle_step(w, inp, np.arange(n))
+    dt = time.perf_counter() - t0
+    n2 = int(min(L, 65536, max(n, n * seconds / max(dt, 1e-6))))
+    lanes = np.arange(n2)
+    t0 = time.perf_counter()
+    oracle_step(w, inp, lanes)
+    dt = time.perf_counter() - t0
+    return w.T * n2 / dt, n2, dt
+
+
+def run_reference(args):
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return
+    import numpy as np
+    from paper_2211_10725_gb300 import workloads as W
+    w = workload(args)
+    inp = oracle_inputs(w, W.make_scan_inputs(w))
+    L = w.B * w.N
+    # size one step's lane sample so that warm-up + steps take about 2 minutes
+    probe = min(L, 2048)
+    t0 = time.perf_counter()
+    oracle_step(w, inp, np.arange(probe))
+    per_lane = (time.perf_counter() - t0) / probe
+    total = max(1, args.steps + args.warmup)
+    n = int(max(64, min(L, 120.0 / total / per_lane)))
+    rng = np.random.default_rng(0)
+    samples = [np.sort(rng.choice(L, n, replace=False)) for _ in range(total)]
+    for i in range(args.warmup):
+        oracle_step(w, inp, samples[i])
+    t0 = time.perf_counter()
+    for i in range(args.steps):
+        oracle_step(w, inp, samples[args.warmup + i])
+    dt = time.perf_counter() - t0
+    value = w.T * n * args.steps / dt
+    line = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT,
+        "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": 1e3 * dt / args.steps, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": {"workload": w.name, "T": w.T, "B": w.B, "N": w.N,
+                   "sample_lanes_per_step": n},
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": 1, "kind": "oracle",
+                         "sample": f"{n} random lanes of {L} per step, all T={w.T} steps, "
+                                   f"float64 numpy oracle fwd+BPTT"},
+        "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+
+
+# ---------------------------------------------------------------------------
+# GPU leg
+# ---------------------------------------------------------------------------
+
+def run_ours(args):
+    import torch
+    import torch.distributed as dist
+
+    from paper_2211_10725_gb300 import snn
+    from paper_2211_10725_gb300 import workloads as W
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1:
+        dist.init_process_group("nccl")
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    w = workload(args)
+    # weak scaling: every rank scans its own batch of the same shape
+    inp = W.make_scan_inputs(w, seed=W.SEED_BASE + w.seed_index + 1000 * rank)
+    d = {k: v.to(dev) for k, v in inp.items()}
+    layer = snn.ScanLayer(w, device=dev)
+    stream = torch.cuda.current_stream(dev)
+
+    def step():
+        layer.forward(d["I"], d["beta"], d["thr"], d.get("alpha"))
+        layer.backward(d["I"], d["beta"], d["thr"], d["grad_spk"], alpha=d.get("alpha"),
+                       want_state_grads=False)
+
+    for _ in range(args.warmup):
+        step()
+    torch.cuda.synchronize()
+    status = layer.status()
+    if status != 0:
+        raise RuntimeError(f"kernel status {status} after warm-up")
+
+    sampler = ClockSampler(local)
+    if rank == 0:
+        sampler.start()
+        time.sleep(0.3)
+    K = args.steps
+    ev = [torch.cuda.Event(enable_timing=True) for _ in range(3 * K + 1)]
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize()
+    t_wall0 = time.time()
+    ev[0].record(stream)
+    for k in range(K):
+        layer.forward(d["I"], d["beta"], d["thr"], d.get("alpha"))
+        ev[3 * k + 1].record(stream)
+        layer.backward(d["I"], d["beta"], d["thr"], d["grad_spk"], alpha=d.get("alpha"),
+                       want_state_grads=False)
+        ev[3 * k + 2].record(stream)
+        ev[3 * k + 3].record(stream)
+    torch.cuda.synchronize()
+    t_wall1 = time.time()
+    if world > 1:
+        dist.barrier()
+    if rank == 0:
+        time.sleep(0.2)
+        sampler.stop()
+    total_ms = ev[0].elapsed_time(ev[3 * K])
+    fwd_ms = sum(ev[3 * k].elapsed_time(ev[3 * k + 1]) for k in range(K)) / K
+    bwd_ms = sum(ev[3 * k + 1].elapsed_time(ev[3 * k + 2]) for k in range(K)) / K
+    if world > 1:
+        t = torch.tensor([total_ms], device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        total_ms = float(t.item())
+    status = layer.status()
+    if status != 0:
+        raise RuntimeError(f"kernel status {status} in the timed region")
+
+    ns_per_step = w.T * w.B * w.N
+    value = world * ns_per_step * K / (total_ms * 1e-3)
+
+    # end to end through the public API with host buffers
+    e2e = None
+    if not args.no_e2e:
+        e2e = run_e2e(args, w, inp, layer, dev, world)
+
+    if rank != 0:
+        if world > 1:
+            dist.destroy_process_group()
+        return
+    fwd_b, bwd_b = algorithmic_bytes(w)
+    peak, peak_kind = hbm_peak()
+    achieved_bwd = bwd_b * ns_per_step / (bwd_ms * 1e-3) / 1e9
+    achieved_path = (fwd_b + bwd_b) * ns_per_step / (total_ms / K * 1e-3) / 1e9
+    kernel_key = f"scan_bwd_staged[{w.neuron},{w.save}]"
+    traffic = profiled_traffic(kernel_key, w.name)
+    clocks = sampler.summary(t_wall0, t_wall1)
+    grads = 2
+    launches_per_step = 2 + sum(1 if m != "scalar" else 2 for m in (w.beta_mode, w.thr_mode)[:grads])
+    cpu = None
+    if not args.no_cpu_baseline and world == 1:
+        v, n, dt = time_oracle(w, inp, args.cpu_seconds)
+        cpu = {"value": v, "unit": UNIT, "cores": 1, "kind": "oracle",
+               "sample": f"first {n} of {w.B * w.N} lanes, all T={w.T} steps, float64 numpy "
+                         f"oracle fwd+BPTT, {dt:.1f} s"}
+    line = {
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": K,
+        "warmup": args.warmup, "ms_per_step": total_ms / K, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
+        "config": {"workload": w.name, "T": w.T, "B": w.B, "N": w.N, "neuron": w.neuron,
+                   "storage": w.io_dtype, "save": w.save, "ckpt_every": w.ckpt_every,
+                   "surrogate": w.surrogate, "params": f"beta {w.beta_mode}, thr {w.thr_mode}",
+                   "l2": "inputs larger than L2 (each [T,B,N] tensor >> 129 MB), no flush",
+                   "parallelism": f"replicas x{world}" if world > 1 else "single GPU"},
+        "roofline": {"bound": "hbm", "kernel": "scan_bwd_staged (+ per-neuron reductions)",
+                     "achieved": achieved_bwd, "peak": peak, "unit": "GB/s",
+                     "frac": achieved_bwd / peak, "peak_kind": peak_kind,
+                     "algorithmic_bytes_per_ns": bwd_b,
+                     "traffic": traffic, "fwd_ms": fwd_ms, "bwd_ms": bwd_ms,
+                     "path_achieved": achieved_path, "path_frac": achieved_path / peak,
+                     "path_bytes_per_ns": fwd_b + bwd_b},
+        "clocks": clocks,
+        "gpu_launches": launches_per_step * K,
+        "cpu_baseline": cpu,
+        "e2e": e2e,
+    }
+    print(json.dumps(line), flush=True)
+    if world > 1:
+        dist.destroy_process_group()
+
+
+def run_e2e(args, w, inp, layer, dev, world):
+    """Same metric through the public API, with the step's inputs copied from
+    pinned host memory and its results read back to pinned host memory."""
+    import torch
+    import torch.distributed as dist
+    hI = inp["I"].pin_memory()
+    hG = inp["grad_spk"].pin_memory()
+    dI = torch.empty_like(hI, device=dev)
+    dG = torch.empty_like(hG, device=dev)
+    beta, thr = inp["beta"].to(dev), inp["thr"].to(dev)
+    alpha = inp["alpha"].to(dev) if "alpha" in inp else None
+    out_spk = torch.empty_like(layer.spk, device="cpu").pin_memory()
+    out_gI = torch.empty_like(layer.grad_I, device="cpu").pin_memory()
+    out_gb = torch.empty_like(layer.grad_beta, device="cpu").pin_memory()
+    out_gt = torch.empty_like(layer.grad_thr, device="cpu").pin_memory()
+    stream = torch.cuda.current_stream(dev)
+
+    def step():
+        dI.copy_(hI, non_blocking=True)
+        dG.copy_(hG, non_blocking=True)
+        layer.forward(dI, beta, thr, alpha)
+        layer.backward(dI, beta, thr, dG, alpha=alpha, want_state_grads=False)
+        out_spk.copy_(layer.spk, non_blocking=True)
+        out_gI.copy_(layer.grad_I, non_blocking=True)
+        out_gb.copy_(layer.grad_beta, non_blocking=True)
+        out_gt.copy_(layer.grad_thr, non_blocking=True)
+
+    K = max(3, min(args.steps, 50))
+    for _ in range(3):
+        step()
+    torch.cuda.synchronize()
+    if world > 1:
+        dist.barrier()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(K):
+        step()
+    e1.record(stream)
+    torch.cuda.synchronize()
+    ms = e0.elapsed_time(e1)
+    if world > 1:
+        t = torch.tensor([ms], device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms = float(t.item())
+    nb = lambda t: t.numel() * t.element_size()
+    return {"value": world * w.T * w.B * w.N * K / (ms * 1e-3), "unit": UNIT,
+            "h2d_bytes_per_step": nb(hI) + nb(hG),
+            "d2h_bytes_per_step": nb(out_spk) + nb(out_gI) + nb(out_gb) + nb(out_gt),
+            "steps": K}
+
+
+def main():
+    args = parse()
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_ours(args)
+
+
+if __name__ == "__main__":
+    main()

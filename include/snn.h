@@ -1,0 +1,231 @@
+/*
+ * snn.h — C ABI of libsnn: the fused temporal scan of spiking-neuron state
+ * equations on one GPU (sm_103a), forward over T steps and the BPTT reverse
+ * scan with a surrogate gradient, plus the dense input-current GEMM.
+ *
+ * Method: arXiv 2211.10725, Sec. III-A/III-B.
+ *   Eq. (3)      z_t = 1 if u_t > u_thr else 0 (strict).
+ *   Eq. (4)      Leaky:     u_t = beta*u_{t-1} + I_t - z_{t-1}*u_thr
+ *   Eqs. (5)(6)  Synaptic:  i_t = alpha*i_{t-1} + I_t,
+ *                           u_t = beta*u_{t-1} + i_t - z_{t-1}*u_thr
+ *   Eqs. (8)(9)  fast-sigmoid surrogate for dz/du (arctan is the other choice)
+ *   Sec. II-A/B  BPTT over the unrolled graph.
+ * I_t = w x_t is the input current; the (1-beta) factor of Eq. (2) is absorbed
+ * into it.  Reset-to-zero (u_t = beta*(1-z_{t-1})*u_{t-1} + I_t, clears only u
+ * in the Synaptic neuron) and "no reset" are extensions the paper names but
+ * does not write out.
+ *
+ * Conventions shared by every entry point
+ * ---------------------------------------
+ * - Tensors of a scan are [T, B, N] row-major with t outermost: lane
+ *   l = b*N + n, element (t, l) at offset t*B*N + l.  Per-lane states and
+ *   their gradients (mem0, syn0, mem_final, grad_mem0, ...) are fp32 [B, N].
+ * - Every pointer argument is a DEVICE pointer unless stated, owned by the
+ *   caller; the library allocates nothing and keeps no state between calls.
+ *   Outputs are overwritten, never accumulated into.
+ * - Calls are asynchronous on `stream` and never synchronise it (except
+ *   snn_workspace_status).  Arguments are checked before anything is
+ *   launched; a failed check returns an error code and launches nothing.
+ * - Device pointers must be 16-byte aligned (SNN_ERR_ALIGNMENT otherwise).
+ *   Shapes whose per-step row (B*N*element size) is a multiple of 16 bytes
+ *   take the TMA-staged kernels; any other shape takes a plain per-lane
+ *   kernel with identical arithmetic.
+ * - Spin-waits inside kernels are bounded (snn_scan_desc.wait_limit_ns); a
+ *   kernel that gives up records SNN_ERR_TIMEOUT in the workspace status word
+ *   and returns.  snn_workspace_status reports it.
+ */
+#ifndef SNN_H_
+#define SNN_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+#if defined(__GNUC__)
+#pragma GCC visibility push(default)
+#endif
+
+/* Same object as cudaStream_t; NULL is the legacy default stream. */
+typedef struct CUstream_st* snn_stream_t;
+
+typedef enum {
+  SNN_OK = 0,
+  SNN_ERR_INVALID_ARG = 1, /* null/inconsistent argument or out-of-range enum  */
+  SNN_ERR_ALIGNMENT = 2,   /* a device pointer is not 16-byte aligned          */
+  SNN_ERR_UNSUPPORTED = 3, /* valid request that this build does not implement */
+  SNN_ERR_WORKSPACE = 4,   /* workspace missing or smaller than required       */
+  SNN_ERR_CUDA = 5,        /* a CUDA runtime call or kernel launch failed      */
+  SNN_ERR_TIMEOUT = 6      /* a bounded in-kernel wait gave up                 */
+} snn_status_t;
+
+typedef enum { SNN_F32 = 0, SNN_BF16 = 1, SNN_F16 = 2 } snn_dtype_t;
+
+typedef enum {
+  SNN_RESET_SUBTRACT = 0, /* Eq. (4): - z_{t-1} * u_thr                       */
+  SNN_RESET_ZERO = 1,     /* u_t = beta*(1 - z_{t-1})*u_{t-1} + input         */
+  SNN_RESET_NONE = 2      /* no reset term                                    */
+} snn_reset_t;
+
+typedef enum {
+  SNN_SG_FAST_SIGMOID = 0, /* dz/du <- 1/(1 + k|u-thr|)^2, k = sg_param (Eq. 9 at k=1) */
+  SNN_SG_ATAN = 1          /* dz/du <- (a/2)/(1 + (pi*a*(u-thr)/2)^2), a = sg_param  */
+} snn_surrogate_t;
+
+typedef enum {
+  SNN_P_SCALAR = 0,     /* one value                                           */
+  SNN_P_PER_NEURON = 1, /* [N], indexed by n                                   */
+  SNN_P_PER_CHANNEL = 2 /* [C], channel of neuron n is (n / HW) % C            */
+} snn_pmode_t;
+
+typedef enum {
+  SNN_SAVE_MEM = 0,      /* BPTT reads the stored mem (and spk) traces          */
+  SNN_SAVE_RECOMPUTE = 1 /* BPTT recomputes u from I and fp32 checkpoints taken
+                            every ckpt_every steps by the forward              */
+} snn_save_t;
+
+/* Debug flags (snn_scan_desc.debug_flags); 0 in normal use. */
+#define SNN_DEBUG_PRODUCER_IDLE 1u /* staged kernels issue no copy, so every
+                                      consumer wait runs out: exercises the
+                                      timeout path without any fault          */
+#define SNN_DEBUG_FORCE_PLAIN 2u   /* take the plain per-lane kernels even
+                                      where the staged ones apply             */
+
+typedef struct snn_scan_desc {
+  int64_t T, B, N;       /* time steps, batch, neurons per sample (C*H*W maps) */
+  int64_t C, HW;         /* per-channel parameters: channel = (n / HW) % C     */
+  int32_t in_dtype;      /* snn_dtype_t of I                                   */
+  int32_t io_dtype;      /* of spk, mem, syn, grad_spk, grad_mem, grad_I       */
+  int32_t reset;         /* snn_reset_t                                        */
+  int32_t detach_reset;  /* 1: z_{t-1} in the reset term is a constant in BPTT */
+  int32_t surrogate;     /* snn_surrogate_t                                    */
+  float sg_param;        /* fast-sigmoid slope k, or arctan alpha              */
+  int32_t beta_mode, thr_mode, alpha_mode; /* snn_pmode_t                      */
+  int32_t save;          /* snn_save_t                                         */
+  int32_t ckpt_every;    /* K >= 1 for SNN_SAVE_RECOMPUTE                      */
+  int32_t reserved0;     /* must be 0                                          */
+  int64_t wait_limit_ns; /* bound on each in-kernel wait; 0 = 2 s              */
+  uint32_t debug_flags;  /* SNN_DEBUG_*                                        */
+  uint32_t reserved1;    /* must be 0                                          */
+} snn_scan_desc;
+
+/* Human-readable name of a status code (static string, never NULL). */
+const char* snn_status_string(snn_status_t status);
+
+/* Library version, as 10000*major + 100*minor + patch. */
+int snn_version(void);
+
+/* sizeof(snn_scan_desc) as compiled into the library (ABI check). */
+size_t snn_scan_desc_size(void);
+
+/* Bytes of device workspace every scan call of `desc` needs (a status word
+ * plus per-lane parameter-gradient partials).  0 if desc is invalid. */
+size_t snn_scan_workspace_bytes(const snn_scan_desc* desc);
+
+/* Number of fp32 elements of the checkpoint buffer for SNN_SAVE_RECOMPUTE:
+ * (ceil(T/K) - 1) * B*N for Leaky, twice that for Synaptic (u then i per
+ * checkpoint).  0 for SNN_SAVE_MEM or an invalid desc. */
+int64_t snn_scan_ckpt_elems(const snn_scan_desc* desc, int synaptic);
+
+/* Zero a workspace (its status word included); asynchronous on stream.
+ * Call once after allocating it. */
+snn_status_t snn_workspace_init(void* ws, size_t ws_bytes, snn_stream_t stream);
+
+/* Synchronise stream, return the sticky status recorded by kernels in ws
+ * (SNN_OK or SNN_ERR_TIMEOUT) and clear it. */
+snn_status_t snn_workspace_status(void* ws, snn_stream_t stream);
+
+/*
+ * Leaky LIF forward, Eqs. (3)-(4), over t = 0..T-1.
+ *   I        [T,B,N] in_dtype            input current w x_t
+ *   beta,thr fp32, shape per beta_mode/thr_mode
+ *   mem0     fp32 [B,N] or NULL          u_{-1}; NULL means u_{-1}=0, z_{-1}=0,
+ *                                        else z_{-1} = [mem0 > thr]
+ *   spk      [T,B,N] io_dtype  (out)     z_t in {0,1}
+ *   mem      [T,B,N] io_dtype  (out)     u_t; required for SNN_SAVE_MEM, else
+ *                                        optional (NULL = not written)
+ *   ckpt     fp32 (out)                  SNN_SAVE_RECOMPUTE: u at the end of every
+ *                                        K-step segment but the last; else NULL
+ *   mem_final fp32 [B,N] (out) or NULL   u_{T-1}
+ *   ws       workspace of snn_scan_workspace_bytes(desc) bytes
+ * State is kept in fp32; the step is evaluated as Eq. (4) is written:
+ * (beta*u_{t-1} + I_t) - z_{t-1}*thr, each operation rounded to nearest.
+ */
+snn_status_t snn_leaky_fwd(const snn_scan_desc* desc, const void* I, const float* beta,
+                           const float* thr, const float* mem0, void* spk, void* mem,
+                           float* ckpt, float* mem_final, void* ws, size_t ws_bytes,
+                           snn_stream_t stream);
+
+/*
+ * Leaky LIF BPTT (Sec. II-A/B) with the surrogate of Sec. III-B.
+ * Inputs of the saved forward:
+ *   SNN_SAVE_MEM:       mem [T,B,N] io_dtype; spk [T,B,N] io_dtype, needed
+ *                       when io_dtype is not fp32 (a rounded mem cannot give
+ *                       back the spike decision), may be NULL for fp32.
+ *   SNN_SAVE_RECOMPUTE: I [T,B,N] in_dtype and ckpt from snn_leaky_fwd.
+ *   beta, thr, mem0 as in the forward.
+ * Upstream gradients:
+ *   grad_spk [T,B,N] io_dtype            dL/dz_t
+ *   grad_mem [T,B,N] io_dtype or NULL    dL/du_t through the mem output
+ *   grad_mem_final fp32 [B,N] or NULL    dL/du_{T-1} through mem_final
+ * Outputs:
+ *   grad_I   [T,B,N] io_dtype            dL/dI_t
+ *   grad_beta, grad_thr fp32, parameter's shape, or NULL; summed over t and
+ *            over the lanes that share the parameter
+ *   grad_mem0 fp32 [B,N] or NULL         dL/du_{-1}
+ * Reverse recurrence, with s_t = surrogate(u_t - thr):
+ *   dz_t = grad_spk_t + [not detach] * (d u_{t+1}/d z_t) * du_{t+1}
+ *   du_t = grad_mem_t + (d u_{t+1}/d u_t) * du_{t+1} + s_t * dz_t
+ * where d u_{t+1}/d u_t = beta (subtract/none) or beta*(1-z_t) (zero) and
+ * d u_{t+1}/d z_t = -thr (subtract), -beta*u_t (zero), 0 (none).
+ * Parameter sums are accumulated in fp32 per lane and reduced across lanes
+ * in fp64 in a fixed order (deterministic).
+ */
+snn_status_t snn_leaky_bwd(const snn_scan_desc* desc, const void* I, const float* ckpt,
+                           const void* mem, const void* spk, const float* beta,
+                           const float* thr, const float* mem0, const void* grad_spk,
+                           const void* grad_mem, const float* grad_mem_final, void* grad_I,
+                           float* grad_beta, float* grad_thr, float* grad_mem0, void* ws,
+                           size_t ws_bytes, snn_stream_t stream);
+
+/*
+ * Current-based (Synaptic) LIF forward, Eqs. (3), (5), (6).  As
+ * snn_leaky_fwd, plus:
+ *   alpha    fp32, shape per alpha_mode  synaptic decay
+ *   syn0     fp32 [B,N] or NULL          i_{-1} (NULL means 0)
+ *   syn      [T,B,N] io_dtype (out) or NULL   i_t; needed by a SNN_SAVE_MEM
+ *                                        backward that asks for grad_alpha
+ *   syn_final fp32 [B,N] (out) or NULL   i_{T-1}
+ * ckpt holds u then i for every checkpoint (2*B*N fp32 each).
+ */
+snn_status_t snn_synaptic_fwd(const snn_scan_desc* desc, const void* I, const float* alpha,
+                              const float* beta, const float* thr, const float* mem0,
+                              const float* syn0, void* spk, void* mem, void* syn,
+                              float* ckpt, float* mem_final, float* syn_final, void* ws,
+                              size_t ws_bytes, snn_stream_t stream);
+
+/*
+ * Synaptic BPTT.  As snn_leaky_bwd, plus:
+ *   syn      [T,B,N] io_dtype            SNN_SAVE_MEM with grad_alpha != NULL
+ *   grad_syn_final fp32 [B,N] or NULL    dL/di_{T-1}
+ *   grad_alpha fp32 or NULL; grad_syn0 fp32 [B,N] or NULL
+ *   di_t = alpha*di_{t+1} + du_t,  grad_I_t = di_t.
+ */
+snn_status_t snn_synaptic_bwd(const snn_scan_desc* desc, const void* I, const float* ckpt,
+                              const void* mem, const void* spk, const void* syn,
+                              const float* alpha, const float* beta, const float* thr,
+                              const float* mem0, const float* syn0, const void* grad_spk,
+                              const void* grad_mem, const float* grad_mem_final,
+                              const float* grad_syn_final, void* grad_I, float* grad_alpha,
+                              float* grad_beta, float* grad_thr, float* grad_mem0,
+                              float* grad_syn0, void* ws, size_t ws_bytes,
+                              snn_stream_t stream);
+
+#if defined(__GNUC__)
+#pragma GCC visibility pop
+#endif
+#ifdef __cplusplus
+}
+#endif
+#endif /* SNN_H_ */

@@ -1,0 +1,12 @@
+// BPTT launchers for the Leaky neuron (store and recompute variants).
+#include "scan_dispatch.cuh"
+
+namespace snn {
+
+cudaError_t launch_scan_bwd_leaky(ScanArgs a, bool recompute, int in_dt, int io_dt, bool staged,
+                                  cudaStream_t stream) {
+  if (recompute) SNN_DTYPE_DISPATCH(in_dt, io_dt, return (bwd_t<false, true, TI, TO>(a, staged, stream)));
+  SNN_DTYPE_DISPATCH(in_dt, io_dt, return (bwd_t<false, false, TI, TO>(a, staged, stream)));
+}
+
+}  // namespace snn

@@ -1,0 +1,76 @@
+// Templated launchers for the scan kernels; each .cu file instantiates one
+// family so the library compiles in parallel.
+#pragma once
+
+#include "scan_host.cuh"
+
+namespace snn {
+
+template <bool SYN, typename TI, typename TO>
+cudaError_t fwd_t(ScanArgs a, bool staged, cudaStream_t st) {
+  if (staged && a.L > 0) {
+    const void* k = (const void*)scan_fwd_staged<SYN, TI, TO>;
+    StagedPlan p;
+    if (plan_staged(k, a.L, a.T, (int)sizeof(TI), 0, &p)) {
+      a.lanes_per_cta = p.lanes_per_cta;
+      a.stages = p.stages;
+      a.stage_bytes = p.stage_bytes;
+      scan_fwd_staged<SYN, TI, TO><<<(unsigned)p.grid, p.threads, p.smem, st>>>(a);
+      return cudaGetLastError();
+    }
+  }
+  if (a.L == 0) return cudaSuccess;
+  scan_fwd_plain<SYN, TI, TO><<<(unsigned)ceil_div(a.L, 256), 256, 0, st>>>(a);
+  return cudaGetLastError();
+}
+
+template <bool SYN, bool RECOMP, typename TI, typename TO>
+cudaError_t bwd_t(ScanArgs a, bool staged, cudaStream_t st) {
+  if (staged && a.L > 0) {
+    const void* k = (const void*)scan_bwd_staged<SYN, RECOMP, TI, TO>;
+    int per_lane, seg;
+    int64_t items;
+    if (RECOMP) {
+      const int fwd_item = (int)sizeof(TI) + 4 * (SYN ? 2 : 1);
+      const int bwd_item = (int)sizeof(TO) * (a.gm ? 2 : 1);
+      per_lane = fwd_item > bwd_item ? fwd_item : bwd_item;
+      seg = VEC * 4 * a.K * (SYN ? 2 : 1);
+      items = 2 * a.T;
+    } else {
+      const int n = 2 + (sizeof(TO) != 4 ? 1 : 0) + ((SYN && a.part_alpha) ? 1 : 0) + (a.gm ? 1 : 0);
+      per_lane = n * (int)sizeof(TO);
+      seg = 0;
+      items = a.T;
+    }
+    StagedPlan p;
+    if (plan_staged(k, a.L, items, per_lane, seg, &p)) {
+      a.lanes_per_cta = p.lanes_per_cta;
+      a.stages = p.stages;
+      a.stage_bytes = p.stage_bytes;
+      scan_bwd_staged<SYN, RECOMP, TI, TO><<<(unsigned)p.grid, p.threads, p.smem, st>>>(a);
+      return cudaGetLastError();
+    }
+  }
+  if (a.L == 0) return cudaSuccess;
+  const int threads = 128;
+  const size_t smem = RECOMP ? (size_t)a.K * threads * 4 * (SYN ? 2 : 1) : 0;
+  const void* k = (const void*)scan_bwd_plain<SYN, RECOMP, TI, TO>;
+  cudaError_t e = ensure_smem(k, smem);
+  if (e != cudaSuccess) return e;
+  scan_bwd_plain<SYN, RECOMP, TI, TO><<<(unsigned)ceil_div(a.L, threads), threads, smem, st>>>(a);
+  return cudaGetLastError();
+}
+
+// dtype codes (snn_dtype_t): 0 f32, 1 bf16, 2 f16.  Instantiated pairs
+// (in, io): (f32,f32) (bf16,bf16) (f16,f16) (f32,bf16) (f32,f16).
+#define SNN_DTYPE_DISPATCH(IN_DT, IO_DT, CALL)                                   \
+  do {                                                                           \
+    if ((IN_DT) == 0 && (IO_DT) == 0) { using TI = float; using TO = float; CALL; } \
+    if ((IN_DT) == 1 && (IO_DT) == 1) { using TI = __nv_bfloat16; using TO = __nv_bfloat16; CALL; } \
+    if ((IN_DT) == 2 && (IO_DT) == 2) { using TI = __half; using TO = __half; CALL; } \
+    if ((IN_DT) == 0 && (IO_DT) == 1) { using TI = float; using TO = __nv_bfloat16; CALL; } \
+    if ((IN_DT) == 0 && (IO_DT) == 2) { using TI = float; using TO = __half; CALL; } \
+    return cudaErrorNotSupported;                                                \
+  } while (0)
+
+}  // namespace snn

@@ -1,0 +1,148 @@
+// Host-side launch planning shared by the scan translation units.
+#pragma once
+
+#include <cuda_runtime.h>
+
+#include <map>
+#include <mutex>
+#include <tuple>
+
+#include "scan_kernels.cuh"
+
+namespace snn {
+
+inline int64_t ceil_div(int64_t a, int64_t b) { return (a + b - 1) / b; }
+inline int64_t round_up(int64_t a, int64_t b) { return ceil_div(a, b) * b; }
+
+struct DeviceInfo {
+  int sms = 0;
+  int smem_per_sm = 0;
+  int smem_optin = 0;
+};
+
+inline cudaError_t device_info(DeviceInfo* out) {
+  static std::mutex mu;
+  static std::map<int, DeviceInfo> cache;
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  std::lock_guard<std::mutex> g(mu);
+  auto it = cache.find(dev);
+  if (it != cache.end()) {
+    *out = it->second;
+    return cudaSuccess;
+  }
+  DeviceInfo d;
+  if ((e = cudaDeviceGetAttribute(&d.sms, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess) return e;
+  if ((e = cudaDeviceGetAttribute(&d.smem_per_sm, cudaDevAttrMaxSharedMemoryPerMultiprocessor, dev)) != cudaSuccess)
+    return e;
+  if ((e = cudaDeviceGetAttribute(&d.smem_optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev)) != cudaSuccess)
+    return e;
+  cache[dev] = d;
+  *out = d;
+  return cudaSuccess;
+}
+
+// Raise a kernel's dynamic shared-memory limit once per (device, kernel).
+inline cudaError_t ensure_smem(const void* kernel, size_t bytes) {
+  static std::mutex mu;
+  static std::map<std::pair<int, const void*>, size_t> done;
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  std::lock_guard<std::mutex> g(mu);
+  size_t& cur = done[{dev, kernel}];
+  if (bytes <= cur || bytes <= 48 * 1024) return cudaSuccess;
+  e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)bytes);
+  if (e == cudaSuccess) cur = bytes;
+  return e;
+}
+
+struct StagedPlan {
+  int lanes_per_cta = 0;
+  int threads = 0;  // consumer warps * 32 + one producer warp
+  int stages = 0;
+  int stage_bytes = 0;
+  size_t smem = 0;
+  int64_t grid = 0;
+};
+
+// Choose a staged launch for L lanes: all CTAs of a wave resident at once
+// (grid = SMs x CTAs-per-SM x waves, lanes split evenly, strip a multiple of
+// 8 lanes so every row copy starts 16-byte aligned), the deepest ring that
+// fits next to the per-thread replay buffer.  Returns false if nothing fits.
+//   stage_bytes_per_lane: bytes one lane contributes to the largest item
+//   seg_bytes_per_thread: replay buffer bytes per consumer thread
+inline bool plan_staged(const void* kernel, int64_t L, int64_t items, int stage_bytes_per_lane,
+                        int seg_bytes_per_thread, StagedPlan* plan) {
+  static std::mutex mu;
+  static std::map<std::tuple<int, const void*, int64_t, int64_t, int, int>, StagedPlan> cache;
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return false;
+  const auto key = std::make_tuple(dev, kernel, L, items, stage_bytes_per_lane, seg_bytes_per_thread);
+  {
+    std::lock_guard<std::mutex> g(mu);
+    auto it = cache.find(key);
+    if (it != cache.end()) {
+      *plan = it->second;
+      return true;
+    }
+  }
+  DeviceInfo d;
+  if (device_info(&d) != cudaSuccess) return false;
+  cudaFuncAttributes fa;
+  if (cudaFuncGetAttributes(&fa, kernel) != cudaSuccess) return false;
+  const int min_stages = (int)(items < 3 ? (items < 1 ? 1 : items) : 3);
+  for (int waves = 1; waves <= 64; ++waves) {
+    for (int cps = 2; cps >= 1; --cps) {
+      const int64_t ctas = (int64_t)d.sms * cps * waves;
+      const int64_t lpc = round_up(ceil_div(L, ctas), 8);
+      const int64_t cthreads = round_up(ceil_div(lpc, VEC), 32);
+      const int threads = (int)cthreads + 32;
+      if (threads > 1024) continue;
+      if ((int64_t)threads * fa.numRegs * cps > 65536) continue;
+      const int64_t stage_bytes = round_up(lpc * stage_bytes_per_lane, 128);
+      const int64_t seg_bytes = cthreads * seg_bytes_per_thread;
+      const int64_t budget = (int64_t)d.smem_per_sm / cps - 1024 - (int64_t)fa.sharedSizeBytes;
+      const int64_t avail = (budget < d.smem_optin ? budget : d.smem_optin) - kBarrierBytes - seg_bytes;
+      if (avail < stage_bytes * min_stages) continue;
+      int64_t stages = avail / stage_bytes;
+      if (stages > kMaxStages) stages = kMaxStages;
+      if (stages > items && items > 0) stages = items;
+      if (stages < 1) stages = 1;
+      StagedPlan p;
+      p.lanes_per_cta = (int)lpc;
+      p.threads = threads;
+      p.stages = (int)stages;
+      p.stage_bytes = (int)stage_bytes;
+      p.smem = (size_t)(kBarrierBytes + stages * stage_bytes + seg_bytes);
+      p.grid = ceil_div(L, lpc);
+      if (ensure_smem(kernel, p.smem) != cudaSuccess) continue;
+      int nb = 0;
+      if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&nb, kernel, threads, p.smem) != cudaSuccess)
+        continue;
+      if (nb < cps) continue;
+      std::lock_guard<std::mutex> g(mu);
+      cache[key] = p;
+      *plan = p;
+      return true;
+    }
+  }
+  return false;
+}
+
+// Entry points of the per-translation-unit dispatchers.  dtype codes follow
+// snn_dtype_t; `staged` selects the TMA-staged kernels (the caller checked
+// row alignment).  Return cudaErrorNotSupported for a combination that is
+// not instantiated.
+cudaError_t launch_scan_fwd(ScanArgs a, bool synaptic, int in_dt, int io_dt, bool staged,
+                            cudaStream_t stream);
+cudaError_t launch_scan_bwd_leaky(ScanArgs a, bool recompute, int in_dt, int io_dt, bool staged,
+                                  cudaStream_t stream);
+cudaError_t launch_scan_bwd_synaptic(ScanArgs a, bool recompute, int in_dt, int io_dt,
+                                     bool staged, cudaStream_t stream);
+cudaError_t launch_param_reduce(const float* part, int64_t B, int64_t N, int64_t C, int64_t HW,
+                                int mode, double* scratch, int scratch_len, float* out,
+                                cudaStream_t stream);
+
+}  // namespace snn

@@ -1,0 +1,272 @@
+"""ctypes binding of libsnn (include/snn.h).
+
+The functions named like the C entry points marshal torch tensors into
+device pointers and call the library; every step of the scan runs in the
+library's CUDA kernels.  PyTorch only allocates memory and supplies the
+current stream.  If the library is missing the binding raises: there is no
+fallback implementation.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import re
+from typing import Optional
+
+import torch
+
+from . import workloads as W
+
+_PKG = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_PKG, "_lib", "libsnn.so")
+HEADER = os.path.join(os.path.dirname(_PKG), "include", "snn.h")
+
+SNN_OK = 0
+STATUS_NAMES = {0: "SNN_OK", 1: "SNN_ERR_INVALID_ARG", 2: "SNN_ERR_ALIGNMENT",
+                3: "SNN_ERR_UNSUPPORTED", 4: "SNN_ERR_WORKSPACE", 5: "SNN_ERR_CUDA",
+                6: "SNN_ERR_TIMEOUT"}
+DTYPE_CODE = {W.F32: 0, W.BF16: 1, W.F16: 2}
+RESET_CODE = {"subtract": 0, "zero": 1, "none": 2}
+SG_CODE = {"fast_sigmoid": 0, "atan": 1}
+PMODE_CODE = {"scalar": 0, "per_neuron": 1, "per_channel": 2}
+SAVE_CODE = {"mem": 0, "recompute": 1}
+DEBUG_PRODUCER_IDLE = 1
+DEBUG_FORCE_PLAIN = 2
+
+
+class SnnError(RuntimeError):
+    def __init__(self, status: int, where: str):
+        self.status = status
+        super().__init__(f"{where}: {STATUS_NAMES.get(status, status)}")
+
+
+class ScanDesc(ctypes.Structure):
+    """Mirror of snn_scan_desc."""
+    _fields_ = [
+        ("T", ctypes.c_int64), ("B", ctypes.c_int64), ("N", ctypes.c_int64),
+        ("C", ctypes.c_int64), ("HW", ctypes.c_int64),
+        ("in_dtype", ctypes.c_int32), ("io_dtype", ctypes.c_int32),
+        ("reset", ctypes.c_int32), ("detach_reset", ctypes.c_int32),
+        ("surrogate", ctypes.c_int32), ("sg_param", ctypes.c_float),
+        ("beta_mode", ctypes.c_int32), ("thr_mode", ctypes.c_int32),
+        ("alpha_mode", ctypes.c_int32), ("save", ctypes.c_int32),
+        ("ckpt_every", ctypes.c_int32), ("reserved0", ctypes.c_int32),
+        ("wait_limit_ns", ctypes.c_int64), ("debug_flags", ctypes.c_uint32),
+        ("reserved1", ctypes.c_uint32),
+    ]
+
+
+_P = ctypes.c_void_p
+_SIGS = {
+    "snn_status_string": ([ctypes.c_int], ctypes.c_char_p),
+    "snn_version": ([], ctypes.c_int),
+    "snn_scan_desc_size": ([], ctypes.c_size_t),
+    "snn_scan_workspace_bytes": ([ctypes.POINTER(ScanDesc)], ctypes.c_size_t),
+    "snn_scan_ckpt_elems": ([ctypes.POINTER(ScanDesc), ctypes.c_int], ctypes.c_int64),
+    "snn_workspace_init": ([_P, ctypes.c_size_t, _P], ctypes.c_int),
+    "snn_workspace_status": ([_P, _P], ctypes.c_int),
+    "snn_leaky_fwd": ([ctypes.POINTER(ScanDesc)] + [_P] * 9 + [ctypes.c_size_t, _P], ctypes.c_int),
+    "snn_leaky_bwd": ([ctypes.POINTER(ScanDesc)] + [_P] * 15 + [ctypes.c_size_t, _P], ctypes.c_int),
+    "snn_synaptic_fwd": ([ctypes.POINTER(ScanDesc)] + [_P] * 13 + [ctypes.c_size_t, _P], ctypes.c_int),
+    "snn_synaptic_bwd": ([ctypes.POINTER(ScanDesc)] + [_P] * 21 + [ctypes.c_size_t, _P], ctypes.c_int),
+}
+
+_lib: Optional[ctypes.CDLL] = None
+
+
+def load_library(path: str = LIB_PATH) -> ctypes.CDLL:
+    """Load libsnn.so (built by paper_2211_10725_gb300.build_lib); raise if absent."""
+    global _lib
+    if _lib is not None:
+        return _lib
+    if not os.path.exists(path):
+        raise RuntimeError(f"libsnn.so not built ({path}); run __graft_entry__.build()")
+    lib = ctypes.CDLL(path)
+    for name, (args, res) in _SIGS.items():
+        fn = getattr(lib, name)
+        fn.argtypes = args
+        fn.restype = res
+    _lib = lib
+    return lib
+
+
+def header_functions(path: str = HEADER) -> list:
+    """Names of the functions include/snn.h declares."""
+    txt = open(path).read()
+    txt = re.sub(r"/\*.*?\*/", "", txt, flags=re.S)
+    return sorted(set(re.findall(r"\b(snn_[a-z0-9_]+)\s*\(", txt)))
+
+
+def status_string(status: int) -> str:
+    return load_library().snn_status_string(status).decode()
+
+
+def _check(status: int, where: str):
+    if status != SNN_OK:
+        raise SnnError(status, where)
+
+
+def _ptr(t) -> Optional[int]:
+    if t is None:
+        return None
+    if isinstance(t, int):
+        return t
+    return t.data_ptr()
+
+
+def _stream(stream) -> Optional[int]:
+    if stream is None:
+        return torch.cuda.current_stream().cuda_stream
+    if isinstance(stream, int):
+        return stream
+    return stream.cuda_stream
+
+
+def make_desc(w: W.ScanWorkload, **over) -> ScanDesc:
+    """Descriptor for a workload (fields can be overridden by keyword)."""
+    d = ScanDesc()
+    d.T, d.B, d.N, d.C, d.HW = w.T, w.B, w.N, w.C, w.HW
+    d.in_dtype, d.io_dtype = DTYPE_CODE[w.in_dtype], DTYPE_CODE[w.io_dtype]
+    d.reset = RESET_CODE[w.reset]
+    d.detach_reset = 1 if w.detach_reset else 0
+    d.surrogate = SG_CODE[w.surrogate]
+    d.sg_param = w.sg_param
+    d.beta_mode, d.thr_mode = PMODE_CODE[w.beta_mode], PMODE_CODE[w.thr_mode]
+    d.alpha_mode = PMODE_CODE[w.alpha_mode]
+    d.save = SAVE_CODE[w.save]
+    d.ckpt_every = w.ckpt_every if w.save == "recompute" else 0
+    for k, v in over.items():
+        setattr(d, k, v)
+    return d
+
+
+# ---------------------------------------------------------------------------
+# Thin wrappers with the C names (tensor -> pointer marshalling only)
+# ---------------------------------------------------------------------------
+
+def snn_scan_workspace_bytes(desc: ScanDesc) -> int:
+    return load_library().snn_scan_workspace_bytes(ctypes.byref(desc))
+
+
+def snn_scan_ckpt_elems(desc: ScanDesc, synaptic: bool) -> int:
+    return load_library().snn_scan_ckpt_elems(ctypes.byref(desc), 1 if synaptic else 0)
+
+
+def snn_workspace_init(ws: torch.Tensor, stream=None):
+    _check(load_library().snn_workspace_init(_ptr(ws), ws.numel() * ws.element_size(),
+                                             _stream(stream)), "snn_workspace_init")
+
+
+def snn_workspace_status(ws: torch.Tensor, stream=None) -> int:
+    return load_library().snn_workspace_status(_ptr(ws), _stream(stream))
+
+
+def snn_leaky_fwd(desc, I, beta, thr, mem0, spk, mem, ckpt, mem_final, ws, stream=None):
+    _check(load_library().snn_leaky_fwd(
+        ctypes.byref(desc), _ptr(I), _ptr(beta), _ptr(thr), _ptr(mem0), _ptr(spk), _ptr(mem),
+        _ptr(ckpt), _ptr(mem_final), _ptr(ws), ws.numel() * ws.element_size(),
+        _stream(stream)), "snn_leaky_fwd")
+
+
+def snn_leaky_bwd(desc, I, ckpt, mem, spk, beta, thr, mem0, grad_spk, grad_mem,
+                  grad_mem_final, grad_I, grad_beta, grad_thr, grad_mem0, ws, stream=None):
+    _check(load_library().snn_leaky_bwd(
+        ctypes.byref(desc), _ptr(I), _ptr(ckpt), _ptr(mem), _ptr(spk), _ptr(beta), _ptr(thr),
+        _ptr(mem0), _ptr(grad_spk), _ptr(grad_mem), _ptr(grad_mem_final), _ptr(grad_I),
+        _ptr(grad_beta), _ptr(grad_thr), _ptr(grad_mem0), _ptr(ws),
+        ws.numel() * ws.element_size(), _stream(stream)), "snn_leaky_bwd")
+
+
+def snn_synaptic_fwd(desc, I, alpha, beta, thr, mem0, syn0, spk, mem, syn, ckpt, mem_final,
+                     syn_final, ws, stream=None):
+    _check(load_library().snn_synaptic_fwd(
+        ctypes.byref(desc), _ptr(I), _ptr(alpha), _ptr(beta), _ptr(thr), _ptr(mem0),
+        _ptr(syn0), _ptr(spk), _ptr(mem), _ptr(syn), _ptr(ckpt), _ptr(mem_final),
+        _ptr(syn_final), _ptr(ws), ws.numel() * ws.element_size(), _stream(stream)),
+        "snn_synaptic_fwd")
+
+
+def snn_synaptic_bwd(desc, I, ckpt, mem, spk, syn, alpha, beta, thr, mem0, syn0, grad_spk,
+                     grad_mem, grad_mem_final, grad_syn_final, grad_I, grad_alpha, grad_beta,
+                     grad_thr, grad_mem0, grad_syn0, ws, stream=None):
+    _check(load_library().snn_synaptic_bwd(
+        ctypes.byref(desc), _ptr(I), _ptr(ckpt), _ptr(mem), _ptr(spk), _ptr(syn), _ptr(alpha),
+        _ptr(beta), _ptr(thr), _ptr(mem0), _ptr(syn0), _ptr(grad_spk), _ptr(grad_mem),
+        _ptr(grad_mem_final), _ptr(grad_syn_final), _ptr(grad_I), _ptr(grad_alpha),
+        _ptr(grad_beta), _ptr(grad_thr), _ptr(grad_mem0), _ptr(grad_syn0), _ptr(ws),
+        ws.numel() * ws.element_size(), _stream(stream)), "snn_synaptic_bwd")
+
+
+# ---------------------------------------------------------------------------
+# A layer object: allocates the buffers of one scan workload on the device
+# ---------------------------------------------------------------------------
+
+class ScanLayer:
+    """Device buffers plus forward/backward calls for one ScanWorkload.
+
+    Inputs are taken as given (already on the device); outputs, checkpoints
+    and the workspace are allocated once with torch and reused.
+    """
+
+    def __init__(self, w: W.ScanWorkload, device="cuda", want_syn: bool = False, **desc_over):
+        self.w = w
+        self.synaptic = w.neuron == "synaptic"
+        self.desc = make_desc(w, **desc_over)
+        self.device = torch.device(device)
+        io = W.TORCH_DTYPE[w.io_dtype]
+        shape = (w.T, w.B, w.N)
+        dev = self.device
+        self.spk = torch.empty(shape, dtype=io, device=dev)
+        need_mem = w.want_mem or w.save == "mem"
+        self.mem = torch.empty(shape, dtype=io, device=dev) if need_mem else None
+        self.syn = torch.empty(shape, dtype=io, device=dev) if (self.synaptic and want_syn) else None
+        nck = snn_scan_ckpt_elems(self.desc, self.synaptic)
+        self.ckpt = torch.empty(max(nck, 1), dtype=torch.float32, device=dev) if nck > 0 else None
+        self.mem_final = torch.empty((w.B, w.N), dtype=torch.float32, device=dev)
+        self.syn_final = torch.empty((w.B, w.N), dtype=torch.float32, device=dev) if self.synaptic else None
+        self.grad_I = torch.empty(shape, dtype=io, device=dev)
+        plen = {"scalar": 1, "per_neuron": w.N, "per_channel": w.C}
+        self.grad_beta = torch.empty(plen[w.beta_mode], dtype=torch.float32, device=dev)
+        self.grad_thr = torch.empty(plen[w.thr_mode], dtype=torch.float32, device=dev)
+        self.grad_alpha = torch.empty(plen[w.alpha_mode], dtype=torch.float32, device=dev) \
+            if self.synaptic else None
+        self.grad_mem0 = torch.empty((w.B, w.N), dtype=torch.float32, device=dev)
+        self.grad_syn0 = torch.empty((w.B, w.N), dtype=torch.float32, device=dev) \
+            if self.synaptic else None
+        nws = snn_scan_workspace_bytes(self.desc)
+        if nws == 0:
+            raise SnnError(1, "snn_scan_workspace_bytes")
+        self.ws = torch.empty(nws, dtype=torch.uint8, device=dev)
+        snn_workspace_init(self.ws)
+
+    def forward(self, I, beta, thr, alpha=None, mem0=None, syn0=None, stream=None):
+        if self.synaptic:
+            snn_synaptic_fwd(self.desc, I, alpha, beta, thr, mem0, syn0, self.spk, self.mem,
+                             self.syn, self.ckpt, self.mem_final, self.syn_final, self.ws, stream)
+        else:
+            snn_leaky_fwd(self.desc, I, beta, thr, mem0, self.spk, self.mem, self.ckpt,
+                          self.mem_final, self.ws, stream)
+        return self.spk
+
+    def backward(self, I, beta, thr, grad_spk, alpha=None, mem0=None, syn0=None, grad_mem=None,
+                 grad_mem_final=None, grad_syn_final=None, want_param_grads=True,
+                 want_state_grads=True, stream=None):
+        gb = self.grad_beta if want_param_grads else None
+        gt = self.grad_thr if want_param_grads else None
+        gm0 = self.grad_mem0 if want_state_grads else None
+        recompute = self.w.save == "recompute"
+        if self.synaptic:
+            ga = self.grad_alpha if (want_param_grads and (recompute or self.syn is not None)) else None
+            gs0 = self.grad_syn0 if want_state_grads else None
+            snn_synaptic_bwd(self.desc, I if recompute else None, self.ckpt, self.mem, self.spk,
+                             self.syn, alpha, beta, thr, mem0, syn0, grad_spk, grad_mem,
+                             grad_mem_final, grad_syn_final, self.grad_I, ga, gb, gt, gm0, gs0,
+                             self.ws, stream)
+        else:
+            snn_leaky_bwd(self.desc, I if recompute else None, self.ckpt, self.mem, self.spk,
+                          beta, thr, mem0, grad_spk, grad_mem, grad_mem_final, self.grad_I, gb,
+                          gt, gm0, self.ws, stream)
+        return self.grad_I
+
+    def status(self, stream=None) -> int:
+        return snn_workspace_status(self.ws, stream)

@@ -1,0 +1,204 @@
+"""Helpers shared by the scan parity tests: run the CPU oracle on the seeded
+inputs of a workload and compare the CUDA results with it.
+
+Comparison protocol
+-------------------
+* Spike decisions are integers decided by floating point, so both sides take
+  them in the kernel's precision: the oracle's float32 evaluation of Eqs.
+  (4)/(6) (``dtype=np.float32``) gives the expected spike train and membrane
+  trace, and the GPU must reproduce both bit for bit.
+* That float32 trace is pinned to the float64 definition: the oracle reruns
+  the scan in float64 with the reset sequence held at the float32 spikes, and
+  every element where the float64 spike would differ must lie within 1e-5 of
+  the threshold (the only places where several answers are correct); mem
+  agrees within rel 1e-5 / abs 1e-6.
+* The backward is a function of the saved forward state (mem, spk): the
+  oracle's float64 BPTT runs on the same saved state the kernel consumes
+  (the float32 trace, rounded to the storage dtype in the store variant) and
+  the kernel's gradients must agree within the stated tolerances.
+"""
+from __future__ import annotations
+
+import numpy as np
+import torch
+
+from oracle import snn_oracle as O
+from paper_2211_10725_gb300 import workloads as W
+
+TOL = {  # (rtol, atol) for values compared elementwise
+    W.F32: (1e-5, 1e-6),
+    W.BF16: (2e-2, 1e-3),
+    W.F16: (2e-2, 1e-3),
+}
+AMBIGUITY = 1e-5   # |u - thr| below which a spike decision may legitimately differ
+
+
+def lanes_2d(x: torch.Tensor, lanes=None) -> np.ndarray:
+    """[T, B, N] tensor (any dtype, any device) -> float64 [T, L'] array."""
+    a = x.detach().to("cpu", torch.float32).numpy().astype(np.float64)
+    a = a.reshape(a.shape[0], -1)
+    return a if lanes is None else a[:, lanes]
+
+
+def lanes_1d(x, lanes=None) -> np.ndarray:
+    a = x.detach().to("cpu", torch.float32).numpy().astype(np.float64).reshape(-1)
+    return a if lanes is None else a[lanes]
+
+
+def round_to(dtype: str, x: np.ndarray) -> np.ndarray:
+    """Round to the storage dtype (library conversion, round to nearest even)."""
+    if dtype == W.F32:
+        return np.asarray(x, dtype=np.float32).astype(np.float64)
+    t = torch.from_numpy(np.asarray(x, dtype=np.float32)).to(W.TORCH_DTYPE[dtype])
+    return t.to(torch.float32).numpy().astype(np.float64)
+
+
+def oracle_expect(w: W.ScanWorkload, inp: dict, lanes=None, backward=True) -> dict:
+    """Oracle results for the workload's inputs on a subset of lanes."""
+    T, B, N, C, HW = w.T, w.B, w.N, w.C, w.HW
+    L = B * N
+    idx = np.arange(L) if lanes is None else np.asarray(lanes)
+    syn = w.neuron == "synaptic"
+
+    def par(name, mode):
+        full = O.lane_param(inp[name].numpy(), B, N, mode, C, HW)
+        return full[idx]
+
+    beta, thr = par("beta", w.beta_mode), par("thr", w.thr_mode)
+    alpha = par("alpha", w.alpha_mode) if syn else None
+    I = lanes_2d(inp["I"], idx)
+    mem0 = lanes_1d(inp["mem0"], idx) if "mem0" in inp else None
+    syn0 = lanes_1d(inp["syn0"], idx) if "syn0" in inp else None
+    f32 = lambda a: None if a is None else np.asarray(a, dtype=np.float32)
+
+    # float32 evaluation: the spike decisions in the kernel's precision
+    if syn:
+        spk32, mem32, syn32 = O.synaptic_forward(f32(I), f32(alpha), f32(beta), f32(thr), w.reset,
+                                                 mem0=f32(mem0), syn0=f32(syn0), dtype=np.float32)
+    else:
+        spk32, mem32 = O.leaky_forward(f32(I), f32(beta), f32(thr), w.reset, mem0=f32(mem0),
+                                       dtype=np.float32)
+        syn32 = None
+    z_m1 = np.zeros(len(idx)) if mem0 is None else (f32(mem0) > f32(thr)).astype(np.float64)
+    z_reset = np.vstack([z_m1[None], spk32[:-1].astype(np.float64)]) if T > 0 else None
+
+    # float64 scan on the same discrete path (reset held at the fp32 spikes)
+    if syn:
+        _, mem64, syn64 = O.synaptic_forward(I, alpha, beta, thr, w.reset, mem0=mem0, syn0=syn0,
+                                             z_reset=z_reset)
+    else:
+        _, mem64 = O.leaky_forward(I, beta, thr, w.reset, mem0=mem0, z_reset=z_reset)
+        syn64 = None
+    out = {"lanes": idx, "spk32": spk32.astype(np.float64), "mem32": mem32.astype(np.float64),
+           "mem64": mem64, "thr": thr, "beta": beta, "alpha": alpha}
+    if syn:
+        out["syn32"], out["syn64"] = syn32.astype(np.float64), syn64
+    if not backward:
+        return out
+
+    # backward on the saved state as the kernel consumes it
+    gs = lanes_2d(inp["grad_spk"], idx)
+    gm = lanes_2d(inp["grad_mem"], idx) if "grad_mem" in inp else None
+    gmf = lanes_1d(inp["grad_mem_final"], idx) if "grad_mem_final" in inp else None
+    gsf = lanes_1d(inp["grad_syn_final"], idx) if "grad_syn_final" in inp else None
+    mem_b = out["mem32"] if w.save == "recompute" else round_to(w.io_dtype, out["mem32"])
+    kw = dict(reset=w.reset, detach=w.detach_reset, sg=w.surrogate, sg_param=w.sg_param,
+              grad_mem=gm, grad_mem_final=gmf, mem0=mem0)
+    if syn:
+        syn_b = out["syn32"] if w.save == "recompute" else round_to(w.io_dtype, out["syn32"])
+        g = O.synaptic_backward(mem_b, out["spk32"], syn_b, gs, alpha, beta, thr, syn0=syn0,
+                                grad_syn_final=gsf, **kw)
+    else:
+        g = O.leaky_backward(mem_b, out["spk32"], gs, beta, thr, **kw)
+    out.update(g)
+    if lanes is None:
+        out["grad_beta"] = O.reduce_lane_grad(g["grad_beta_lane"], B, N, w.beta_mode, C, HW)
+        out["grad_thr"] = O.reduce_lane_grad(g["grad_thr_lane"], B, N, w.thr_mode, C, HW)
+        if syn:
+            out["grad_alpha"] = O.reduce_lane_grad(g["grad_alpha_lane"], B, N, w.alpha_mode, C, HW)
+    return out
+
+
+def check_spikes_and_mem(w, ref, spk_gpu, mem_gpu=None, syn_gpu=None, lanes=None):
+    """Bit-exact spikes and trace against the fp32 evaluation; fp32 trace
+    within tolerance of the float64 scan on the same spike path."""
+    spk = lanes_2d(spk_gpu, lanes)
+    mism = np.argwhere(spk != ref["spk32"])
+    assert mism.size == 0, f"{len(mism)} spike mismatches, first at {mism[:5].tolist()}"
+    # the fp32 spike path is a valid one: the float64 decision differs only
+    # within AMBIGUITY of the threshold
+    z64 = (ref["mem64"] > ref["thr"][None]).astype(np.float64)
+    diff = z64 != ref["spk32"]
+    if diff.any():
+        margin = np.abs(ref["mem64"] - ref["thr"][None])[diff]
+        assert margin.max() < AMBIGUITY, f"fp32 spike off the fp64 path by {margin.max()}"
+    np.testing.assert_allclose(ref["mem32"], ref["mem64"], rtol=1e-5, atol=1e-6)
+    if mem_gpu is not None:
+        m = lanes_2d(mem_gpu, lanes)
+        expect = round_to(w.io_dtype, ref["mem32"])
+        bad = np.argwhere(m != expect)
+        assert bad.size == 0, f"{len(bad)} mem mismatches, first {bad[:5].tolist()}"
+    if syn_gpu is not None:
+        s = lanes_2d(syn_gpu, lanes)
+        expect = round_to(w.io_dtype, ref["syn32"])
+        assert np.array_equal(s, expect)
+        np.testing.assert_allclose(ref["syn32"], ref["syn64"], rtol=1e-5, atol=1e-6)
+    return int(diff.sum())
+
+
+def assert_close(name, got, ref, rtol, atol):
+    got = np.asarray(got, dtype=np.float64)
+    ref = np.asarray(ref, dtype=np.float64)
+    err = np.abs(got - ref)
+    lim = atol + rtol * np.abs(ref)
+    bad = err > lim
+    if bad.any():
+        i = np.unravel_index(np.argmax(err - lim), err.shape)
+        raise AssertionError(f"{name}: {bad.sum()} / {bad.size} beyond tolerance; worst at {i}: "
+                             f"got {got[i]!r} ref {ref[i]!r} (rtol {rtol}, atol {atol})")
+
+
+def check_param_grad(name, got, ref, lane_partials, B, N, mode, C, HW, rtol=1e-5):
+    """A reduced parameter gradient: relative to its value, with an absolute
+    floor proportional to the sum of |per-lane partials| it reduces (fp32
+    accumulation over t within a lane, fp64 across lanes)."""
+    scale = O.reduce_lane_grad(np.abs(lane_partials), B, N, mode, C, HW)
+    assert_close(name, got, ref, rtol, rtol * scale + 1e-6)
+
+
+def run_gpu(w: W.ScanWorkload, inp: dict, device="cuda", **desc_over):
+    """Forward + backward of one workload through the C ABI; returns the
+    ScanLayer holding every output (on the device)."""
+    from paper_2211_10725_gb300 import snn
+    d = {k: v.to(device) for k, v in inp.items()}
+    layer = snn.ScanLayer(w, device=device, want_syn=True, **desc_over)
+    layer.forward(d["I"], d["beta"], d["thr"], d.get("alpha"), d.get("mem0"), d.get("syn0"))
+    layer.backward(d["I"], d["beta"], d["thr"], d["grad_spk"], alpha=d.get("alpha"),
+                   mem0=d.get("mem0"), syn0=d.get("syn0"), grad_mem=d.get("grad_mem"),
+                   grad_mem_final=d.get("grad_mem_final"),
+                   grad_syn_final=d.get("grad_syn_final"))
+    torch.cuda.synchronize()
+    return layer
+
+
+def check_all(w: W.ScanWorkload, inp: dict, layer, ref: dict, lanes=None):
+    """Every output of a run against the oracle (ref from oracle_expect)."""
+    syn = w.neuron == "synaptic"
+    amb = check_spikes_and_mem(w, ref, layer.spk, layer.mem, layer.syn if syn else None, lanes)
+    rtol, atol = TOL[w.io_dtype]
+    assert_close("grad_I", lanes_2d(layer.grad_I, lanes), ref["grad_I"], rtol, atol)
+    f_rtol, f_atol = TOL[W.F32]
+    assert np.array_equal(lanes_1d(layer.mem_final, lanes), ref["mem32"][-1]) if w.T > 0 else True
+    assert_close("grad_mem0", lanes_1d(layer.grad_mem0, lanes), ref["grad_mem0"], f_rtol, f_atol)
+    if syn:
+        assert_close("grad_syn0", lanes_1d(layer.grad_syn0, lanes), ref["grad_syn0"], f_rtol, f_atol)
+    if lanes is None:
+        B, N, C, HW = w.B, w.N, w.C, w.HW
+        check_param_grad("grad_beta", lanes_1d(layer.grad_beta), ref["grad_beta"],
+                         ref["grad_beta_lane"], B, N, w.beta_mode, C, HW)
+        check_param_grad("grad_thr", lanes_1d(layer.grad_thr), ref["grad_thr"],
+                         ref["grad_thr_lane"], B, N, w.thr_mode, C, HW)
+        if syn:
+            check_param_grad("grad_alpha", lanes_1d(layer.grad_alpha), ref["grad_alpha"],
+                             ref["grad_alpha_lane"], B, N, w.alpha_mode, C, HW)
+    return amb

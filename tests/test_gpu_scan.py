@@ -1,0 +1,136 @@
+"""Parity of the CUDA scan (through the C ABI) with the CPU oracle.
+
+Small cases sweep every mode (neuron, reset, detach, surrogate, parameter
+layout, save variant, dtype pair, optional inputs) over shapes that span
+several CTAs with a ragged last strip and shapes whose rows are not 16-byte
+multiples (the plain per-lane kernels).  Full-size cases run each workload
+in the launch configuration the benchmark times.
+"""
+import numpy as np
+import pytest
+import torch
+
+from paper_2211_10725_gb300 import snn
+from paper_2211_10725_gb300 import workloads as W
+from tests import scan_harness as H
+from oracle import snn_oracle as O
+
+pytestmark = pytest.mark.gpu
+
+SHAPES = [(1, 1, 7), (2, 3, 5), (5, 2, 64), (33, 5, 1000), (17, 4, 2048), (9, 3, 1368)]
+CHANNELS = {7: (7, 1), 5: (5, 1), 64: (4, 16), 1000: (10, 100), 2048: (8, 256), 1368: (6, 228)}
+DTYPES = [(W.F32, W.F32), (W.BF16, W.BF16), (W.F16, W.F16), (W.F32, W.BF16)]
+RESETS = ["subtract", "zero", "none"]
+MODES = ["scalar", "per_neuron", "per_channel"]
+
+
+def small_case(i):
+    T, B, N = SHAPES[i % len(SHAPES)]
+    C, HW = CHANNELS[N]
+    in_dt, io_dt = DTYPES[(i // 5) % len(DTYPES)]
+    save = ["mem", "recompute"][(i // 3) % 2]
+    w = W.ScanWorkload(
+        name=f"small{i}", neuron=["leaky", "synaptic"][(i // 11) % 2], T=T, B=B, N=N, C=C, HW=HW,
+        in_dtype=in_dt, io_dtype=io_dt, i_mean=0.5, i_std=0.6,
+        beta=("uniform", 0.5, 0.95), thr=("uniform", 0.6, 1.4), alpha=("uniform", 0.3, 0.9),
+        beta_mode=MODES[(i // 7) % 3], thr_mode=MODES[(i // 2) % 3], alpha_mode=MODES[i % 3],
+        reset=RESETS[i % 3], detach_reset=(i % 2 == 0),
+        surrogate=["fast_sigmoid", "atan"][(i // 2) % 2], sg_param=[25.0, 2.0][(i // 2) % 2],
+        save=save, ckpt_every=[1, 3, 4, 8][(i // 4) % 4], want_mem=True, seed_index=100 + i)
+    opts = dict(with_mem0=(i % 4 == 0), with_grad_mem=(i % 5 == 1), with_grad_final=(i % 3 == 0))
+    return w, opts
+
+
+@pytest.mark.parametrize("i", range(72))
+def test_small_cases(i, cuda_device):
+    w, opts = small_case(i)
+    inp = W.make_scan_inputs(w, **opts)
+    layer = H.run_gpu(w, inp)
+    assert layer.status() == 0
+    H.check_all(w, inp, layer, H.oracle_expect(w, inp))
+
+
+@pytest.mark.parametrize("i", [3, 4, 15, 16, 27, 28, 40, 51, 63])
+def test_staged_and_plain_kernels_agree(i, cuda_device):
+    w, opts = small_case(i)
+    inp = W.make_scan_inputs(w, **opts)
+    a = H.run_gpu(w, inp)
+    b = H.run_gpu(w, inp, debug_flags=snn.DEBUG_FORCE_PLAIN)
+    assert torch.equal(a.spk, b.spk) and torch.equal(a.mem, b.mem)
+    assert torch.equal(a.mem_final, b.mem_final)
+    if a.ckpt is not None:
+        assert torch.equal(a.ckpt, b.ckpt)
+    H.assert_close("grad_I", H.lanes_2d(a.grad_I), H.lanes_2d(b.grad_I), 1e-6, 1e-7)
+
+
+def test_backward_is_deterministic(cuda_device):
+    w = W.SYNAPTIC_C2.scaled(T=20, B=16)
+    inp = W.make_scan_inputs(w)
+    a = H.run_gpu(w, inp)
+    g1 = (a.grad_beta.clone(), a.grad_thr.clone(), a.grad_I.clone())
+    a.backward(*[v.cuda() for v in (inp["I"], inp["beta"], inp["thr"], inp["grad_spk"])],
+               alpha=inp["alpha"].cuda())
+    torch.cuda.synchronize()
+    assert torch.equal(g1[0], a.grad_beta) and torch.equal(g1[1], a.grad_thr)
+    assert torch.equal(g1[2], a.grad_I)
+
+
+def test_empty_inputs(cuda_device):
+    # B = 0: nothing to scan; parameter gradients are zero-filled
+    w = W.LEAKY_C1.scaled(B=0)
+    inp = W.make_scan_inputs(w)
+    layer = H.run_gpu(w, inp)
+    assert float(layer.grad_beta.abs().sum()) == 0.0
+    # T = 0: final state is the initial state, grad_mem0 is grad_mem_final
+    w = W.LEAKY_C1.scaled(T=0, B=2, N=64)
+    inp = W.make_scan_inputs(w, with_mem0=True, with_grad_final=True)
+    layer = H.run_gpu(w, inp)
+    assert torch.equal(layer.mem_final.cpu(), inp["mem0"])
+    assert torch.equal(layer.grad_mem0.cpu(), inp["grad_mem_final"])
+    assert float(layer.grad_beta.abs().sum()) == 0.0
+
+
+def test_wait_timeout_reports_status_and_context_survives(cuda_device):
+    # the producer issues nothing, so the consumers' bounded wait runs out
+    w = W.LEAKY_C1.scaled(T=8, B=4, N=1024)
+    inp = W.make_scan_inputs(w)
+    layer = H.run_gpu(w, inp, debug_flags=snn.DEBUG_PRODUCER_IDLE, wait_limit_ns=2_000_000)
+    assert layer.status() == 6          # SNN_ERR_TIMEOUT, read and cleared
+    assert layer.status() == 0
+    ok = H.run_gpu(w, inp)
+    assert ok.status() == 0
+    H.check_all(w, inp, ok, H.oracle_expect(w, inp))
+
+
+# ---------------------------------------------------------------------------
+# Full-size workloads
+# ---------------------------------------------------------------------------
+
+@pytest.mark.parametrize("name", ["leaky_T25_B128_N1000", "synaptic_T100_B128_N4096",
+                                  "conv_lif_T25_B128_C12x24x24", "conv_lif_T25_B128_C64x8x8"])
+def test_full_size_workloads(name, cuda_device):
+    w = W.SCAN_WORKLOADS[name]
+    inp = W.make_scan_inputs(w)
+    layer = H.run_gpu(w, inp)
+    assert layer.status() == 0
+    H.check_all(w, inp, layer, H.oracle_expect(w, inp))
+
+
+@pytest.mark.parametrize("save", ["recompute", "mem"])
+def test_full_size_large_bf16(save, cuda_device):
+    # T=500, B=64, N=8192, bf16 storage; the oracle recomputes a sample of
+    # neurons (all 64 samples of each, so per-neuron gradients are exact sums)
+    w = W.BIG_C5.scaled(save=save)
+    inp = W.make_scan_inputs(w)
+    layer = H.run_gpu(w, inp)
+    assert layer.status() == 0
+    rng = np.random.default_rng(5)
+    ns = np.sort(rng.choice(w.N, 24, replace=False))
+    ns = np.unique(np.concatenate([ns, [0, 7, w.N - 1]]))
+    lanes = (np.arange(w.B)[:, None] * w.N + ns[None, :]).reshape(-1)
+    ref = H.oracle_expect(w, inp, lanes=lanes)
+    H.check_all(w, inp, layer, ref, lanes=lanes)
+    for pname, mode in (("beta", w.beta_mode), ("thr", w.thr_mode)):
+        part = ref[f"grad_{pname}_lane"].reshape(w.B, len(ns))
+        got = H.lanes_1d(getattr(layer, f"grad_{pname}"))[ns]
+        H.assert_close(f"grad_{pname}", got, part.sum(0), 1e-5, 1e-5 * np.abs(part).sum(0) + 1e-6)
