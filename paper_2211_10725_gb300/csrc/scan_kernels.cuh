@@ -318,8 +318,6 @@ __global__ void __launch_bounds__(1024) scan_fwd_staged(const ScanArgs a) {
     }
     float x[VEC];
     if (active) Elem<TI>::load4(reinterpret_cast<const TI*>(ring + (size_t)s * a.stage_bytes) + c * VEC, x);
-    __syncwarp();
-    if (lid == 0) mbar_arrive(&empty[s]);
     if (active) {
       float zf[VEC];
 #pragma unroll
@@ -340,6 +338,11 @@ __global__ void __launch_bounds__(1024) scan_fwd_staged(const ScanArgs a) {
         }
       }
     }
+    // Release the stage only after its values were consumed: the stores
+    // above depend on them, so every lane's shared-memory read has completed
+    // before the producer may refill the stage with a bulk copy.
+    __syncwarp();
+    if (lid == 0) mbar_arrive(&empty[s]);
   }
   if (active) {
     if (a.mem_final) Elem<float>::store4(a.mem_final + l, u);
@@ -459,6 +462,9 @@ __global__ void __launch_bounds__(1024) scan_bwd_staged(const ScanArgs a) {
     base = ring + (size_t)s * a.stage_bytes;
     return true;
   };
+  // Called only once the values read from item jj's stage have been consumed
+  // (outputs computed and stored), so the reads have completed before the
+  // producer may overwrite the stage.
   auto release_item = [&](int64_t jj) {
     __syncwarp();
     if (lid == 0) mbar_arrive(&empty[(int)(jj % S)]);
@@ -476,7 +482,6 @@ __global__ void __launch_bounds__(1024) scan_bwd_staged(const ScanArgs a) {
         if (want_syn) Elem<TO>::load4(reinterpret_cast<const TO*>(base + t_syn * io_stride) + c * VEC, ii);
         if (a.gm) Elem<TO>::load4(reinterpret_cast<const TO*>(base + t_gm_store * io_stride) + c * VEC, gmv);
       }
-      release_item(j);
       if (active) {
         float out[VEC];
         const bool last = (t == a.T - 1);
@@ -489,6 +494,7 @@ __global__ void __launch_bounds__(1024) scan_bwd_staged(const ScanArgs a) {
         }
         Elem<TO>::store4(gI + t * a.L + l, out);
       }
+      release_item(j);  // after the values read from the stage were consumed
     }
   } else {
     for (int k = a.nseg - 1; k >= 0 && ok; --k) {
@@ -519,7 +525,6 @@ __global__ void __launch_bounds__(1024) scan_bwd_staged(const ScanArgs a) {
             }
           }
         }
-        release_item(j);
         if (active) {
 #pragma unroll
           for (int v = 0; v < VEC; ++v)
@@ -528,6 +533,7 @@ __global__ void __launch_bounds__(1024) scan_bwd_staged(const ScanArgs a) {
           Elem<float>::store4(su, u);
           if (SYN) Elem<float>::store4(su + seg_plane, ii);
         }
+        release_item(j);
       }
       if (!ok) break;
       // reverse steps over the segment
@@ -539,7 +545,6 @@ __global__ void __launch_bounds__(1024) scan_bwd_staged(const ScanArgs a) {
           Elem<TO>::load4(reinterpret_cast<const TO*>(base) + c * VEC, g);
           if (a.gm) Elem<TO>::load4(reinterpret_cast<const TO*>(base + io_stride) + c * VEC, gmv);
         }
-        release_item(j);
         if (active) {
           const float* su = seg + ((size_t)(t - t0) * nthr + c) * VEC;
           float uu[VEC], iv[VEC], out[VEC];
@@ -554,6 +559,7 @@ __global__ void __launch_bounds__(1024) scan_bwd_staged(const ScanArgs a) {
           }
           Elem<TO>::store4(gI + t * a.L + l, out);
         }
+        release_item(j);
       }
     }
   }

@@ -134,3 +134,19 @@ def test_full_size_large_bf16(save, cuda_device):
         part = ref[f"grad_{pname}_lane"].reshape(w.B, len(ns))
         got = H.lanes_1d(getattr(layer, f"grad_{pname}"))[ns]
         H.assert_close(f"grad_{pname}", got, part.sum(0), 1e-5, 1e-5 * np.abs(part).sum(0) + 1e-6)
+
+
+@pytest.mark.parametrize("neuron,dt,save", [("leaky", W.F32, "mem"), ("synaptic", W.F32, "mem"),
+                                            ("leaky", W.BF16, "recompute"),
+                                            ("synaptic", W.F16, "recompute")])
+def test_ring_wraps_with_many_warps(neuron, dt, save, cuda_device):
+    # T well beyond the ring depth and strips of hundreds of lanes per CTA, so
+    # every stage is refilled many times while a dozen consumer warps read it
+    w = W.SYNAPTIC_C2.scaled(name="wrap", neuron=neuron, T=120, B=64, N=4096, in_dtype=dt,
+                             io_dtype=dt, save=save, ckpt_every=8)
+    inp = W.make_scan_inputs(w)
+    layer = H.run_gpu(w, inp)
+    assert layer.status() == 0
+    rng = np.random.default_rng(9)
+    lanes = np.sort(rng.choice(w.B * w.N, 20000, replace=False))
+    H.check_all(w, inp, layer, H.oracle_expect(w, inp, lanes=lanes), lanes=lanes)
