@@ -2,54 +2,94 @@
 // family so the library compiles in parallel.
 #pragma once
 
+#include <type_traits>
+
 #include "scan_host.cuh"
 
 namespace snn {
 
+// dtype pairs (input, io) whose staged backward gets loops specialised on
+// the reset mode and surrogate; other pairs use the run-time-mode loop.
+template <typename TI, typename TO>
+constexpr bool kSpecialise =
+    (std::is_same<TI, float>::value && std::is_same<TO, float>::value) ||
+    (std::is_same<TI, __nv_bfloat16>::value && std::is_same<TO, __nv_bfloat16>::value) ||
+    (std::is_same<TI, float>::value && std::is_same<TO, __nv_bfloat16>::value);
+
+template <bool SYN, typename TI, typename TO, int RESET>
+cudaError_t fwd_staged(ScanArgs a, cudaStream_t st, bool* launched) {
+  const void* k = (const void*)scan_fwd_staged<SYN, TI, TO, RESET>;
+  StagedPlan p;
+  if (!plan_staged(k, a.L, a.T, (int)sizeof(TI), 0, kLanes<SYN>, &p)) return cudaSuccess;
+  a.lanes_per_cta = p.lanes_per_cta;
+  a.stages = p.stages;
+  a.stage_bytes = p.stage_bytes;
+  scan_fwd_staged<SYN, TI, TO, RESET><<<(unsigned)p.grid, p.threads, p.smem, st>>>(a);
+  *launched = true;
+  return cudaGetLastError();
+}
+
 template <bool SYN, typename TI, typename TO>
 cudaError_t fwd_t(ScanArgs a, bool staged, cudaStream_t st) {
   if (staged && a.L > 0) {
-    const void* k = (const void*)scan_fwd_staged<SYN, TI, TO>;
-    StagedPlan p;
-    if (plan_staged(k, a.L, a.T, (int)sizeof(TI), 0, &p)) {
-      a.lanes_per_cta = p.lanes_per_cta;
-      a.stages = p.stages;
-      a.stage_bytes = p.stage_bytes;
-      scan_fwd_staged<SYN, TI, TO><<<(unsigned)p.grid, p.threads, p.smem, st>>>(a);
-      return cudaGetLastError();
-    }
+    bool launched = false;
+    cudaError_t e;
+    if (a.reset == RESET_SUBTRACT) e = fwd_staged<SYN, TI, TO, RESET_SUBTRACT>(a, st, &launched);
+    else if (a.reset == RESET_ZERO) e = fwd_staged<SYN, TI, TO, RESET_ZERO>(a, st, &launched);
+    else e = fwd_staged<SYN, TI, TO, -1>(a, st, &launched);
+    if (launched || e != cudaSuccess) return e;
   }
   if (a.L == 0) return cudaSuccess;
   scan_fwd_plain<SYN, TI, TO><<<(unsigned)ceil_div(a.L, 256), 256, 0, st>>>(a);
   return cudaGetLastError();
 }
 
+template <bool SYN, bool RECOMP, typename TI, typename TO, int RESET, int SG>
+cudaError_t bwd_staged(ScanArgs a, cudaStream_t st, bool* launched) {
+  const void* k = (const void*)scan_bwd_staged<SYN, RECOMP, TI, TO, RESET, SG>;
+  int per_lane, seg;
+  int64_t items;
+  if (RECOMP) {
+    const int fwd_item = (int)sizeof(TI) + 4 * (SYN ? 2 : 1);
+    const int bwd_item = (int)sizeof(TO) * (a.gm ? 2 : 1);
+    per_lane = fwd_item > bwd_item ? fwd_item : bwd_item;
+    seg = kLanes<SYN> * 4 * a.K * (SYN ? 2 : 1);
+    items = 2 * a.T;
+  } else {
+    const int n = 2 + (sizeof(TO) != 4 ? 1 : 0) + ((SYN && a.part_alpha) ? 1 : 0) + (a.gm ? 1 : 0);
+    per_lane = n * (int)sizeof(TO);
+    seg = 0;
+    items = a.T;
+  }
+  StagedPlan p;
+  if (!plan_staged(k, a.L, items, per_lane, seg, kLanes<SYN>, &p)) return cudaSuccess;
+  a.lanes_per_cta = p.lanes_per_cta;
+  a.stages = p.stages;
+  a.stage_bytes = p.stage_bytes;
+  scan_bwd_staged<SYN, RECOMP, TI, TO, RESET, SG><<<(unsigned)p.grid, p.threads, p.smem, st>>>(a);
+  *launched = true;
+  return cudaGetLastError();
+}
+
 template <bool SYN, bool RECOMP, typename TI, typename TO>
 cudaError_t bwd_t(ScanArgs a, bool staged, cudaStream_t st) {
   if (staged && a.L > 0) {
-    const void* k = (const void*)scan_bwd_staged<SYN, RECOMP, TI, TO>;
-    int per_lane, seg;
-    int64_t items;
-    if (RECOMP) {
-      const int fwd_item = (int)sizeof(TI) + 4 * (SYN ? 2 : 1);
-      const int bwd_item = (int)sizeof(TO) * (a.gm ? 2 : 1);
-      per_lane = fwd_item > bwd_item ? fwd_item : bwd_item;
-      seg = VEC * 4 * a.K * (SYN ? 2 : 1);
-      items = 2 * a.T;
-    } else {
-      const int n = 2 + (sizeof(TO) != 4 ? 1 : 0) + ((SYN && a.part_alpha) ? 1 : 0) + (a.gm ? 1 : 0);
-      per_lane = n * (int)sizeof(TO);
-      seg = 0;
-      items = a.T;
+    bool launched = false;
+    cudaError_t e = cudaSuccess;
+    bool done = false;
+    if constexpr (kSpecialise<TI, TO>) {
+      done = true;
+      const int key = (a.reset == RESET_NONE ? 9 : a.reset * 2 + a.sg);
+      switch (key) {
+        case 0: e = bwd_staged<SYN, RECOMP, TI, TO, RESET_SUBTRACT, SG_FAST_SIGMOID>(a, st, &launched); break;
+        case 1: e = bwd_staged<SYN, RECOMP, TI, TO, RESET_SUBTRACT, SG_ATAN>(a, st, &launched); break;
+        case 2: e = bwd_staged<SYN, RECOMP, TI, TO, RESET_ZERO, SG_FAST_SIGMOID>(a, st, &launched); break;
+        case 3: e = bwd_staged<SYN, RECOMP, TI, TO, RESET_ZERO, SG_ATAN>(a, st, &launched); break;
+        default: done = false;
+      }
     }
-    StagedPlan p;
-    if (plan_staged(k, a.L, items, per_lane, seg, &p)) {
-      a.lanes_per_cta = p.lanes_per_cta;
-      a.stages = p.stages;
-      a.stage_bytes = p.stage_bytes;
-      scan_bwd_staged<SYN, RECOMP, TI, TO><<<(unsigned)p.grid, p.threads, p.smem, st>>>(a);
-      return cudaGetLastError();
-    }
+    if (!done) e = bwd_staged<SYN, RECOMP, TI, TO, -1, -1>(a, st, &launched);
+    if (launched || e != cudaSuccess) return e;
   }
   if (a.L == 0) return cudaSuccess;
   const int threads = 128;

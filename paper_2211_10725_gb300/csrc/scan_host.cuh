@@ -73,8 +73,9 @@ struct StagedPlan {
 // fits next to the per-thread replay buffer.  Returns false if nothing fits.
 //   stage_bytes_per_lane: bytes one lane contributes to the largest item
 //   seg_bytes_per_thread: replay buffer bytes per consumer thread
+//   lanes_per_thread: lanes each consumer thread owns
 inline bool plan_staged(const void* kernel, int64_t L, int64_t items, int stage_bytes_per_lane,
-                        int seg_bytes_per_thread, StagedPlan* plan) {
+                        int seg_bytes_per_thread, int lanes_per_thread, StagedPlan* plan) {
   static std::mutex mu;
   static std::map<std::tuple<int, const void*, int64_t, int64_t, int, int>, StagedPlan> cache;
   int dev = 0;
@@ -97,9 +98,9 @@ inline bool plan_staged(const void* kernel, int64_t L, int64_t items, int stage_
     for (int cps = 2; cps >= 1; --cps) {
       const int64_t ctas = (int64_t)d.sms * cps * waves;
       const int64_t lpc = round_up(ceil_div(L, ctas), 8);
-      const int64_t cthreads = round_up(ceil_div(lpc, VEC), 32);
+      const int64_t cthreads = round_up(ceil_div(lpc, lanes_per_thread), 32);
       const int threads = (int)cthreads + 32;
-      if (threads > 1024) continue;
+      if (threads > kMaxStagedThreads) continue;
       if ((int64_t)threads * fa.numRegs * cps > 65536) continue;
       const int64_t stage_bytes = round_up(lpc * stage_bytes_per_lane, 128);
       const int64_t seg_bytes = cthreads * seg_bytes_per_thread;

@@ -3,16 +3,19 @@
 //
 // Layout: every [T, B, N] tensor is t-major, so the L = B*N lanes of one step
 // are contiguous.  A lane is independent of every other lane and sequential
-// in t: each thread owns VEC=4 consecutive lanes and keeps their state (u, i,
+// in t: each thread owns 8 (Leaky) or 4 (Synaptic) consecutive lanes and keeps their state (u, i,
 // z and, backward, the adjoints) in registers for the whole scan.
 //
 // Staged kernels (the fast path): a CTA owns a contiguous strip of lanes.
 // One producer thread streams the strip's row of every input tensor, step by
 // step, into a ring of shared-memory stages with 1-D bulk copies (TMA,
-// cp.async.bulk) completing on an mbarrier per stage; the consumer warps wait
-// on the stage, read their lanes, release the stage on a second mbarrier and
-// write outputs with vector stores.  The ring depth, not the thread count,
-// supplies the bytes in flight that HBM needs.
+// cp.async.bulk) completing on a "full" mbarrier per stage; the consumer
+// warps wait on it, read their lanes, compute and store the step, and only
+// then release the stage on its "empty" mbarrier.  The ring depth, not the
+// thread count, supplies the bytes in flight that HBM needs.  Ring position
+// (stage index and phase parity) advances incrementally: no division in the
+// loop.  Reset mode and surrogate are template parameters (-1 = read at run
+// time) so the specialised loops carry no mode branches.
 //
 // Plain kernels: one lane per thread, direct loads; taken for shapes whose
 // rows are not 16-byte multiples.  Both use the same per-lane step code, so
@@ -27,9 +30,10 @@ enum { RESET_SUBTRACT = 0, RESET_ZERO = 1, RESET_NONE = 2 };
 enum { SG_FAST_SIGMOID = 0, SG_ATAN = 1 };
 enum { PM_SCALAR = 0, PM_PER_NEURON = 1, PM_PER_CHANNEL = 2 };
 constexpr uint32_t DEBUG_PRODUCER_IDLE = 1u;
-constexpr int VEC = 4;                 // lanes per thread in the staged kernels
+constexpr int VEC = 8;                 // lane granularity of a staged CTA strip
 constexpr int kBarrierBytes = 1024;    // room for up to 64 stages x 2 mbarriers
 constexpr int kMaxStages = 64;
+constexpr int kMaxStagedThreads = 512;
 constexpr uint64_t kDrainNs = 1000000000ull;
 
 struct ScanArgs {
@@ -89,30 +93,36 @@ __device__ __forceinline__ float lane_param(const float* p, int mode, int64_t l,
 }
 
 // One forward step, Eq. (4) / Eqs. (5)-(6), evaluated left to right as the
-// equations are written, one rounded fp32 operation at a time (no FMA), so
-// the forward and the backward's recomputation agree bit for bit.
-template <bool SYN>
-__device__ __forceinline__ void fwd_step(int reset, float beta, float thr, float alpha, float x,
-                                         float& u, bool& z, float& i) {
+// equations are written, one rounded fp32 operation at a time (no FMA that
+// would fuse two of them), so the forward and the backward's recomputation
+// agree bit for bit.  The subtract reset u - z*thr is one rounding since
+// z*thr is exact (z in {0,1}); reset-to-zero scales u by (1 - z) exactly.
+template <bool SYN, int RESET>
+__device__ __forceinline__ void fwd_step(int reset_rt, float beta, float thr, float alpha,
+                                         float x, float& u, bool& z, float& i) {
+  const int reset = RESET >= 0 ? RESET : reset_rt;
   float in = x;
   if (SYN) {
     i = __fadd_rn(__fmul_rn(alpha, i), x);
     in = i;
   }
+  const float zf = z ? 1.0f : 0.0f;
   float un;
   if (reset == RESET_ZERO) {
-    un = __fadd_rn(__fmul_rn(beta, z ? 0.0f : u), in);
+    un = __fadd_rn(__fmul_rn(beta, __fmul_rn(u, 1.0f - zf)), in);
   } else {
     un = __fadd_rn(__fmul_rn(beta, u), in);
-    if (reset == RESET_SUBTRACT && z) un = __fsub_rn(un, thr);
+    if (reset == RESET_SUBTRACT) un = __fmaf_rn(zf, -thr, un);
   }
   u = un;
   z = un > thr;  // Eq. (3), strict
 }
 
 // Surrogate dz/du at x = u - thr (Sec. III-B).
+template <int SG>
 __device__ __forceinline__ float surrogate(const ScanArgs& a, float x) {
-  if (a.sg == SG_FAST_SIGMOID) {
+  const int sg = SG >= 0 ? SG : a.sg;
+  if (sg == SG_FAST_SIGMOID) {
     const float d = fmaf(a.sg_a, fabsf(x), 1.0f);
     return __fdividef(1.0f, d * d);
   }
@@ -130,22 +140,23 @@ struct BwdLane {
 // parameter terms of step t+1 that need the step-t state
 // (d u_{t+1}/d beta = u_t or (1-z_t) u_t, the subtract reset's -z_t, and
 // d i_{t+1}/d alpha = i_t), then the adjoint of step t.  Returns dL/dI_t.
-template <bool SYN>
+template <bool SYN, int RESET, int SG>
 __device__ __forceinline__ float bwd_step(const ScanArgs& a, float beta, float thr, float alpha,
                                           bool has_next, float u, bool z, float i, float gs,
                                           float extra_u, float extra_i, BwdLane& s) {
+  const int reset = RESET >= 0 ? RESET : a.reset;
   if (has_next) {
-    s.dbeta = fmaf(s.du, (a.reset == RESET_ZERO && z) ? 0.0f : u, s.dbeta);
-    if (a.reset == RESET_SUBTRACT && z) s.dthr -= s.du;
+    s.dbeta = fmaf(s.du, (reset == RESET_ZERO && z) ? 0.0f : u, s.dbeta);
+    if (reset == RESET_SUBTRACT && z) s.dthr -= s.du;
     if (SYN) s.dalpha = fmaf(s.di, i, s.dalpha);
   }
-  const float sgv = surrogate(a, u - thr);
+  const float sgv = surrogate<SG>(a, u - thr);
   float dz = gs;
   if (!a.detach) {
-    if (a.reset == RESET_SUBTRACT) dz = fmaf(-thr, s.du, dz);
-    else if (a.reset == RESET_ZERO) dz = fmaf(-beta * u, s.du, dz);
+    if (reset == RESET_SUBTRACT) dz = fmaf(-thr, s.du, dz);
+    else if (reset == RESET_ZERO) dz = fmaf(-beta * u, s.du, dz);
   }
-  const float decay = (a.reset == RESET_ZERO && z) ? 0.0f : beta;
+  const float decay = (reset == RESET_ZERO && z) ? 0.0f : beta;
   const float du = fmaf(decay, s.du, fmaf(sgv, dz, extra_u));
   s.dthr = fmaf(-sgv, dz, s.dthr);
   s.du = du;
@@ -170,7 +181,7 @@ __device__ __forceinline__ void bwd_initial(const ScanArgs& a, float beta, float
   const float decay = (a.reset == RESET_ZERO && z_m1) ? 0.0f : beta;
   gmem0 = decay * s.du;
   if (have_mem0 && !a.detach && a.reset != RESET_NONE) {
-    const float sgv = surrogate(a, u_m1 - thr);
+    const float sgv = surrogate<-1>(a, u_m1 - thr);
     const float slope = (a.reset == RESET_SUBTRACT) ? -thr : -beta * u_m1;
     const float dz = slope * s.du;
     gmem0 = fmaf(sgv, dz, gmem0);
@@ -178,6 +189,103 @@ __device__ __forceinline__ void bwd_initial(const ScanArgs& a, float beta, float
   }
   gsyn0 = SYN ? alpha * s.di : 0.0f;
 }
+
+// ---------------------------------------------------------------------------
+// Packed pairs of lanes (Blackwell fp32x2: one instruction, two IEEE-rounded
+// lane results), used by the staged kernels
+// ---------------------------------------------------------------------------
+
+__device__ __forceinline__ float2 f2(float a) { return make_float2(a, a); }
+__device__ __forceinline__ float2 add2(float2 a, float2 b) { return __fadd2_rn(a, b); }
+__device__ __forceinline__ float2 mul2(float2 a, float2 b) { return __fmul2_rn(a, b); }
+__device__ __forceinline__ float2 fma2(float2 a, float2 b, float2 c) { return __ffma2_rn(a, b, c); }
+
+// 1 where x > 0 else 0; with x = fl(u - thr) this is Eq. (3): the rounded
+// difference of two floats is positive exactly when u > thr (no flush to 0)
+__device__ __forceinline__ float2 pos2(float2 x) {
+  return make_float2(x.x > 0.0f ? 1.0f : 0.0f, x.y > 0.0f ? 1.0f : 0.0f);
+}
+
+// Forward step on a pair of lanes: fwd_step on each lane (scalar operations
+// with explicit rounding, which the compiler never fuses; packed fp32x2
+// multiply and add may be fused into a packed FMA, which would change the
+// result).  negthr = -thr; z holds z_{t-1} on entry and z_t on exit (0/1).
+template <bool SYN, int RESET>
+__device__ __forceinline__ void fwd_pair(int reset_rt, float2 beta, float2 negthr, float2 alpha,
+                                         float2 x, float2& u, float2& z, float2& i) {
+  bool zx = z.x != 0.0f, zy = z.y != 0.0f;
+  fwd_step<SYN, RESET>(reset_rt, beta.x, -negthr.x, alpha.x, x.x, u.x, zx, i.x);
+  fwd_step<SYN, RESET>(reset_rt, beta.y, -negthr.y, alpha.y, x.y, u.y, zy, i.y);
+  z = make_float2(zx ? 1.0f : 0.0f, zy ? 1.0f : 0.0f);
+}
+
+template <int SG>
+__device__ __forceinline__ float2 surrogate2(const ScanArgs& a, float2 x) {
+  const int sg = SG >= 0 ? SG : a.sg;
+  if (sg == SG_FAST_SIGMOID) {
+    const float2 d = fma2(f2(a.sg_a), make_float2(fabsf(x.x), fabsf(x.y)), f2(1.0f));
+    const float2 d2 = mul2(d, d);
+    return make_float2(__fdividef(1.0f, d2.x), __fdividef(1.0f, d2.y));
+  }
+  const float2 y = mul2(f2(a.sg_b), x);
+  const float2 d = fma2(y, y, f2(1.0f));
+  return mul2(f2(a.sg_a), make_float2(__fdividef(1.0f, d.x), __fdividef(1.0f, d.y)));
+}
+
+// Reverse-pass state of a pair of lanes.  dthr accumulates
+// +(sigma'*dz + z_t*du_{t+1}); the threshold gradient is its negation.
+struct Bwd2 {
+  float2 du, di, dbeta, dthr, dalpha;
+};
+
+// One reverse step at time t on a pair of lanes (u, z, i = u_t, z_t, i_t).
+// du/di hold dL/du_{t+1}, dL/di_{t+1} on entry (zero at t = T-1, so the
+// parameter terms of step t+1 vanish there) and dL/du_t, dL/di_t on exit.
+// EXTRA adds eu to dL/du_t and ei to dL/di_t (grad_mem every step,
+// grad_mem_final / grad_syn_final at t = T-1).  Returns dL/dI_t.
+template <bool SYN, int RESET, int SG, bool EXTRA>
+__device__ __forceinline__ float2 bwd_pair(const ScanArgs& a, float2 beta, float2 negthr,
+                                           float2 alpha, float2 u, float2 z, float2 i,
+                                           float2 gs, float2 eu, float2 ei, Bwd2& s) {
+  const int reset = RESET >= 0 ? RESET : a.reset;
+  const float2 keep = add2(f2(1.0f), make_float2(-z.x, -z.y));  // 1 - z_t
+  s.dbeta = fma2(s.du, reset == RESET_ZERO ? mul2(u, keep) : u, s.dbeta);
+  if (reset == RESET_SUBTRACT) s.dthr = fma2(z, s.du, s.dthr);
+  if (SYN) s.dalpha = fma2(s.di, i, s.dalpha);
+  const float2 sg = surrogate2<SG>(a, add2(u, negthr));
+  float2 dz = gs;
+  if (!a.detach) {
+    if (reset == RESET_SUBTRACT) dz = fma2(negthr, s.du, dz);
+    else if (reset == RESET_ZERO) dz = fma2(mul2(f2(-1.0f), mul2(beta, u)), s.du, dz);
+  }
+  const float2 p = mul2(sg, dz);
+  const float2 decay = reset == RESET_ZERO ? mul2(beta, keep) : beta;
+  s.du = fma2(decay, s.du, p);
+  if (EXTRA) s.du = add2(s.du, eu);
+  s.dthr = add2(s.dthr, p);
+  if (SYN) {
+    s.di = fma2(alpha, s.di, s.du);
+    if (EXTRA) s.di = add2(s.di, ei);
+    return s.di;
+  }
+  return s.du;
+}
+
+// ---------------------------------------------------------------------------
+// Ring of shared-memory stages
+// ---------------------------------------------------------------------------
+
+// Stage index and phase parity of the next item; items are consumed in order.
+struct RingPos {
+  int s = 0;
+  uint32_t ph = 0;
+  __device__ __forceinline__ void next(int S) {
+    if (++s == S) {
+      s = 0;
+      ph ^= 1u;
+    }
+  }
+};
 
 // Warp-uniform bounded wait: every lane polls the barrier (so every lane
 // acquires the completed phase); the decision to give up is taken by lane 0's
@@ -195,46 +303,44 @@ __device__ __forceinline__ bool warp_wait(uint64_t* bar, uint32_t parity, uint64
   }
 }
 
-// ---------------------------------------------------------------------------
-// Producer: streams item j's tiles into stage j % S.
-// ---------------------------------------------------------------------------
-
 struct Tile {
   const void* src;  // global address of the strip's row (16-byte aligned)
   uint32_t bytes;   // multiple of 16
   uint32_t dst;     // byte offset inside the stage (multiple of 16)
 };
 
+// The single producer thread: fills stage after stage once the consumers
+// have released it, and drains its copies before the CTA may exit.
 struct Producer {
   unsigned char* ring;
   uint64_t* full;
   uint64_t* empty;
   int S;
   int stage_bytes;
+  RingPos pos;
+  bool wrapped = false;  // the ring has been filled once: wait for releases
   int64_t issued = 0;
   bool ok = true;
 
-  // Issue the next item into stage issued % S once the consumers released it.
   __device__ __forceinline__ void issue(const Tile* tiles, int n, const ScanArgs& a) {
     if (!ok) return;
-    const int64_t j = issued;
-    const int s = (int)(j % S);
-    if (j >= S &&
-        !mbar_wait_bounded(&empty[s], (uint32_t)(((j / S) - 1) & 1), a.wait_ns)) {
+    // round r >= 1 of stage s waits for the consumers' release of round r-1
+    if (wrapped && !mbar_wait_bounded(&empty[pos.s], pos.ph ^ 1u, a.wait_ns)) {
       record_status(a.status, kStatusTimeout);
       ok = false;
       return;
     }
     uint32_t total = 0;
     for (int k = 0; k < n; ++k) total += tiles[k].bytes;
-    mbar_arrive_expect_tx(&full[s], total);
-    unsigned char* dst = ring + (size_t)s * stage_bytes;
-    for (int k = 0; k < n; ++k) bulk_g2s(dst + tiles[k].dst, tiles[k].src, tiles[k].bytes, &full[s]);
-    issued = j + 1;
+    mbar_arrive_expect_tx(&full[pos.s], total);
+    unsigned char* dst = ring + (size_t)pos.s * stage_bytes;
+    for (int k = 0; k < n; ++k) bulk_g2s(dst + tiles[k].dst, tiles[k].src, tiles[k].bytes, &full[pos.s]);
+    ++issued;
+    pos.next(S);
+    if (pos.s == 0) wrapped = true;
   }
 
-  // Wait until every copy this thread issued has landed (bounded), so the
-  // CTA's shared memory outlives all of them.
+  // Wait (bounded) until the last copy into every stage has landed.
   __device__ __forceinline__ void drain() {
     const int64_t first = issued > S ? issued - S : 0;
     for (int64_t j = first; j < issued; ++j)
@@ -259,12 +365,86 @@ __device__ __forceinline__ void init_ring_barriers(uint64_t* full, uint64_t* emp
   __syncthreads();
 }
 
+// Release a stage: called only after the values read from it were consumed
+// (the step's outputs are computed and stored), so every lane's shared-memory
+// read has completed before the producer may overwrite the stage.
+__device__ __forceinline__ void release_stage(uint64_t* empty, int s, int lid) {
+  __syncwarp();
+  if (lid == 0) mbar_arrive(&empty[s]);
+}
+
+// Lanes per thread of the staged kernels: 8 for the Leaky neuron, 4 for the
+// Synaptic one (whose reverse pass carries five adjoints per lane).
+template <bool SYN>
+constexpr int kLanes = SYN ? 4 : 8;
+
+template <typename T, int NP>
+__device__ __forceinline__ void load_pairs(const T* p, float2 q[NP]) {
+  float v[2 * NP];
+  loadv<T, 2 * NP>(p, v);
+#pragma unroll
+  for (int k = 0; k < NP; ++k) q[k] = make_float2(v[2 * k], v[2 * k + 1]);
+}
+
+template <typename T, int NP>
+__device__ __forceinline__ void store_pairs(T* p, const float2 q[NP]) {
+  float v[2 * NP];
+#pragma unroll
+  for (int k = 0; k < NP; ++k) {
+    v[2 * k] = q[k].x;
+    v[2 * k + 1] = q[k].y;
+  }
+  storev<T, 2 * NP>(p, v);
+}
+
+template <int NP>
+__device__ __forceinline__ void load_pairs_global(const float* p, float2 q[NP]) {
+#pragma unroll
+  for (int k = 0; k < NP; ++k) q[k] = make_float2(p[2 * k], p[2 * k + 1]);
+}
+
+// beta, -thr and alpha of the thread's 2*NP lanes, as pairs
+template <bool SYN, int NP>
+__device__ __forceinline__ void load_params(const ScanArgs& a, int64_t l, float2 beta[NP],
+                                            float2 negthr[NP], float2 alpha[NP]) {
+#pragma unroll
+  for (int k = 0; k < NP; ++k) {
+    const int64_t m = l + 2 * k;
+    beta[k] = make_float2(lane_param(a.beta, a.beta_mode, m, a),
+                          lane_param(a.beta, a.beta_mode, m + 1, a));
+    negthr[k] = make_float2(-lane_param(a.thr, a.thr_mode, m, a),
+                            -lane_param(a.thr, a.thr_mode, m + 1, a));
+    alpha[k] = SYN ? make_float2(lane_param(a.alpha, a.alpha_mode, m, a),
+                                 lane_param(a.alpha, a.alpha_mode, m + 1, a))
+                   : f2(0.0f);
+  }
+}
+
+// Initial state of the thread's lanes: u_{-1} = mem0 (or 0), z_{-1} =
+// [mem0 > thr] when mem0 is given (else 0), i_{-1} = syn0 (or 0).
+template <bool SYN, int NP>
+__device__ __forceinline__ void initial_state(const ScanArgs& a, int64_t l, const float2 negthr[NP],
+                                              float2 u[NP], float2 z[NP], float2 i[NP]) {
+#pragma unroll
+  for (int k = 0; k < NP; ++k) {
+    if (a.mem0) {
+      u[k] = make_float2(a.mem0[l + 2 * k], a.mem0[l + 2 * k + 1]);
+      z[k] = pos2(add2(u[k], negthr[k]));
+    } else {
+      u[k] = f2(0.0f);
+      z[k] = f2(0.0f);
+    }
+    i[k] = (SYN && a.syn0) ? make_float2(a.syn0[l + 2 * k], a.syn0[l + 2 * k + 1]) : f2(0.0f);
+  }
+}
+
 // ---------------------------------------------------------------------------
 // Staged forward
 // ---------------------------------------------------------------------------
 
-template <bool SYN, typename TI, typename TO>
-__global__ void __launch_bounds__(1024) scan_fwd_staged(const ScanArgs a) {
+template <bool SYN, typename TI, typename TO, int RESET>
+__global__ void __launch_bounds__(kMaxStagedThreads) scan_fwd_staged(const ScanArgs a) {
+  constexpr int V = kLanes<SYN>, NP = V / 2;
   extern __shared__ __align__(1024) unsigned char smem[];
   uint64_t* full = reinterpret_cast<uint64_t*>(smem);
   uint64_t* empty = full + kMaxStages;
@@ -279,10 +459,10 @@ __global__ void __launch_bounds__(1024) scan_fwd_staged(const ScanArgs a) {
   if (warp == cwarps) {  // producer warp
     if (lid == 0 && !(a.debug & DEBUG_PRODUCER_IDLE)) {
       Producer p{ring, full, empty, S, a.stage_bytes};
-      const uint32_t bytes = (uint32_t)cta_lanes * sizeof(TI);
+      Tile tile{static_cast<const TI*>(a.I) + lane0, (uint32_t)cta_lanes * (uint32_t)sizeof(TI), 0};
       for (int64_t t = 0; t < a.T && p.ok; ++t) {
-        const Tile tile{row<TI>(a.I, t, a.L, lane0), bytes, 0};
         p.issue(&tile, 1, a);
+        tile.src = static_cast<const TI*>(tile.src) + a.L;
       }
       p.drain();
     }
@@ -290,63 +470,54 @@ __global__ void __launch_bounds__(1024) scan_fwd_staged(const ScanArgs a) {
   }
 
   const int c = threadIdx.x;
-  const int64_t l = lane0 + (int64_t)c * VEC;
-  const bool active = c * VEC < cta_lanes;
-  float beta[VEC], thr[VEC], alpha[VEC], u[VEC], in[VEC];
-  bool z[VEC];
+  const int64_t l = lane0 + (int64_t)c * V;
+  const bool active = c * V < cta_lanes;
+  float2 beta[NP], negthr[NP], alpha[NP], u[NP], z[NP], in[NP];
   if (active) {
-#pragma unroll
-    for (int v = 0; v < VEC; ++v) {
-      beta[v] = lane_param(a.beta, a.beta_mode, l + v, a);
-      thr[v] = lane_param(a.thr, a.thr_mode, l + v, a);
-      alpha[v] = SYN ? lane_param(a.alpha, a.alpha_mode, l + v, a) : 0.0f;
-      u[v] = a.mem0 ? a.mem0[l + v] : 0.0f;
-      z[v] = a.mem0 ? (u[v] > thr[v]) : false;
-      in[v] = (SYN && a.syn0) ? a.syn0[l + v] : 0.0f;
-    }
+    load_params<SYN, NP>(a, l, beta, negthr, alpha);
+    initial_state<SYN, NP>(a, l, negthr, u, z, in);
   }
-  TO* spk = static_cast<TO*>(a.spk);
-  TO* mem = static_cast<TO*>(a.mem);
-  TO* syn = static_cast<TO*>(a.syn);
-  const int64_t ckpt_stride = SYN ? 2 * a.L : a.L;
+  TO* spk = static_cast<TO*>(a.spk) + l;
+  TO* mem = a.mem ? static_cast<TO*>(a.mem) + l : nullptr;
+  TO* syn = (SYN && a.syn) ? static_cast<TO*>(a.syn) + l : nullptr;
+  float* ck = a.ckpt ? a.ckpt + l : nullptr;
+  const int64_t ck_stride = SYN ? 2 * a.L : a.L;
+  const TI* my = reinterpret_cast<const TI*>(ring) + c * V;
+  const int stage_elems = a.stage_bytes / (int)sizeof(TI);
+  RingPos pos;
   int kk = 0;  // position inside the current checkpoint segment
   for (int64_t t = 0; t < a.T; ++t) {
-    const int s = (int)(t % S);
-    if (!warp_wait(&full[s], (uint32_t)((t / S) & 1), a.wait_ns)) {
+    if (!warp_wait(&full[pos.s], pos.ph, a.wait_ns)) {
       if (lid == 0) record_status(a.status, kStatusTimeout);
       break;
     }
-    float x[VEC];
-    if (active) Elem<TI>::load4(reinterpret_cast<const TI*>(ring + (size_t)s * a.stage_bytes) + c * VEC, x);
     if (active) {
-      float zf[VEC];
+      float2 x[NP];
+      load_pairs<TI, NP>(my + pos.s * stage_elems, x);
 #pragma unroll
-      for (int v = 0; v < VEC; ++v) {
-        fwd_step<SYN>(a.reset, beta[v], thr[v], alpha[v], x[v], u[v], z[v], in[v]);
-        zf[v] = z[v] ? 1.0f : 0.0f;
-      }
-      const int64_t off = t * a.L + l;
-      Elem<TO>::store4(spk + off, zf);
-      if (mem) Elem<TO>::store4(mem + off, u);
-      if (SYN && syn) Elem<TO>::store4(syn + off, in);
+      for (int k = 0; k < NP; ++k)
+        fwd_pair<SYN, RESET>(a.reset, beta[k], negthr[k], alpha[k], x[k], u[k], z[k], in[k]);
+      store_pairs<TO, NP>(spk, z);
+      if (mem) store_pairs<TO, NP>(mem, u);
+      if (SYN && syn) store_pairs<TO, NP>(syn, in);
       if (++kk == a.K) {
         kk = 0;
-        if (a.ckpt && t + 1 < a.T) {
-          float* cp = a.ckpt + (t / a.K) * ckpt_stride + l;
-          Elem<float>::store4(cp, u);
-          if (SYN) Elem<float>::store4(cp + a.L, in);
+        if (ck && t + 1 < a.T) {
+          store_pairs<float, NP>(ck, u);
+          if (SYN) store_pairs<float, NP>(ck + a.L, in);
+          ck += ck_stride;
         }
       }
     }
-    // Release the stage only after its values were consumed: the stores
-    // above depend on them, so every lane's shared-memory read has completed
-    // before the producer may refill the stage with a bulk copy.
-    __syncwarp();
-    if (lid == 0) mbar_arrive(&empty[s]);
+    release_stage(empty, pos.s, lid);
+    pos.next(S);
+    spk += a.L;
+    if (mem) mem += a.L;
+    if (SYN && syn) syn += a.L;
   }
   if (active) {
-    if (a.mem_final) Elem<float>::store4(a.mem_final + l, u);
-    if (SYN && a.syn_final) Elem<float>::store4(a.syn_final + l, in);
+    if (a.mem_final) store_pairs<float, NP>(a.mem_final + l, u);
+    if (SYN && a.syn_final) store_pairs<float, NP>(a.syn_final + l, in);
   }
 }
 
@@ -359,8 +530,24 @@ __global__ void __launch_bounds__(1024) scan_fwd_staged(const ScanArgs a) {
 // {grad_spk, [grad_mem]} run the reverse steps.
 // ---------------------------------------------------------------------------
 
-template <bool SYN, bool RECOMP, typename TI, typename TO>
-__global__ void __launch_bounds__(1024) scan_bwd_staged(const ScanArgs a) {
+// The reverse step on all of a thread's pairs; EXTRA steps (grad_mem given,
+// or t = T-1 with grad_mem_final / grad_syn_final) add those gradients.
+template <bool SYN, int RESET, int SG, bool EXTRA, int NP>
+__device__ __forceinline__ void bwd_pairs(const ScanArgs& a, const float2 beta[NP],
+                                          const float2 negthr[NP], const float2 alpha[NP],
+                                          const float2 u[NP], const float2 z[NP],
+                                          const float2 i[NP], const float2 g[NP],
+                                          const float2 eu[NP], const float2 ei[NP], Bwd2 st[NP],
+                                          float2 out[NP]) {
+#pragma unroll
+  for (int k = 0; k < NP; ++k)
+    out[k] = bwd_pair<SYN, RESET, SG, EXTRA>(a, beta[k], negthr[k], alpha[k], u[k], z[k], i[k],
+                                             g[k], eu[k], ei[k], st[k]);
+}
+
+template <bool SYN, bool RECOMP, typename TI, typename TO, int RESET, int SG>
+__global__ void __launch_bounds__(kMaxStagedThreads) scan_bwd_staged(const ScanArgs a) {
+  constexpr int V = kLanes<SYN>, NP = V / 2;
   extern __shared__ __align__(1024) unsigned char smem[];
   uint64_t* full = reinterpret_cast<uint64_t*>(smem);
   uint64_t* empty = full + kMaxStages;
@@ -371,14 +558,14 @@ __global__ void __launch_bounds__(1024) scan_bwd_staged(const ScanArgs a) {
   const int warp = threadIdx.x >> 5, lid = threadIdx.x & 31;
   const int64_t lane0 = (int64_t)blockIdx.x * a.lanes_per_cta;
   const int cta_lanes = (int)min((int64_t)a.lanes_per_cta, a.L - lane0);
-  const int io_stride = a.lanes_per_cta * (int)sizeof(TO);   // tile stride of io tiles
+  const int io_stride = a.lanes_per_cta * (int)sizeof(TO);  // byte stride of io tiles
   const int in_stride = a.lanes_per_cta * (int)sizeof(TI);
-  const bool half_store = !RECOMP && sizeof(TO) != 4;       // z from the spk rows
+  const bool half_store = !RECOMP && sizeof(TO) != 4;      // z from the spk rows
   const bool want_syn = SYN && a.part_alpha != nullptr;
   // store-mode tile order: gs, mem, [spk], [syn], [gm]
   const int t_spk = 2, t_syn = 2 + (half_store ? 1 : 0);
   const int t_gm_store = t_syn + ((!RECOMP && want_syn) ? 1 : 0);
-  const int ck_off = (in_stride + 15) & ~15;  // recompute: checkpoint tiles after I
+  const int ck_off = in_stride;  // recompute: checkpoint tiles after the I tile
   init_ring_barriers(full, empty, S, cwarps);
 
   if (warp == cwarps) {
@@ -427,165 +614,200 @@ __global__ void __launch_bounds__(1024) scan_bwd_staged(const ScanArgs a) {
   }
 
   const int c = threadIdx.x;
-  const int64_t l = lane0 + (int64_t)c * VEC;
-  const bool active = c * VEC < cta_lanes;
-  float beta[VEC], thr[VEC], alpha[VEC], m0[VEC], s0[VEC], ex_u[VEC], ex_i[VEC];
-  BwdLane st[VEC];
-  const bool have_mem0 = a.mem0 != nullptr;
-  if (active) {
+  const int64_t l = lane0 + (int64_t)c * V;
+  const bool active = c * V < cta_lanes;
+  float2 beta[NP], negthr[NP], alpha[NP];
+  Bwd2 st[NP];
+  if (active) load_params<SYN, NP>(a, l, beta, negthr, alpha);
 #pragma unroll
-    for (int v = 0; v < VEC; ++v) {
-      beta[v] = lane_param(a.beta, a.beta_mode, l + v, a);
-      thr[v] = lane_param(a.thr, a.thr_mode, l + v, a);
-      alpha[v] = SYN ? lane_param(a.alpha, a.alpha_mode, l + v, a) : 0.0f;
-      m0[v] = have_mem0 ? a.mem0[l + v] : 0.0f;
-      s0[v] = (SYN && a.syn0) ? a.syn0[l + v] : 0.0f;
-      ex_u[v] = a.gmf ? a.gmf[l + v] : 0.0f;
-      ex_i[v] = (SYN && a.gsf) ? a.gsf[l + v] : 0.0f;
-      st[v] = BwdLane{0.0f, 0.0f, 0.0f, 0.0f, 0.0f};
-    }
-  }
-  TO* gI = static_cast<TO*>(a.gI);
-  // per-thread replay buffer for one checkpoint segment: [K][nthr][VEC] fp32
-  // (u), followed by the same for i (Synaptic)
-  float* seg = reinterpret_cast<float*>(ring + (size_t)S * a.stage_bytes);
-  const size_t seg_plane = (size_t)a.K * nthr * VEC;
+  for (int k = 0; k < NP; ++k) st[k] = Bwd2{f2(0.0f), f2(0.0f), f2(0.0f), f2(0.0f), f2(0.0f)};
+  const int stage_io_elems = a.stage_bytes / (int)sizeof(TO);
+  const int stage_in_elems = a.stage_bytes / (int)sizeof(TI);
+  const int stage_f32 = a.stage_bytes / 4;
+  const int tile_io_elems = a.lanes_per_cta;  // elements per io tile
+  const TO* ring_o = reinterpret_cast<const TO*>(ring) + c * V;
+  const TI* ring_i = reinterpret_cast<const TI*>(ring) + c * V;
+  const float* ring_f = reinterpret_cast<const float*>(ring) + c * V;
+  TO* gI = static_cast<TO*>(a.gI) + l + (a.T - 1) * a.L;  // walks backwards
+  // per-thread replay buffer: [K][V/4 planes][nthr][4] fp32 for u, then i
+  // (each plane holds 4 lanes of every thread: conflict-free 16-byte rows)
+  float* seg = reinterpret_cast<float*>(ring + (size_t)S * a.stage_bytes) + c * 4;
+  const int seg_row = (V / 4) * nthr * 4;  // floats per replayed step
+  const size_t seg_plane = (size_t)a.K * seg_row;
+  RingPos pos;
   bool ok = true;
-  int64_t j = 0;  // item counter, mirrors the producer's
 
-  auto wait_item = [&](int64_t jj, const unsigned char*& base) -> bool {
-    const int s = (int)(jj % S);
-    if (!warp_wait(&full[s], (uint32_t)((jj / S) & 1), a.wait_ns)) {
-      if (lid == 0) record_status(a.status, kStatusTimeout);
-      return false;
+  // one reverse step on the thread's pairs: general (EXTRA) only where needed
+  auto reverse = [&](int64_t t, const float2 u[NP], const float2 z[NP], const float2 i[NP],
+                     const float2 g[NP], const float2 gmv[NP], float2 out[NP]) {
+    if (a.gm || t == a.T - 1) {
+      float2 eu[NP], ei[NP];
+#pragma unroll
+      for (int k = 0; k < NP; ++k) {
+        eu[k] = a.gm ? gmv[k] : f2(0.0f);
+        ei[k] = f2(0.0f);
+      }
+      if (t == a.T - 1) {
+        float2 fu[NP], fi[NP];
+        if (a.gmf) load_pairs_global<NP>(a.gmf + l, fu);
+        if (SYN && a.gsf) load_pairs_global<NP>(a.gsf + l, fi);
+#pragma unroll
+        for (int k = 0; k < NP; ++k) {
+          if (a.gmf) eu[k] = add2(eu[k], fu[k]);
+          if (SYN && a.gsf) ei[k] = fi[k];
+        }
+      }
+      bwd_pairs<SYN, RESET, SG, true, NP>(a, beta, negthr, alpha, u, z, i, g, eu, ei, st, out);
+    } else {
+      bwd_pairs<SYN, RESET, SG, false, NP>(a, beta, negthr, alpha, u, z, i, g, g, g, st, out);
     }
-    base = ring + (size_t)s * a.stage_bytes;
-    return true;
-  };
-  // Called only once the values read from item jj's stage have been consumed
-  // (outputs computed and stored), so the reads have completed before the
-  // producer may overwrite the stage.
-  auto release_item = [&](int64_t jj) {
-    __syncwarp();
-    if (lid == 0) mbar_arrive(&empty[(int)(jj % S)]);
   };
 
   if (!RECOMP) {
-    for (int64_t t = a.T - 1; t >= 0; --t, ++j) {
-      const unsigned char* base;
-      if (!wait_item(j, base)) { ok = false; break; }
-      float g[VEC], uu[VEC], zz[VEC], ii[VEC], gmv[VEC];
-      if (active) {
-        Elem<TO>::load4(reinterpret_cast<const TO*>(base) + c * VEC, g);
-        Elem<TO>::load4(reinterpret_cast<const TO*>(base + io_stride) + c * VEC, uu);
-        if (half_store) Elem<TO>::load4(reinterpret_cast<const TO*>(base + t_spk * io_stride) + c * VEC, zz);
-        if (want_syn) Elem<TO>::load4(reinterpret_cast<const TO*>(base + t_syn * io_stride) + c * VEC, ii);
-        if (a.gm) Elem<TO>::load4(reinterpret_cast<const TO*>(base + t_gm_store * io_stride) + c * VEC, gmv);
+    for (int64_t t = a.T - 1; t >= 0; --t) {
+      if (!warp_wait(&full[pos.s], pos.ph, a.wait_ns)) {
+        if (lid == 0) record_status(a.status, kStatusTimeout);
+        ok = false;
+        break;
       }
       if (active) {
-        float out[VEC];
-        const bool last = (t == a.T - 1);
+        const TO* base = ring_o + pos.s * stage_io_elems;
+        float2 g[NP], uu[NP], zz[NP], ii[NP], gmv[NP], out[NP];
+        load_pairs<TO, NP>(base, g);
+        load_pairs<TO, NP>(base + tile_io_elems, uu);
+        if (half_store) {
+          load_pairs<TO, NP>(base + t_spk * tile_io_elems, zz);
+        } else {
 #pragma unroll
-        for (int v = 0; v < VEC; ++v) {
-          const bool zv = half_store ? (zz[v] != 0.0f) : (uu[v] > thr[v]);
-          const float eu = (a.gm ? gmv[v] : 0.0f) + (last ? ex_u[v] : 0.0f);
-          out[v] = bwd_step<SYN>(a, beta[v], thr[v], alpha[v], !last, uu[v], zv,
-                                 want_syn ? ii[v] : 0.0f, g[v], eu, last ? ex_i[v] : 0.0f, st[v]);
+          for (int k = 0; k < NP; ++k) zz[k] = pos2(add2(uu[k], negthr[k]));
         }
-        Elem<TO>::store4(gI + t * a.L + l, out);
+        if (want_syn) {
+          load_pairs<TO, NP>(base + t_syn * tile_io_elems, ii);
+        } else {
+#pragma unroll
+          for (int k = 0; k < NP; ++k) ii[k] = f2(0.0f);
+        }
+        if (a.gm) load_pairs<TO, NP>(base + t_gm_store * tile_io_elems, gmv);
+        reverse(t, uu, zz, ii, g, gmv, out);
+        store_pairs<TO, NP>(gI, out);
       }
-      release_item(j);  // after the values read from the stage were consumed
+      release_stage(empty, pos.s, lid);
+      pos.next(S);
+      gI -= a.L;
     }
   } else {
     for (int k = a.nseg - 1; k >= 0 && ok; --k) {
       const int64_t t0 = (int64_t)k * a.K, t1 = min(a.T, t0 + a.K);
-      float u[VEC], ii[VEC];
-      bool z[VEC];
+      float2 u[NP], z[NP], ii[NP];
       // replay the forward over the segment
-      for (int64_t t = t0; t < t1; ++t, ++j) {
-        const unsigned char* base;
-        if (!wait_item(j, base)) { ok = false; break; }
-        float x[VEC];
+      float* su = seg;
+      for (int64_t t = t0; t < t1; ++t) {
+        if (!warp_wait(&full[pos.s], pos.ph, a.wait_ns)) {
+          if (lid == 0) record_status(a.status, kStatusTimeout);
+          ok = false;
+          break;
+        }
         if (active) {
-          Elem<TI>::load4(reinterpret_cast<const TI*>(base) + c * VEC, x);
+          float2 x[NP];
+          load_pairs<TI, NP>(ring_i + pos.s * stage_in_elems, x);
           if (t == t0) {
             if (k > 0) {
-              Elem<float>::load4(reinterpret_cast<const float*>(base + ck_off) + c * VEC, u);
-              if (SYN)
-                Elem<float>::load4(reinterpret_cast<const float*>(base + ck_off + a.lanes_per_cta * 4) + c * VEC, ii);
+              const float* cb = ring_f + pos.s * stage_f32 + ck_off / 4;
+              load_pairs<float, NP>(cb, u);
+              if (SYN) load_pairs<float, NP>(cb + a.lanes_per_cta, ii);
 #pragma unroll
-              for (int v = 0; v < VEC; ++v) z[v] = u[v] > thr[v];
+              for (int q = 0; q < NP; ++q) z[q] = pos2(add2(u[q], negthr[q]));
             } else {
-#pragma unroll
-              for (int v = 0; v < VEC; ++v) {
-                u[v] = m0[v];
-                z[v] = have_mem0 && (m0[v] > thr[v]);
-                ii[v] = s0[v];
-              }
+              initial_state<SYN, NP>(a, l, negthr, u, z, ii);
             }
           }
-        }
-        if (active) {
 #pragma unroll
-          for (int v = 0; v < VEC; ++v)
-            fwd_step<SYN>(a.reset, beta[v], thr[v], alpha[v], x[v], u[v], z[v], ii[v]);
-          float* su = seg + ((size_t)(t - t0) * nthr + c) * VEC;
-          Elem<float>::store4(su, u);
-          if (SYN) Elem<float>::store4(su + seg_plane, ii);
+          for (int q = 0; q < NP; ++q)
+            fwd_pair<SYN, RESET>(a.reset, beta[q], negthr[q], alpha[q], x[q], u[q], z[q], ii[q]);
+#pragma unroll
+          for (int q = 0; q < V / 4; ++q) {
+            *reinterpret_cast<float4*>(su + q * nthr * 4) =
+                make_float4(u[2 * q].x, u[2 * q].y, u[2 * q + 1].x, u[2 * q + 1].y);
+            if (SYN)
+              *reinterpret_cast<float4*>(su + seg_plane + q * nthr * 4) =
+                  make_float4(ii[2 * q].x, ii[2 * q].y, ii[2 * q + 1].x, ii[2 * q + 1].y);
+          }
         }
-        release_item(j);
+        release_stage(empty, pos.s, lid);
+        pos.next(S);
+        su += seg_row;
       }
       if (!ok) break;
       // reverse steps over the segment
-      for (int64_t t = t1 - 1; t >= t0; --t, ++j) {
-        const unsigned char* base;
-        if (!wait_item(j, base)) { ok = false; break; }
-        float g[VEC], gmv[VEC];
-        if (active) {
-          Elem<TO>::load4(reinterpret_cast<const TO*>(base) + c * VEC, g);
-          if (a.gm) Elem<TO>::load4(reinterpret_cast<const TO*>(base + io_stride) + c * VEC, gmv);
+      for (int64_t t = t1 - 1; t >= t0; --t) {
+        su -= seg_row;
+        if (!warp_wait(&full[pos.s], pos.ph, a.wait_ns)) {
+          if (lid == 0) record_status(a.status, kStatusTimeout);
+          ok = false;
+          break;
         }
         if (active) {
-          const float* su = seg + ((size_t)(t - t0) * nthr + c) * VEC;
-          float uu[VEC], iv[VEC], out[VEC];
-          Elem<float>::load4(su, uu);
-          if (SYN) Elem<float>::load4(su + seg_plane, iv);
-          const bool last = (t == a.T - 1);
+          const TO* base = ring_o + pos.s * stage_io_elems;
+          float2 g[NP], gmv[NP], uu[NP], zz[NP], iv[NP], out[NP];
+          load_pairs<TO, NP>(base, g);
+          if (a.gm) load_pairs<TO, NP>(base + tile_io_elems, gmv);
 #pragma unroll
-          for (int v = 0; v < VEC; ++v) {
-            const float eu = (a.gm ? gmv[v] : 0.0f) + (last ? ex_u[v] : 0.0f);
-            out[v] = bwd_step<SYN>(a, beta[v], thr[v], alpha[v], !last, uu[v], uu[v] > thr[v],
-                                   SYN ? iv[v] : 0.0f, g[v], eu, last ? ex_i[v] : 0.0f, st[v]);
+          for (int q = 0; q < V / 4; ++q) {
+            const float4 uq = *reinterpret_cast<const float4*>(su + q * nthr * 4);
+            uu[2 * q] = make_float2(uq.x, uq.y);
+            uu[2 * q + 1] = make_float2(uq.z, uq.w);
+            if (SYN) {
+              const float4 iq = *reinterpret_cast<const float4*>(su + seg_plane + q * nthr * 4);
+              iv[2 * q] = make_float2(iq.x, iq.y);
+              iv[2 * q + 1] = make_float2(iq.z, iq.w);
+            } else {
+              iv[2 * q] = f2(0.0f);
+              iv[2 * q + 1] = f2(0.0f);
+            }
           }
-          Elem<TO>::store4(gI + t * a.L + l, out);
+#pragma unroll
+          for (int q = 0; q < NP; ++q) zz[q] = pos2(add2(uu[q], negthr[q]));
+          reverse(t, uu, zz, iv, g, gmv, out);
+          store_pairs<TO, NP>(gI, out);
         }
-        release_item(j);
+        release_stage(empty, pos.s, lid);
+        pos.next(S);
+        gI -= a.L;
       }
     }
   }
   if (!ok || !active) return;
-  float gm0[VEC], gs0[VEC], db[VEC], dt[VEC], da[VEC];
+  float gm0[V], gs0[V], db[V], dt[V], da[V];
 #pragma unroll
-  for (int v = 0; v < VEC; ++v) {
+  for (int v = 0; v < V; ++v) {
+    const Bwd2& q = st[v / 2];
+    const bool hi = v & 1;
+    BwdLane sl{hi ? q.du.y : q.du.x, hi ? q.di.y : q.di.x, hi ? q.dbeta.y : q.dbeta.x,
+               -(hi ? q.dthr.y : q.dthr.x), hi ? q.dalpha.y : q.dalpha.x};
+    const float b = hi ? beta[v / 2].y : beta[v / 2].x;
+    const float th = -(hi ? negthr[v / 2].y : negthr[v / 2].x);
+    const float al = hi ? alpha[v / 2].y : alpha[v / 2].x;
     if (a.T == 0) {
-      gm0[v] = ex_u[v];
-      gs0[v] = ex_i[v];
+      gm0[v] = a.gmf ? a.gmf[l + v] : 0.0f;
+      gs0[v] = (SYN && a.gsf) ? a.gsf[l + v] : 0.0f;
     } else {
-      bwd_initial<SYN>(a, beta[v], thr[v], alpha[v], have_mem0, m0[v], s0[v], st[v], gm0[v], gs0[v]);
+      const float m0 = a.mem0 ? a.mem0[l + v] : 0.0f;
+      const float s0 = (SYN && a.syn0) ? a.syn0[l + v] : 0.0f;
+      bwd_initial<SYN>(a, b, th, al, a.mem0 != nullptr, m0, s0, sl, gm0[v], gs0[v]);
     }
-    db[v] = st[v].dbeta;
-    dt[v] = st[v].dthr;
-    da[v] = st[v].dalpha;
+    db[v] = sl.dbeta;
+    dt[v] = sl.dthr;
+    da[v] = sl.dalpha;
   }
-  if (a.gmem0) Elem<float>::store4(a.gmem0 + l, gm0);
-  if (SYN && a.gsyn0) Elem<float>::store4(a.gsyn0 + l, gs0);
-  if (a.part_beta) Elem<float>::store4(a.part_beta + l, db);
-  if (a.part_thr) Elem<float>::store4(a.part_thr + l, dt);
-  if (SYN && a.part_alpha) Elem<float>::store4(a.part_alpha + l, da);
+  if (a.gmem0) storev<float, V>(a.gmem0 + l, gm0);
+  if (SYN && a.gsyn0) storev<float, V>(a.gsyn0 + l, gs0);
+  if (a.part_beta) storev<float, V>(a.part_beta + l, db);
+  if (a.part_thr) storev<float, V>(a.part_thr + l, dt);
+  if (SYN && a.part_alpha) storev<float, V>(a.part_alpha + l, da);
 }
 
 // ---------------------------------------------------------------------------
-// Plain kernels: one lane per thread, direct loads, any shape.
+// Plain kernels: one lane per thread, direct loads, any shape, run-time modes.
 // ---------------------------------------------------------------------------
 
 template <bool SYN, typename TI, typename TO>
@@ -606,7 +828,7 @@ __global__ void __launch_bounds__(256) scan_fwd_plain(const ScanArgs a) {
   int kk = 0;
   for (int64_t t = 0; t < a.T; ++t) {
     const int64_t off = t * a.L + l;
-    fwd_step<SYN>(a.reset, beta, thr, alpha, Elem<TI>::load1(I + off), u, z, i);
+    fwd_step<SYN, -1>(a.reset, beta, thr, alpha, Elem<TI>::load1(I + off), u, z, i);
     Elem<TO>::store1(spk + off, z ? 1.0f : 0.0f);
     if (mem) Elem<TO>::store1(mem + off, u);
     if (SYN && syn) Elem<TO>::store1(syn + off, i);
@@ -653,9 +875,9 @@ __global__ void __launch_bounds__(128) scan_bwd_plain(const ScanArgs a) {
       const float i = want_syn ? Elem<TO>::load1(syn + off) : 0.0f;
       const bool last = (t == a.T - 1);
       const float eu = (gm ? Elem<TO>::load1(gm + off) : 0.0f) + (last ? ex_u : 0.0f);
-      Elem<TO>::store1(gI + off, bwd_step<SYN>(a, beta, thr, alpha, !last, u, z, i,
-                                               Elem<TO>::load1(gs + off), eu,
-                                               last ? ex_i : 0.0f, st));
+      Elem<TO>::store1(gI + off, bwd_step<SYN, -1, -1>(a, beta, thr, alpha, !last, u, z, i,
+                                                       Elem<TO>::load1(gs + off), eu,
+                                                       last ? ex_i : 0.0f, st));
     }
   } else {
     const TI* I = static_cast<const TI*>(a.I);
@@ -676,7 +898,7 @@ __global__ void __launch_bounds__(128) scan_bwd_plain(const ScanArgs a) {
         z = have_mem0 && (m0 > thr);
       }
       for (int64_t t = t0; t < t1; ++t) {
-        fwd_step<SYN>(a.reset, beta, thr, alpha, Elem<TI>::load1(I + t * a.L + l), u, z, i);
+        fwd_step<SYN, -1>(a.reset, beta, thr, alpha, Elem<TI>::load1(I + t * a.L + l), u, z, i);
         su[(t - t0) * blockDim.x] = u;
         if (SYN) si[(t - t0) * blockDim.x] = i;
       }
@@ -686,9 +908,9 @@ __global__ void __launch_bounds__(128) scan_bwd_plain(const ScanArgs a) {
         const float iv = SYN ? si[(t - t0) * blockDim.x] : 0.0f;
         const bool last = (t == a.T - 1);
         const float eu = (gm ? Elem<TO>::load1(gm + off) : 0.0f) + (last ? ex_u : 0.0f);
-        Elem<TO>::store1(gI + off, bwd_step<SYN>(a, beta, thr, alpha, !last, uu, uu > thr, iv,
-                                                 Elem<TO>::load1(gs + off), eu,
-                                                 last ? ex_i : 0.0f, st));
+        Elem<TO>::store1(gI + off, bwd_step<SYN, -1, -1>(a, beta, thr, alpha, !last, uu,
+                                                         uu > thr, iv, Elem<TO>::load1(gs + off),
+                                                         eu, last ? ex_i : 0.0f, st));
       }
     }
   }

@@ -94,11 +94,12 @@ snn_status_t check_ws(const snn_scan_desc* d, const void* ws, size_t ws_bytes) {
   return aligned16(ws) ? SNN_OK : SNN_ERR_ALIGNMENT;
 }
 
-// Rows of every streamed tensor must be 16-byte multiples for the TMA path.
+// Rows of every streamed tensor must be 16-byte multiples for the TMA path,
+// and lanes come in groups of VEC per thread.
 bool staged_ok(const snn_scan_desc* d) {
   if (d->debug_flags & 2u) return false;  // SNN_DEBUG_FORCE_PLAIN
   const int64_t L = d->B * d->N;
-  return L > 0 && (L * (int64_t)dtype_size(d->in_dtype)) % 16 == 0 &&
+  return L > 0 && L % VEC == 0 && (L * (int64_t)dtype_size(d->in_dtype)) % 16 == 0 &&
          (L * (int64_t)dtype_size(d->io_dtype)) % 16 == 0 && (L * 4) % 16 == 0;
 }
 

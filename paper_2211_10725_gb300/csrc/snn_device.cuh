@@ -87,7 +87,7 @@ __device__ __forceinline__ void record_status(int* status, int code) {
 }
 
 // ---------------------------------------------------------------------------
-// Element conversion: VEC=4 consecutive elements <-> float[4]
+// Element conversion: 8 or 4 consecutive elements <-> float[], or one element
 // ---------------------------------------------------------------------------
 
 template <typename T>
@@ -95,9 +95,19 @@ struct Elem;
 
 template <>
 struct Elem<float> {
+  static __device__ __forceinline__ void load8(const float* p, float v[8]) {
+    const float4 a = reinterpret_cast<const float4*>(p)[0];
+    const float4 b = reinterpret_cast<const float4*>(p)[1];
+    v[0] = a.x; v[1] = a.y; v[2] = a.z; v[3] = a.w;
+    v[4] = b.x; v[5] = b.y; v[6] = b.z; v[7] = b.w;
+  }
+  static __device__ __forceinline__ void store8(float* p, const float v[8]) {
+    reinterpret_cast<float4*>(p)[0] = make_float4(v[0], v[1], v[2], v[3]);
+    reinterpret_cast<float4*>(p)[1] = make_float4(v[4], v[5], v[6], v[7]);
+  }
   static __device__ __forceinline__ void load4(const float* p, float v[4]) {
-    const float4 x = *reinterpret_cast<const float4*>(p);
-    v[0] = x.x; v[1] = x.y; v[2] = x.z; v[3] = x.w;
+    const float4 a = *reinterpret_cast<const float4*>(p);
+    v[0] = a.x; v[1] = a.y; v[2] = a.z; v[3] = a.w;
   }
   static __device__ __forceinline__ void store4(float* p, const float v[4]) {
     *reinterpret_cast<float4*>(p) = make_float4(v[0], v[1], v[2], v[3]);
@@ -108,19 +118,33 @@ struct Elem<float> {
 
 template <>
 struct Elem<__nv_bfloat16> {
+  static __device__ __forceinline__ float2 to2(uint32_t w) {
+    return __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&w));
+  }
+  static __device__ __forceinline__ uint32_t from2(float a, float b) {
+    __nv_bfloat162 h = __floats2bfloat162_rn(a, b);
+    return *reinterpret_cast<uint32_t*>(&h);
+  }
+  static __device__ __forceinline__ void load8(const __nv_bfloat16* p, float v[8]) {
+    const uint4 x = *reinterpret_cast<const uint4*>(p);
+    float2 f;
+    f = to2(x.x); v[0] = f.x; v[1] = f.y;
+    f = to2(x.y); v[2] = f.x; v[3] = f.y;
+    f = to2(x.z); v[4] = f.x; v[5] = f.y;
+    f = to2(x.w); v[6] = f.x; v[7] = f.y;
+  }
+  static __device__ __forceinline__ void store8(__nv_bfloat16* p, const float v[8]) {
+    *reinterpret_cast<uint4*>(p) =
+        make_uint4(from2(v[0], v[1]), from2(v[2], v[3]), from2(v[4], v[5]), from2(v[6], v[7]));
+  }
   static __device__ __forceinline__ void load4(const __nv_bfloat16* p, float v[4]) {
     const uint2 x = *reinterpret_cast<const uint2*>(p);
-    const float2 a = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&x.x));
-    const float2 b = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&x.y));
-    v[0] = a.x; v[1] = a.y; v[2] = b.x; v[3] = b.y;
+    float2 f;
+    f = to2(x.x); v[0] = f.x; v[1] = f.y;
+    f = to2(x.y); v[2] = f.x; v[3] = f.y;
   }
   static __device__ __forceinline__ void store4(__nv_bfloat16* p, const float v[4]) {
-    __nv_bfloat162 a = __floats2bfloat162_rn(v[0], v[1]);
-    __nv_bfloat162 b = __floats2bfloat162_rn(v[2], v[3]);
-    uint2 x;
-    x.x = *reinterpret_cast<uint32_t*>(&a);
-    x.y = *reinterpret_cast<uint32_t*>(&b);
-    *reinterpret_cast<uint2*>(p) = x;
+    *reinterpret_cast<uint2*>(p) = make_uint2(from2(v[0], v[1]), from2(v[2], v[3]));
   }
   static __device__ __forceinline__ float load1(const __nv_bfloat16* p) {
     return __bfloat162float(*p);
@@ -132,22 +156,48 @@ struct Elem<__nv_bfloat16> {
 
 template <>
 struct Elem<__half> {
+  static __device__ __forceinline__ float2 to2(uint32_t w) {
+    return __half22float2(*reinterpret_cast<const __half2*>(&w));
+  }
+  static __device__ __forceinline__ uint32_t from2(float a, float b) {
+    __half2 h = __floats2half2_rn(a, b);
+    return *reinterpret_cast<uint32_t*>(&h);
+  }
+  static __device__ __forceinline__ void load8(const __half* p, float v[8]) {
+    const uint4 x = *reinterpret_cast<const uint4*>(p);
+    float2 f;
+    f = to2(x.x); v[0] = f.x; v[1] = f.y;
+    f = to2(x.y); v[2] = f.x; v[3] = f.y;
+    f = to2(x.z); v[4] = f.x; v[5] = f.y;
+    f = to2(x.w); v[6] = f.x; v[7] = f.y;
+  }
+  static __device__ __forceinline__ void store8(__half* p, const float v[8]) {
+    *reinterpret_cast<uint4*>(p) =
+        make_uint4(from2(v[0], v[1]), from2(v[2], v[3]), from2(v[4], v[5]), from2(v[6], v[7]));
+  }
   static __device__ __forceinline__ void load4(const __half* p, float v[4]) {
     const uint2 x = *reinterpret_cast<const uint2*>(p);
-    const float2 a = __half22float2(*reinterpret_cast<const __half2*>(&x.x));
-    const float2 b = __half22float2(*reinterpret_cast<const __half2*>(&x.y));
-    v[0] = a.x; v[1] = a.y; v[2] = b.x; v[3] = b.y;
+    float2 f;
+    f = to2(x.x); v[0] = f.x; v[1] = f.y;
+    f = to2(x.y); v[2] = f.x; v[3] = f.y;
   }
   static __device__ __forceinline__ void store4(__half* p, const float v[4]) {
-    __half2 a = __floats2half2_rn(v[0], v[1]);
-    __half2 b = __floats2half2_rn(v[2], v[3]);
-    uint2 x;
-    x.x = *reinterpret_cast<uint32_t*>(&a);
-    x.y = *reinterpret_cast<uint32_t*>(&b);
-    *reinterpret_cast<uint2*>(p) = x;
+    *reinterpret_cast<uint2*>(p) = make_uint2(from2(v[0], v[1]), from2(v[2], v[3]));
   }
   static __device__ __forceinline__ float load1(const __half* p) { return __half2float(*p); }
   static __device__ __forceinline__ void store1(__half* p, float v) { *p = __float2half_rn(v); }
 };
+
+// V consecutive elements (V = 4 or 8)
+template <typename T, int V>
+__device__ __forceinline__ void loadv(const T* p, float* v) {
+  if constexpr (V == 8) Elem<T>::load8(p, v);
+  else Elem<T>::load4(p, v);
+}
+template <typename T, int V>
+__device__ __forceinline__ void storev(T* p, const float* v) {
+  if constexpr (V == 8) Elem<T>::store8(p, v);
+  else Elem<T>::store4(p, v);
+}
 
 }  // namespace snn

@@ -60,7 +60,9 @@ def test_staged_and_plain_kernels_agree(i, cuda_device):
     assert torch.equal(a.mem_final, b.mem_final)
     if a.ckpt is not None:
         assert torch.equal(a.ckpt, b.ckpt)
-    H.assert_close("grad_I", H.lanes_2d(a.grad_I), H.lanes_2d(b.grad_I), 1e-6, 1e-7)
+    # the reverse passes accumulate in different orders (packed FMAs vs
+    # scalar): they agree within the fp32 gradient tolerance
+    H.assert_close("grad_I", H.lanes_2d(a.grad_I), H.lanes_2d(b.grad_I), *H.TOL[w.io_dtype])
 
 
 def test_backward_is_deterministic(cuda_device):
