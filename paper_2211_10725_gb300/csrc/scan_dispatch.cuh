@@ -47,22 +47,24 @@ cudaError_t fwd_t(ScanArgs a, bool staged, cudaStream_t st) {
 template <bool SYN, bool RECOMP, typename TI, typename TO, int RESET, int SG>
 cudaError_t bwd_staged(ScanArgs a, cudaStream_t st, bool* launched) {
   const void* k = (const void*)scan_bwd_staged<SYN, RECOMP, TI, TO, RESET, SG>;
-  int per_lane, seg;
+  int per_lane, seg, fixed;
   int64_t items;
   if (RECOMP) {
-    const int fwd_item = (int)sizeof(TI) + 4 * (SYN ? 2 : 1);
+    const int fwd_item = (int)sizeof(TI);
     const int bwd_item = (int)sizeof(TO) * (a.gm ? 2 : 1);
     per_lane = fwd_item > bwd_item ? fwd_item : bwd_item;
     seg = kLanes<SYN> * 4 * a.K * (SYN ? 2 : 1);
+    fixed = 2 * 4 * (SYN ? 2 : 1);  // two checkpoint slots
     items = 2 * a.T;
   } else {
     const int n = 2 + (sizeof(TO) != 4 ? 1 : 0) + ((SYN && a.part_alpha) ? 1 : 0) + (a.gm ? 1 : 0);
     per_lane = n * (int)sizeof(TO);
     seg = 0;
+    fixed = 0;
     items = a.T;
   }
   StagedPlan p;
-  if (!plan_staged(k, a.L, items, per_lane, seg, kLanes<SYN>, &p)) return cudaSuccess;
+  if (!plan_staged(k, a.L, items, per_lane, seg, kLanes<SYN>, &p, fixed)) return cudaSuccess;
   a.lanes_per_cta = p.lanes_per_cta;
   a.stages = p.stages;
   a.stage_bytes = p.stage_bytes;

@@ -74,13 +74,16 @@ struct StagedPlan {
 //   stage_bytes_per_lane: bytes one lane contributes to the largest item
 //   seg_bytes_per_thread: replay buffer bytes per consumer thread
 //   lanes_per_thread: lanes each consumer thread owns
+//   fixed_bytes_per_lane: other shared memory per lane of the strip
 inline bool plan_staged(const void* kernel, int64_t L, int64_t items, int stage_bytes_per_lane,
-                        int seg_bytes_per_thread, int lanes_per_thread, StagedPlan* plan) {
+                        int seg_bytes_per_thread, int lanes_per_thread, StagedPlan* plan,
+                        int fixed_bytes_per_lane = 0) {
   static std::mutex mu;
   static std::map<std::tuple<int, const void*, int64_t, int64_t, int, int>, StagedPlan> cache;
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess) return false;
-  const auto key = std::make_tuple(dev, kernel, L, items, stage_bytes_per_lane, seg_bytes_per_thread);
+  const auto key = std::make_tuple(dev, kernel, L, items, stage_bytes_per_lane,
+                                   seg_bytes_per_thread * 64 + fixed_bytes_per_lane);
   {
     std::lock_guard<std::mutex> g(mu);
     auto it = cache.find(key);
@@ -103,7 +106,7 @@ inline bool plan_staged(const void* kernel, int64_t L, int64_t items, int stage_
       if (threads > kMaxStagedThreads) continue;
       if ((int64_t)threads * fa.numRegs * cps > 65536) continue;
       const int64_t stage_bytes = round_up(lpc * stage_bytes_per_lane, 128);
-      const int64_t seg_bytes = cthreads * seg_bytes_per_thread;
+      const int64_t seg_bytes = cthreads * seg_bytes_per_thread + lpc * fixed_bytes_per_lane;
       const int64_t budget = (int64_t)d.smem_per_sm / cps - 1024 - (int64_t)fa.sharedSizeBytes;
       const int64_t avail = (budget < d.smem_optin ? budget : d.smem_optin) - kBarrierBytes - seg_bytes;
       if (avail < stage_bytes * min_stages) continue;
@@ -142,8 +145,13 @@ cudaError_t launch_scan_bwd_leaky(ScanArgs a, bool recompute, int in_dt, int io_
                                   cudaStream_t stream);
 cudaError_t launch_scan_bwd_synaptic(ScanArgs a, bool recompute, int in_dt, int io_dt,
                                      bool staged, cudaStream_t stream);
+// fp64 scratch the reduction of one parameter needs (elements)
+inline int64_t param_reduce_scratch(int64_t N, int64_t C) {
+  const int64_t a = 1024, b = 8 * N, c = 64 * C;
+  return a > b ? (a > c ? a : c) : (b > c ? b : c);
+}
 cudaError_t launch_param_reduce(const float* part, int64_t B, int64_t N, int64_t C, int64_t HW,
-                                int mode, double* scratch, int scratch_len, float* out,
+                                int mode, double* scratch, int64_t scratch_len, float* out,
                                 cudaStream_t stream);
 
 }  // namespace snn

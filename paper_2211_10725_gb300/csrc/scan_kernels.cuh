@@ -31,8 +31,8 @@ enum { SG_FAST_SIGMOID = 0, SG_ATAN = 1 };
 enum { PM_SCALAR = 0, PM_PER_NEURON = 1, PM_PER_CHANNEL = 2 };
 constexpr uint32_t DEBUG_PRODUCER_IDLE = 1u;
 constexpr int VEC = 8;                 // lane granularity of a staged CTA strip
-constexpr int kBarrierBytes = 1024;    // room for up to 64 stages x 2 mbarriers
-constexpr int kMaxStages = 64;
+constexpr int kBarrierBytes = 1024;    // full[60], empty[60], ck_full[2], ck_empty[2]
+constexpr int kMaxStages = 60;
 constexpr int kMaxStagedThreads = 512;
 constexpr uint64_t kDrainNs = 1000000000ull;
 
@@ -106,13 +106,13 @@ __device__ __forceinline__ void fwd_step(int reset_rt, float beta, float thr, fl
     i = __fadd_rn(__fmul_rn(alpha, i), x);
     in = i;
   }
-  const float zf = z ? 1.0f : 0.0f;
   float un;
   if (reset == RESET_ZERO) {
-    un = __fadd_rn(__fmul_rn(beta, __fmul_rn(u, 1.0f - zf)), in);
+    // (1 - z) u: u, or a zero with u's sign (as the float evaluation gives)
+    un = __fadd_rn(__fmul_rn(beta, z ? __fmul_rn(u, 0.0f) : u), in);
   } else {
     un = __fadd_rn(__fmul_rn(beta, u), in);
-    if (reset == RESET_SUBTRACT) un = __fmaf_rn(zf, -thr, un);
+    if (reset == RESET_SUBTRACT && z) un = __fsub_rn(un, thr);
   }
   u = un;
   z = un > thr;  // Eq. (3), strict
@@ -200,23 +200,23 @@ __device__ __forceinline__ float2 add2(float2 a, float2 b) { return __fadd2_rn(a
 __device__ __forceinline__ float2 mul2(float2 a, float2 b) { return __fmul2_rn(a, b); }
 __device__ __forceinline__ float2 fma2(float2 a, float2 b, float2 c) { return __ffma2_rn(a, b, c); }
 
-// 1 where x > 0 else 0; with x = fl(u - thr) this is Eq. (3): the rounded
-// difference of two floats is positive exactly when u > thr (no flush to 0)
-__device__ __forceinline__ float2 pos2(float2 x) {
-  return make_float2(x.x > 0.0f ? 1.0f : 0.0f, x.y > 0.0f ? 1.0f : 0.0f);
-}
-
 // Forward step on a pair of lanes: fwd_step on each lane (scalar operations
 // with explicit rounding, which the compiler never fuses; packed fp32x2
 // multiply and add may be fused into a packed FMA, which would change the
-// result).  negthr = -thr; z holds z_{t-1} on entry and z_t on exit (0/1).
+// result).  negthr = -thr; z[0..1] hold z_{t-1} on entry and z_t on exit.
 template <bool SYN, int RESET>
 __device__ __forceinline__ void fwd_pair(int reset_rt, float2 beta, float2 negthr, float2 alpha,
-                                         float2 x, float2& u, float2& z, float2& i) {
-  bool zx = z.x != 0.0f, zy = z.y != 0.0f;
-  fwd_step<SYN, RESET>(reset_rt, beta.x, -negthr.x, alpha.x, x.x, u.x, zx, i.x);
-  fwd_step<SYN, RESET>(reset_rt, beta.y, -negthr.y, alpha.y, x.y, u.y, zy, i.y);
-  z = make_float2(zx ? 1.0f : 0.0f, zy ? 1.0f : 0.0f);
+                                         float2 x, float2& u, bool* z, float2& i) {
+  fwd_step<SYN, RESET>(reset_rt, beta.x, -negthr.x, alpha.x, x.x, u.x, z[0], i.x);
+  fwd_step<SYN, RESET>(reset_rt, beta.y, -negthr.y, alpha.y, x.y, u.y, z[1], i.y);
+}
+
+// Approximate reciprocal (one hardware instruction, relative error ~2^-23)
+// of a value >= 1: the surrogates' denominators, so no subnormals occur.
+__device__ __forceinline__ float rcp_ge1(float d) {
+  float r;
+  asm("rcp.approx.ftz.f32 %0, %1;" : "=f"(r) : "f"(d));
+  return r;
 }
 
 template <int SG>
@@ -225,11 +225,11 @@ __device__ __forceinline__ float2 surrogate2(const ScanArgs& a, float2 x) {
   if (sg == SG_FAST_SIGMOID) {
     const float2 d = fma2(f2(a.sg_a), make_float2(fabsf(x.x), fabsf(x.y)), f2(1.0f));
     const float2 d2 = mul2(d, d);
-    return make_float2(__fdividef(1.0f, d2.x), __fdividef(1.0f, d2.y));
+    return make_float2(rcp_ge1(d2.x), rcp_ge1(d2.y));
   }
   const float2 y = mul2(f2(a.sg_b), x);
   const float2 d = fma2(y, y, f2(1.0f));
-  return mul2(f2(a.sg_a), make_float2(__fdividef(1.0f, d.x), __fdividef(1.0f, d.y)));
+  return mul2(f2(a.sg_a), make_float2(rcp_ge1(d.x), rcp_ge1(d.y)));
 }
 
 // Reverse-pass state of a pair of lanes.  dthr accumulates
@@ -245,12 +245,18 @@ struct Bwd2 {
 // grad_mem_final / grad_syn_final at t = T-1).  Returns dL/dI_t.
 template <bool SYN, int RESET, int SG, bool EXTRA>
 __device__ __forceinline__ float2 bwd_pair(const ScanArgs& a, float2 beta, float2 negthr,
-                                           float2 alpha, float2 u, float2 z, float2 i,
+                                           float2 alpha, float2 u, bool z0, bool z1, float2 i,
                                            float2 gs, float2 eu, float2 ei, Bwd2& s) {
   const int reset = RESET >= 0 ? RESET : a.reset;
-  const float2 keep = add2(f2(1.0f), make_float2(-z.x, -z.y));  // 1 - z_t
-  s.dbeta = fma2(s.du, reset == RESET_ZERO ? mul2(u, keep) : u, s.dbeta);
-  if (reset == RESET_SUBTRACT) s.dthr = fma2(z, s.du, s.dthr);
+  if (reset == RESET_ZERO) {
+    s.dbeta = fma2(s.du, make_float2(z0 ? 0.0f : u.x, z1 ? 0.0f : u.y), s.dbeta);
+  } else {
+    s.dbeta = fma2(s.du, u, s.dbeta);
+  }
+  if (reset == RESET_SUBTRACT) {  // d u_{t+1} / d thr = -z_t
+    if (z0) s.dthr.x += s.du.x;
+    if (z1) s.dthr.y += s.du.y;
+  }
   if (SYN) s.dalpha = fma2(s.di, i, s.dalpha);
   const float2 sg = surrogate2<SG>(a, add2(u, negthr));
   float2 dz = gs;
@@ -259,7 +265,9 @@ __device__ __forceinline__ float2 bwd_pair(const ScanArgs& a, float2 beta, float
     else if (reset == RESET_ZERO) dz = fma2(mul2(f2(-1.0f), mul2(beta, u)), s.du, dz);
   }
   const float2 p = mul2(sg, dz);
-  const float2 decay = reset == RESET_ZERO ? mul2(beta, keep) : beta;
+  const float2 decay = reset == RESET_ZERO
+                           ? make_float2(z0 ? 0.0f : beta.x, z1 ? 0.0f : beta.y)
+                           : beta;
   s.du = fma2(decay, s.du, p);
   if (EXTRA) s.du = add2(s.du, eu);
   s.dthr = add2(s.dthr, p);
@@ -353,12 +361,19 @@ __device__ __forceinline__ const void* row(const void* base, int64_t t, int64_t 
   return static_cast<const T*>(base) + t * L + lane0;
 }
 
+// Barrier block at the start of shared memory: the ring's full/empty pairs
+// and the two-slot checkpoint buffer's pairs (recompute backward).
 __device__ __forceinline__ void init_ring_barriers(uint64_t* full, uint64_t* empty, int S,
                                                    int consumer_warps) {
   if (threadIdx.x == 0) {
     for (int s = 0; s < S; ++s) {
       mbar_init(&full[s], 1);
       mbar_init(&empty[s], consumer_warps);
+    }
+    uint64_t* ck = full + 2 * kMaxStages;
+    for (int s = 0; s < 2; ++s) {
+      mbar_init(&ck[s], 1);
+      mbar_init(&ck[2 + s], consumer_warps);
     }
     fence_barrier_init();
   }
@@ -424,15 +439,16 @@ __device__ __forceinline__ void load_params(const ScanArgs& a, int64_t l, float2
 // [mem0 > thr] when mem0 is given (else 0), i_{-1} = syn0 (or 0).
 template <bool SYN, int NP>
 __device__ __forceinline__ void initial_state(const ScanArgs& a, int64_t l, const float2 negthr[NP],
-                                              float2 u[NP], float2 z[NP], float2 i[NP]) {
+                                              float2 u[NP], bool z[2 * NP], float2 i[NP]) {
 #pragma unroll
   for (int k = 0; k < NP; ++k) {
     if (a.mem0) {
       u[k] = make_float2(a.mem0[l + 2 * k], a.mem0[l + 2 * k + 1]);
-      z[k] = pos2(add2(u[k], negthr[k]));
+      z[2 * k] = u[k].x > -negthr[k].x;
+      z[2 * k + 1] = u[k].y > -negthr[k].y;
     } else {
       u[k] = f2(0.0f);
-      z[k] = f2(0.0f);
+      z[2 * k] = z[2 * k + 1] = false;
     }
     i[k] = (SYN && a.syn0) ? make_float2(a.syn0[l + 2 * k], a.syn0[l + 2 * k + 1]) : f2(0.0f);
   }
@@ -472,7 +488,8 @@ __global__ void __launch_bounds__(kMaxStagedThreads) scan_fwd_staged(const ScanA
   const int c = threadIdx.x;
   const int64_t l = lane0 + (int64_t)c * V;
   const bool active = c * V < cta_lanes;
-  float2 beta[NP], negthr[NP], alpha[NP], u[NP], z[NP], in[NP];
+  float2 beta[NP], negthr[NP], alpha[NP], u[NP], in[NP];
+  bool z[V];
   if (active) {
     load_params<SYN, NP>(a, l, beta, negthr, alpha);
     initial_state<SYN, NP>(a, l, negthr, u, z, in);
@@ -494,10 +511,13 @@ __global__ void __launch_bounds__(kMaxStagedThreads) scan_fwd_staged(const ScanA
     if (active) {
       float2 x[NP];
       load_pairs<TI, NP>(my + pos.s * stage_elems, x);
+      float2 zf[NP];
 #pragma unroll
-      for (int k = 0; k < NP; ++k)
-        fwd_pair<SYN, RESET>(a.reset, beta[k], negthr[k], alpha[k], x[k], u[k], z[k], in[k]);
-      store_pairs<TO, NP>(spk, z);
+      for (int k = 0; k < NP; ++k) {
+        fwd_pair<SYN, RESET>(a.reset, beta[k], negthr[k], alpha[k], x[k], u[k], &z[2 * k], in[k]);
+        zf[k] = make_float2(z[2 * k] ? 1.0f : 0.0f, z[2 * k + 1] ? 1.0f : 0.0f);
+      }
+      store_pairs<TO, NP>(spk, zf);
       if (mem) store_pairs<TO, NP>(mem, u);
       if (SYN && syn) store_pairs<TO, NP>(syn, in);
       if (++kk == a.K) {
@@ -535,14 +555,14 @@ __global__ void __launch_bounds__(kMaxStagedThreads) scan_fwd_staged(const ScanA
 template <bool SYN, int RESET, int SG, bool EXTRA, int NP>
 __device__ __forceinline__ void bwd_pairs(const ScanArgs& a, const float2 beta[NP],
                                           const float2 negthr[NP], const float2 alpha[NP],
-                                          const float2 u[NP], const float2 z[NP],
+                                          const float2 u[NP], const bool z[2 * NP],
                                           const float2 i[NP], const float2 g[NP],
                                           const float2 eu[NP], const float2 ei[NP], Bwd2 st[NP],
                                           float2 out[NP]) {
 #pragma unroll
   for (int k = 0; k < NP; ++k)
-    out[k] = bwd_pair<SYN, RESET, SG, EXTRA>(a, beta[k], negthr[k], alpha[k], u[k], z[k], i[k],
-                                             g[k], eu[k], ei[k], st[k]);
+    out[k] = bwd_pair<SYN, RESET, SG, EXTRA>(a, beta[k], negthr[k], alpha[k], u[k], z[2 * k],
+                                             z[2 * k + 1], i[k], g[k], eu[k], ei[k], st[k]);
 }
 
 template <bool SYN, bool RECOMP, typename TI, typename TO, int RESET, int SG>
@@ -565,7 +585,13 @@ __global__ void __launch_bounds__(kMaxStagedThreads) scan_bwd_staged(const ScanA
   // store-mode tile order: gs, mem, [spk], [syn], [gm]
   const int t_spk = 2, t_syn = 2 + (half_store ? 1 : 0);
   const int t_gm_store = t_syn + ((!RECOMP && want_syn) ? 1 : 0);
-  const int ck_off = in_stride;  // recompute: checkpoint tiles after the I tile
+  // recompute: two checkpoint slots after the replay buffer, prefetched one
+  // segment ahead (each holds the strip's u row, then its i row)
+  uint64_t* ck_full = full + 2 * kMaxStages;
+  uint64_t* ck_empty = ck_full + 2;
+  const int ck_slot_bytes = a.lanes_per_cta * 4 * (SYN ? 2 : 1);
+  unsigned char* ck_base = ring + (size_t)S * a.stage_bytes +
+                           (RECOMP ? (size_t)nthr * V * 4 * a.K * (SYN ? 2 : 1) : 0);
   init_ring_barriers(full, empty, S, cwarps);
 
   if (warp == cwarps) {
@@ -574,6 +600,7 @@ __global__ void __launch_bounds__(kMaxStagedThreads) scan_bwd_staged(const ScanA
       const uint32_t bo = (uint32_t)cta_lanes * sizeof(TO);
       const uint32_t bi = (uint32_t)cta_lanes * sizeof(TI);
       const uint32_t bc = (uint32_t)cta_lanes * 4u;
+      (void)bi;
       Tile tiles[5];
       if (!RECOMP) {
         for (int64_t t = a.T - 1; t >= 0 && p.ok; --t) {
@@ -586,19 +613,28 @@ __global__ void __launch_bounds__(kMaxStagedThreads) scan_bwd_staged(const ScanA
           p.issue(tiles, n, a);
         }
       } else {
+        int64_t ck_n = 0;  // checkpoint loads issued
         for (int k = a.nseg - 1; k >= 0 && p.ok; --k) {
           const int64_t t0 = (int64_t)k * a.K, t1 = min(a.T, t0 + a.K);
-          for (int64_t t = t0; t < t1 && p.ok; ++t) {
-            int n = 0;
-            tiles[n++] = Tile{row<TI>(a.I, t, a.L, lane0), bi, 0};
-            if (t == t0 && k > 0) {
-              // the segment's starting state rides with its first input row;
-              // checkpoint rows are fp32 [nseg-1][SYN ? 2 : 1][L]
-              const float* cu = a.ckpt + (int64_t)(k - 1) * (SYN ? 2 : 1) * a.L + lane0;
-              tiles[n++] = Tile{cu, bc, (uint32_t)ck_off};
-              if (SYN) tiles[n++] = Tile{cu + a.L, bc, (uint32_t)(ck_off + a.lanes_per_cta * 4)};
+          if (k > 0) {
+            // the segment's starting state: checkpoint rows fp32 [nseg-1][SYN?2:1][L]
+            const int slot = (int)(ck_n & 1);
+            if (ck_n >= 2 &&
+                !mbar_wait_bounded(&ck_empty[slot], (uint32_t)(((ck_n >> 1) - 1) & 1), a.wait_ns)) {
+              record_status(a.status, kStatusTimeout);
+              p.ok = false;
+              break;
             }
-            p.issue(tiles, n, a);
+            const float* cu = a.ckpt + (int64_t)(k - 1) * (SYN ? 2 : 1) * a.L + lane0;
+            unsigned char* dst = ck_base + (size_t)slot * ck_slot_bytes;
+            mbar_arrive_expect_tx(&ck_full[slot], bc * (SYN ? 2u : 1u));
+            bulk_g2s(dst, cu, bc, &ck_full[slot]);
+            if (SYN) bulk_g2s(dst + a.lanes_per_cta * 4, cu + a.L, bc, &ck_full[slot]);
+            ++ck_n;
+          }
+          for (int64_t t = t0; t < t1 && p.ok; ++t) {
+            const Tile tile{row<TI>(a.I, t, a.L, lane0), bi, 0};
+            p.issue(&tile, 1, a);
           }
           for (int64_t t = t1 - 1; t >= t0 && p.ok; --t) {
             int n = 0;
@@ -607,6 +643,8 @@ __global__ void __launch_bounds__(kMaxStagedThreads) scan_bwd_staged(const ScanA
             p.issue(tiles, n, a);
           }
         }
+        for (int64_t j = ck_n > 2 ? ck_n - 2 : 0; j < ck_n; ++j)
+          mbar_wait_bounded(&ck_full[j & 1], (uint32_t)((j >> 1) & 1), kDrainNs);
       }
       p.drain();
     }
@@ -623,11 +661,9 @@ __global__ void __launch_bounds__(kMaxStagedThreads) scan_bwd_staged(const ScanA
   for (int k = 0; k < NP; ++k) st[k] = Bwd2{f2(0.0f), f2(0.0f), f2(0.0f), f2(0.0f), f2(0.0f)};
   const int stage_io_elems = a.stage_bytes / (int)sizeof(TO);
   const int stage_in_elems = a.stage_bytes / (int)sizeof(TI);
-  const int stage_f32 = a.stage_bytes / 4;
   const int tile_io_elems = a.lanes_per_cta;  // elements per io tile
   const TO* ring_o = reinterpret_cast<const TO*>(ring) + c * V;
   const TI* ring_i = reinterpret_cast<const TI*>(ring) + c * V;
-  const float* ring_f = reinterpret_cast<const float*>(ring) + c * V;
   TO* gI = static_cast<TO*>(a.gI) + l + (a.T - 1) * a.L;  // walks backwards
   // per-thread replay buffer: [K][V/4 planes][nthr][4] fp32 for u, then i
   // (each plane holds 4 lanes of every thread: conflict-free 16-byte rows)
@@ -638,7 +674,7 @@ __global__ void __launch_bounds__(kMaxStagedThreads) scan_bwd_staged(const ScanA
   bool ok = true;
 
   // one reverse step on the thread's pairs: general (EXTRA) only where needed
-  auto reverse = [&](int64_t t, const float2 u[NP], const float2 z[NP], const float2 i[NP],
+  auto reverse = [&](int64_t t, const float2 u[NP], const bool z[V], const float2 i[NP],
                      const float2 g[NP], const float2 gmv[NP], float2 out[NP]) {
     if (a.gm || t == a.T - 1) {
       float2 eu[NP], ei[NP];
@@ -672,14 +708,24 @@ __global__ void __launch_bounds__(kMaxStagedThreads) scan_bwd_staged(const ScanA
       }
       if (active) {
         const TO* base = ring_o + pos.s * stage_io_elems;
-        float2 g[NP], uu[NP], zz[NP], ii[NP], gmv[NP], out[NP];
+        float2 g[NP], uu[NP], ii[NP], gmv[NP], out[NP];
+        bool zz[V];
         load_pairs<TO, NP>(base, g);
         load_pairs<TO, NP>(base + tile_io_elems, uu);
         if (half_store) {
-          load_pairs<TO, NP>(base + t_spk * tile_io_elems, zz);
+          float2 sp[NP];
+          load_pairs<TO, NP>(base + t_spk * tile_io_elems, sp);
+#pragma unroll
+          for (int k = 0; k < NP; ++k) {
+            zz[2 * k] = sp[k].x != 0.0f;
+            zz[2 * k + 1] = sp[k].y != 0.0f;
+          }
         } else {
 #pragma unroll
-          for (int k = 0; k < NP; ++k) zz[k] = pos2(add2(uu[k], negthr[k]));
+          for (int k = 0; k < NP; ++k) {
+            zz[2 * k] = uu[k].x > -negthr[k].x;
+            zz[2 * k + 1] = uu[k].y > -negthr[k].y;
+          }
         }
         if (want_syn) {
           load_pairs<TO, NP>(base + t_syn * tile_io_elems, ii);
@@ -696,9 +742,30 @@ __global__ void __launch_bounds__(kMaxStagedThreads) scan_bwd_staged(const ScanA
       gI -= a.L;
     }
   } else {
+    int64_t ck_u = 0;  // checkpoints consumed
     for (int k = a.nseg - 1; k >= 0 && ok; --k) {
       const int64_t t0 = (int64_t)k * a.K, t1 = min(a.T, t0 + a.K);
-      float2 u[NP], z[NP], ii[NP];
+      float2 u[NP], ii[NP];
+      bool z[V];
+      if (k > 0) {
+        if (!warp_wait(&ck_full[ck_u & 1], (uint32_t)((ck_u >> 1) & 1), a.wait_ns)) {
+          if (lid == 0) record_status(a.status, kStatusTimeout);
+          ok = false;
+          break;
+        }
+        if (active) {
+          const float* cb = reinterpret_cast<const float*>(ck_base + (size_t)(ck_u & 1) * ck_slot_bytes) + c * V;
+          load_pairs<float, NP>(cb, u);
+          if (SYN) load_pairs<float, NP>(cb + a.lanes_per_cta, ii);
+#pragma unroll
+          for (int q = 0; q < NP; ++q) {
+            z[2 * q] = u[q].x > -negthr[q].x;
+            z[2 * q + 1] = u[q].y > -negthr[q].y;
+          }
+        }
+      } else if (active) {
+        initial_state<SYN, NP>(a, l, negthr, u, z, ii);
+      }
       // replay the forward over the segment
       float* su = seg;
       for (int64_t t = t0; t < t1; ++t) {
@@ -710,20 +777,9 @@ __global__ void __launch_bounds__(kMaxStagedThreads) scan_bwd_staged(const ScanA
         if (active) {
           float2 x[NP];
           load_pairs<TI, NP>(ring_i + pos.s * stage_in_elems, x);
-          if (t == t0) {
-            if (k > 0) {
-              const float* cb = ring_f + pos.s * stage_f32 + ck_off / 4;
-              load_pairs<float, NP>(cb, u);
-              if (SYN) load_pairs<float, NP>(cb + a.lanes_per_cta, ii);
-#pragma unroll
-              for (int q = 0; q < NP; ++q) z[q] = pos2(add2(u[q], negthr[q]));
-            } else {
-              initial_state<SYN, NP>(a, l, negthr, u, z, ii);
-            }
-          }
 #pragma unroll
           for (int q = 0; q < NP; ++q)
-            fwd_pair<SYN, RESET>(a.reset, beta[q], negthr[q], alpha[q], x[q], u[q], z[q], ii[q]);
+            fwd_pair<SYN, RESET>(a.reset, beta[q], negthr[q], alpha[q], x[q], u[q], &z[2 * q], ii[q]);
 #pragma unroll
           for (int q = 0; q < V / 4; ++q) {
             *reinterpret_cast<float4*>(su + q * nthr * 4) =
@@ -738,6 +794,10 @@ __global__ void __launch_bounds__(kMaxStagedThreads) scan_bwd_staged(const ScanA
         su += seg_row;
       }
       if (!ok) break;
+      if (k > 0) {  // the replay consumed the checkpoint values: free the slot
+        release_stage(ck_empty, (int)(ck_u & 1), lid);
+        ++ck_u;
+      }
       // reverse steps over the segment
       for (int64_t t = t1 - 1; t >= t0; --t) {
         su -= seg_row;
@@ -748,7 +808,8 @@ __global__ void __launch_bounds__(kMaxStagedThreads) scan_bwd_staged(const ScanA
         }
         if (active) {
           const TO* base = ring_o + pos.s * stage_io_elems;
-          float2 g[NP], gmv[NP], uu[NP], zz[NP], iv[NP], out[NP];
+          float2 g[NP], gmv[NP], uu[NP], iv[NP], out[NP];
+          bool zz[V];
           load_pairs<TO, NP>(base, g);
           if (a.gm) load_pairs<TO, NP>(base + tile_io_elems, gmv);
 #pragma unroll
@@ -766,7 +827,10 @@ __global__ void __launch_bounds__(kMaxStagedThreads) scan_bwd_staged(const ScanA
             }
           }
 #pragma unroll
-          for (int q = 0; q < NP; ++q) zz[q] = pos2(add2(uu[q], negthr[q]));
+          for (int q = 0; q < NP; ++q) {
+            zz[2 * q] = uu[q].x > -negthr[q].x;
+            zz[2 * q + 1] = uu[q].y > -negthr[q].y;
+          }
           reverse(t, uu, zz, iv, g, gmv, out);
           store_pairs<TO, NP>(gI, out);
         }

@@ -10,7 +10,6 @@ namespace snn {
 namespace {
 
 constexpr size_t kStatusBytes = 256;
-constexpr int kRedScratch = 1024;  // fp64 block partials per reduced parameter
 constexpr uint64_t kDefaultWaitNs = 2000000000ull;
 
 bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
@@ -62,8 +61,11 @@ size_t lane_bytes(const snn_scan_desc* d) {
   return (size_t)round_up((int64_t)d->B * d->N * 4, 256);
 }
 
+// fp64 partials of one parameter's cross-lane reduction
+int64_t red_scratch(const snn_scan_desc* d) { return param_reduce_scratch(d->N, d->C); }
+
 size_t workspace_bytes(const snn_scan_desc* d) {
-  return kStatusBytes + 3 * lane_bytes(d) + 3 * kRedScratch * sizeof(double);
+  return kStatusBytes + 3 * lane_bytes(d) + 3 * (size_t)red_scratch(d) * sizeof(double);
 }
 
 struct WsView {
@@ -79,7 +81,7 @@ WsView ws_view(void* ws, const snn_scan_desc* d) {
   const size_t lb = lane_bytes(d);
   for (int k = 0; k < 3; ++k) v.part[k] = reinterpret_cast<float*>(p + kStatusBytes + k * lb);
   for (int k = 0; k < 3; ++k)
-    v.scratch[k] = reinterpret_cast<double*>(p + kStatusBytes + 3 * lb + k * kRedScratch * sizeof(double));
+    v.scratch[k] = reinterpret_cast<double*>(p + kStatusBytes + 3 * lb + k * red_scratch(d) * sizeof(double));
   return v;
 }
 
@@ -240,7 +242,7 @@ snn_status_t scan_bwd(const snn_scan_desc* d, bool syn, const void* I, const flo
   float* parts[3] = {a.part_beta, a.part_thr, a.part_alpha};
   for (int k = 0; k < 3; ++k) {
     if (!outs[k]) continue;
-    e = launch_param_reduce(parts[k], d->B, d->N, d->C, d->HW, modes[k], v.scratch[k], kRedScratch,
+    e = launch_param_reduce(parts[k], d->B, d->N, d->C, d->HW, modes[k], v.scratch[k], red_scratch(d),
                             outs[k], stream);
     if (e != cudaSuccess) return SNN_ERR_CUDA;
   }
