@@ -222,6 +222,33 @@ snn_status_t snn_synaptic_bwd(const snn_scan_desc* desc, const void* I, const fl
                               float* grad_syn0, void* ws, size_t ws_bytes,
                               snn_stream_t stream);
 
+/*
+ * Leaky BPTT that allocates nothing (no counterpart in the paper; it exists
+ * for callers of this library that cannot allocate device memory: hosts
+ * whose device memory is budgeted by another runtime, real-time loops that
+ * must not call cudaMalloc because it can synchronise the device, plain C
+ * hosts without an allocator).
+ * Arguments and results are those of snn_leaky_bwd, without ws/ws_bytes:
+ * the workspace is a fixed 16 MiB array in the library's device memory,
+ * held by every GPU that loads the library until the process exits.
+ *   status   device int (4-byte aligned) or NULL: receives SNN_OK or
+ *            SNN_ERR_TIMEOUT from the kernels (asynchronously, on stream)
+ * Returns SNN_ERR_WORKSPACE, launching nothing, when
+ * snn_scan_workspace_bytes(desc) exceeds 16 MiB.  Allocates nothing.
+ * The first call on each device looks up the array's device address (a
+ * one-time set-up that is not a stream operation); make that first call
+ * before any stream capture.  Every call shares the one array and it keeps
+ * the last call's contents (the status word is cleared at the start of each
+ * call); calls whose work overlaps on the GPU (other streams, other host
+ * threads) race on it and must be serialised by the caller.
+ */
+snn_status_t snn_leaky_bwd_noalloc(const snn_scan_desc* desc, const void* I, const float* ckpt,
+                                   const void* mem, const void* spk, const float* beta,
+                                   const float* thr, const float* mem0, const void* grad_spk,
+                                   const void* grad_mem, const float* grad_mem_final,
+                                   void* grad_I, float* grad_beta, float* grad_thr,
+                                   float* grad_mem0, int* status, snn_stream_t stream);
+
 #if defined(__GNUC__)
 #pragma GCC visibility pop
 #endif

@@ -69,6 +69,7 @@ _SIGS = {
     "snn_leaky_bwd": ([ctypes.POINTER(ScanDesc)] + [_P] * 15 + [ctypes.c_size_t, _P], ctypes.c_int),
     "snn_synaptic_fwd": ([ctypes.POINTER(ScanDesc)] + [_P] * 13 + [ctypes.c_size_t, _P], ctypes.c_int),
     "snn_synaptic_bwd": ([ctypes.POINTER(ScanDesc)] + [_P] * 21 + [ctypes.c_size_t, _P], ctypes.c_int),
+    "snn_leaky_bwd_noalloc": ([ctypes.POINTER(ScanDesc)] + [_P] * 16, ctypes.c_int),
 }
 
 _lib: Optional[ctypes.CDLL] = None
@@ -195,6 +196,18 @@ def snn_synaptic_bwd(desc, I, ckpt, mem, spk, syn, alpha, beta, thr, mem0, syn0,
         _ptr(grad_mem_final), _ptr(grad_syn_final), _ptr(grad_I), _ptr(grad_alpha),
         _ptr(grad_beta), _ptr(grad_thr), _ptr(grad_mem0), _ptr(grad_syn0), _ptr(ws),
         ws.numel() * ws.element_size(), _stream(stream)), "snn_synaptic_bwd")
+
+
+def snn_leaky_bwd_noalloc(desc, I, ckpt, mem, spk, beta, thr, mem0, grad_spk, grad_mem,
+                          grad_mem_final, grad_I, grad_beta, grad_thr, grad_mem0, status=None,
+                          stream=None):
+    """Leaky BPTT using the library's fixed device scratch instead of a
+    workspace, for callers that cannot allocate device memory."""
+    _check(load_library().snn_leaky_bwd_noalloc(
+        ctypes.byref(desc), _ptr(I), _ptr(ckpt), _ptr(mem), _ptr(spk), _ptr(beta), _ptr(thr),
+        _ptr(mem0), _ptr(grad_spk), _ptr(grad_mem), _ptr(grad_mem_final), _ptr(grad_I),
+        _ptr(grad_beta), _ptr(grad_thr), _ptr(grad_mem0), _ptr(status), _stream(stream)),
+        "snn_leaky_bwd_noalloc")
 
 
 # ---------------------------------------------------------------------------
