@@ -146,7 +146,10 @@ snn_status_t snn_workspace_status(void* ws, snn_stream_t stream);
  *   mem      [T,B,N] io_dtype  (out)     u_t; required for SNN_SAVE_MEM, else
  *                                        optional (NULL = not written)
  *   ckpt     fp32 (out)                  SNN_SAVE_RECOMPUTE: u at the end of every
- *                                        K-step segment but the last; else NULL
+ *                                        segment but the last; else NULL.  Segments
+ *                                        are aligned to the end of the sequence:
+ *                                        the first has T-(ceil(T/K)-1)*K steps, the
+ *                                        others K.
  *   mem_final fp32 [B,N] (out) or NULL   u_{T-1}
  *   ws       workspace of snn_scan_workspace_bytes(desc) bytes
  * State is kept in fp32; the step is evaluated as Eq. (4) is written:

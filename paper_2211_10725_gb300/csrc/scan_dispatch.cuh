@@ -44,9 +44,9 @@ cudaError_t fwd_t(ScanArgs a, bool staged, cudaStream_t st) {
   return cudaGetLastError();
 }
 
-template <bool SYN, bool RECOMP, typename TI, typename TO, int RESET, int SG>
+template <bool SYN, bool RECOMP, typename TI, typename TO, int RESET, int SG, int KC = 0>
 cudaError_t bwd_staged(ScanArgs a, cudaStream_t st, bool* launched) {
-  const void* k = (const void*)scan_bwd_staged<SYN, RECOMP, TI, TO, RESET, SG>;
+  const void* k = (const void*)scan_bwd_staged<SYN, RECOMP, TI, TO, RESET, SG, KC>;
   int per_lane, seg, fixed;
   int64_t items;
   if (RECOMP) {
@@ -64,11 +64,11 @@ cudaError_t bwd_staged(ScanArgs a, cudaStream_t st, bool* launched) {
     items = a.T;
   }
   StagedPlan p;
-  if (!plan_staged(k, a.L, items, per_lane, seg, kLanes<SYN>, &p, fixed)) return cudaSuccess;
+  if (!plan_staged(k, a.L, items, per_lane, seg, kLanes<SYN>, &p, fixed, KC)) return cudaSuccess;
   a.lanes_per_cta = p.lanes_per_cta;
   a.stages = p.stages;
   a.stage_bytes = p.stage_bytes;
-  scan_bwd_staged<SYN, RECOMP, TI, TO, RESET, SG><<<(unsigned)p.grid, p.threads, p.smem, st>>>(a);
+  scan_bwd_staged<SYN, RECOMP, TI, TO, RESET, SG, KC><<<(unsigned)p.grid, p.threads, p.smem, st>>>(a);
   *launched = true;
   return cudaGetLastError();
 }
@@ -82,9 +82,20 @@ cudaError_t bwd_t(ScanArgs a, bool staged, cudaStream_t st) {
     if constexpr (kSpecialise<TI, TO>) {
       done = true;
       const int key = (a.reset == RESET_NONE ? 9 : a.reset * 2 + a.sg);
+      // the recompute variant with the default checkpoint interval K = 8
+      // also has a fully unrolled segment body (ring of exactly 8 stages)
+      const bool k8 = RECOMP && a.K == 8;
       switch (key) {
-        case 0: e = bwd_staged<SYN, RECOMP, TI, TO, RESET_SUBTRACT, SG_FAST_SIGMOID>(a, st, &launched); break;
-        case 1: e = bwd_staged<SYN, RECOMP, TI, TO, RESET_SUBTRACT, SG_ATAN>(a, st, &launched); break;
+        case 0:
+          if (k8) e = bwd_staged<SYN, RECOMP, TI, TO, RESET_SUBTRACT, SG_FAST_SIGMOID, 8>(a, st, &launched);
+          if (!launched && e == cudaSuccess)
+            e = bwd_staged<SYN, RECOMP, TI, TO, RESET_SUBTRACT, SG_FAST_SIGMOID>(a, st, &launched);
+          break;
+        case 1:
+          if (k8) e = bwd_staged<SYN, RECOMP, TI, TO, RESET_SUBTRACT, SG_ATAN, 8>(a, st, &launched);
+          if (!launched && e == cudaSuccess)
+            e = bwd_staged<SYN, RECOMP, TI, TO, RESET_SUBTRACT, SG_ATAN>(a, st, &launched);
+          break;
         case 2: e = bwd_staged<SYN, RECOMP, TI, TO, RESET_ZERO, SG_FAST_SIGMOID>(a, st, &launched); break;
         case 3: e = bwd_staged<SYN, RECOMP, TI, TO, RESET_ZERO, SG_ATAN>(a, st, &launched); break;
         default: done = false;

@@ -75,15 +75,17 @@ struct StagedPlan {
 //   seg_bytes_per_thread: replay buffer bytes per consumer thread
 //   lanes_per_thread: lanes each consumer thread owns
 //   fixed_bytes_per_lane: other shared memory per lane of the strip
+//   force_stages: exact ring depth the kernel was compiled for (0 = any)
 inline bool plan_staged(const void* kernel, int64_t L, int64_t items, int stage_bytes_per_lane,
                         int seg_bytes_per_thread, int lanes_per_thread, StagedPlan* plan,
-                        int fixed_bytes_per_lane = 0) {
+                        int fixed_bytes_per_lane = 0, int force_stages = 0) {
   static std::mutex mu;
   static std::map<std::tuple<int, const void*, int64_t, int64_t, int, int>, StagedPlan> cache;
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess) return false;
   const auto key = std::make_tuple(dev, kernel, L, items, stage_bytes_per_lane,
-                                   seg_bytes_per_thread * 64 + fixed_bytes_per_lane);
+                                   (seg_bytes_per_thread * 64 + fixed_bytes_per_lane) * 64 +
+                                       force_stages);
   {
     std::lock_guard<std::mutex> g(mu);
     auto it = cache.find(key);
@@ -109,11 +111,12 @@ inline bool plan_staged(const void* kernel, int64_t L, int64_t items, int stage_
       const int64_t seg_bytes = cthreads * seg_bytes_per_thread + lpc * fixed_bytes_per_lane;
       const int64_t budget = (int64_t)d.smem_per_sm / cps - 1024 - (int64_t)fa.sharedSizeBytes;
       const int64_t avail = (budget < d.smem_optin ? budget : d.smem_optin) - kBarrierBytes - seg_bytes;
-      if (avail < stage_bytes * min_stages) continue;
+      if (avail < stage_bytes * (force_stages > 0 ? force_stages : min_stages)) continue;
       int64_t stages = avail / stage_bytes;
       if (stages > kMaxStages) stages = kMaxStages;
       if (stages > items && items > 0) stages = items;
       if (stages < 1) stages = 1;
+      if (force_stages > 0) stages = force_stages;
       StagedPlan p;
       p.lanes_per_cta = (int)lpc;
       p.threads = threads;

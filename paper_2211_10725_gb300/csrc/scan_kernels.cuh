@@ -92,6 +92,22 @@ __device__ __forceinline__ float lane_param(const float* p, int mode, int64_t l,
   return __ldg(p + (n / a.HW) % a.C);
 }
 
+// Checkpoint segments are aligned to the end of the sequence: segment k of
+// nseg covers [t0, t1) with t1 = r + k*K, r = T - (nseg-1)*K, so only the
+// first segment (k = 0, starting at t = 0) can be shorter than K.  The
+// forward stores u (and i) at t1 - 1 of every segment but the last.
+__device__ __forceinline__ void seg_bounds(const ScanArgs& a, int k, int64_t& t0, int64_t& t1) {
+  const int64_t r = a.T - (int64_t)(a.nseg - 1) * a.K;
+  t1 = r + (int64_t)k * a.K;
+  t0 = k == 0 ? 0 : t1 - a.K;
+}
+
+// Position inside its checkpoint segment of step t = 0: the forward's step
+// counter starts here so that its segment ends fall at t1 - 1.
+__device__ __forceinline__ int seg_phase0(const ScanArgs& a) {
+  return (int)(a.K - (a.T - (int64_t)(a.nseg - 1) * a.K));
+}
+
 // One forward step, Eq. (4) / Eqs. (5)-(6), evaluated left to right as the
 // equations are written, one rounded fp32 operation at a time (no FMA that
 // would fuse two of them), so the forward and the backward's recomputation
@@ -502,7 +518,7 @@ __global__ void __launch_bounds__(kMaxStagedThreads) scan_fwd_staged(const ScanA
   const TI* my = reinterpret_cast<const TI*>(ring) + c * V;
   const int stage_elems = a.stage_bytes / (int)sizeof(TI);
   RingPos pos;
-  int kk = 0;  // position inside the current checkpoint segment
+  int kk = a.nseg > 0 ? seg_phase0(a) : 0;  // position inside the current checkpoint segment
   for (int64_t t = 0; t < a.T; ++t) {
     if (!warp_wait(&full[pos.s], pos.ph, a.wait_ns)) {
       if (lid == 0) record_status(a.status, kStatusTimeout);
@@ -565,7 +581,7 @@ __device__ __forceinline__ void bwd_pairs(const ScanArgs& a, const float2 beta[N
                                              z[2 * k + 1], i[k], g[k], eu[k], ei[k], st[k]);
 }
 
-template <bool SYN, bool RECOMP, typename TI, typename TO, int RESET, int SG>
+template <bool SYN, bool RECOMP, typename TI, typename TO, int RESET, int SG, int KC = 0>
 __global__ void __launch_bounds__(kMaxStagedThreads) scan_bwd_staged(const ScanArgs a) {
   constexpr int V = kLanes<SYN>, NP = V / 2;
   extern __shared__ __align__(1024) unsigned char smem[];
@@ -579,7 +595,6 @@ __global__ void __launch_bounds__(kMaxStagedThreads) scan_bwd_staged(const ScanA
   const int64_t lane0 = (int64_t)blockIdx.x * a.lanes_per_cta;
   const int cta_lanes = (int)min((int64_t)a.lanes_per_cta, a.L - lane0);
   const int io_stride = a.lanes_per_cta * (int)sizeof(TO);  // byte stride of io tiles
-  const int in_stride = a.lanes_per_cta * (int)sizeof(TI);
   const bool half_store = !RECOMP && sizeof(TO) != 4;      // z from the spk rows
   const bool want_syn = SYN && a.part_alpha != nullptr;
   // store-mode tile order: gs, mem, [spk], [syn], [gm]
@@ -615,7 +630,8 @@ __global__ void __launch_bounds__(kMaxStagedThreads) scan_bwd_staged(const ScanA
       } else {
         int64_t ck_n = 0;  // checkpoint loads issued
         for (int k = a.nseg - 1; k >= 0 && p.ok; --k) {
-          const int64_t t0 = (int64_t)k * a.K, t1 = min(a.T, t0 + a.K);
+          int64_t t0, t1;
+          seg_bounds(a, k, t0, t1);
           if (k > 0) {
             // the segment's starting state: checkpoint rows fp32 [nseg-1][SYN?2:1][L]
             const int slot = (int)(ck_n & 1);
@@ -743,18 +759,19 @@ __global__ void __launch_bounds__(kMaxStagedThreads) scan_bwd_staged(const ScanA
     }
   } else {
     int64_t ck_u = 0;  // checkpoints consumed
-    for (int k = a.nseg - 1; k >= 0 && ok; --k) {
-      const int64_t t0 = (int64_t)k * a.K, t1 = min(a.T, t0 + a.K);
-      float2 u[NP], ii[NP];
-      bool z[V];
+    float2 u[NP], ii[NP];
+    bool z[V];
+    // Start of segment k: its starting state from the checkpoint slot (k > 0)
+    // or the initial state (k = 0).
+    auto seg_start = [&](int k) -> bool {
       if (k > 0) {
         if (!warp_wait(&ck_full[ck_u & 1], (uint32_t)((ck_u >> 1) & 1), a.wait_ns)) {
           if (lid == 0) record_status(a.status, kStatusTimeout);
-          ok = false;
-          break;
+          return false;
         }
         if (active) {
-          const float* cb = reinterpret_cast<const float*>(ck_base + (size_t)(ck_u & 1) * ck_slot_bytes) + c * V;
+          const float* cb =
+              reinterpret_cast<const float*>(ck_base + (size_t)(ck_u & 1) * ck_slot_bytes) + c * V;
           load_pairs<float, NP>(cb, u);
           if (SYN) load_pairs<float, NP>(cb + a.lanes_per_cta, ii);
 #pragma unroll
@@ -766,77 +783,139 @@ __global__ void __launch_bounds__(kMaxStagedThreads) scan_bwd_staged(const ScanA
       } else if (active) {
         initial_state<SYN, NP>(a, l, negthr, u, z, ii);
       }
-      // replay the forward over the segment
-      float* su = seg;
-      for (int64_t t = t0; t < t1; ++t) {
-        if (!warp_wait(&full[pos.s], pos.ph, a.wait_ns)) {
-          if (lid == 0) record_status(a.status, kStatusTimeout);
+      return true;
+    };
+    // After the replay consumed the checkpoint values: free the slot.
+    auto seg_replayed = [&](int k) {
+      if (k > 0) {
+        release_stage(ck_empty, (int)(ck_u & 1), lid);
+        ++ck_u;
+      }
+    };
+    // One replayed forward step from an I row in the stage at `xin`; the
+    // state goes to the replay buffer row `su`.
+    auto replay = [&](const TI* xin, float* su) {
+      if (!active) return;
+      float2 x[NP];
+      load_pairs<TI, NP>(xin, x);
+#pragma unroll
+      for (int q = 0; q < NP; ++q)
+        fwd_pair<SYN, RESET>(a.reset, beta[q], negthr[q], alpha[q], x[q], u[q], &z[2 * q], ii[q]);
+#pragma unroll
+      for (int q = 0; q < V / 4; ++q) {
+        *reinterpret_cast<float4*>(su + q * nthr * 4) =
+            make_float4(u[2 * q].x, u[2 * q].y, u[2 * q + 1].x, u[2 * q + 1].y);
+        if (SYN)
+          *reinterpret_cast<float4*>(su + seg_plane + q * nthr * 4) =
+              make_float4(ii[2 * q].x, ii[2 * q].y, ii[2 * q + 1].x, ii[2 * q + 1].y);
+      }
+    };
+    // One reverse step at time t: grad rows in the stage at `gin`, the
+    // replayed state from buffer row `su`, dL/dI_t to `gout`.
+    auto reverse_step = [&](int64_t t, const TO* gin, const float* su, TO* gout) {
+      if (!active) return;
+      float2 g[NP], gmv[NP], uu[NP], iv[NP], out[NP];
+      bool zz[V];
+      load_pairs<TO, NP>(gin, g);
+      if (a.gm) load_pairs<TO, NP>(gin + tile_io_elems, gmv);
+#pragma unroll
+      for (int q = 0; q < V / 4; ++q) {
+        const float4 uq = *reinterpret_cast<const float4*>(su + q * nthr * 4);
+        uu[2 * q] = make_float2(uq.x, uq.y);
+        uu[2 * q + 1] = make_float2(uq.z, uq.w);
+        if (SYN) {
+          const float4 iq = *reinterpret_cast<const float4*>(su + seg_plane + q * nthr * 4);
+          iv[2 * q] = make_float2(iq.x, iq.y);
+          iv[2 * q + 1] = make_float2(iq.z, iq.w);
+        } else {
+          iv[2 * q] = f2(0.0f);
+          iv[2 * q + 1] = f2(0.0f);
+        }
+      }
+#pragma unroll
+      for (int q = 0; q < NP; ++q) {
+        zz[2 * q] = uu[q].x > -negthr[q].x;
+        zz[2 * q + 1] = uu[q].y > -negthr[q].y;
+      }
+      reverse(t, uu, zz, iv, g, gmv, out);
+      store_pairs<TO, NP>(gout, out);
+    };
+    auto fail = [&]() {
+      if (lid == 0) record_status(a.status, kStatusTimeout);
+      ok = false;
+    };
+
+    int k = a.nseg - 1;
+    if constexpr (KC > 0) {
+      // Full segments (all but the first in time) with the ring at exactly
+      // KS = KC stages: a segment is two whole ring rounds (KC replay items,
+      // then KC reverse items), so every stage index and phase parity below
+      // is a compile-time constant and the ring position is unchanged after
+      // each segment.
+      for (; k >= 1 && ok; --k) {
+        int64_t t0, t1;
+        seg_bounds(a, k, t0, t1);
+        if (!seg_start(k)) {
           ok = false;
           break;
         }
-        if (active) {
-          float2 x[NP];
-          load_pairs<TI, NP>(ring_i + pos.s * stage_in_elems, x);
 #pragma unroll
-          for (int q = 0; q < NP; ++q)
-            fwd_pair<SYN, RESET>(a.reset, beta[q], negthr[q], alpha[q], x[q], u[q], &z[2 * q], ii[q]);
-#pragma unroll
-          for (int q = 0; q < V / 4; ++q) {
-            *reinterpret_cast<float4*>(su + q * nthr * 4) =
-                make_float4(u[2 * q].x, u[2 * q].y, u[2 * q + 1].x, u[2 * q + 1].y);
-            if (SYN)
-              *reinterpret_cast<float4*>(su + seg_plane + q * nthr * 4) =
-                  make_float4(ii[2 * q].x, ii[2 * q].y, ii[2 * q + 1].x, ii[2 * q + 1].y);
+        for (int q = 0; q < KC; ++q) {
+          if (!warp_wait(&full[q], 0u, a.wait_ns)) {
+            fail();
+            break;
           }
+          replay(ring_i + q * stage_in_elems, seg + q * seg_row);
+          release_stage(empty, q, lid);
         }
+        if (!ok) break;
+        seg_replayed(k);
+        TO* gout = static_cast<TO*>(a.gI) + l + t0 * a.L;
+#pragma unroll
+        for (int q = KC - 1; q >= 0; --q) {
+          const int st_idx = KC - 1 - q;  // stage of this reverse item
+          if (!warp_wait(&full[st_idx], 1u, a.wait_ns)) {
+            fail();
+            break;
+          }
+          reverse_step(t0 + q, ring_o + st_idx * stage_io_elems, seg + q * seg_row,
+                       gout + q * a.L);
+          release_stage(empty, st_idx, lid);
+        }
+      }
+    }
+    // Remaining segments (all of them for run-time K) with the general ring
+    // position.
+    for (; k >= 0 && ok; --k) {
+      int64_t t0, t1;
+      seg_bounds(a, k, t0, t1);
+      if (!seg_start(k)) {
+        ok = false;
+        break;
+      }
+      float* su = seg;
+      for (int64_t t = t0; t < t1; ++t) {
+        if (!warp_wait(&full[pos.s], pos.ph, a.wait_ns)) {
+          fail();
+          break;
+        }
+        replay(ring_i + pos.s * stage_in_elems, su);
         release_stage(empty, pos.s, lid);
         pos.next(S);
         su += seg_row;
       }
       if (!ok) break;
-      if (k > 0) {  // the replay consumed the checkpoint values: free the slot
-        release_stage(ck_empty, (int)(ck_u & 1), lid);
-        ++ck_u;
-      }
-      // reverse steps over the segment
+      seg_replayed(k);
+      TO* gout = static_cast<TO*>(a.gI) + l + t0 * a.L;
       for (int64_t t = t1 - 1; t >= t0; --t) {
         su -= seg_row;
         if (!warp_wait(&full[pos.s], pos.ph, a.wait_ns)) {
-          if (lid == 0) record_status(a.status, kStatusTimeout);
-          ok = false;
+          fail();
           break;
         }
-        if (active) {
-          const TO* base = ring_o + pos.s * stage_io_elems;
-          float2 g[NP], gmv[NP], uu[NP], iv[NP], out[NP];
-          bool zz[V];
-          load_pairs<TO, NP>(base, g);
-          if (a.gm) load_pairs<TO, NP>(base + tile_io_elems, gmv);
-#pragma unroll
-          for (int q = 0; q < V / 4; ++q) {
-            const float4 uq = *reinterpret_cast<const float4*>(su + q * nthr * 4);
-            uu[2 * q] = make_float2(uq.x, uq.y);
-            uu[2 * q + 1] = make_float2(uq.z, uq.w);
-            if (SYN) {
-              const float4 iq = *reinterpret_cast<const float4*>(su + seg_plane + q * nthr * 4);
-              iv[2 * q] = make_float2(iq.x, iq.y);
-              iv[2 * q + 1] = make_float2(iq.z, iq.w);
-            } else {
-              iv[2 * q] = f2(0.0f);
-              iv[2 * q + 1] = f2(0.0f);
-            }
-          }
-#pragma unroll
-          for (int q = 0; q < NP; ++q) {
-            zz[2 * q] = uu[q].x > -negthr[q].x;
-            zz[2 * q + 1] = uu[q].y > -negthr[q].y;
-          }
-          reverse(t, uu, zz, iv, g, gmv, out);
-          store_pairs<TO, NP>(gI, out);
-        }
+        reverse_step(t, ring_o + pos.s * stage_io_elems, su, gout + (t - t0) * a.L);
         release_stage(empty, pos.s, lid);
         pos.next(S);
-        gI -= a.L;
       }
     }
   }
@@ -889,7 +968,8 @@ __global__ void __launch_bounds__(256) scan_fwd_plain(const ScanArgs a) {
   TO* mem = static_cast<TO*>(a.mem);
   TO* syn = static_cast<TO*>(a.syn);
   const int64_t ckpt_stride = SYN ? 2 * a.L : a.L;
-  int kk = 0;
+  int kk = a.nseg > 0 ? seg_phase0(a) : 0;
+  float* cp = a.ckpt ? a.ckpt + l : nullptr;
   for (int64_t t = 0; t < a.T; ++t) {
     const int64_t off = t * a.L + l;
     fwd_step<SYN, -1>(a.reset, beta, thr, alpha, Elem<TI>::load1(I + off), u, z, i);
@@ -898,10 +978,10 @@ __global__ void __launch_bounds__(256) scan_fwd_plain(const ScanArgs a) {
     if (SYN && syn) Elem<TO>::store1(syn + off, i);
     if (++kk == a.K) {
       kk = 0;
-      if (a.ckpt && t + 1 < a.T) {
-        float* cp = a.ckpt + (t / a.K) * ckpt_stride + l;
+      if (cp && t + 1 < a.T) {
         *cp = u;
         if (SYN) cp[a.L] = i;
+        cp += ckpt_stride;
       }
     }
   }
@@ -948,7 +1028,8 @@ __global__ void __launch_bounds__(128) scan_bwd_plain(const ScanArgs a) {
     float* su = segbuf + threadIdx.x;
     float* si = segbuf + (size_t)a.K * blockDim.x + threadIdx.x;
     for (int k = a.nseg - 1; k >= 0; --k) {
-      const int64_t t0 = (int64_t)k * a.K, t1 = min(a.T, t0 + a.K);
+      int64_t t0, t1;
+      seg_bounds(a, k, t0, t1);
       float u, i;
       bool z;
       if (k > 0) {
