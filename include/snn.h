@@ -226,6 +226,48 @@ snn_status_t snn_synaptic_bwd(const snn_scan_desc* desc, const void* I, const fl
                               snn_stream_t stream);
 
 /*
+ * Dense-layer input current, the synaptic operation w.x of Fig. 3 (Sec. III,
+ * "the current injection term is replaced with a weighted input"), for all
+ * T*B rows at once on the tcgen05 tensor cores:
+ *   I[M, N] = X[M, K] * W[N, K]^T
+ *   X  bf16 [M, K] row-major (M = T*B rows of layer input, e.g. spikes)
+ *   W  bf16 [N, K] row-major (N outputs, K inputs; no bias)
+ *   I  fp32 [M, N] row-major (out), fp32 accumulation
+ *   ws device workspace of at least 256 bytes (status word, as for the scans)
+ * K must be a multiple of 8 (16-byte rows for the tensor memory accelerator),
+ * else SNN_ERR_UNSUPPORTED.  K = 0 writes zeros.
+ */
+snn_status_t snn_dense_layer_fwd(int64_t M, int64_t K, int64_t N, const void* X, const void* W,
+                                 float* I, void* ws, size_t ws_bytes, snn_stream_t stream);
+
+/* Workspace bytes of snn_dense_layer_bwd (transposed operand copies). */
+size_t snn_dense_workspace_bytes(int64_t M, int64_t K, int64_t N);
+
+/*
+ * Backward of snn_dense_layer_fwd, given dI = dL/dI (bf16 [M, N], e.g. the
+ * grad_I of a scan with bf16 io):
+ *   dX bf16 [M, K] (out, or NULL) = dI * W          (input gradient)
+ *   dW fp32 [N, K] (out, or NULL) = dI^T * X        (weight gradient)
+ * M, K and N must be multiples of 8.  ws: snn_dense_workspace_bytes(M,K,N).
+ */
+snn_status_t snn_dense_layer_bwd(int64_t M, int64_t K, int64_t N, const void* X, const void* W,
+                                 const void* dI, void* dX, float* dW, void* ws, size_t ws_bytes,
+                                 snn_stream_t stream);
+
+/*
+ * Rate-coded readout loss (Sec. V-A: the predicted class is the output
+ * neuron that fires most): cross-entropy of the spike counts over T.
+ *   spk   [T, B, ld] in `dtype` (snn_dtype_t); the first C of ld neurons are
+ *         the classes (C <= 1024)
+ *   labels int32 [B];  loss fp32 [1] (out) = mean_b CE(sum_t spk[:, b, :C], y_b)
+ *   grad_spk [T, B, ld] (out) = (softmax - onehot) / B for every t; 0 for
+ *         neurons C..ld-1
+ */
+snn_status_t snn_rate_ce_loss(int64_t T, int64_t B, int64_t C, int64_t ld, int32_t dtype,
+                              const void* spk, const int32_t* labels, float* loss,
+                              void* grad_spk, snn_stream_t stream);
+
+/*
  * Leaky BPTT that allocates nothing (no counterpart in the paper; it exists
  * for callers of this library that cannot allocate device memory: hosts
  * whose device memory is budgeted by another runtime, real-time loops that

@@ -1,0 +1,452 @@
+// Dense-layer input current on the 5th-generation tensor cores: the synaptic
+// operation w.x of the paper's Fig. 3 batched over all T*B rows,
+//   D[M, N] = A[M, K] * B[N, K]^T,   A, B bf16 row-major (K contiguous),
+// fp32 accumulation in tensor memory, fp32 or bf16 output.
+//
+// One CTA computes a 128 x BN tile.  Warp 0 (one thread) streams 128x64 and
+// BNx64 operand tiles into a 4-stage shared-memory ring with TMA (128-byte
+// swizzle); warp 1 allocates the TMEM accumulator and one thread issues
+// tcgen05.mma (M=128, N=BN, K=16 per instruction) as stages land, freeing
+// each stage through tcgen05.commit; warps 2-5 read the accumulator back
+// with tcgen05.ld (each warp its 32-lane quarter) and store it.  Every wait
+// is bounded; a kernel that gives up records SNN_ERR_TIMEOUT and still
+// drains its copies and frees its TMEM.
+//
+// The backward products dX = dI*W and dW = dI^T*X use the same kernel on
+// transposed copies (made by a tiled transpose kernel) so both operands stay
+// K-major.
+#include <cuda.h>
+#include <cudaTypedefs.h>
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+
+#include <climits>
+#include <cstdint>
+#include <mutex>
+
+#include "scan_host.cuh"
+#include "snn.h"
+
+namespace snn {
+namespace gemm {
+
+constexpr int BM = 128;
+constexpr int BK = 64;  // 64 bf16 = 128 bytes: one swizzle atom row
+constexpr int kStages = 4;
+constexpr int kThreads = 192;
+constexpr uint64_t kDefaultWaitNs = 2000000000ull;
+constexpr uint64_t kDrainWaitNs = 1000000000ull;
+
+struct GemmArgs {
+  int M, N, K;
+  void* D;
+  int64_t ldd;  // row stride of D in elements
+  int* status;
+  uint64_t wait_ns;
+};
+
+// ---------------------------------------------------------------------------
+// PTX wrappers: TMA, tcgen05
+// ---------------------------------------------------------------------------
+
+__device__ __forceinline__ void tma_load_2d(void* dst, const CUtensorMap* map, int x, int y,
+                                            uint64_t* bar) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], [%4];" ::"r"(
+          smem_u32(dst)),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(smem_u32(bar))
+      : "memory");
+}
+
+__device__ __forceinline__ void tc_fence_before() {
+  asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+}
+__device__ __forceinline__ void tc_fence_after() {
+  asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+}
+
+// Shared-memory matrix descriptor of a K-major operand tile in the 128-byte
+// swizzled layout TMA writes: rows of 128 bytes, 8-row (1024-byte) atoms.
+__device__ __forceinline__ uint64_t sdesc_sw128(const void* tile) {
+  const uint32_t addr = smem_u32(tile);
+  uint64_t d = 0;
+  d |= (uint64_t)((addr >> 4) & 0x3FFFu);      // start address
+  d |= (uint64_t)(16u >> 4) << 16;              // leading byte offset (unused here)
+  d |= (uint64_t)(1024u >> 4) << 32;            // stride byte offset: one 8-row atom
+  d |= (uint64_t)1 << 46;                       // descriptor version
+  d |= (uint64_t)2 << 61;                       // 128-byte swizzle
+  return d;
+}
+
+// Instruction descriptor: bf16 x bf16 -> fp32, both operands K-major.
+__host__ __device__ constexpr uint32_t idesc_bf16(int m, int n) {
+  return (1u << 4)                         // D format: f32
+         | (1u << 7)                       // A format: bf16
+         | (1u << 10)                      // B format: bf16
+         | ((uint32_t)(n >> 3) << 17)      // N / 8
+         | ((uint32_t)(m >> 4) << 24);     // M / 16
+}
+
+__device__ __forceinline__ void tc_mma(uint32_t tmem_d, uint64_t adesc, uint64_t bdesc,
+                                       uint32_t idesc, uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "setp.ne.b32 p, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(tmem_d),
+      "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+
+// Arrive on `bar` once every tcgen05.mma this thread issued has completed.
+__device__ __forceinline__ void tc_commit(uint64_t* bar) {
+  asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
+                   smem_u32(bar))
+               : "memory");
+}
+
+__device__ __forceinline__ void tmem_alloc(uint32_t* slot, uint32_t ncols) {
+  asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(slot)),
+               "r"(ncols)
+               : "memory");
+  asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+}
+
+__device__ __forceinline__ void tmem_dealloc(uint32_t taddr, uint32_t ncols) {
+  asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(ncols)
+               : "memory");
+}
+
+// 32 lanes x 16 consecutive 32-bit columns of TMEM -> 16 registers per thread.
+__device__ __forceinline__ void tmem_ld16(uint32_t taddr, uint32_t r[16]) {
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, "
+      "%12, %13, %14, %15}, [%16];"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
+        "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]),
+        "=r"(r[14]), "=r"(r[15])
+      : "r"(taddr));
+  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+}
+
+// Bounded wait taken by a whole warp; the give-up decision is warp-uniform.
+__device__ __forceinline__ bool warp_wait_uniform(uint64_t* bar, uint32_t parity, uint64_t limit_ns) {
+  bool done = mbar_try_wait(bar, parity);
+  if (__all_sync(0xffffffffu, done)) return true;
+  const uint64_t t0 = globaltimer_ns();
+  while (true) {
+    if (!done) done = mbar_try_wait(bar, parity);
+    if (__all_sync(0xffffffffu, done)) return true;
+    uint64_t el = globaltimer_ns() - t0;
+    el = __shfl_sync(0xffffffffu, el, 0);
+    if (el > limit_ns) return false;
+  }
+}
+
+template <int BN>
+__host__ __device__ constexpr uint32_t tmem_cols() {
+  return BN <= 32 ? 32u : (uint32_t)BN;
+}
+
+template <int BN>
+__host__ __device__ constexpr size_t smem_bytes() {
+  return 1024 /* alignment slack */ + (size_t)kStages * (BM * BK * 2 + BN * BK * 2) + 256;
+}
+
+// ---------------------------------------------------------------------------
+// Kernel
+// ---------------------------------------------------------------------------
+
+template <int BN, bool OUT_BF16>
+__global__ void __launch_bounds__(kThreads, 1)
+    gemm_tn_tcgen05(const __grid_constant__ CUtensorMap ta, const __grid_constant__ CUtensorMap tb,
+                    const GemmArgs g) {
+  static_assert(BN % 16 == 0 && BN >= 16 && BN <= 256, "UMMA N for M=128");
+  constexpr int A_BYTES = BM * BK * 2;
+  constexpr int B_BYTES = BN * BK * 2;
+  constexpr uint32_t TCOLS = tmem_cols<BN>();
+  extern __shared__ unsigned char smem_raw[];
+  unsigned char* smem =
+      reinterpret_cast<unsigned char*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  unsigned char* sA = smem;
+  unsigned char* sB = smem + kStages * A_BYTES;
+  uint64_t* full = reinterpret_cast<uint64_t*>(sB + kStages * B_BYTES);
+  uint64_t* empty = full + kStages;
+  uint64_t* accum = empty + kStages;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(accum + 1);
+  const int warp = threadIdx.x >> 5, lid = threadIdx.x & 31;
+  const int m0 = blockIdx.y * BM, n0 = blockIdx.x * BN;
+  const int nk = (g.K + BK - 1) / BK;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < kStages; ++s) {
+      mbar_init(&full[s], 1);
+      mbar_init(&empty[s], 1);
+    }
+    mbar_init(accum, 1);
+    fence_barrier_init();
+  }
+  if (warp == 1) tmem_alloc(tmem_slot, TCOLS);
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+
+  if (warp == 0) {
+    if (lid == 0) {
+      int issued = 0;
+      for (int kb = 0; kb < nk; ++kb) {
+        const int s = kb % kStages;
+        if (kb >= kStages &&
+            !mbar_wait_bounded(&empty[s], (uint32_t)(((kb / kStages) - 1) & 1), g.wait_ns)) {
+          record_status(g.status, kStatusTimeout);
+          break;
+        }
+        mbar_arrive_expect_tx(&full[s], A_BYTES + B_BYTES);
+        tma_load_2d(sA + s * A_BYTES, &ta, kb * BK, m0, &full[s]);
+        tma_load_2d(sB + s * B_BYTES, &tb, kb * BK, n0, &full[s]);
+        ++issued;
+      }
+      // every copy this thread issued has landed before the CTA may exit
+      for (int j = issued > kStages ? issued - kStages : 0; j < issued; ++j)
+        mbar_wait_bounded(&full[j % kStages], (uint32_t)((j / kStages) & 1), kDrainWaitNs);
+    }
+  } else if (warp == 1) {
+    if (lid == 0) {
+      constexpr uint32_t idesc = idesc_bf16(BM, BN);
+      for (int kb = 0; kb < nk; ++kb) {
+        const int s = kb % kStages;
+        if (!mbar_wait_bounded(&full[s], (uint32_t)((kb / kStages) & 1), g.wait_ns)) {
+          record_status(g.status, kStatusTimeout);
+          break;
+        }
+        tc_fence_after();
+        const uint64_t da = sdesc_sw128(sA + s * A_BYTES);
+        const uint64_t db = sdesc_sw128(sB + s * B_BYTES);
+#pragma unroll
+        for (int kk = 0; kk < BK / 16; ++kk)  // 16 bf16 = 32 bytes further along K
+          tc_mma(tmem, da + 2 * kk, db + 2 * kk, idesc, (kb | kk) != 0 ? 1u : 0u);
+        tc_commit(&empty[s]);  // the stage is free once these MMAs are done
+      }
+      tc_commit(accum);  // the accumulator is final once every MMA is done
+    }
+  } else {
+    // epilogue: warp w reads TMEM lanes 32*(w%4) .. +32, i.e. tile rows
+    const int q = warp & 3;
+    const bool ok = warp_wait_uniform(accum, 0u, g.wait_ns);
+    tc_fence_after();
+    if (ok) {
+      const int row = m0 + q * 32 + lid;
+#pragma unroll 1
+      for (int c = 0; c < BN; c += 16) {
+        uint32_t r[16];
+        tmem_ld16(tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)c, r);
+        const int col = n0 + c;
+        if (row < g.M && col < g.N) {
+          if (OUT_BF16) {
+            __nv_bfloat16* d = static_cast<__nv_bfloat16*>(g.D) + (int64_t)row * g.ldd + col;
+            if (col + 16 <= g.N && (((int64_t)row * g.ldd + col) & 7) == 0) {
+              uint4 v[2];
+              uint32_t* w = reinterpret_cast<uint32_t*>(v);
+#pragma unroll
+              for (int j = 0; j < 8; ++j) {
+                __nv_bfloat162 h = __floats2bfloat162_rn(__uint_as_float(r[2 * j]), __uint_as_float(r[2 * j + 1]));
+                w[j] = *reinterpret_cast<uint32_t*>(&h);
+              }
+              reinterpret_cast<uint4*>(d)[0] = v[0];
+              reinterpret_cast<uint4*>(d)[1] = v[1];
+            } else {
+              for (int j = 0; j < 16 && col + j < g.N; ++j) d[j] = __float2bfloat16_rn(__uint_as_float(r[j]));
+            }
+          } else {
+            float* d = static_cast<float*>(g.D) + (int64_t)row * g.ldd + col;
+            if (col + 16 <= g.N && (((int64_t)row * g.ldd + col) & 3) == 0) {
+#pragma unroll
+              for (int j = 0; j < 4; ++j)
+                reinterpret_cast<float4*>(d)[j] =
+                    make_float4(__uint_as_float(r[4 * j]), __uint_as_float(r[4 * j + 1]),
+                                __uint_as_float(r[4 * j + 2]), __uint_as_float(r[4 * j + 3]));
+            } else {
+              for (int j = 0; j < 16 && col + j < g.N; ++j) d[j] = __uint_as_float(r[j]);
+            }
+          }
+        }
+      }
+    } else if (lid == 0) {
+      record_status(g.status, kStatusTimeout);
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem, TCOLS);
+  }
+}
+
+// bf16 [R, C] row-major -> [C, R] row-major, 32x32 tiles through shared memory.
+__global__ void __launch_bounds__(256) transpose_bf16(const __nv_bfloat16* in, __nv_bfloat16* out,
+                                                      int R, int C) {
+  __shared__ __nv_bfloat16 tile[32][34];
+  const int bx = blockIdx.x * 32, by = blockIdx.y * 32;
+  const int tx = threadIdx.x & 31, ty = threadIdx.x >> 5;  // 32 x 8
+  for (int j = ty; j < 32; j += 8) {
+    const int r = by + j, c = bx + tx;
+    if (r < R && c < C) tile[j][tx] = in[(int64_t)r * C + c];
+  }
+  __syncthreads();
+  for (int j = ty; j < 32; j += 8) {
+    const int r = bx + j, c = by + tx;  // output row = input column
+    if (r < C && c < R) out[(int64_t)r * R + c] = tile[tx][j];
+  }
+}
+
+// ---------------------------------------------------------------------------
+// Host side
+// ---------------------------------------------------------------------------
+
+PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
+  static std::once_flag once;
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  std::call_once(once, [] {
+    cudaDriverEntryPointQueryResult q;
+    void* p = nullptr;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault,
+                                         &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+  });
+  return fn;
+}
+
+// Tensor map of a bf16 row-major [rows, cols] matrix read as box_rows x 64
+// tiles with 128-byte swizzle; out-of-range elements read as zero.
+bool make_map(CUtensorMap* map, const void* base, int64_t rows, int64_t cols, int box_rows) {
+  auto fn = encode_fn();
+  if (!fn) return false;
+  const cuuint64_t dims[2] = {(cuuint64_t)cols, (cuuint64_t)rows};
+  const cuuint64_t strides[1] = {(cuuint64_t)cols * 2};
+  const cuuint32_t box[2] = {(cuuint32_t)BK, (cuuint32_t)box_rows};
+  const cuuint32_t estr[2] = {1, 1};
+  return fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box,
+            estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+            CU_TENSOR_MAP_L2_PROMOTION_L2_128B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+template <int BN, bool OUT_BF16>
+cudaError_t launch_bn(const CUtensorMap& ta, const CUtensorMap& tb, const GemmArgs& g,
+                      cudaStream_t st) {
+  const void* k = (const void*)gemm_tn_tcgen05<BN, OUT_BF16>;
+  const cudaError_t attr = ensure_smem(k, smem_bytes<BN>());  // once per device
+  if (attr != cudaSuccess) return attr;
+  const dim3 grid((unsigned)((g.N + BN - 1) / BN), (unsigned)((g.M + BM - 1) / BM));
+  gemm_tn_tcgen05<BN, OUT_BF16><<<grid, kThreads, smem_bytes<BN>(), st>>>(ta, tb, g);
+  return cudaGetLastError();
+}
+
+// D[M, N] = A[M, K] * B[N, K]^T with the widest N tile that the output needs.
+template <bool OUT_BF16>
+cudaError_t gemm_tn(const void* A, const void* B, void* D, int M, int N, int K, int* status,
+                    cudaStream_t st) {
+  int bn = 128;
+  if (N <= 16) bn = 16;
+  else if (N <= 32) bn = 32;
+  else if (N <= 64) bn = 64;
+  CUtensorMap ta, tb;
+  if (!make_map(&ta, A, M, K, BM) || !make_map(&tb, B, N, K, bn)) return cudaErrorInvalidValue;
+  GemmArgs g{M, N, K, D, (int64_t)N, status, kDefaultWaitNs};
+  switch (bn) {
+    case 16: return launch_bn<16, OUT_BF16>(ta, tb, g, st);
+    case 32: return launch_bn<32, OUT_BF16>(ta, tb, g, st);
+    case 64: return launch_bn<64, OUT_BF16>(ta, tb, g, st);
+    default: return launch_bn<128, OUT_BF16>(ta, tb, g, st);
+  }
+}
+
+cudaError_t transpose(const void* in, void* out, int R, int C, cudaStream_t st) {
+  if (R == 0 || C == 0) return cudaSuccess;
+  const dim3 grid((unsigned)((C + 31) / 32), (unsigned)((R + 31) / 32));
+  transpose_bf16<<<grid, 256, 0, st>>>(static_cast<const __nv_bfloat16*>(in),
+                                       static_cast<__nv_bfloat16*>(out), R, C);
+  return cudaGetLastError();
+}
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+size_t round256(size_t b) { return (b + 255) & ~size_t(255); }
+
+snn_status_t check_dims(int64_t M, int64_t K, int64_t N) {
+  if (M < 0 || K < 0 || N < 0) return SNN_ERR_INVALID_ARG;
+  if (M > INT_MAX / 2 || K > INT_MAX / 2 || N > INT_MAX / 2) return SNN_ERR_INVALID_ARG;
+  return SNN_OK;
+}
+
+}  // namespace gemm
+}  // namespace snn
+
+using namespace snn::gemm;
+
+extern "C" {
+
+size_t snn_dense_workspace_bytes(int64_t M, int64_t K, int64_t N) {
+  if (check_dims(M, K, N) != SNN_OK) return 0;
+  return 256 + round256((size_t)K * N * 2) + round256((size_t)N * M * 2) +
+         round256((size_t)K * M * 2);
+}
+
+snn_status_t snn_dense_layer_fwd(int64_t M, int64_t K, int64_t N, const void* X, const void* W,
+                                 float* I, void* ws, size_t ws_bytes, snn_stream_t stream) {
+  snn_status_t s = check_dims(M, K, N);
+  if (s != SNN_OK) return s;
+  if (K % 8 != 0) return SNN_ERR_UNSUPPORTED;  // TMA needs 16-byte row strides
+  if ((M > 0 && N > 0) && (!X || !W || !I)) return SNN_ERR_INVALID_ARG;
+  if (!aligned16(X) || !aligned16(W) || !aligned16(I) || !aligned16(ws)) return SNN_ERR_ALIGNMENT;
+  if (!ws || ws_bytes < 256) return SNN_ERR_WORKSPACE;
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  if (M == 0 || N == 0) return SNN_OK;
+  if (K == 0)
+    return cudaMemsetAsync(I, 0, (size_t)M * N * sizeof(float), st) == cudaSuccess ? SNN_OK : SNN_ERR_CUDA;
+  const cudaError_t e = gemm_tn<false>(X, W, I, (int)M, (int)N, (int)K, static_cast<int*>(ws), st);
+  return e == cudaSuccess ? SNN_OK : (e == cudaErrorInvalidValue ? SNN_ERR_UNSUPPORTED : SNN_ERR_CUDA);
+}
+
+snn_status_t snn_dense_layer_bwd(int64_t M, int64_t K, int64_t N, const void* X, const void* W,
+                                 const void* dI, void* dX, float* dW, void* ws, size_t ws_bytes,
+                                 snn_stream_t stream) {
+  snn_status_t s = check_dims(M, K, N);
+  if (s != SNN_OK) return s;
+  if (K % 8 != 0 || N % 8 != 0 || M % 8 != 0) return SNN_ERR_UNSUPPORTED;
+  if (!dI || (!dX && !dW)) return SNN_ERR_INVALID_ARG;
+  if ((dX && !W) || (dW && !X)) return SNN_ERR_INVALID_ARG;
+  const void* ptrs[6] = {X, W, dI, dX, dW, ws};
+  for (const void* p : ptrs)
+    if (!aligned16(p)) return SNN_ERR_ALIGNMENT;
+  if (!ws || ws_bytes < snn_dense_workspace_bytes(M, K, N)) return SNN_ERR_WORKSPACE;
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  unsigned char* w = static_cast<unsigned char*>(ws);
+  int* status = reinterpret_cast<int*>(w);
+  void* Wt = w + 256;                                       // [K, N]
+  void* dIt = w + 256 + round256((size_t)K * N * 2);       // [N, M]
+  void* Xt = static_cast<unsigned char*>(dIt) + round256((size_t)N * M * 2);  // [K, M]
+  cudaError_t e = cudaSuccess;
+  if (dX && M > 0 && K > 0) {
+    if (N == 0) {
+      e = cudaMemsetAsync(dX, 0, (size_t)M * K * 2, st);
+    } else {
+      e = transpose(W, Wt, (int)N, (int)K, st);
+      if (e == cudaSuccess) e = gemm_tn<true>(dI, Wt, dX, (int)M, (int)K, (int)N, status, st);
+    }
+    if (e != cudaSuccess) return e == cudaErrorInvalidValue ? SNN_ERR_UNSUPPORTED : SNN_ERR_CUDA;
+  }
+  if (dW && N > 0 && K > 0) {
+    if (M == 0) {
+      e = cudaMemsetAsync(dW, 0, (size_t)N * K * sizeof(float), st);
+    } else {
+      e = transpose(dI, dIt, (int)M, (int)N, st);
+      if (e == cudaSuccess) e = transpose(X, Xt, (int)M, (int)K, st);
+      if (e == cudaSuccess) e = gemm_tn<false>(dIt, Xt, dW, (int)N, (int)K, (int)M, status, st);
+    }
+    if (e != cudaSuccess) return e == cudaErrorInvalidValue ? SNN_ERR_UNSUPPORTED : SNN_ERR_CUDA;
+  }
+  return SNN_OK;
+}
+
+}  // extern "C"

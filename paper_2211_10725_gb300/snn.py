@@ -70,6 +70,10 @@ _SIGS = {
     "snn_synaptic_fwd": ([ctypes.POINTER(ScanDesc)] + [_P] * 13 + [ctypes.c_size_t, _P], ctypes.c_int),
     "snn_synaptic_bwd": ([ctypes.POINTER(ScanDesc)] + [_P] * 21 + [ctypes.c_size_t, _P], ctypes.c_int),
     "snn_leaky_bwd_noalloc": ([ctypes.POINTER(ScanDesc)] + [_P] * 16, ctypes.c_int),
+    "snn_dense_layer_fwd": ([ctypes.c_int64] * 3 + [_P] * 4 + [ctypes.c_size_t, _P], ctypes.c_int),
+    "snn_dense_workspace_bytes": ([ctypes.c_int64] * 3, ctypes.c_size_t),
+    "snn_dense_layer_bwd": ([ctypes.c_int64] * 3 + [_P] * 6 + [ctypes.c_size_t, _P], ctypes.c_int),
+    "snn_rate_ce_loss": ([ctypes.c_int64] * 4 + [ctypes.c_int32] + [_P] * 4 + [_P], ctypes.c_int),
 }
 
 _lib: Optional[ctypes.CDLL] = None
@@ -208,6 +212,36 @@ def snn_leaky_bwd_noalloc(desc, I, ckpt, mem, spk, beta, thr, mem0, grad_spk, gr
         _ptr(mem0), _ptr(grad_spk), _ptr(grad_mem), _ptr(grad_mem_final), _ptr(grad_I),
         _ptr(grad_beta), _ptr(grad_thr), _ptr(grad_mem0), _ptr(status), _stream(stream)),
         "snn_leaky_bwd_noalloc")
+
+
+def snn_dense_workspace_bytes(M: int, K: int, N: int) -> int:
+    return load_library().snn_dense_workspace_bytes(M, K, N)
+
+
+def snn_dense_layer_fwd(X, W, I, ws, stream=None):
+    """I[M, N] = X[M, K] @ W[N, K]^T on the tensor cores (bf16 in, fp32 out)."""
+    M, K = X.shape[-2], X.shape[-1]
+    N = W.shape[0]
+    _check(load_library().snn_dense_layer_fwd(M, K, N, _ptr(X), _ptr(W), _ptr(I), _ptr(ws),
+                                              ws.numel() * ws.element_size(), _stream(stream)),
+           "snn_dense_layer_fwd")
+
+
+def snn_dense_layer_bwd(X, W, dI, dX, dW, ws, stream=None):
+    """dX = dI @ W (bf16) and dW = dI^T @ X (fp32); either output may be None."""
+    M, K = X.shape[-2], X.shape[-1]
+    N = W.shape[0]
+    _check(load_library().snn_dense_layer_bwd(M, K, N, _ptr(X), _ptr(W), _ptr(dI), _ptr(dX),
+                                              _ptr(dW), _ptr(ws), ws.numel() * ws.element_size(),
+                                              _stream(stream)), "snn_dense_layer_bwd")
+
+
+def snn_rate_ce_loss(spk, labels, C, loss, grad_spk, stream=None):
+    """Cross-entropy on output spike counts; spk/grad_spk [T, B, ld]."""
+    T, B, ld = spk.shape
+    dt = {torch.float32: 0, torch.bfloat16: 1, torch.float16: 2}[spk.dtype]
+    _check(load_library().snn_rate_ce_loss(T, B, C, ld, dt, _ptr(spk), _ptr(labels), _ptr(loss),
+                                           _ptr(grad_spk), _stream(stream)), "snn_rate_ce_loss")
 
 
 # ---------------------------------------------------------------------------
