@@ -386,3 +386,76 @@ def rate_ce_loss(spk_out, labels):
     onehot[np.arange(B), y] = 1.0
     g = (p - onehot) / B
     return loss, np.broadcast_to(g, (T, B, C)).copy()
+
+
+# ---------------------------------------------------------------------------
+# The dense SNN of Tab. I: dense layers feeding Leaky layers (Sec. V-A)
+# ---------------------------------------------------------------------------
+
+def dsnn_forward(X, Ws, T: int, B: int, beta: float, thr: float, dtype=np.float32):
+    """Forward pass of a stack of dense -> Leaky layers.
+
+    X: [T*B, K_0] input spikes (row t*B + b); Ws[l]: [N_l, K_l] with
+    K_{l+1} = N_l.  Layer l: I_l = in_l W_l^T over all T*B rows
+    (``dense_forward``, the synaptic operation of Fig. 3), then Eq. (4) with
+    reset by subtraction over t (``leaky_forward``) in ``dtype``, the
+    precision in which the spike decisions are taken; the spikes of layer l
+    are the input of layer l + 1.
+
+    Returns dict of per-layer lists: ``ins`` [T*B, K_l], ``I`` [T*B, N_l]
+    (float64), ``spk`` and ``mem`` [T, B*N_l] (float64 copies of the
+    ``dtype`` trace).
+    """
+    x = np.asarray(X, dtype=np.float64)
+    out = {"ins": [], "I": [], "spk": [], "mem": []}
+    for Wl in Ws:
+        n = Wl.shape[0]
+        I = dense_forward(x, Wl)
+        L = B * n
+        spk, mem = leaky_forward(I.astype(dtype).reshape(T, L), np.full(L, beta, dtype),
+                                 np.full(L, thr, dtype), "subtract", dtype=dtype)
+        out["ins"].append(x)
+        out["I"].append(I)
+        out["spk"].append(spk.astype(np.float64))
+        out["mem"].append(mem.astype(np.float64))
+        x = out["spk"][-1].reshape(T * B, n)
+    return out
+
+
+def dsnn_backward(fwd, Ws, labels, T: int, B: int, beta: float, thr: float,
+                  sg_param: float, store=None):
+    """Loss and BPTT of ``dsnn_forward``.
+
+    The loss is ``rate_ce_loss`` on the last layer's spikes.  Then, from the
+    top layer down: ``leaky_backward`` (detached reset, fast-sigmoid
+    surrogate of slope ``sg_param``) on the layer's saved trace turns the
+    spike gradient into dL/dI_l; ``dense_backward`` turns that into dL/dW_l
+    and dL/din_l, which is the spike gradient of layer l - 1.
+
+    ``store(x)`` rounds a value at each point where the path keeps it in a
+    storage format (the loss gradient, every dL/dI_l and dL/din_l); None
+    keeps float64 throughout.
+
+    Returns dict: ``loss``, ``grad_out`` [T, B, C], and per-layer lists
+    ``grad_spk`` [T, B*N_l], ``grad_I`` [T*B, N_l], ``dW`` [N_l, K_l].
+    """
+    keep = (lambda a: a) if store is None else store
+    nl = len(Ws)
+    C = Ws[-1].shape[0]
+    loss, g_out = rate_ce_loss(fwd["spk"][-1].reshape(T, B, C), labels)
+    g_out = keep(g_out)
+    gs = g_out.reshape(T, B * C)
+    res = {"loss": loss, "grad_out": g_out, "grad_spk": [None] * nl,
+           "grad_I": [None] * nl, "dW": [None] * nl}
+    for l in range(nl - 1, -1, -1):
+        n = Ws[l].shape[0]
+        L = B * n
+        res["grad_spk"][l] = gs
+        g = leaky_backward(fwd["mem"][l], fwd["spk"][l], gs, np.full(L, beta), np.full(L, thr),
+                           reset="subtract", detach=True, sg="fast_sigmoid", sg_param=sg_param)
+        dI = keep(g["grad_I"]).reshape(T * B, n)
+        dX, dW = dense_backward(fwd["ins"][l], Ws[l], dI)
+        res["grad_I"][l] = dI
+        res["dW"][l] = dW
+        gs = keep(dX).reshape(T, B * Ws[l].shape[1])
+    return res

@@ -395,3 +395,60 @@ def test_rate_ce_loss_matches_torch_autograd():
     ref.backward()
     assert abs(loss - ref.item()) < 1e-12
     np.testing.assert_allclose(g, ts.grad.numpy(), rtol=1e-12, atol=1e-14)
+
+
+class _SpikeFastSigmoid(torch.autograd.Function):
+    """Heaviside forward (Eq. 3) with the fast-sigmoid derivative of slope k
+    in the backward: written directly in torch so that autograd, not the
+    oracle's hand-written reverse recurrence, does the chain rule."""
+
+    @staticmethod
+    def forward(ctx, x, k):
+        ctx.save_for_backward(x)
+        ctx.k = k
+        return (x > 0).to(x.dtype)
+
+    @staticmethod
+    def backward(ctx, g):
+        (x,) = ctx.saved_tensors
+        return g / (1.0 + ctx.k * x.abs()) ** 2, None
+
+
+@pytest.mark.parametrize("k", [1.0, 5.0])
+def test_dsnn_matches_torch_autograd(k):
+    """The 3-layer dense SNN (dense -> Eq. 4 per layer, rate-coded CE) against
+    a torch float64 network differentiated by autograd with the reset
+    detached: spikes, loss and every dW agree."""
+    rng = np.random.default_rng(13)
+    T, B, sizes, beta, thr = 5, 4, (12, 9, 7, 5), 0.85, 1.0
+    X = (rng.uniform(0, 1, (T * B, sizes[0])) < 0.4).astype(np.float64)
+    Ws = [rng.uniform(-1.2, 1.2, (o, i)) for i, o in zip(sizes[:-1], sizes[1:])]
+    y = rng.integers(0, sizes[-1], B)
+    fwd = O.dsnn_forward(X, Ws, T, B, beta, thr, dtype=np.float64)
+    res = O.dsnn_backward(fwd, Ws, y, T, B, beta, thr, k)
+
+    tW = [torch.tensor(w, requires_grad=True) for w in Ws]
+    x = torch.tensor(X)
+    spikes = []
+    for w in tW:
+        cur = (x @ w.T).reshape(T, B, -1)
+        u = torch.zeros(B, w.shape[0], dtype=torch.float64)
+        z = torch.zeros_like(u)
+        zs = []
+        for t in range(T):
+            u = beta * u + cur[t] - z.detach() * thr
+            z = _SpikeFastSigmoid.apply(u - thr, k)
+            zs.append(z)
+        s = torch.stack(zs)
+        spikes.append(s)
+        x = s.reshape(T * B, -1)
+    loss = torch.nn.functional.cross_entropy(spikes[-1].sum(0), torch.tensor(y))
+    loss.backward()
+
+    for l, s in enumerate(spikes):
+        assert np.array_equal(fwd["spk"][l], s.detach().numpy().reshape(T, -1))
+    assert all(0 < f.mean() < 1 for f in fwd["spk"])   # every layer spikes, not saturated
+    assert abs(res["loss"] - loss.item()) < 1e-12
+    for l, w in enumerate(tW):
+        assert np.abs(w.grad.numpy()).max() > 1e-4      # a gradient reaches every layer
+        np.testing.assert_allclose(res["dW"][l], w.grad.numpy(), rtol=1e-10, atol=1e-14)
