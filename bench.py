@@ -24,6 +24,9 @@ import time
 
 ROOT = os.path.dirname(os.path.abspath(__file__))
 sys.path.insert(0, ROOT)
+# the oracle legs are timed on one host core: keep numpy's BLAS to one thread
+for _var in ("OPENBLAS_NUM_THREADS", "MKL_NUM_THREADS", "OMP_NUM_THREADS"):
+    os.environ.setdefault(_var, "1")
 
 METRIC = "neuron-steps/sec (fwd+BPTT) on 1 GB300; achieved HBM GB/s vs roofline"
 UNIT = "neuron-steps/s"
@@ -40,7 +43,9 @@ def parse():
     p.add_argument("--workload", default=DEFAULT_WORKLOAD)
     # store (mem + spk saved) is the faster variant on GB300; recompute moves
     # fewer bytes but its reverse pass is instruction-bound
-    p.add_argument("--save", default="mem", choices=["mem", "recompute"])
+    p.add_argument("--save", default=None, choices=["mem", "recompute"])
+    p.add_argument("--no-graph", action="store_true",
+                   help="dense-SNN workload: launch the step eagerly, not as a CUDA graph")
     p.add_argument("--no-e2e", action="store_true")
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--cpu-seconds", type=float, default=15.0)
@@ -50,9 +55,12 @@ def parse():
 def workload(args):
     from paper_2211_10725_gb300 import workloads as W
     w = W.SCAN_WORKLOADS[args.workload]
-    if args.save:
-        w = w.scaled(save=args.save)
-    return w
+    return w.scaled(save=args.save or "mem")
+
+
+def is_dense(args):
+    from paper_2211_10725_gb300 import workloads as W
+    return args.workload == W.DSNN_C3.name
 
 
 # ---------------------------------------------------------------------------
@@ -234,9 +242,58 @@ def time_oracle(w, inp, seconds):
     return w.T * done / t_total, done, t_total
 
 
+def run_dense_reference(args):
+    """The oracle's dense-SNN forward + loss + BPTT on a bounded sample of
+    the batch per step (samples are independent until the dW sums)."""
+    import numpy as np
+    from oracle import snn_oracle as O
+    from paper_2211_10725_gb300 import workloads as W
+    w = W.DSNN_C3
+    inp = W.make_dense_inputs(w)
+    Ws = [x.float().numpy().astype(np.float64) for x in inp["W"]]
+    X = inp["X"].float().numpy().astype(np.float64)          # [T, B, K0]
+    y = inp["labels"].numpy().astype(np.int64)
+
+    def one(bs):
+        xb = X[:, bs].reshape(w.T * len(bs), -1)
+        fwd = O.dsnn_forward(xb, Ws, w.T, len(bs), w.beta, w.thr)
+        O.dsnn_backward(fwd, Ws, y[bs], w.T, len(bs), w.beta, w.thr, w.sg_param)
+
+    t0 = time.perf_counter()
+    one(np.arange(8))
+    per_sample = (time.perf_counter() - t0) / 8
+    total = max(1, args.steps + args.warmup)
+    n = int(max(1, min(w.B, 120.0 / total / per_sample)))
+    rng = np.random.default_rng(0)
+    samples = [np.sort(rng.choice(w.B, n, replace=False)) for _ in range(total)]
+    for i in range(args.warmup):
+        one(samples[i])
+    t0 = time.perf_counter()
+    for i in range(args.steps):
+        one(samples[args.warmup + i])
+    dt = time.perf_counter() - t0
+    value = w.T * n * sum(w.sizes[1:]) * args.steps / dt
+    line = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT,
+        "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": 1e3 * dt / args.steps, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": {"workload": w.name, "sizes": list(w.sizes), "T": w.T, "B": w.B,
+                   "sample_batch_per_step": n},
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": 1, "kind": "oracle",
+                         "sample": f"{n} random samples of {w.B} per step, all T={w.T} steps, "
+                                   f"float64 oracle forward+loss+BPTT (no optimiser)"},
+        "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+
+
 def run_reference(args):
     rank = int(os.environ.get("RANK", "0"))
     if rank != 0:
+        return
+    if is_dense(args):
+        run_dense_reference(args)
         return
     import numpy as np
     from paper_2211_10725_gb300 import workloads as W
@@ -406,6 +463,247 @@ def run_ours(args):
         dist.destroy_process_group()
 
 
+# ---------------------------------------------------------------------------
+# Dense SNN training step (784-1000-1000-10, T=25, B=128)
+# ---------------------------------------------------------------------------
+
+def tensor_peak(sustained):
+    key = "bf16_tflops_sustained" if sustained else "bf16_tflops"
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            return float(json.load(f)[key]), "measured"
+    except Exception:
+        return (1700.0 if sustained else 1900.0), "fallback"
+
+
+def dense_flops(w):
+    """Algorithmic GEMM flops of one training step (unpadded layer sizes):
+    forward I = X W^T per layer, dW per layer, dX for every layer but the
+    first."""
+    M = w.T * w.B
+    fwd = sum(2 * M * k * n for k, n in zip(w.sizes[:-1], w.sizes[1:]))
+    dx = sum(2 * M * k * n for k, n in zip(w.sizes[1:-1], w.sizes[2:]))
+    return fwd, fwd, dx
+
+
+def _timing_events(external):
+    import torch
+    if external:
+        return torch.cuda.Event(enable_timing=True, external=True)
+    return torch.cuda.Event(enable_timing=True)
+
+
+def run_dense(args):
+    import torch
+    import torch.distributed as dist
+
+    from paper_2211_10725_gb300 import workloads as W
+    from paper_2211_10725_gb300.dsnn import DenseSNN
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1:
+        dist.init_process_group("nccl")
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    w = W.DSNN_C3
+    save = args.save or "recompute"
+    inp = W.make_dense_inputs(w, seed=W.SEED_BASE + w.seed_index + 1000 * rank)
+    net = DenseSNN(w, inp["W"], device=dev, save=save)
+    X = inp["X"].reshape(w.T * w.B, -1).to(dev)
+    labels = inp["labels"].to(dev)
+    stream = torch.cuda.Stream(dev)
+    names = [n for n, _ in net.ops(X, labels)]
+
+    with torch.cuda.stream(stream):
+        for _ in range(args.warmup):
+            net.train_step(X, labels)
+    stream.synchronize()
+    for layer in net.layers:
+        if layer.status() != 0:
+            raise RuntimeError("kernel status after warm-up")
+
+    # one step as a CUDA graph, with a timing event between consecutive ops
+    graph, evs = None, None
+    if not args.no_graph:
+        try:
+            evs = [_timing_events(True) for _ in range(len(names) + 1)]
+            graph = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(graph, stream=stream):
+                evs[0].record()
+                for i, (_, call) in enumerate(net.ops(X, labels)):
+                    call()
+                    evs[i + 1].record()
+        except TypeError:
+            graph, evs = None, None   # no graph-capturable timing events in this torch
+    if graph is None:
+        evs = [_timing_events(False) for _ in range(len(names) + 1)]
+
+    def launch():
+        if graph is not None:
+            graph.replay()
+        else:
+            evs[0].record(stream)
+            for i, (_, call) in enumerate(net.ops(X, labels, stream)):
+                call()
+                evs[i + 1].record(stream)
+
+    with torch.cuda.stream(stream):
+        for _ in range(3):
+            launch()
+    stream.synchronize()
+
+    sampler = ClockSampler(local)
+    if rank == 0:
+        sampler.start()
+        time.sleep(0.3)
+    K = args.steps
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    per_op = [0.0] * len(names)
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize()
+    t_wall0 = time.time()
+    with torch.cuda.stream(stream):
+        e0.record(stream)
+        for _ in range(K):
+            launch()
+        e1.record(stream)
+    torch.cuda.synchronize()
+    t_wall1 = time.time()
+    # per-op durations of the last step of the timed region
+    per_op = [evs[i].elapsed_time(evs[i + 1]) for i in range(len(names))]
+    if world > 1:
+        dist.barrier()
+    if rank == 0:
+        time.sleep(0.2)
+        sampler.stop()
+    total_ms = e0.elapsed_time(e1)
+    if world > 1:
+        t = torch.tensor([total_ms], device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        total_ms = float(t.item())
+    for layer in net.layers:
+        if layer.status() != 0:
+            raise RuntimeError("kernel status in the timed region")
+    loss = float(net.loss.item())
+    if not (loss == loss):
+        raise RuntimeError("loss is NaN")
+
+    ns_per_step = w.T * w.B * sum(w.sizes[1:])
+    ms = total_ms / K
+    value = world * ns_per_step / (ms * 1e-3)
+    e2e = None if args.no_e2e else run_dense_e2e(args, w, inp, net, dev, world)
+    if rank != 0:
+        if world > 1:
+            dist.destroy_process_group()
+        return
+    fwd_f, dw_f, dx_f = dense_flops(w)
+    op_ms = dict(zip(names, per_op))
+    gemm_fwd_ms = sum(v for k, v in op_ms.items() if k.startswith("dense_fwd"))
+    peak, peak_kind = tensor_peak(sustained=True)
+    achieved = fwd_f / (gemm_fwd_ms * 1e-3) / 1e12
+    clocks = sampler.summary(t_wall0, t_wall1)
+    cpu = None
+    if not args.no_cpu_baseline and world == 1:
+        cpu = time_dense_oracle(w, inp, args.cpu_seconds)
+    # launches of our kernels per step: per forward GEMM 1, per forward scan
+    # 1, the loss 1, per scan BPTT 1, per dense backward 3 transposes + 2
+    # GEMMs (the first layer: 2 + 1), AdamW 1
+    nl = len(w.sizes) - 1
+    launches = nl + nl + 1 + nl + (5 * (nl - 1) + 3) + 1
+    line = {
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": K,
+        "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+        "config": {"workload": w.name, "sizes": list(w.sizes), "T": w.T, "B": w.B,
+                   "step": "forward GEMMs + Leaky scans, rate-coded CE loss, BPTT scans, "
+                           "dense backward (dX, dW), AdamW",
+                   "neuron_steps_per_step": ns_per_step, "save": save,
+                   "launch": "CUDA graph replay" if graph is not None else "eager",
+                   "l2": "working set (~70 MB) fits in L2; no flush between steps",
+                   "parallelism": f"replicas x{world}" if world > 1 else "single GPU"},
+        "images_per_s": world * w.B / (ms * 1e-3),
+        "roofline": {"bound": "tensor", "kernel": "gemm_tn_tcgen05 (forward GEMMs)",
+                     "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
+                     "frac": achieved / peak, "peak_kind": f"{peak_kind} sustained bf16",
+                     "traffic": None, "flops_per_step": {"fwd": fwd_f, "dW": dw_f, "dX": dx_f},
+                     "op_ms_last_step": op_ms,
+                     "timing": "timing events between the ops of the step, read after the "
+                               "last step of the timed region"},
+        "clocks": clocks,
+        "gpu_launches": launches * K,
+        "cpu_baseline": cpu,
+        "e2e": e2e,
+    }
+    print(json.dumps(line), flush=True)
+    if world > 1:
+        dist.destroy_process_group()
+
+
+def time_dense_oracle(w, inp, seconds):
+    """The oracle's forward + loss + BPTT of the dense SNN (float64 GEMMs,
+    float32 spike decisions) on the full batch, repeated for about `seconds`."""
+    import numpy as np
+    from oracle import snn_oracle as O
+    Ws = [x.float().numpy().astype(np.float64) for x in inp["W"]]
+    X = inp["X"].float().numpy().astype(np.float64).reshape(w.T * w.B, -1)
+    y = inp["labels"].numpy().astype(np.int64)
+    n, t_total = 0, 0.0
+    while t_total < seconds or n == 0:
+        t0 = time.perf_counter()
+        fwd = O.dsnn_forward(X, Ws, w.T, w.B, w.beta, w.thr)
+        O.dsnn_backward(fwd, Ws, y, w.T, w.B, w.beta, w.thr, w.sg_param)
+        t_total += time.perf_counter() - t0
+        n += 1
+    ns = w.T * w.B * sum(w.sizes[1:])
+    return {"value": ns * n / t_total, "unit": UNIT, "cores": 1, "kind": "oracle",
+            "sample": f"{n} full forward+loss+BPTT passes of the oracle (no optimiser), "
+                      f"{t_total:.1f} s, BLAS on one thread"}
+
+
+def run_dense_e2e(args, w, inp, net, dev, world):
+    """Training steps through the public API with the batch copied from
+    pinned host memory each step and the loss read back."""
+    import torch
+    import torch.distributed as dist
+    hX = inp["X"].reshape(w.T * w.B, -1).pin_memory()
+    hy = inp["labels"].pin_memory()
+    dX = torch.empty_like(hX, device=dev)
+    dy = torch.empty_like(hy, device=dev)
+    out = torch.empty(1, dtype=torch.float32).pin_memory()
+    stream = torch.cuda.current_stream(dev)
+
+    def step():
+        dX.copy_(hX, non_blocking=True)
+        dy.copy_(hy, non_blocking=True)
+        net.train_step(dX, dy)
+        out.copy_(net.loss, non_blocking=True)
+
+    K = max(3, min(args.steps, 200))
+    for _ in range(3):
+        step()
+    torch.cuda.synchronize()
+    if world > 1:
+        dist.barrier()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(K):
+        step()
+    e1.record(stream)
+    torch.cuda.synchronize()
+    ms = e0.elapsed_time(e1)
+    if world > 1:
+        t = torch.tensor([ms], device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms = float(t.item())
+    nb = lambda t: t.numel() * t.element_size()
+    return {"value": world * w.T * w.B * sum(w.sizes[1:]) * K / (ms * 1e-3), "unit": UNIT,
+            "h2d_bytes_per_step": nb(hX) + nb(hy), "d2h_bytes_per_step": nb(out), "steps": K,
+            "launch": "eager"}
+
+
 def run_e2e(args, w, inp, layer, dev, world):
     """Same metric through the public API, with the step's inputs copied from
     pinned host memory and its results read back to pinned host memory."""
@@ -461,6 +759,8 @@ def main():
     args = parse()
     if args.impl == "reference":
         run_reference(args)
+    elif is_dense(args):
+        run_dense(args)
     else:
         run_ours(args)
 

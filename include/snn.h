@@ -268,6 +268,29 @@ snn_status_t snn_rate_ce_loss(int64_t T, int64_t B, int64_t C, int64_t ld, int32
                               void* grad_spk, snn_stream_t stream);
 
 /*
+ * AdamW update of n fp32 master weights (the optimiser of the paper's
+ * training runs, Sec. V; decoupled weight decay):
+ *   m <- beta1 m + (1 - beta1) g ;  v <- beta2 v + (1 - beta2) g^2
+ *   w <- w (1 - lr weight_decay) - lr / (1 - beta1^step) * m / (sqrt(v / (1 - beta2^step)) + eps)
+ *   w, m, v  fp32 [n] (in/out, device);  grad fp32 [n] (in)
+ *   w_bf16   bf16 [n] (out, or NULL): the updated weights rounded to bf16
+ *            (round to nearest even) for the next forward GEMM
+ *   step     1 for the first update (used when step_counter is NULL)
+ *   step_counter  device int64 [2], or NULL: {updates done, 0}, zeroed by the
+ *            caller before the first update.  The launch then uses step =
+ *            step_counter[0] + 1 and advances step_counter[0] itself, so a
+ *            captured CUDA graph replays successive steps.  One counter per
+ *            parameter buffer; launches sharing a counter must not overlap.
+ * All pointers 16-byte aligned (SNN_ERR_ALIGNMENT); step < 1 without a
+ * counter, beta outside (0, 1) or eps <= 0 give SNN_ERR_INVALID_ARG.
+ * Asynchronous on stream.
+ */
+snn_status_t snn_adamw_step(int64_t n, float* w, void* w_bf16, const float* grad, float* m,
+                            float* v, float lr, float beta1, float beta2, float eps,
+                            float weight_decay, int64_t step, int64_t* step_counter,
+                            snn_stream_t stream);
+
+/*
  * Leaky BPTT that allocates nothing (no counterpart in the paper; it exists
  * for callers of this library that cannot allocate device memory: hosts
  * whose device memory is budgeted by another runtime, real-time loops that

@@ -459,3 +459,21 @@ def dsnn_backward(fwd, Ws, labels, T: int, B: int, beta: float, thr: float,
         res["dW"][l] = dW
         gs = keep(dX).reshape(T, B * Ws[l].shape[1])
     return res
+
+
+# ---------------------------------------------------------------------------
+# Optimiser of the training runs (Sec. V): AdamW
+# ---------------------------------------------------------------------------
+
+def adamw_step(w, g, m, v, lr, beta1, beta2, eps, weight_decay, step):
+    """One AdamW update (Adam with decoupled weight decay, Loshchilov and
+    Hutter): moment estimates, their bias corrections 1 - beta^step, and a
+    decay of w by lr * weight_decay applied beside the Adam step.  Float64.
+    Returns (w, m, v)."""
+    w, g, m, v = (np.asarray(a, dtype=np.float64) for a in (w, g, m, v))
+    m = beta1 * m + (1.0 - beta1) * g
+    v = beta2 * v + (1.0 - beta2) * g * g
+    m_hat = m / (1.0 - beta1 ** step)
+    v_hat = v / (1.0 - beta2 ** step)
+    w = w - lr * weight_decay * w - lr * m_hat / (np.sqrt(v_hat) + eps)
+    return w, m, v

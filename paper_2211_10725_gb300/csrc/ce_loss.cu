@@ -14,63 +14,98 @@
 namespace snn {
 namespace {
 
-constexpr int kCeThreads = 256;
+constexpr int kCeThreads = 1024;
+constexpr int kCeWarps = kCeThreads / 32;
 constexpr int kMaxClasses = 1024;
+constexpr int kCountSlots = 8192;  // shared-memory counts per chunk of samples
 
-// One block: thread b handles samples b, b + blockDim, ...; the loss is a
-// fixed-order fp64 block sum (deterministic).
+__device__ __forceinline__ float warp_max(float v) {
+  for (int o = 16; o > 0; o >>= 1) v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, o));
+  return v;
+}
+
+__device__ __forceinline__ float warp_sum(float v) {
+  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  return v;
+}
+
+// One block, samples in chunks of Bc = kCountSlots / C:
+//   1. every thread sums spk over t for (b, c) pairs of the chunk, t in a
+//      fixed order (8 independent loads in flight), into shared counts;
+//   2. warp w takes the chunk's samples w, w + 32, ...: softmax over the
+//      classes with lanes over c, the sample's loss added to the warp's sum
+//      in sample order, the gradient row written back over the counts;
+//   3. every thread writes gradients of (b, c) pairs for every t, so that
+//      the threads of a warp store a contiguous run of each row.
+// The softmax runs in float (double arithmetic is slow on this part); each
+// warp adds its samples' losses in double, and the 32 warp sums are added in
+// warp order: the loss is deterministic.
 template <typename T>
 __global__ void __launch_bounds__(kCeThreads) rate_ce_kernel(int64_t Tn, int64_t B, int64_t C,
                                                              int64_t ld, const T* spk,
                                                              const int* labels, float* loss,
                                                              T* grad) {
-  __shared__ double sh[kCeThreads];
+  __shared__ float cnt[kCountSlots];
+  __shared__ double warp_loss[kCeWarps];
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int64_t Bc = kCountSlots / C;
+  const float inv_b = 1.0f / (float)(B > 0 ? B : 1);
   double acc = 0.0;
-  for (int64_t b = threadIdx.x; b < B; b += blockDim.x) {
-    float cnt[32];
-    float m = -1e30f;
-    const int y = labels[b];
-    // classes in chunks of 32 registers: pass 1 max, pass 2 sum, pass 3 grads
-    for (int64_t c0 = 0; c0 < C; c0 += 32) {
-      for (int j = 0; j < 32 && c0 + j < C; ++j) {
-        float s = 0.0f;
-        for (int64_t t = 0; t < Tn; ++t) s += Elem<T>::load1(spk + (t * B + b) * ld + c0 + j);
-        m = fmaxf(m, s);
+  for (int64_t b0 = 0; b0 < B; b0 += Bc) {
+    const int64_t nb = min(Bc, B - b0);
+    for (int64_t e = threadIdx.x; e < nb * C; e += kCeThreads) {
+      const int64_t b = b0 + e / C, c = e % C;
+      const T* p = spk + b * ld + c;
+      const int64_t step = B * ld;
+      float s = 0.0f;
+      int64_t t = 0;
+      for (; t + 8 <= Tn; t += 8) {
+        float v[8];
+#pragma unroll
+        for (int k = 0; k < 8; ++k) v[k] = Elem<T>::load1(p + (t + k) * step);
+#pragma unroll
+        for (int k = 0; k < 8; ++k) s += v[k];
       }
+      for (; t < Tn; ++t) s += Elem<T>::load1(p + t * step);
+      cnt[e] = s;
     }
-    double sum = 0.0;
-    float cy = 0.0f;
-    for (int64_t c0 = 0; c0 < C; c0 += 32) {
-      for (int j = 0; j < 32 && c0 + j < C; ++j) {
-        float s = 0.0f;
-        for (int64_t t = 0; t < Tn; ++t) s += Elem<T>::load1(spk + (t * B + b) * ld + c0 + j);
-        cnt[j] = s;
-        sum += exp((double)(s - m));
-        if (c0 + j == y) cy = s;
+    __syncthreads();
+    for (int64_t j = warp; j < nb; j += kCeWarps) {
+      float* row = cnt + j * C;
+      const int y = labels[b0 + j];
+      float m = -1e30f;
+      for (int64_t c = lane; c < C; c += 32) m = fmaxf(m, row[c]);
+      m = warp_max(m);
+      float se = 0.0f, cy = 0.0f;
+      for (int64_t c = lane; c < C; c += 32) {
+        se += expf(row[c] - m);
+        if (c == y) cy = row[c];
       }
+      se = warp_sum(se);
+      cy = warp_sum(cy);
+      // loss = (m - count_y) + log(sum_c exp(count_c - m)); softmax_c =
+      // exp(count_c - m) / sum, both relative to the largest count
+      acc += (double)(m - cy) + (double)logf(se);
+      __syncwarp();
+      for (int64_t c = lane; c < C; c += 32)
+        row[c] = (expf(row[c] - m) / se - (c == y ? 1.0f : 0.0f)) * inv_b;
     }
-    const double lse = (double)m + log(sum);
-    acc += lse - (double)cy;
-    for (int64_t c0 = 0; c0 < C; c0 += 32) {
-      for (int j = 0; j < 32 && c0 + j < C; ++j) {
-        float s = 0.0f;
-        for (int64_t t = 0; t < Tn; ++t) s += Elem<T>::load1(spk + (t * B + b) * ld + c0 + j);
-        cnt[j] = s;
-        const double p = exp((double)s - lse);
-        const float gv = (float)((p - (c0 + j == y ? 1.0 : 0.0)) / (double)B);
-        for (int64_t t = 0; t < Tn; ++t) Elem<T>::store1(grad + (t * B + b) * ld + c0 + j, gv);
-      }
+    __syncthreads();
+    for (int64_t r = threadIdx.x; r < nb * ld; r += kCeThreads) {
+      const int64_t j = r / ld, c = r - j * ld;
+      const float g = c < C ? cnt[j * C + c] : 0.0f;
+      T* q = grad + b0 * ld + r;
+      for (int64_t t = 0; t < Tn; ++t) Elem<T>::store1(q + t * B * ld, g);
     }
-    for (int64_t c = C; c < ld; ++c)
-      for (int64_t t = 0; t < Tn; ++t) Elem<T>::store1(grad + (t * B + b) * ld + c, 0.0f);
-  }
-  sh[threadIdx.x] = acc;
-  __syncthreads();
-  for (int s = blockDim.x / 2; s > 0; s >>= 1) {
-    if ((int)threadIdx.x < s) sh[threadIdx.x] += sh[threadIdx.x + s];
     __syncthreads();
   }
-  if (threadIdx.x == 0) loss[0] = (float)(sh[0] / (double)(B > 0 ? B : 1));
+  if (lane == 0) warp_loss[warp] = acc;
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    double total = 0.0;
+    for (int w = 0; w < kCeWarps; ++w) total += warp_loss[w];
+    loss[0] = (float)(total / (double)(B > 0 ? B : 1));
+  }
 }
 
 }  // namespace

@@ -1,9 +1,11 @@
 """The paper's dense SNN (Tab. I "DSNN", here 784-1000-1000-10 Leaky layers)
 as one training step through the C ABI: per layer the input current of all
 T*B rows in one tensor-core GEMM (the synaptic operation of Fig. 3), then
-the fused Leaky scan; the rate-coded cross-entropy loss (Sec. V-A); and the
-BPTT reverse pass back through every scan and GEMM.  Only the sequencing of
-library calls lives here; every step runs in libsnn's kernels.
+the fused Leaky scan; the rate-coded cross-entropy loss (Sec. V-A); the
+BPTT reverse pass back through every scan and GEMM; and the AdamW update of
+the weights (fp32 master copy, bf16 copy for the GEMMs).  Only the
+sequencing of library calls lives here; every step runs in libsnn's
+kernels.
 
 Layer widths are padded to a multiple of 8 neurons (zero weight rows, so
 the 10-neuron output layer has 16) because the GEMM's TMA tiles need row
@@ -27,23 +29,41 @@ def _pad8(n: int) -> int:
 
 
 class DenseSNN:
-    """Buffers and calls of one DSNN training step (forward, loss, BPTT)."""
+    """Buffers and calls of one DSNN training step (forward, loss, BPTT,
+    AdamW update)."""
 
-    def __init__(self, w: W.DenseWorkload, weights, device="cuda", save: str = "recompute"):
+    def __init__(self, w: W.DenseWorkload, weights, device="cuda", save: str = "recompute",
+                 lr: float = 1e-3, betas=(0.9, 0.999), eps: float = 1e-8,
+                 weight_decay: float = 1e-2):
         self.w = w
         self.save = save
+        self.lr, self.betas, self.eps, self.weight_decay = lr, betas, eps, weight_decay
         self.device = torch.device(device)
         dev = self.device
         T, B = w.T, w.B
         self.M = T * B
         self.sizes = list(w.sizes)
         self.padded = [self.sizes[0]] + [_pad8(n) for n in self.sizes[1:]]
-        self.W = []
+        # all layers' weights in one flat buffer per quantity (bf16 copy for
+        # the GEMMs, fp32 master, AdamW moments, dW), so that one launch
+        # updates every layer; each layer's [N_pad, K_pad] block starts on a
+        # 64-element boundary
+        shapes = [(self.padded[l + 1], self.padded[l]) for l in range(len(weights))]
+        offs = [0]
+        for n_out, k_in in shapes:
+            offs.append(offs[-1] + n_out * k_in)
+        host = torch.zeros(offs[-1], dtype=torch.bfloat16)
         for l, Wl in enumerate(weights):
             n_out, k_in = Wl.shape
-            Wp = torch.zeros((self.padded[l + 1], self.padded[l]), dtype=torch.bfloat16)
-            Wp[:n_out, :k_in] = Wl
-            self.W.append(Wp.to(dev))
+            host[offs[l]:offs[l + 1]].view(shapes[l])[:n_out, :k_in] = Wl
+        self.W_flat = host.to(dev)
+        self.W32_flat = self.W_flat.float()
+        self.m_flat = torch.zeros_like(self.W32_flat)
+        self.v_flat = torch.zeros_like(self.W32_flat)
+        self.dW_flat = torch.zeros_like(self.W32_flat)
+        self.step_counter = torch.zeros(2, dtype=torch.int64, device=dev)
+        self.W = [self.W_flat[offs[l]:offs[l + 1]].view(shapes[l]) for l in range(len(shapes))]
+        self.dW = [self.dW_flat[offs[l]:offs[l + 1]].view(shapes[l]) for l in range(len(shapes))]
         self.layers, self.I = [], []
         for l in range(len(weights)):
             n = self.padded[l + 1]
@@ -64,8 +84,6 @@ class DenseSNN:
         self.grad_out = torch.empty((T, B, self.padded[-1]), dtype=torch.bfloat16, device=dev)
         self.grad_in = [torch.empty((self.M, self.padded[l]), dtype=torch.bfloat16, device=dev)
                         for l in range(1, len(weights))]
-        self.dW = [torch.empty((self.padded[l + 1], self.padded[l]), dtype=torch.float32,
-                               device=dev) for l in range(len(weights))]
 
     def layer_input(self, l, X):
         """[T*B, K] bf16 input of layer l: the data for l = 0, else the spikes
@@ -74,32 +92,59 @@ class DenseSNN:
 
     def forward(self, X, labels, stream=None):
         """X: bf16 [T*B, 784] spikes on the device; labels int32 [B]."""
-        for l, layer in enumerate(self.layers):
-            snn.snn_dense_layer_fwd(self.layer_input(l, X), self.W[l], self.I[l], self.ws_fwd,
-                                    stream)
-            layer.forward(self.I[l].view(self.w.T, self.w.B, -1), self.beta, self.thr,
-                          stream=stream)
-        snn.snn_rate_ce_loss(self.layers[-1].spk, labels, self.sizes[-1], self.loss,
-                             self.grad_out, stream)
+        for _, call in self.ops(X, labels, stream)[: 2 * len(self.layers) + 1]:
+            call()
         return self.loss
 
     def backward(self, X, stream=None):
-        grad = self.grad_out
-        for l in range(len(self.layers) - 1, -1, -1):
-            layer = self.layers[l]
-            layer.backward(self.I[l].view(self.w.T, self.w.B, -1), self.beta, self.thr, grad,
-                           want_param_grads=False, want_state_grads=False, stream=stream)
-            dX = self.grad_in[l - 1] if l > 0 else None
-            snn.snn_dense_layer_bwd(self.layer_input(l, X), self.W[l],
-                                    layer.grad_I.view(self.M, -1), dX, self.dW[l],
-                                    self.ws_bwd[l], stream)
-            if l > 0:
-                grad = dX.view(self.w.T, self.w.B, -1)
+        """BPTT from the loss gradient of the last forward; returns dW."""
+        for _, call in self.ops(X, None, stream)[2 * len(self.layers) + 1: -1]:
+            call()
         return self.dW
 
+    def update(self, stream=None):
+        """AdamW on every layer in one launch; rewrites the bf16 weights the
+        GEMMs read.  The step number lives on the device (graph-replayable)."""
+        snn.snn_adamw_step(self.W32_flat, self.W_flat, self.dW_flat, self.m_flat, self.v_flat,
+                           self.lr, self.betas[0], self.betas[1], self.eps, self.weight_decay,
+                           step_counter=self.step_counter, stream=stream)
+
+    def ops(self, X, labels, stream=None):
+        """The training step as a list of (name, call) in launch order: per
+        layer the forward GEMM and scan, the loss, per layer from the top the
+        scan BPTT and the dense backward, then the AdamW update."""
+        T, B = self.w.T, self.w.B
+        out = []
+        for l, layer in enumerate(self.layers):
+            out.append((f"dense_fwd{l}", lambda l=l: snn.snn_dense_layer_fwd(
+                self.layer_input(l, X), self.W[l], self.I[l], self.ws_fwd, stream)))
+            out.append((f"scan_fwd{l}", lambda l=l, layer=layer: layer.forward(
+                self.I[l].view(T, B, -1), self.beta, self.thr, stream=stream)))
+        out.append(("ce_loss", lambda: snn.snn_rate_ce_loss(
+            self.layers[-1].spk, labels, self.sizes[-1], self.loss, self.grad_out, stream)))
+        for l in range(len(self.layers) - 1, -1, -1):
+            grad = self.grad_out if l == len(self.layers) - 1 else \
+                self.grad_in[l].view(T, B, -1)
+            dX = self.grad_in[l - 1] if l > 0 else None
+            out.append((f"scan_bwd{l}", lambda l=l, grad=grad: self.layers[l].backward(
+                self.I[l].view(T, B, -1), self.beta, self.thr, grad, want_param_grads=False,
+                want_state_grads=False, stream=stream)))
+            out.append((f"dense_bwd{l}", lambda l=l, dX=dX: snn.snn_dense_layer_bwd(
+                self.layer_input(l, X), self.W[l], self.layers[l].grad_I.view(self.M, -1), dX,
+                self.dW[l], self.ws_bwd[l], stream)))
+        out.append(("adamw", lambda: self.update(stream)))
+        return out
+
     def step(self, X, labels, stream=None):
+        """Forward, loss and BPTT (weights unchanged); returns the dW list."""
         self.forward(X, labels, stream)
         return self.backward(X, stream)
+
+    def train_step(self, X, labels, stream=None):
+        """One full training step: forward, loss, BPTT and the AdamW update."""
+        for _, call in self.ops(X, labels, stream):
+            call()
+        return self.loss
 
     def weight_grads(self):
         """dW of each layer without the padding rows/columns."""

@@ -74,6 +74,8 @@ _SIGS = {
     "snn_dense_workspace_bytes": ([ctypes.c_int64] * 3, ctypes.c_size_t),
     "snn_dense_layer_bwd": ([ctypes.c_int64] * 3 + [_P] * 6 + [ctypes.c_size_t, _P], ctypes.c_int),
     "snn_rate_ce_loss": ([ctypes.c_int64] * 4 + [ctypes.c_int32] + [_P] * 4 + [_P], ctypes.c_int),
+    "snn_adamw_step": ([ctypes.c_int64] + [_P] * 5 + [ctypes.c_float] * 5 + [ctypes.c_int64] +
+                       [_P, _P], ctypes.c_int),
 }
 
 _lib: Optional[ctypes.CDLL] = None
@@ -242,6 +244,21 @@ def snn_rate_ce_loss(spk, labels, C, loss, grad_spk, stream=None):
     dt = {torch.float32: 0, torch.bfloat16: 1, torch.float16: 2}[spk.dtype]
     _check(load_library().snn_rate_ce_loss(T, B, C, ld, dt, _ptr(spk), _ptr(labels), _ptr(loss),
                                            _ptr(grad_spk), _stream(stream)), "snn_rate_ce_loss")
+
+
+def snn_adamw_step(w, w_bf16, grad, m, v, lr, beta1=0.9, beta2=0.999, eps=1e-8,
+                   weight_decay=1e-2, step=1, step_counter=None, stream=None):
+    """AdamW update in place of fp32 w, m, v from grad (same numel); writes
+    the bf16 copy of the new weights to w_bf16 unless it is None.  With a
+    device int64 [2] step_counter the step number is read from (and advanced
+    on) the device instead of taken from ``step``."""
+    n = w.numel()
+    for t in (grad, m, v) + ((w_bf16,) if w_bf16 is not None else ()):
+        if t.numel() != n:
+            raise ValueError("snn_adamw_step: tensors differ in size")
+    _check(load_library().snn_adamw_step(n, _ptr(w), _ptr(w_bf16), _ptr(grad), _ptr(m), _ptr(v),
+                                         lr, beta1, beta2, eps, weight_decay, step,
+                                         _ptr(step_counter), _stream(stream)), "snn_adamw_step")
 
 
 # ---------------------------------------------------------------------------

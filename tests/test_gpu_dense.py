@@ -68,10 +68,13 @@ def test_dense_argument_checks(cuda_device):
     assert lib.snn_dense_layer_bwd(8, 16, 10, 16, 16, 16, 16, 16, 16, 1 << 20, None) == 3
 
 
+# (T, B, C, ld): the 3-layer network's readout; more classes than a warp's
+# lanes with samples in several shared-memory chunks; the largest class count
+@pytest.mark.parametrize("T,B,C,ld", [(25, 128, 10, 16), (7, 300, 100, 104), (3, 20, 1024, 1032),
+                                      (1, 1, 1, 8)])
 @pytest.mark.parametrize("dtype", [torch.float32, torch.bfloat16])
-def test_rate_ce_loss(dtype, cuda_device):
-    T, B, C, ld = 25, 128, 10, 16
-    g = torch.Generator().manual_seed(3)
+def test_rate_ce_loss(T, B, C, ld, dtype, cuda_device):
+    g = torch.Generator().manual_seed(3 + B)
     spk = (torch.rand((T, B, ld), generator=g) < 0.3).to(dtype)
     labels = torch.randint(0, C, (B,), generator=g, dtype=torch.int32)
     loss = torch.zeros(1, dtype=torch.float32, device=cuda_device)

@@ -452,3 +452,24 @@ def test_dsnn_matches_torch_autograd(k):
     for l, w in enumerate(tW):
         assert np.abs(w.grad.numpy()).max() > 1e-4      # a gradient reaches every layer
         np.testing.assert_allclose(res["dW"][l], w.grad.numpy(), rtol=1e-10, atol=1e-14)
+
+
+def test_adamw_matches_torch_optim():
+    """Three AdamW steps of the oracle against torch.optim.AdamW (the library
+    routine) on float64 parameters."""
+    rng = np.random.default_rng(14)
+    n = 257
+    w0 = rng.normal(0, 1, n)
+    grads = [rng.normal(0, 1, n) * s for s in (1.0, 1e-3, 10.0)]
+    lr, b1, b2, eps, wd = 1e-2, 0.9, 0.999, 1e-8, 0.05
+    p = torch.tensor(w0, requires_grad=True)
+    opt = torch.optim.AdamW([p], lr=lr, betas=(b1, b2), eps=eps, weight_decay=wd)
+    w, m, v = w0.copy(), np.zeros(n), np.zeros(n)
+    for k, g in enumerate(grads, start=1):
+        p.grad = torch.tensor(g)
+        opt.step()
+        w, m, v = O.adamw_step(w, g, m, v, lr, b1, b2, eps, wd, k)
+        np.testing.assert_allclose(w, p.detach().numpy(), rtol=1e-12, atol=1e-14)
+    st = opt.state[p]
+    np.testing.assert_allclose(m, st["exp_avg"].numpy(), rtol=1e-12)
+    np.testing.assert_allclose(v, st["exp_avg_sq"].numpy(), rtol=1e-12)
