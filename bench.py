@@ -75,17 +75,18 @@ def algorithmic_bytes(w):
     """Bytes per neuron-step the contract must touch (fwd, bwd).
 
     Forward: read I, write spk (+ mem if requested).  Backward: read
-    grad_spk, read the cheaper saved state (I for recompute, mem (+spk for
-    half storage) for store), write grad_I.  Checkpoints, parameters and
-    reductions are excluded (they are overhead, not contract)."""
+    grad_spk, read the cheaper saved state (I for recompute; mem for store,
+    plus for half storage the spike bits the forward wrote, 1/8 byte),
+    write grad_I.  Checkpoints, parameters and reductions are excluded (they
+    are overhead, not contract)."""
     ei, eo = esize(w.in_dtype), esize(w.io_dtype)
     fwd = ei + eo + (eo if (w.want_mem or w.save == "mem") else 0)
-    if w.neuron == "synaptic" and w.save == "mem":
-        fwd += 0
     if w.save == "recompute":
         bwd = eo + ei + eo
     else:
-        bwd = eo + eo + eo + (eo if eo != 4 else 0)
+        bits = 0.125 if eo != 4 else 0.0
+        fwd += bits
+        bwd = eo + eo + eo + bits
     return fwd, bwd
 
 

@@ -123,9 +123,17 @@ size_t snn_scan_desc_size(void);
  * plus per-lane parameter-gradient partials).  0 if desc is invalid. */
 size_t snn_scan_workspace_bytes(const snn_scan_desc* desc);
 
-/* Number of fp32 elements of the checkpoint buffer for SNN_SAVE_RECOMPUTE:
- * (ceil(T/K) - 1) * B*N for Leaky, twice that for Synaptic (u then i per
- * checkpoint).  0 for SNN_SAVE_MEM or an invalid desc. */
+/* Number of fp32 elements of the ckpt buffer passed to the forward and the
+ * backward of one sequence:
+ *   SNN_SAVE_RECOMPUTE: (ceil(T/K) - 1) * B*N for Leaky, twice that for
+ *     Synaptic (u then i per checkpoint);
+ *   SNN_SAVE_MEM with a bf16/fp16 io_dtype: T rows of ceil(B*N/8) bytes
+ *     rounded up to 16, in fp32 units: the spike bits (bit k of byte j of
+ *     row t is z_t of lane 8j + k).  Optional: given to both calls, the
+ *     backward reads 1 bit per neuron-step instead of the 16-bit spk row
+ *     (used when B*N is a multiple of 8; otherwise spk is read);
+ *   SNN_SAVE_MEM with fp32 io: 0.
+ * 0 for an invalid desc. */
 int64_t snn_scan_ckpt_elems(const snn_scan_desc* desc, int synaptic);
 
 /* Zero a workspace (its status word included); asynchronous on stream.
@@ -146,10 +154,11 @@ snn_status_t snn_workspace_status(void* ws, snn_stream_t stream);
  *   mem      [T,B,N] io_dtype  (out)     u_t; required for SNN_SAVE_MEM, else
  *                                        optional (NULL = not written)
  *   ckpt     fp32 (out)                  SNN_SAVE_RECOMPUTE: u at the end of every
- *                                        segment but the last; else NULL.  Segments
- *                                        are aligned to the end of the sequence:
- *                                        the first has T-(ceil(T/K)-1)*K steps, the
- *                                        others K.
+ *                                        segment but the last.  Segments are aligned
+ *                                        to the end of the sequence: the first has
+ *                                        T-(ceil(T/K)-1)*K steps, the others K.
+ *                                        SNN_SAVE_MEM, half io: the spike bits, or
+ *                                        NULL (see snn_scan_ckpt_elems).
  *   mem_final fp32 [B,N] (out) or NULL   u_{T-1}
  *   ws       workspace of snn_scan_workspace_bytes(desc) bytes
  * State is kept in fp32; the step is evaluated as Eq. (4) is written:
@@ -165,7 +174,9 @@ snn_status_t snn_leaky_fwd(const snn_scan_desc* desc, const void* I, const float
  * Inputs of the saved forward:
  *   SNN_SAVE_MEM:       mem [T,B,N] io_dtype; spk [T,B,N] io_dtype, needed
  *                       when io_dtype is not fp32 (a rounded mem cannot give
- *                       back the spike decision), may be NULL for fp32.
+ *                       back the spike decision) unless the forward wrote the
+ *                       spike bits to ckpt and B*N is a multiple of 8; may be
+ *                       NULL for fp32.  ckpt: the forward's spike bits or NULL.
  *   SNN_SAVE_RECOMPUTE: I [T,B,N] in_dtype and ckpt from snn_leaky_fwd.
  *   beta, thr, mem0 as in the forward.
  * Upstream gradients:

@@ -54,6 +54,10 @@ struct ScanArgs {
   void* mem;
   void* syn;
   float* ckpt;  // forward: written; backward: read
+  // store mode, half io: spike bits (bit k of byte j of row t = z_t of lane
+  // 8j + k), rows of bits_row bytes; forward: written; backward: read
+  unsigned char* bits;
+  int64_t bits_row;
   float* mem_final;
   float* syn_final;
   // backward
@@ -515,6 +519,9 @@ __global__ void __launch_bounds__(kMaxStagedThreads) scan_fwd_staged(const ScanA
   TO* syn = (SYN && a.syn) ? static_cast<TO*>(a.syn) + l : nullptr;
   float* ck = a.ckpt ? a.ckpt + l : nullptr;
   const int64_t ck_stride = SYN ? 2 * a.L : a.L;
+  // spike bits: one byte per thread and step (Leaky, 8 lanes), or one per
+  // pair of threads (Synaptic, 4 lanes each: the even thread stores)
+  unsigned char* bits = a.bits ? a.bits + lane0 / 8 + (SYN ? c / 2 : c) : nullptr;
   const TI* my = reinterpret_cast<const TI*>(ring) + c * V;
   const int stage_elems = a.stage_bytes / (int)sizeof(TI);
   RingPos pos;
@@ -524,6 +531,7 @@ __global__ void __launch_bounds__(kMaxStagedThreads) scan_fwd_staged(const ScanA
       if (lid == 0) record_status(a.status, kStatusTimeout);
       break;
     }
+    unsigned zbits = 0;
     if (active) {
       float2 x[NP];
       load_pairs<TI, NP>(my + pos.s * stage_elems, x);
@@ -533,6 +541,8 @@ __global__ void __launch_bounds__(kMaxStagedThreads) scan_fwd_staged(const ScanA
         fwd_pair<SYN, RESET>(a.reset, beta[k], negthr[k], alpha[k], x[k], u[k], &z[2 * k], in[k]);
         zf[k] = make_float2(z[2 * k] ? 1.0f : 0.0f, z[2 * k + 1] ? 1.0f : 0.0f);
       }
+#pragma unroll
+      for (int k = 0; k < V; ++k) zbits |= (z[k] ? 1u : 0u) << k;
       store_pairs<TO, NP>(spk, zf);
       if (mem) store_pairs<TO, NP>(mem, u);
       if (SYN && syn) store_pairs<TO, NP>(syn, in);
@@ -544,6 +554,15 @@ __global__ void __launch_bounds__(kMaxStagedThreads) scan_fwd_staged(const ScanA
           ck += ck_stride;
         }
       }
+    }
+    if (bits) {
+      if (SYN) {
+        const unsigned hi = __shfl_down_sync(0xffffffffu, zbits, 1);
+        if (active && !(c & 1)) *bits = (unsigned char)(zbits | (hi << 4));
+      } else if (active) {
+        *bits = (unsigned char)zbits;
+      }
+      bits += a.bits_row;
     }
     release_stage(empty, pos.s, lid);
     pos.next(S);
@@ -596,6 +615,10 @@ __global__ void __launch_bounds__(kMaxStagedThreads) scan_bwd_staged(const ScanA
   const int cta_lanes = (int)min((int64_t)a.lanes_per_cta, a.L - lane0);
   const int io_stride = a.lanes_per_cta * (int)sizeof(TO);  // byte stride of io tiles
   const bool half_store = !RECOMP && sizeof(TO) != 4;      // z from the spk rows
+  const bool use_bits = half_store && a.bits != nullptr;    // ... or from the bit rows
+  // the bit row of the strip starts at byte lane0/8, copied from the 16-byte
+  // boundary below it: the consumer skips bits_skew bytes
+  const int bits_skew = (int)((lane0 / 8) & 15);
   const bool want_syn = SYN && a.part_alpha != nullptr;
   // store-mode tile order: gs, mem, [spk], [syn], [gm]
   const int t_spk = 2, t_syn = 2 + (half_store ? 1 : 0);
@@ -622,7 +645,13 @@ __global__ void __launch_bounds__(kMaxStagedThreads) scan_bwd_staged(const ScanA
           int n = 0;
           tiles[n] = Tile{row<TO>(a.gs, t, a.L, lane0), bo, (uint32_t)(n * io_stride)}; ++n;
           tiles[n] = Tile{row<TO>(a.mem_in, t, a.L, lane0), bo, (uint32_t)(n * io_stride)}; ++n;
-          if (half_store) { tiles[n] = Tile{row<TO>(a.spk_in, t, a.L, lane0), bo, (uint32_t)(n * io_stride)}; ++n; }
+          if (use_bits) {
+            const unsigned char* src = a.bits + t * a.bits_row + lane0 / 8 - bits_skew;
+            const uint32_t nb = (uint32_t)(bits_skew + cta_lanes / 8 + 15) & ~15u;
+            tiles[n] = Tile{src, nb, (uint32_t)(n * io_stride)}; ++n;
+          } else if (half_store) {
+            tiles[n] = Tile{row<TO>(a.spk_in, t, a.L, lane0), bo, (uint32_t)(n * io_stride)}; ++n;
+          }
           if (want_syn) { tiles[n] = Tile{row<TO>(a.syn_in, t, a.L, lane0), bo, (uint32_t)(n * io_stride)}; ++n; }
           if (a.gm) { tiles[n] = Tile{row<TO>(a.gm, t, a.L, lane0), bo, (uint32_t)(n * io_stride)}; ++n; }
           p.issue(tiles, n, a);
@@ -728,7 +757,13 @@ __global__ void __launch_bounds__(kMaxStagedThreads) scan_bwd_staged(const ScanA
         bool zz[V];
         load_pairs<TO, NP>(base, g);
         load_pairs<TO, NP>(base + tile_io_elems, uu);
-        if (half_store) {
+        if (use_bits) {
+          const unsigned char* bb = reinterpret_cast<const unsigned char*>(base - c * V) +
+                                    t_spk * io_stride + bits_skew + (SYN ? c / 2 : c);
+          const unsigned zb = SYN ? (unsigned)(*bb >> ((c & 1) * 4)) : (unsigned)*bb;
+#pragma unroll
+          for (int k = 0; k < V; ++k) zz[k] = (zb >> k) & 1u;
+        } else if (half_store) {
           float2 sp[NP];
           load_pairs<TO, NP>(base + t_spk * tile_io_elems, sp);
 #pragma unroll

@@ -98,6 +98,10 @@ snn_status_t check_ws(const snn_scan_desc* d, const void* ws, size_t ws_bytes) {
 
 // Rows of every streamed tensor must be 16-byte multiples for the TMA path,
 // and lanes come in groups of VEC per thread.
+// Bytes per time step of the spike-bit rows (store mode, half io): one bit
+// per lane, rows padded to 16 bytes.
+int64_t spike_bits_row(const snn_scan_desc* d) { return round_up(ceil_div(d->B * d->N, 8), 16); }
+
 bool staged_ok(const snn_scan_desc* d) {
   if (d->debug_flags & 2u) return false;  // SNN_DEBUG_FORCE_PLAIN
   const int64_t L = d->B * d->N;
@@ -172,9 +176,14 @@ snn_status_t scan_fwd(const snn_scan_desc* d, bool syn, const void* I, const flo
   a.mem = mem;
   a.syn = syn ? synout : nullptr;
   a.ckpt = recompute ? ckpt : nullptr;
+  const bool staged = staged_ok(d);
+  if (!recompute && d->io_dtype != SNN_F32 && ckpt && staged) {
+    a.bits = reinterpret_cast<unsigned char*>(ckpt);
+    a.bits_row = spike_bits_row(d);
+  }
   a.mem_final = mem_final;
   a.syn_final = syn ? syn_final : nullptr;
-  return cuda_status(launch_scan_fwd(a, syn, d->in_dtype, d->io_dtype, staged_ok(d), stream));
+  return cuda_status(launch_scan_fwd(a, syn, d->in_dtype, d->io_dtype, staged, stream));
 }
 
 snn_status_t scan_bwd(const snn_scan_desc* d, bool syn, const void* I, const float* ckpt,
@@ -194,7 +203,9 @@ snn_status_t scan_bwd(const snn_scan_desc* d, bool syn, const void* I, const flo
   if (recompute && snn_scan_ckpt_elems(d, syn) > 0 && !ckpt) return SNN_ERR_INVALID_ARG;
   if (n > 0 && !recompute) {
     if (!mem) return SNN_ERR_INVALID_ARG;
-    if (d->io_dtype != SNN_F32 && !spk) return SNN_ERR_INVALID_ARG;
+    // a rounded mem cannot give back the spike: spk rows, or the bit rows
+    // (which only the staged kernels read)
+    if (d->io_dtype != SNN_F32 && !spk && !(ckpt && staged_ok(d))) return SNN_ERR_INVALID_ARG;
     if (syn && grad_alpha && !synin) return SNN_ERR_INVALID_ARG;
   }
   if ((s = check_ptrs({I, ckpt, mem, spk, synin, alpha, beta, thr, mem0, syn0, grad_spk, grad_mem,
@@ -224,6 +235,10 @@ snn_status_t scan_bwd(const snn_scan_desc* d, bool syn, const void* I, const flo
   a.ckpt = recompute ? const_cast<float*>(ckpt) : nullptr;
   a.mem_in = recompute ? nullptr : mem;
   a.spk_in = (!recompute && d->io_dtype != SNN_F32) ? spk : nullptr;
+  if (!recompute && d->io_dtype != SNN_F32 && ckpt && staged_ok(d)) {
+    a.bits = reinterpret_cast<unsigned char*>(const_cast<float*>(ckpt));
+    a.bits_row = spike_bits_row(d);
+  }
   a.syn_in = (syn && !recompute && grad_alpha) ? synin : nullptr;
   a.gs = grad_spk;
   a.gm = grad_mem;
@@ -279,7 +294,11 @@ size_t snn_scan_workspace_bytes(const snn_scan_desc* desc) {
 }
 
 int64_t snn_scan_ckpt_elems(const snn_scan_desc* desc, int synaptic) {
-  if (check_desc(desc) != SNN_OK || desc->save != SNN_SAVE_RECOMPUTE) return 0;
+  if (check_desc(desc) != SNN_OK) return 0;
+  if (desc->save != SNN_SAVE_RECOMPUTE) {
+    if (desc->io_dtype == SNN_F32) return 0;
+    return desc->T * spike_bits_row(desc) / 4;  // spike bits, in fp32 units
+  }
   const int64_t nseg = ceil_div(desc->T, desc->ckpt_every);
   const int64_t n = nseg > 1 ? (nseg - 1) * desc->B * desc->N : 0;
   return synaptic ? 2 * n : n;

@@ -58,11 +58,66 @@ def test_staged_and_plain_kernels_agree(i, cuda_device):
     b = H.run_gpu(w, inp, debug_flags=snn.DEBUG_FORCE_PLAIN)
     assert torch.equal(a.spk, b.spk) and torch.equal(a.mem, b.mem)
     assert torch.equal(a.mem_final, b.mem_final)
-    if a.ckpt is not None:
+    if w.save == "recompute" and a.ckpt is not None:
         assert torch.equal(a.ckpt, b.ckpt)
     # the reverse passes accumulate in different orders (packed FMAs vs
     # scalar): they agree within the fp32 gradient tolerance
     H.assert_close("grad_I", H.lanes_2d(a.grad_I), H.lanes_2d(b.grad_I), *H.TOL[w.io_dtype])
+
+
+def _unpack_bits(ckpt, T, L):
+    """Spike bits (bit k of byte j of row t = lane 8j + k; rows padded to 16
+    bytes) as a [T, L] 0/1 array."""
+    row = ((L + 7) // 8 + 15) // 16 * 16
+    raw = ckpt.cpu().view(torch.uint8).numpy()[: T * row].reshape(T, row)[:, : (L + 7) // 8]
+    return np.unpackbits(raw, axis=1, bitorder="little")[:, :L].astype(np.float64)
+
+
+@pytest.mark.parametrize("neuron", ["leaky", "synaptic"])
+@pytest.mark.parametrize("io", [W.BF16, W.F16])
+@pytest.mark.parametrize("T,B,N", [(9, 3, 1368), (4, 7, 1000), (3, 1, 8)])
+def test_store_mode_spike_bits(neuron, io, T, B, N, cuda_device):
+    """Store mode with half io: the forward's spike bits equal spk, and the
+    backward from the bits (spk not passed) equals the backward from spk."""
+    w = W.ScanWorkload(name="bits", neuron=neuron, T=T, B=B, N=N, in_dtype=io, io_dtype=io,
+                       save="mem", surrogate="atan", sg_param=2.0, reset="zero",
+                       beta=("uniform", 0.5, 0.95), thr=("uniform", 0.6, 1.4), i_mean=0.5,
+                       beta_mode="per_neuron", seed_index=7)
+    inp = W.make_scan_inputs(w)
+    d = {k: v.to(cuda_device) for k, v in inp.items()}
+    layer = snn.ScanLayer(w, device=cuda_device, want_syn=True)
+    assert layer.ckpt is not None      # the bit rows
+    layer.forward(d["I"], d["beta"], d["thr"], d.get("alpha"))
+    torch.cuda.synchronize()
+    bits = _unpack_bits(layer.ckpt, T, B * N)
+    assert np.array_equal(bits, H.lanes_2d(layer.spk))
+    spk = layer.spk
+    layer.spk = None                   # the backward must not need it
+    try:
+        layer.backward(d["I"], d["beta"], d["thr"], d["grad_spk"], alpha=d.get("alpha"))
+    finally:
+        layer.spk = spk
+    g_bits = layer.grad_I.clone()
+    gb_bits = layer.grad_beta.clone()
+    ckpt = layer.ckpt
+    layer.ckpt = None                  # now from the spk rows
+    layer.backward(d["I"], d["beta"], d["thr"], d["grad_spk"], alpha=d.get("alpha"))
+    layer.ckpt = ckpt
+    torch.cuda.synchronize()
+    assert layer.status() == 0
+    assert torch.equal(g_bits, layer.grad_I)
+    assert torch.equal(gb_bits, layer.grad_beta)
+    H.check_all(w, inp, layer, H.oracle_expect(w, inp))
+
+
+def test_store_mode_without_spk_or_bits_is_rejected(cuda_device):
+    w = W.LEAKY_C1.scaled(io_dtype=W.BF16, in_dtype=W.BF16, T=3, B=2, N=16)
+    layer = snn.ScanLayer(w, device=cuda_device)
+    inp = {k: v.to(cuda_device) for k, v in W.make_scan_inputs(w).items()}
+    layer.forward(inp["I"], inp["beta"], inp["thr"])
+    layer.spk, layer.ckpt = None, None
+    with pytest.raises(snn.SnnError):
+        layer.backward(inp["I"], inp["beta"], inp["thr"], inp["grad_spk"])
 
 
 def test_backward_is_deterministic(cuda_device):
