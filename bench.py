@@ -515,11 +515,26 @@ def run_dense(args):
     X = inp["X"].reshape(w.T * w.B, -1).to(dev)
     labels = inp["labels"].to(dev)
     stream = torch.cuda.Stream(dev)
-    names = [n for n, _ in net.ops(X, labels)]
+    if world > 1:
+        # data parallel: this rank's 128 samples are its shard of a global
+        # batch of world * 128; dW and the loss are summed over the ranks
+        # (NCCL) before the AdamW update
+        from paper_2211_10725_gb300.data_parallel import allreduce_sum_
+        net.batch_total = world * w.B
+
+    def step_ops(st=None):
+        ops = net.ops(X, labels, st)
+        if world > 1:
+            ops.insert(len(ops) - 1, ("allreduce_dW", lambda: allreduce_sum_([net.dW_flat,
+                                                                             net.loss])))
+        return ops
+
+    names = [n for n, _ in step_ops()]
 
     with torch.cuda.stream(stream):
         for _ in range(args.warmup):
-            net.train_step(X, labels)
+            for _, call in step_ops():
+                call()
     stream.synchronize()
     for layer in net.layers:
         if layer.status() != 0:
@@ -527,13 +542,13 @@ def run_dense(args):
 
     # one step as a CUDA graph, with a timing event between consecutive ops
     graph, evs = None, None
-    if not args.no_graph:
+    if not args.no_graph and world == 1:
         try:
             evs = [_timing_events(True) for _ in range(len(names) + 1)]
             graph = torch.cuda.CUDAGraph()
             with torch.cuda.graph(graph, stream=stream):
                 evs[0].record()
-                for i, (_, call) in enumerate(net.ops(X, labels)):
+                for i, (_, call) in enumerate(step_ops()):
                     call()
                     evs[i + 1].record()
         except TypeError:
@@ -546,7 +561,7 @@ def run_dense(args):
             graph.replay()
         else:
             evs[0].record(stream)
-            for i, (_, call) in enumerate(net.ops(X, labels, stream)):
+            for i, (_, call) in enumerate(step_ops(stream)):
                 call()
                 evs[i + 1].record(stream)
 
@@ -624,7 +639,8 @@ def run_dense(args):
                    "neuron_steps_per_step": ns_per_step, "save": save,
                    "launch": "CUDA graph replay" if graph is not None else "eager",
                    "l2": "working set (~70 MB) fits in L2; no flush between steps",
-                   "parallelism": f"replicas x{world}" if world > 1 else "single GPU"},
+                   "parallelism": (f"data parallel x{world} (global batch {world * w.B}, "
+                                   "dW all-reduced over NCCL)") if world > 1 else "single GPU"},
         "images_per_s": world * w.B / (ms * 1e-3),
         "roofline": {"bound": "tensor", "kernel": "gemm_tn_tcgen05 (forward GEMMs)",
                      "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
@@ -676,10 +692,16 @@ def run_dense_e2e(args, w, inp, net, dev, world):
     out = torch.empty(1, dtype=torch.float32).pin_memory()
     stream = torch.cuda.current_stream(dev)
 
+    if world > 1:
+        from paper_2211_10725_gb300.data_parallel import DataParallelDenseSNN
+        train = DataParallelDenseSNN(net, world * w.B).train_step
+    else:
+        train = net.train_step
+
     def step():
         dX.copy_(hX, non_blocking=True)
         dy.copy_(hy, non_blocking=True)
-        net.train_step(dX, dy)
+        train(dX, dy)
         out.copy_(net.loss, non_blocking=True)
 
     K = max(3, min(args.steps, 200))

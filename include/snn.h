@@ -270,12 +270,17 @@ snn_status_t snn_dense_layer_bwd(int64_t M, int64_t K, int64_t N, const void* X,
  * neuron that fires most): cross-entropy of the spike counts over T.
  *   spk   [T, B, ld] in `dtype` (snn_dtype_t); the first C of ld neurons are
  *         the classes (C <= 1024)
- *   labels int32 [B];  loss fp32 [1] (out) = mean_b CE(sum_t spk[:, b, :C], y_b)
- *   grad_spk [T, B, ld] (out) = (softmax - onehot) / B for every t; 0 for
- *         neurons C..ld-1
+ *   labels int32 [B]
+ *   batch_total  the batch the mean is taken over: 0 for B; the global batch
+ *         (>= B) when these B samples are one data-parallel shard, so that
+ *         the shards' losses and gradients add up to the global ones
+ *   loss  fp32 [1] (out) = sum_b CE(sum_t spk[:, b, :C], y_b) / batch_total
+ *   grad_spk [T, B, ld] (out) = (softmax - onehot) / batch_total for every
+ *         t; 0 for neurons C..ld-1
+ * Deterministic (fixed summation order).
  */
-snn_status_t snn_rate_ce_loss(int64_t T, int64_t B, int64_t C, int64_t ld, int32_t dtype,
-                              const void* spk, const int32_t* labels, float* loss,
+snn_status_t snn_rate_ce_loss(int64_t T, int64_t B, int64_t C, int64_t ld, int64_t batch_total,
+                              int32_t dtype, const void* spk, const int32_t* labels, float* loss,
                               void* grad_spk, snn_stream_t stream);
 
 /*

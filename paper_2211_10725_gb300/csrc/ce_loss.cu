@@ -2,8 +2,11 @@
 // neuron with the most spikes): cross-entropy on the spike counts over T,
 // and its gradient with respect to every output spike.
 //   counts[b, c] = sum_t spk[t, b, c]
-//   loss = mean_b ( logsumexp_c counts[b, :] - counts[b, y_b] )
-//   dL/dspk[t, b, c] = (softmax(counts[b, :])_c - [c == y_b]) / B   (same for all t)
+//   loss = sum_b ( logsumexp_c counts[b, :] - counts[b, y_b] ) / B_norm
+//   dL/dspk[t, b, c] = (softmax(counts[b, :])_c - [c == y_b]) / B_norm   (same for all t)
+// B_norm is the batch the mean is taken over: B, or the global batch when
+// B samples are one data-parallel shard (the shards' results then add up to
+// the global loss and gradient).
 #include <cuda_bf16.h>
 #include <cuda_fp16.h>
 #include <cuda_runtime.h>
@@ -42,14 +45,14 @@ __device__ __forceinline__ float warp_sum(float v) {
 // warp order: the loss is deterministic.
 template <typename T>
 __global__ void __launch_bounds__(kCeThreads) rate_ce_kernel(int64_t Tn, int64_t B, int64_t C,
-                                                             int64_t ld, const T* spk,
+                                                             int64_t ld, int64_t Bn, const T* spk,
                                                              const int* labels, float* loss,
                                                              T* grad) {
   __shared__ float cnt[kCountSlots];
   __shared__ double warp_loss[kCeWarps];
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const int64_t Bc = kCountSlots / C;
-  const float inv_b = 1.0f / (float)(B > 0 ? B : 1);
+  const float inv_b = 1.0f / (float)Bn;
   double acc = 0.0;
   for (int64_t b0 = 0; b0 < B; b0 += Bc) {
     const int64_t nb = min(Bc, B - b0);
@@ -104,32 +107,35 @@ __global__ void __launch_bounds__(kCeThreads) rate_ce_kernel(int64_t Tn, int64_t
   if (threadIdx.x == 0) {
     double total = 0.0;
     for (int w = 0; w < kCeWarps; ++w) total += warp_loss[w];
-    loss[0] = (float)(total / (double)(B > 0 ? B : 1));
+    loss[0] = (float)(total / (double)Bn);
   }
 }
 
 }  // namespace
 }  // namespace snn
 
-extern "C" snn_status_t snn_rate_ce_loss(int64_t T, int64_t B, int64_t C, int64_t ld, int32_t dtype,
-                                         const void* spk, const int32_t* labels, float* loss,
-                                         void* grad_spk, snn_stream_t stream) {
+extern "C" snn_status_t snn_rate_ce_loss(int64_t T, int64_t B, int64_t C, int64_t ld,
+                                         int64_t batch_total, int32_t dtype, const void* spk,
+                                         const int32_t* labels, float* loss, void* grad_spk,
+                                         snn_stream_t stream) {
   if (T < 0 || B < 0 || C < 1 || ld < C || C > snn::kMaxClasses) return SNN_ERR_INVALID_ARG;
+  const int64_t Bn = batch_total > 0 ? batch_total : (B > 0 ? B : 1);
+  if (batch_total > 0 && batch_total < B) return SNN_ERR_INVALID_ARG;
   if (!loss || (T > 0 && B > 0 && (!spk || !labels || !grad_spk))) return SNN_ERR_INVALID_ARG;
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
   switch (dtype) {
     case SNN_F32:
       snn::rate_ce_kernel<float><<<1, snn::kCeThreads, 0, st>>>(
-          T, B, C, ld, static_cast<const float*>(spk), labels, loss, static_cast<float*>(grad_spk));
+          T, B, C, ld, Bn, static_cast<const float*>(spk), labels, loss, static_cast<float*>(grad_spk));
       break;
     case SNN_BF16:
       snn::rate_ce_kernel<__nv_bfloat16><<<1, snn::kCeThreads, 0, st>>>(
-          T, B, C, ld, static_cast<const __nv_bfloat16*>(spk), labels, loss,
+          T, B, C, ld, Bn, static_cast<const __nv_bfloat16*>(spk), labels, loss,
           static_cast<__nv_bfloat16*>(grad_spk));
       break;
     case SNN_F16:
       snn::rate_ce_kernel<__half><<<1, snn::kCeThreads, 0, st>>>(
-          T, B, C, ld, static_cast<const __half*>(spk), labels, loss, static_cast<__half*>(grad_spk));
+          T, B, C, ld, Bn, static_cast<const __half*>(spk), labels, loss, static_cast<__half*>(grad_spk));
       break;
     default:
       return SNN_ERR_INVALID_ARG;

@@ -38,6 +38,9 @@ class DenseSNN:
         self.w = w
         self.save = save
         self.lr, self.betas, self.eps, self.weight_decay = lr, betas, eps, weight_decay
+        # batch the loss is averaged over (the global batch under data
+        # parallelism; None: this replica's batch)
+        self.batch_total = None
         self.device = torch.device(device)
         dev = self.device
         T, B = w.T, w.B
@@ -121,7 +124,8 @@ class DenseSNN:
             out.append((f"scan_fwd{l}", lambda l=l, layer=layer: layer.forward(
                 self.I[l].view(T, B, -1), self.beta, self.thr, stream=stream)))
         out.append(("ce_loss", lambda: snn.snn_rate_ce_loss(
-            self.layers[-1].spk, labels, self.sizes[-1], self.loss, self.grad_out, stream)))
+            self.layers[-1].spk, labels, self.sizes[-1], self.loss, self.grad_out, stream,
+            batch_total=self.batch_total)))
         for l in range(len(self.layers) - 1, -1, -1):
             grad = self.grad_out if l == len(self.layers) - 1 else \
                 self.grad_in[l].view(T, B, -1)

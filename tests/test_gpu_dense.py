@@ -88,3 +88,24 @@ def test_rate_ce_loss(T, B, C, ld, dtype, cuda_device):
     np.testing.assert_allclose(got[:, :, :C], rg, rtol=1e-5 if dtype == torch.float32 else 2e-2,
                                atol=tol)
     assert np.all(got[:, :, C:] == 0)
+
+
+def test_rate_ce_loss_shard_normalisation(cuda_device):
+    """A shard of a larger batch: loss and gradient are averaged over the
+    global batch, so they are the shard's own values times B / batch_total."""
+    T, B, C, ld, total = 25, 64, 10, 16, 256
+    g = torch.Generator().manual_seed(5)
+    spk = (torch.rand((T, B, ld), generator=g) < 0.3).to(torch.float32)
+    labels = torch.randint(0, C, (B,), generator=g, dtype=torch.int32)
+    loss = torch.zeros(1, dtype=torch.float32, device=cuda_device)
+    grad = torch.full((T, B, ld), float("nan"), dtype=torch.float32, device=cuda_device)
+    snn.snn_rate_ce_loss(spk.to(cuda_device), labels.to(cuda_device), C, loss, grad,
+                         batch_total=total)
+    torch.cuda.synchronize()
+    rl, rg = O.rate_ce_loss(_np(spk[:, :, :C]), labels.numpy())
+    k = B / total
+    assert abs(loss.item() - rl * k) <= 1e-6 * max(1.0, abs(rl))
+    np.testing.assert_allclose(_np(grad.cpu())[:, :, :C], rg * k, rtol=1e-5, atol=1e-8)
+    lib = snn.load_library()
+    assert lib.snn_rate_ce_loss(T, B, C, ld, B - 1, 0, grad.data_ptr(), labels.data_ptr(),
+                                loss.data_ptr(), grad.data_ptr(), None) == 1
