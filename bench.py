@@ -13,7 +13,6 @@ workload instead.
 from __future__ import annotations
 
 import argparse
-import glob
 import hashlib
 import json
 import os
@@ -100,9 +99,14 @@ def hbm_peak():
         return FALLBACK_HBM_GBS, "fallback"
 
 
+SCAN_SOURCES = ("scan_kernels.cuh", "scan_dispatch.cuh", "scan_host.cuh", "snn_device.cuh",
+                "scan_fwd.cu", "scan_bwd_leaky.cu", "scan_bwd_synaptic.cu", "snn_api.cu")
+
+
 def kernel_source_hash():
+    """Hash of the sources the scan kernels are built from (and launched by)."""
     h = hashlib.sha256()
-    for f in sorted(glob.glob(os.path.join(ROOT, "paper_2211_10725_gb300", "csrc", "*"))):
+    for f in sorted(os.path.join(ROOT, "paper_2211_10725_gb300", "csrc", n) for n in SCAN_SOURCES):
         with open(f, "rb") as fh:
             h.update(os.path.basename(f).encode())
             h.update(fh.read())
