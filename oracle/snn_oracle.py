@@ -12,6 +12,8 @@ What it computes (arXiv 2211.10725, Sec. III-A and III-B):
            (the input current I_t = w x_t is given; (1-beta) is absorbed in it)
 * Eqs. (5)-(6) current-based (Synaptic) LIF
            i_t = alpha*i_{t-1} + I_t,   u_t = beta*u_{t-1} + i_t - z_{t-1}*u_thr
+* Eq. (7)  recurrent Leaky LIF (one-to-one recurrent weight v)
+           u_t = beta*u_{t-1} + w x_t + z_{t-1}*(v - u_thr)
 * Eqs. (8)-(9) fast-sigmoid surrogate, and an arctan surrogate, substituted
   for dz/du in the backward pass (Sec. III-B).
 * BPTT over the unrolled graph (Sec. II-A, II-B; Fig. 2): the exact reverse
@@ -24,7 +26,9 @@ Synaptic neuron); the fast-sigmoid slope k gives dz/du <- 1/(1+k|u-thr|)^2
 (k=1 is Eq. 9); arctan gives (a/2)/(1+(pi*a*(u-thr)/2)^2); a detached reset
 treats z_{t-1} in the reset term as a constant; initial state u_{-1}=i_{-1}=0,
 z_{-1}=0, or z_{-1}=[mem0 > thr] when mem0 is given; grad_mem_final is the
-gradient of the loss with respect to the returned final state u_{T-1}.
+gradient of the loss with respect to the returned final state u_{T-1}; in
+Eq. (7) a detached reset detaches only the -z*u_thr part: the recurrent
+connection z*v always carries gradient.
 
 Arrays are lane-major per time step: ``I[t, l]`` with lane l = b*N + n.  The
 arithmetic runs in float64 unless ``dtype=np.float32`` is asked for; in that
@@ -164,6 +168,39 @@ def leaky_forward(I, beta, thr, reset: str = "subtract", mem0=None,
     return spk, mem
 
 
+def rleaky_forward(I, v, beta, thr, mem0=None, dtype=np.float64, spike_fn=None,
+                   z_reset=None):
+    """Recurrent Leaky LIF over T steps (Eqs. 3, 7): the spike of step t-1
+    returns through the one-to-one weight v and the reset subtracts thr.
+
+    I: [T, L]; v, beta, thr: [L].  Returns (spk [T, L], mem [T, L]).  Each
+    step is (beta*u + I_t) + z_{t-1}*(v - thr), evaluated in ``dtype``.
+    With z_reset (test-only), the reset part uses the given constant
+    z_{t-1} while the recurrent part uses the live spike: u = beta*u + I_t +
+    z_{t-1}*v - zr*thr.
+    """
+    I = np.asarray(I, dtype=dtype)
+    T, L = I.shape
+    v = np.asarray(v, dtype=dtype).reshape(L)
+    beta = np.asarray(beta, dtype=dtype).reshape(L)
+    thr = np.asarray(thr, dtype=dtype).reshape(L)
+    spike = spike_fn if spike_fn is not None else (lambda u: heaviside(u, thr))
+    u_prev, z_prev = _initial(L, dtype, mem0, thr, spike)
+    vmt = v - thr
+    spk = np.zeros((T, L), dtype=dtype)
+    mem = np.zeros((T, L), dtype=dtype)
+    for t in range(T):
+        if z_reset is None:
+            u = beta * u_prev + I[t] + z_prev * vmt
+        else:
+            zr = np.asarray(z_reset[t], dtype=dtype)
+            u = beta * u_prev + I[t] + z_prev * v - zr * thr
+        z = spike(u)
+        mem[t], spk[t] = u, z
+        u_prev, z_prev = u, z
+    return spk, mem
+
+
 def synaptic_forward(I, alpha, beta, thr, reset: str = "subtract", mem0=None,
                      syn0=None, dtype=np.float64, spike_fn=None, z_reset=None):
     """Current-based LIF over T steps (Eqs. 3, 5, 6).
@@ -205,7 +242,7 @@ def synaptic_forward(I, alpha, beta, thr, reset: str = "subtract", mem0=None,
 
 def _bptt(mem, spk, grad_spk, beta, thr, reset, detach, sg, sg_param,
           grad_mem=None, grad_mem_final=None, mem0=None,
-          syn=None, alpha=None, syn0=None, grad_syn_final=None, z_init=None):
+          syn=None, alpha=None, syn0=None, grad_syn_final=None, z_init=None, vrec=None):
     """Shared reverse pass for the Leaky (syn is None) and Synaptic neurons.
 
     The pass differentiates along the given trajectory (mem u_t, spk z_t),
@@ -219,7 +256,9 @@ def _bptt(mem, spk, grad_spk, beta, thr, reset, detach, sg, sg_param,
       dI_t  = du_t (Leaky) or di_t (Synaptic)
 
     with d u_{t+1}/d u_t = beta (subtract, none) or beta*(1-z_t) (zero) and
-    d u_{t+1}/d z_t = -thr (subtract), -beta*u_t (zero), 0 (none).
+    d u_{t+1}/d z_t = -thr (subtract), -beta*u_t (zero), 0 (none).  The
+    recurrent neuron (vrec = v, Eq. 7, subtract) adds v to d u_{t+1}/d z_t
+    outside the detach factor, and dv += z_{t-1} * du_t.
     Parameter gradients, per lane, summed over t:
       dbeta  += du_t * d u_t/d beta   = du_t * u_{t-1}  (or (1-z_{t-1})*u_{t-1})
       dthr   += -sigma'_t * dz_t  -  [subtract] z_{t-1} * du_t
@@ -265,6 +304,13 @@ def _bptt(mem, spk, grad_spk, beta, thr, reset, detach, sg, sg_param,
             return -beta * u_at(t)
         return np.zeros(L)
 
+    if vrec is not None:
+        vrec = np.asarray(vrec, dtype=np.float64).reshape(L)
+        dv = np.zeros(L)
+
+    def rec_slope():     # d u_{t+1} / d z_t through the recurrent weight
+        return vrec if vrec is not None else 0.0
+
     dI = np.zeros((T, L))
     dbeta = np.zeros(L)
     dthr = np.zeros(L)
@@ -273,7 +319,7 @@ def _bptt(mem, spk, grad_spk, beta, thr, reset, detach, sg, sg_param,
     di_next = np.zeros(L)
     for t in range(T - 1, -1, -1):
         s = surrogate_grad(mem[t] - thr, sg, sg_param)
-        dz = gs[t] + (0.0 if detach else 1.0) * reset_slope(t) * du_next
+        dz = gs[t] + ((0.0 if detach else 1.0) * reset_slope(t) + rec_slope()) * du_next
         du = decay(t) * du_next + s * dz
         if gm is not None:
             du = du + gm[t]
@@ -282,6 +328,8 @@ def _bptt(mem, spk, grad_spk, beta, thr, reset, detach, sg, sg_param,
         dthr += -s * dz
         if reset == "subtract":
             dthr += -z_at(t - 1) * du
+        if vrec is not None:
+            dv += z_at(t - 1) * du
         if reset == "zero":
             dbeta += du * (1.0 - z_at(t - 1)) * u_at(t - 1)
         else:
@@ -301,7 +349,7 @@ def _bptt(mem, spk, grad_spk, beta, thr, reset, detach, sg, sg_param,
     dmem0 = decay(-1) * du_next
     if have_mem0:
         s = surrogate_grad(u_m1 - thr, sg, sg_param)
-        dz = (0.0 if detach else 1.0) * reset_slope(-1) * du_next
+        dz = ((0.0 if detach else 1.0) * reset_slope(-1) + rec_slope()) * du_next
         dmem0 = dmem0 + s * dz
         dthr += -s * dz
     out = {"grad_I": dI, "grad_beta_lane": dbeta, "grad_thr_lane": dthr,
@@ -309,6 +357,8 @@ def _bptt(mem, spk, grad_spk, beta, thr, reset, detach, sg, sg_param,
     if synaptic:
         out["grad_alpha_lane"] = dalpha
         out["grad_syn0"] = alpha * di_next
+    if vrec is not None:
+        out["grad_v_lane"] = dv
     return out
 
 
@@ -321,6 +371,16 @@ def leaky_backward(mem, spk, grad_spk, beta, thr, reset="subtract", detach=True,
     grad_mem0 [L] (all float64)."""
     return _bptt(mem, spk, grad_spk, beta, thr, reset, detach, sg, sg_param,
                  grad_mem, grad_mem_final, mem0, z_init=z_init)
+
+
+def rleaky_backward(mem, spk, grad_spk, v, beta, thr, detach=True, sg="fast_sigmoid",
+                    sg_param=25.0, grad_mem=None, grad_mem_final=None, mem0=None,
+                    z_init=None):
+    """BPTT for the recurrent Leaky neuron (Eq. 7) along (mem, spk).
+
+    Adds grad_v_lane [L] to the Leaky outputs."""
+    return _bptt(mem, spk, grad_spk, beta, thr, "subtract", detach, sg, sg_param,
+                 grad_mem, grad_mem_final, mem0, z_init=z_init, vrec=v)
 
 
 def synaptic_backward(mem, spk, syn, grad_spk, alpha, beta, thr, reset="subtract",

@@ -473,3 +473,91 @@ def test_adamw_matches_torch_optim():
     st = opt.state[p]
     np.testing.assert_allclose(m, st["exp_avg"].numpy(), rtol=1e-12)
     np.testing.assert_allclose(v, st["exp_avg_sq"].numpy(), rtol=1e-12)
+
+
+# ---------------------------------------------------------------------------
+# Recurrent Leaky neuron (Eq. 7)
+# ---------------------------------------------------------------------------
+
+@pytest.mark.parametrize("dtype,tol", [(np.float64, 1e-12), (np.float32, 1e-6)])
+def test_hand_trace_rleaky(dtype, tol):
+    # beta 0.5, thr 1, v 0.25: a spike feeds back v - thr = -0.75 at t+1.
+    #  t0: 1.5 -> fire;  t1: 0.75 + 0.2 - 0.75 = 0.2;  t2: 0.1 + 1.0 = 1.1 -> fire;
+    #  t3: 0.55 + 0 - 0.75 = -0.2;  t4: -0.1 + 0.9 = 0.8
+    I = np.array([1.5, 0.2, 1.0, 0.0, 0.9])[:, None]
+    spk, mem = O.rleaky_forward(I, [0.25], [0.5], [1.0], dtype=dtype)
+    np.testing.assert_allclose(mem[:, 0], [1.5, 0.2, 1.1, -0.2, 0.8], rtol=tol, atol=tol)
+    assert spk[:, 0].tolist() == [1, 0, 1, 0, 0]
+
+
+def test_rleaky_special_cases_reduce_to_leaky():
+    """v = 0 is the Leaky neuron with reset by subtraction; v = thr with the
+    reset not detached is the Leaky neuron without reset (forward and
+    BPTT); the recurrent weight's gradient is the reset term's with the
+    opposite sign."""
+    rng = np.random.default_rng(21)
+    T, L = 9, 6
+    I = rng.normal(0.6, 0.7, (T, L))
+    beta, thr = rng.uniform(0.5, 0.95, L), rng.uniform(0.7, 1.2, L)
+    gs, gm = rng.normal(0, 1, (T, L)), rng.normal(0, 0.5, (T, L))
+    kw = dict(sg="atan", sg_param=2.0, grad_mem=gm)
+    s0, m0 = O.rleaky_forward(I, np.zeros(L), beta, thr)
+    s1, m1 = O.leaky_forward(I, beta, thr, "subtract")
+    assert np.array_equal(s0, s1) and np.array_equal(m0, m1)
+    for detach in (True, False):
+        g0 = O.rleaky_backward(m0, s0, gs, np.zeros(L), beta, thr, detach=detach, **kw)
+        g1 = O.leaky_backward(m1, s1, gs, beta, thr, "subtract", detach=detach, **kw)
+        for k in ("grad_I", "grad_beta_lane", "grad_thr_lane", "grad_mem0"):
+            np.testing.assert_allclose(g0[k], g1[k], rtol=1e-13, atol=1e-15)
+    s2, m2 = O.rleaky_forward(I, thr, beta, thr)
+    s3, m3 = O.leaky_forward(I, beta, thr, "none")
+    assert np.array_equal(s2, s3)
+    np.testing.assert_allclose(m2, m3, rtol=0, atol=1e-14)
+    g2 = O.rleaky_backward(m2, s2, gs, thr, beta, thr, detach=False, **kw)
+    g3 = O.leaky_backward(m3, s3, gs, beta, thr, "none", detach=False, **kw)
+    np.testing.assert_allclose(g2["grad_I"], g3["grad_I"], rtol=1e-12, atol=1e-14)
+    np.testing.assert_allclose(g2["grad_beta_lane"], g3["grad_beta_lane"], rtol=1e-12, atol=1e-14)
+    # thr enters both the spike and (v - thr): the none-reset thr gradient
+    # plus the reset term's, which is -dv
+    np.testing.assert_allclose(g2["grad_thr_lane"], g3["grad_thr_lane"] - g2["grad_v_lane"],
+                               rtol=1e-12, atol=1e-14)
+
+
+@pytest.mark.parametrize("detach", [True, False])
+@pytest.mark.parametrize("sg,k", [("fast_sigmoid", 2.0), ("atan", 2.0)])
+def test_rleaky_bptt_matches_finite_differences(detach, sg, k):
+    rng = np.random.default_rng(31 + int(detach) + 2 * (sg == "atan"))
+    T, L = 5, 3
+    p = {"I": rng.normal(0.6, 0.6, (T, L)), "beta": rng.uniform(0.5, 0.95, L),
+         "thr": rng.uniform(0.7, 1.2, L), "mem0": rng.normal(0.5, 0.5, L),
+         "v": rng.uniform(-0.6, 0.6, L)}
+    gs, gm, gmf = rng.normal(0, 1, (T, L)), rng.normal(0, 0.5, (T, L)), rng.normal(0, 1, L)
+    f = lambda thr: (lambda u: O.smooth_spike(u - thr, sg, k))
+
+    def loss(q, z_reset):
+        spk, mem = O.rleaky_forward(q["I"], q["v"], q["beta"], q["thr"], mem0=q["mem0"],
+                                    spike_fn=f(q["thr"]), z_reset=z_reset)
+        return (gs * spk).sum() + (gm * mem).sum() + (gmf * mem[-1]).sum(), spk, mem
+
+    _, spk, mem = loss(p, None)
+    z_init = O.smooth_spike(p["mem0"] - p["thr"], sg, k)
+    z_reset = np.vstack([z_init[None], spk[:-1]]) if detach else None
+    g = O.rleaky_backward(mem, spk, gs, p["v"], p["beta"], p["thr"], detach=detach, sg=sg,
+                          sg_param=k, grad_mem=gm, grad_mem_final=gmf, mem0=p["mem0"],
+                          z_init=z_init)
+    h = 1e-6
+
+    def fd(name, idx):
+        q = {kk: vv.copy() for kk, vv in p.items()}
+        q[name][idx] += h
+        lp = loss(q, z_reset)[0]
+        q[name][idx] -= 2 * h
+        return (lp - loss(q, z_reset)[0]) / (2 * h)
+
+    for t in range(T):
+        for l in range(L):
+            np.testing.assert_allclose(g["grad_I"][t, l], fd("I", (t, l)), rtol=1e-6, atol=1e-8)
+    for pname, gname in [("beta", "grad_beta_lane"), ("thr", "grad_thr_lane"),
+                         ("mem0", "grad_mem0"), ("v", "grad_v_lane")]:
+        for l in range(L):
+            np.testing.assert_allclose(g[gname][l], fd(pname, l), rtol=1e-6, atol=1e-8)
