@@ -101,7 +101,8 @@ typedef struct snn_scan_desc {
   int32_t detach_reset;  /* 1: z_{t-1} in the reset term is a constant in BPTT */
   int32_t surrogate;     /* snn_surrogate_t                                    */
   float sg_param;        /* fast-sigmoid slope k, or arctan alpha              */
-  int32_t beta_mode, thr_mode, alpha_mode; /* snn_pmode_t                      */
+  int32_t beta_mode, thr_mode, alpha_mode; /* snn_pmode_t; alpha_mode is the
+                            layout of alpha (Synaptic) or of v (recurrent)     */
   int32_t save;          /* snn_save_t                                         */
   int32_t ckpt_every;    /* K >= 1 for SNN_SAVE_RECOMPUTE                      */
   int32_t reserved0;     /* must be 0                                          */
@@ -264,6 +265,36 @@ size_t snn_dense_workspace_bytes(int64_t M, int64_t K, int64_t N);
 snn_status_t snn_dense_layer_bwd(int64_t M, int64_t K, int64_t N, const void* X, const void* W,
                                  const void* dI, void* dX, float* dW, void* ws, size_t ws_bytes,
                                  snn_stream_t stream);
+
+/*
+ * Recurrent Leaky LIF forward, Eqs. (3) and (7): the spike of step t-1 is
+ * fed back through a one-to-one recurrent weight v,
+ *   u_t = beta*u_{t-1} + I_t + z_{t-1}*(v - thr),
+ * evaluated as (beta*u_{t-1} + I_t) + z_{t-1}*(v - thr), each operation
+ * rounded to nearest.  Arguments as snn_leaky_fwd, plus:
+ *   v        fp32, shape per desc->alpha_mode (scalar, [N] or [C])
+ * desc->reset must be SNN_RESET_SUBTRACT (Eq. 7 resets by subtraction),
+ * else SNN_ERR_UNSUPPORTED.
+ */
+snn_status_t snn_rleaky_fwd(const snn_scan_desc* desc, const void* I, const float* v,
+                            const float* beta, const float* thr, const float* mem0, void* spk,
+                            void* mem, float* ckpt, float* mem_final, void* ws, size_t ws_bytes,
+                            snn_stream_t stream);
+
+/*
+ * Recurrent Leaky LIF BPTT.  Arguments as snn_leaky_bwd, plus v and
+ *   grad_v   fp32, v's shape, or NULL: dL/dv summed over t and the lanes
+ *            sharing v (d u_{t+1}/d v = z_t).
+ * The recurrent connection always carries gradient; detach_reset detaches
+ * only the -z_{t-1}*thr part:
+ *   dz_t = grad_spk_t + (v - [not detach]*thr) * du_{t+1}.
+ */
+snn_status_t snn_rleaky_bwd(const snn_scan_desc* desc, const void* I, const float* ckpt,
+                            const void* mem, const void* spk, const float* v, const float* beta,
+                            const float* thr, const float* mem0, const void* grad_spk,
+                            const void* grad_mem, const float* grad_mem_final, void* grad_I,
+                            float* grad_v, float* grad_beta, float* grad_thr, float* grad_mem0,
+                            void* ws, size_t ws_bytes, snn_stream_t stream);
 
 /*
  * Rate-coded readout loss (Sec. V-A: the predicted class is the output

@@ -169,7 +169,7 @@ def leaky_forward(I, beta, thr, reset: str = "subtract", mem0=None,
 
 
 def rleaky_forward(I, v, beta, thr, mem0=None, dtype=np.float64, spike_fn=None,
-                   z_reset=None):
+                   z_reset=None, z_path=None):
     """Recurrent Leaky LIF over T steps (Eqs. 3, 7): the spike of step t-1
     returns through the one-to-one weight v and the reset subtracts thr.
 
@@ -177,7 +177,8 @@ def rleaky_forward(I, v, beta, thr, mem0=None, dtype=np.float64, spike_fn=None,
     step is (beta*u + I_t) + z_{t-1}*(v - thr), evaluated in ``dtype``.
     With z_reset (test-only), the reset part uses the given constant
     z_{t-1} while the recurrent part uses the live spike: u = beta*u + I_t +
-    z_{t-1}*v - zr*thr.
+    z_{t-1}*v - zr*thr.  With z_path ([T, L], row t = z_{t-1}; test-only)
+    both parts follow the given spike sequence.
     """
     I = np.asarray(I, dtype=dtype)
     T, L = I.shape
@@ -190,7 +191,9 @@ def rleaky_forward(I, v, beta, thr, mem0=None, dtype=np.float64, spike_fn=None,
     spk = np.zeros((T, L), dtype=dtype)
     mem = np.zeros((T, L), dtype=dtype)
     for t in range(T):
-        if z_reset is None:
+        if z_path is not None:
+            u = beta * u_prev + I[t] + np.asarray(z_path[t], dtype=dtype) * vmt
+        elif z_reset is None:
             u = beta * u_prev + I[t] + z_prev * vmt
         else:
             zr = np.asarray(z_reset[t], dtype=dtype)

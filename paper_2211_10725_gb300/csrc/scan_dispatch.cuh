@@ -16,15 +16,15 @@ constexpr bool kSpecialise =
     (std::is_same<TI, __nv_bfloat16>::value && std::is_same<TO, __nv_bfloat16>::value) ||
     (std::is_same<TI, float>::value && std::is_same<TO, __nv_bfloat16>::value);
 
-template <bool SYN, typename TI, typename TO, int RESET>
+template <bool SYN, typename TI, typename TO, int RESET, bool REC = false>
 cudaError_t fwd_staged(ScanArgs a, cudaStream_t st, bool* launched) {
-  const void* k = (const void*)scan_fwd_staged<SYN, TI, TO, RESET>;
+  const void* k = (const void*)scan_fwd_staged<SYN, TI, TO, RESET, REC>;
   StagedPlan p;
   if (!plan_staged(k, a.L, a.T, (int)sizeof(TI), 0, kLanes<SYN>, &p)) return cudaSuccess;
   a.lanes_per_cta = p.lanes_per_cta;
   a.stages = p.stages;
   a.stage_bytes = p.stage_bytes;
-  scan_fwd_staged<SYN, TI, TO, RESET><<<(unsigned)p.grid, p.threads, p.smem, st>>>(a);
+  scan_fwd_staged<SYN, TI, TO, RESET, REC><<<(unsigned)p.grid, p.threads, p.smem, st>>>(a);
   *launched = true;
   return cudaGetLastError();
 }
@@ -34,7 +34,8 @@ cudaError_t fwd_t(ScanArgs a, bool staged, cudaStream_t st) {
   if (staged && a.L > 0) {
     bool launched = false;
     cudaError_t e;
-    if (a.reset == RESET_SUBTRACT) e = fwd_staged<SYN, TI, TO, RESET_SUBTRACT>(a, st, &launched);
+    if (!SYN && a.rec) e = fwd_staged<false, TI, TO, RESET_SUBTRACT, true>(a, st, &launched);
+    else if (a.reset == RESET_SUBTRACT) e = fwd_staged<SYN, TI, TO, RESET_SUBTRACT>(a, st, &launched);
     else if (a.reset == RESET_ZERO) e = fwd_staged<SYN, TI, TO, RESET_ZERO>(a, st, &launched);
     else e = fwd_staged<SYN, TI, TO, -1>(a, st, &launched);
     if (launched || e != cudaSuccess) return e;
@@ -44,9 +45,10 @@ cudaError_t fwd_t(ScanArgs a, bool staged, cudaStream_t st) {
   return cudaGetLastError();
 }
 
-template <bool SYN, bool RECOMP, typename TI, typename TO, int RESET, int SG, int KC = 0>
+template <bool SYN, bool RECOMP, typename TI, typename TO, int RESET, int SG, int KC = 0,
+          bool REC = false>
 cudaError_t bwd_staged(ScanArgs a, cudaStream_t st, bool* launched) {
-  const void* k = (const void*)scan_bwd_staged<SYN, RECOMP, TI, TO, RESET, SG, KC>;
+  const void* k = (const void*)scan_bwd_staged<SYN, RECOMP, TI, TO, RESET, SG, KC, REC>;
   int per_lane, seg, fixed;
   int64_t items;
   if (RECOMP) {
@@ -68,7 +70,8 @@ cudaError_t bwd_staged(ScanArgs a, cudaStream_t st, bool* launched) {
   a.lanes_per_cta = p.lanes_per_cta;
   a.stages = p.stages;
   a.stage_bytes = p.stage_bytes;
-  scan_bwd_staged<SYN, RECOMP, TI, TO, RESET, SG, KC><<<(unsigned)p.grid, p.threads, p.smem, st>>>(a);
+  scan_bwd_staged<SYN, RECOMP, TI, TO, RESET, SG, KC, REC><<<(unsigned)p.grid, p.threads, p.smem,
+                                                             st>>>(a);
   *launched = true;
   return cudaGetLastError();
 }
@@ -79,7 +82,10 @@ cudaError_t bwd_t(ScanArgs a, bool staged, cudaStream_t st) {
     bool launched = false;
     cudaError_t e = cudaSuccess;
     bool done = false;
-    if constexpr (kSpecialise<TI, TO>) {
+    if (!SYN && a.rec) {  // recurrent Leaky neuron: reset by subtraction (Eq. 7)
+      e = bwd_staged<false, RECOMP, TI, TO, RESET_SUBTRACT, -1, 0, true>(a, st, &launched);
+      done = true;
+    } else if constexpr (kSpecialise<TI, TO>) {
       done = true;
       const int key = (a.reset == RESET_NONE ? 9 : a.reset * 2 + a.sg);
       // the recompute variant with the default checkpoint interval K = 8

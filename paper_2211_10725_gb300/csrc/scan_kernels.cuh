@@ -41,6 +41,7 @@ struct ScanArgs {
   int K;      // checkpoint interval (recompute); T in store mode
   int nseg;   // ceil(T / K)
   int reset, detach, sg;
+  int rec;           // recurrent Leaky neuron (Eq. 7): alpha holds v, part_alpha dv
   float sg_a, sg_b;  // fast sigmoid: a = slope; atan: a = alpha/2, b = pi*alpha/2
   int beta_mode, thr_mode, alpha_mode;
   const float* beta;
@@ -117,10 +118,12 @@ __device__ __forceinline__ int seg_phase0(const ScanArgs& a) {
 // would fuse two of them), so the forward and the backward's recomputation
 // agree bit for bit.  The subtract reset u - z*thr is one rounding since
 // z*thr is exact (z in {0,1}); reset-to-zero scales u by (1 - z) exactly.
-template <bool SYN, int RESET>
+template <bool SYN, int RESET, int REC = 0>
 __device__ __forceinline__ void fwd_step(int reset_rt, float beta, float thr, float alpha,
-                                         float x, float& u, bool& z, float& i) {
+                                         float x, float& u, bool& z, float& i,
+                                         bool rec_rt = false) {
   const int reset = RESET >= 0 ? RESET : reset_rt;
+  const bool rec = REC > 0 || (REC < 0 && rec_rt);  // Eq. (7): alpha is v
   float in = x;
   if (SYN) {
     i = __fadd_rn(__fmul_rn(alpha, i), x);
@@ -132,7 +135,7 @@ __device__ __forceinline__ void fwd_step(int reset_rt, float beta, float thr, fl
     un = __fadd_rn(__fmul_rn(beta, z ? __fmul_rn(u, 0.0f) : u), in);
   } else {
     un = __fadd_rn(__fmul_rn(beta, u), in);
-    if (reset == RESET_SUBTRACT && z) un = __fsub_rn(un, thr);
+    if (reset == RESET_SUBTRACT && z) un = rec ? __fadd_rn(un, __fsub_rn(alpha, thr)) : __fsub_rn(un, thr);
   }
   u = un;
   z = un > thr;  // Eq. (3), strict
@@ -169,6 +172,7 @@ __device__ __forceinline__ float bwd_step(const ScanArgs& a, float beta, float t
     s.dbeta = fmaf(s.du, (reset == RESET_ZERO && z) ? 0.0f : u, s.dbeta);
     if (reset == RESET_SUBTRACT && z) s.dthr -= s.du;
     if (SYN) s.dalpha = fmaf(s.di, i, s.dalpha);
+    if (!SYN && a.rec && z) s.dalpha += s.du;  // dv: d u_{t+1} / d v = z_t
   }
   const float sgv = surrogate<SG>(a, u - thr);
   float dz = gs;
@@ -176,6 +180,7 @@ __device__ __forceinline__ float bwd_step(const ScanArgs& a, float beta, float t
     if (reset == RESET_SUBTRACT) dz = fmaf(-thr, s.du, dz);
     else if (reset == RESET_ZERO) dz = fmaf(-beta * u, s.du, dz);
   }
+  if (!SYN && a.rec) dz = fmaf(alpha, s.du, dz);  // the recurrent connection, never detached
   const float decay = (reset == RESET_ZERO && z) ? 0.0f : beta;
   const float du = fmaf(decay, s.du, fmaf(sgv, dz, extra_u));
   s.dthr = fmaf(-sgv, dz, s.dthr);
@@ -195,14 +200,18 @@ __device__ __forceinline__ void bwd_initial(const ScanArgs& a, float beta, float
                                             float i_m1, BwdLane& s, float& gmem0,
                                             float& gsyn0) {
   const bool z_m1 = have_mem0 && (u_m1 > thr);
+  const bool rec = !SYN && a.rec;
   s.dbeta = fmaf(s.du, (a.reset == RESET_ZERO && z_m1) ? 0.0f : u_m1, s.dbeta);
   if (a.reset == RESET_SUBTRACT && z_m1) s.dthr -= s.du;
   if (SYN) s.dalpha = fmaf(s.di, i_m1, s.dalpha);
+  if (rec && z_m1) s.dalpha += s.du;
   const float decay = (a.reset == RESET_ZERO && z_m1) ? 0.0f : beta;
   gmem0 = decay * s.du;
-  if (have_mem0 && !a.detach && a.reset != RESET_NONE) {
+  if (have_mem0 && ((!a.detach && a.reset != RESET_NONE) || rec)) {
     const float sgv = surrogate<-1>(a, u_m1 - thr);
-    const float slope = (a.reset == RESET_SUBTRACT) ? -thr : -beta * u_m1;
+    float slope = 0.0f;
+    if (!a.detach && a.reset != RESET_NONE) slope = (a.reset == RESET_SUBTRACT) ? -thr : -beta * u_m1;
+    if (rec) slope += alpha;
     const float dz = slope * s.du;
     gmem0 = fmaf(sgv, dz, gmem0);
     s.dthr = fmaf(-sgv, dz, s.dthr);
@@ -224,11 +233,11 @@ __device__ __forceinline__ float2 fma2(float2 a, float2 b, float2 c) { return __
 // with explicit rounding, which the compiler never fuses; packed fp32x2
 // multiply and add may be fused into a packed FMA, which would change the
 // result).  negthr = -thr; z[0..1] hold z_{t-1} on entry and z_t on exit.
-template <bool SYN, int RESET>
+template <bool SYN, int RESET, int REC = 0>
 __device__ __forceinline__ void fwd_pair(int reset_rt, float2 beta, float2 negthr, float2 alpha,
                                          float2 x, float2& u, bool* z, float2& i) {
-  fwd_step<SYN, RESET>(reset_rt, beta.x, -negthr.x, alpha.x, x.x, u.x, z[0], i.x);
-  fwd_step<SYN, RESET>(reset_rt, beta.y, -negthr.y, alpha.y, x.y, u.y, z[1], i.y);
+  fwd_step<SYN, RESET, REC>(reset_rt, beta.x, -negthr.x, alpha.x, x.x, u.x, z[0], i.x);
+  fwd_step<SYN, RESET, REC>(reset_rt, beta.y, -negthr.y, alpha.y, x.y, u.y, z[1], i.y);
 }
 
 // Approximate reciprocal (one hardware instruction, relative error ~2^-23)
@@ -263,7 +272,7 @@ struct Bwd2 {
 // parameter terms of step t+1 vanish there) and dL/du_t, dL/di_t on exit.
 // EXTRA adds eu to dL/du_t and ei to dL/di_t (grad_mem every step,
 // grad_mem_final / grad_syn_final at t = T-1).  Returns dL/dI_t.
-template <bool SYN, int RESET, int SG, bool EXTRA>
+template <bool SYN, int RESET, int SG, bool EXTRA, bool REC = false>
 __device__ __forceinline__ float2 bwd_pair(const ScanArgs& a, float2 beta, float2 negthr,
                                            float2 alpha, float2 u, bool z0, bool z1, float2 i,
                                            float2 gs, float2 eu, float2 ei, Bwd2& s) {
@@ -277,6 +286,10 @@ __device__ __forceinline__ float2 bwd_pair(const ScanArgs& a, float2 beta, float
     if (z0) s.dthr.x += s.du.x;
     if (z1) s.dthr.y += s.du.y;
   }
+  if (REC) {  // d u_{t+1} / d v = z_t (Eq. 7)
+    if (z0) s.dalpha.x += s.du.x;
+    if (z1) s.dalpha.y += s.du.y;
+  }
   if (SYN) s.dalpha = fma2(s.di, i, s.dalpha);
   const float2 sg = surrogate2<SG>(a, add2(u, negthr));
   float2 dz = gs;
@@ -284,6 +297,7 @@ __device__ __forceinline__ float2 bwd_pair(const ScanArgs& a, float2 beta, float
     if (reset == RESET_SUBTRACT) dz = fma2(negthr, s.du, dz);
     else if (reset == RESET_ZERO) dz = fma2(mul2(f2(-1.0f), mul2(beta, u)), s.du, dz);
   }
+  if (REC) dz = fma2(alpha, s.du, dz);  // the recurrent connection, never detached
   const float2 p = mul2(sg, dz);
   const float2 decay = reset == RESET_ZERO
                            ? make_float2(z0 ? 0.0f : beta.x, z1 ? 0.0f : beta.y)
@@ -439,7 +453,7 @@ __device__ __forceinline__ void load_pairs_global(const float* p, float2 q[NP]) 
 }
 
 // beta, -thr and alpha of the thread's 2*NP lanes, as pairs
-template <bool SYN, int NP>
+template <bool SYN, int NP>  // SYN: also load the third parameter (alpha, or v)
 __device__ __forceinline__ void load_params(const ScanArgs& a, int64_t l, float2 beta[NP],
                                             float2 negthr[NP], float2 alpha[NP]) {
 #pragma unroll
@@ -478,7 +492,7 @@ __device__ __forceinline__ void initial_state(const ScanArgs& a, int64_t l, cons
 // Staged forward
 // ---------------------------------------------------------------------------
 
-template <bool SYN, typename TI, typename TO, int RESET>
+template <bool SYN, typename TI, typename TO, int RESET, bool REC = false>
 __global__ void __launch_bounds__(kMaxStagedThreads) scan_fwd_staged(const ScanArgs a) {
   constexpr int V = kLanes<SYN>, NP = V / 2;
   extern __shared__ __align__(1024) unsigned char smem[];
@@ -511,7 +525,7 @@ __global__ void __launch_bounds__(kMaxStagedThreads) scan_fwd_staged(const ScanA
   float2 beta[NP], negthr[NP], alpha[NP], u[NP], in[NP];
   bool z[V];
   if (active) {
-    load_params<SYN, NP>(a, l, beta, negthr, alpha);
+    load_params<SYN || REC, NP>(a, l, beta, negthr, alpha);
     initial_state<SYN, NP>(a, l, negthr, u, z, in);
   }
   TO* spk = static_cast<TO*>(a.spk) + l;
@@ -538,7 +552,8 @@ __global__ void __launch_bounds__(kMaxStagedThreads) scan_fwd_staged(const ScanA
       float2 zf[NP];
 #pragma unroll
       for (int k = 0; k < NP; ++k) {
-        fwd_pair<SYN, RESET>(a.reset, beta[k], negthr[k], alpha[k], x[k], u[k], &z[2 * k], in[k]);
+        fwd_pair<SYN, RESET, REC ? 1 : 0>(a.reset, beta[k], negthr[k], alpha[k], x[k], u[k],
+                                          &z[2 * k], in[k]);
         zf[k] = make_float2(z[2 * k] ? 1.0f : 0.0f, z[2 * k + 1] ? 1.0f : 0.0f);
       }
 #pragma unroll
@@ -587,7 +602,7 @@ __global__ void __launch_bounds__(kMaxStagedThreads) scan_fwd_staged(const ScanA
 
 // The reverse step on all of a thread's pairs; EXTRA steps (grad_mem given,
 // or t = T-1 with grad_mem_final / grad_syn_final) add those gradients.
-template <bool SYN, int RESET, int SG, bool EXTRA, int NP>
+template <bool SYN, int RESET, int SG, bool EXTRA, int NP, bool REC = false>
 __device__ __forceinline__ void bwd_pairs(const ScanArgs& a, const float2 beta[NP],
                                           const float2 negthr[NP], const float2 alpha[NP],
                                           const float2 u[NP], const bool z[2 * NP],
@@ -596,11 +611,13 @@ __device__ __forceinline__ void bwd_pairs(const ScanArgs& a, const float2 beta[N
                                           float2 out[NP]) {
 #pragma unroll
   for (int k = 0; k < NP; ++k)
-    out[k] = bwd_pair<SYN, RESET, SG, EXTRA>(a, beta[k], negthr[k], alpha[k], u[k], z[2 * k],
-                                             z[2 * k + 1], i[k], g[k], eu[k], ei[k], st[k]);
+    out[k] = bwd_pair<SYN, RESET, SG, EXTRA, REC>(a, beta[k], negthr[k], alpha[k], u[k],
+                                                  z[2 * k], z[2 * k + 1], i[k], g[k], eu[k],
+                                                  ei[k], st[k]);
 }
 
-template <bool SYN, bool RECOMP, typename TI, typename TO, int RESET, int SG, int KC = 0>
+template <bool SYN, bool RECOMP, typename TI, typename TO, int RESET, int SG, int KC = 0,
+          bool REC = false>
 __global__ void __launch_bounds__(kMaxStagedThreads) scan_bwd_staged(const ScanArgs a) {
   constexpr int V = kLanes<SYN>, NP = V / 2;
   extern __shared__ __align__(1024) unsigned char smem[];
@@ -701,7 +718,7 @@ __global__ void __launch_bounds__(kMaxStagedThreads) scan_bwd_staged(const ScanA
   const bool active = c * V < cta_lanes;
   float2 beta[NP], negthr[NP], alpha[NP];
   Bwd2 st[NP];
-  if (active) load_params<SYN, NP>(a, l, beta, negthr, alpha);
+  if (active) load_params<SYN || REC, NP>(a, l, beta, negthr, alpha);
 #pragma unroll
   for (int k = 0; k < NP; ++k) st[k] = Bwd2{f2(0.0f), f2(0.0f), f2(0.0f), f2(0.0f), f2(0.0f)};
   const int stage_io_elems = a.stage_bytes / (int)sizeof(TO);
@@ -738,9 +755,11 @@ __global__ void __launch_bounds__(kMaxStagedThreads) scan_bwd_staged(const ScanA
           if (SYN && a.gsf) ei[k] = fi[k];
         }
       }
-      bwd_pairs<SYN, RESET, SG, true, NP>(a, beta, negthr, alpha, u, z, i, g, eu, ei, st, out);
+      bwd_pairs<SYN, RESET, SG, true, NP, REC>(a, beta, negthr, alpha, u, z, i, g, eu, ei, st,
+                                               out);
     } else {
-      bwd_pairs<SYN, RESET, SG, false, NP>(a, beta, negthr, alpha, u, z, i, g, g, g, st, out);
+      bwd_pairs<SYN, RESET, SG, false, NP, REC>(a, beta, negthr, alpha, u, z, i, g, g, g, st,
+                                                out);
     }
   };
 
@@ -835,7 +854,8 @@ __global__ void __launch_bounds__(kMaxStagedThreads) scan_bwd_staged(const ScanA
       load_pairs<TI, NP>(xin, x);
 #pragma unroll
       for (int q = 0; q < NP; ++q)
-        fwd_pair<SYN, RESET>(a.reset, beta[q], negthr[q], alpha[q], x[q], u[q], &z[2 * q], ii[q]);
+        fwd_pair<SYN, RESET, REC ? 1 : 0>(a.reset, beta[q], negthr[q], alpha[q], x[q], u[q],
+                                          &z[2 * q], ii[q]);
 #pragma unroll
       for (int q = 0; q < V / 4; ++q) {
         *reinterpret_cast<float4*>(su + q * nthr * 4) =
@@ -981,7 +1001,7 @@ __global__ void __launch_bounds__(kMaxStagedThreads) scan_bwd_staged(const ScanA
   if (SYN && a.gsyn0) storev<float, V>(a.gsyn0 + l, gs0);
   if (a.part_beta) storev<float, V>(a.part_beta + l, db);
   if (a.part_thr) storev<float, V>(a.part_thr + l, dt);
-  if (SYN && a.part_alpha) storev<float, V>(a.part_alpha + l, da);
+  if ((SYN || REC) && a.part_alpha) storev<float, V>(a.part_alpha + l, da);
 }
 
 // ---------------------------------------------------------------------------
@@ -994,7 +1014,7 @@ __global__ void __launch_bounds__(256) scan_fwd_plain(const ScanArgs a) {
   if (l >= a.L) return;
   const float beta = lane_param(a.beta, a.beta_mode, l, a);
   const float thr = lane_param(a.thr, a.thr_mode, l, a);
-  const float alpha = SYN ? lane_param(a.alpha, a.alpha_mode, l, a) : 0.0f;
+  const float alpha = (SYN || a.rec) ? lane_param(a.alpha, a.alpha_mode, l, a) : 0.0f;
   float u = a.mem0 ? a.mem0[l] : 0.0f;
   bool z = a.mem0 ? (u > thr) : false;
   float i = (SYN && a.syn0) ? a.syn0[l] : 0.0f;
@@ -1007,7 +1027,8 @@ __global__ void __launch_bounds__(256) scan_fwd_plain(const ScanArgs a) {
   float* cp = a.ckpt ? a.ckpt + l : nullptr;
   for (int64_t t = 0; t < a.T; ++t) {
     const int64_t off = t * a.L + l;
-    fwd_step<SYN, -1>(a.reset, beta, thr, alpha, Elem<TI>::load1(I + off), u, z, i);
+    fwd_step<SYN, -1, -1>(a.reset, beta, thr, alpha, Elem<TI>::load1(I + off), u, z, i,
+                          a.rec != 0);
     Elem<TO>::store1(spk + off, z ? 1.0f : 0.0f);
     if (mem) Elem<TO>::store1(mem + off, u);
     if (SYN && syn) Elem<TO>::store1(syn + off, i);
@@ -1031,7 +1052,7 @@ __global__ void __launch_bounds__(128) scan_bwd_plain(const ScanArgs a) {
   if (l >= a.L) return;
   const float beta = lane_param(a.beta, a.beta_mode, l, a);
   const float thr = lane_param(a.thr, a.thr_mode, l, a);
-  const float alpha = SYN ? lane_param(a.alpha, a.alpha_mode, l, a) : 0.0f;
+  const float alpha = (SYN || a.rec) ? lane_param(a.alpha, a.alpha_mode, l, a) : 0.0f;
   const bool have_mem0 = a.mem0 != nullptr;
   const float m0 = have_mem0 ? a.mem0[l] : 0.0f;
   const float s0 = (SYN && a.syn0) ? a.syn0[l] : 0.0f;
@@ -1078,7 +1099,8 @@ __global__ void __launch_bounds__(128) scan_bwd_plain(const ScanArgs a) {
         z = have_mem0 && (m0 > thr);
       }
       for (int64_t t = t0; t < t1; ++t) {
-        fwd_step<SYN, -1>(a.reset, beta, thr, alpha, Elem<TI>::load1(I + t * a.L + l), u, z, i);
+        fwd_step<SYN, -1, -1>(a.reset, beta, thr, alpha, Elem<TI>::load1(I + t * a.L + l), u,
+                              z, i, a.rec != 0);
         su[(t - t0) * blockDim.x] = u;
         if (SYN) si[(t - t0) * blockDim.x] = i;
       }
@@ -1105,7 +1127,7 @@ __global__ void __launch_bounds__(128) scan_bwd_plain(const ScanArgs a) {
   if (SYN && a.gsyn0) a.gsyn0[l] = gs0;
   if (a.part_beta) a.part_beta[l] = st.dbeta;
   if (a.part_thr) a.part_thr[l] = st.dthr;
-  if (SYN && a.part_alpha) a.part_alpha[l] = st.dalpha;
+  if ((SYN || a.rec) && a.part_alpha) a.part_alpha[l] = st.dalpha;
 }
 
 }  // namespace snn

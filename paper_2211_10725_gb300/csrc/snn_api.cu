@@ -149,15 +149,20 @@ snn_status_t cuda_status(cudaError_t e) {
   return SNN_ERR_CUDA;
 }
 
-snn_status_t scan_fwd(const snn_scan_desc* d, bool syn, const void* I, const float* alpha,
+// Neuron kinds of the shared scan paths.
+enum Neuron { kLeaky = 0, kSynaptic = 1, kRecurrentLeaky = 2 };
+
+snn_status_t scan_fwd(const snn_scan_desc* d, int neuron, const void* I, const float* alpha,
                       const float* beta, const float* thr, const float* mem0, const float* syn0,
                       void* spk, void* mem, void* synout, float* ckpt, float* mem_final,
                       float* syn_final, void* ws, size_t ws_bytes, cudaStream_t stream) {
   snn_status_t s = check_desc(d);
   if (s != SNN_OK) return s;
+  const bool syn = neuron == kSynaptic, rec = neuron == kRecurrentLeaky;
   const int64_t n = d->T * d->B * d->N;
   const bool recompute = d->save == SNN_SAVE_RECOMPUTE;
-  if (!beta || !thr || (syn && !alpha)) return SNN_ERR_INVALID_ARG;
+  if (!beta || !thr || ((syn || rec) && !alpha)) return SNN_ERR_INVALID_ARG;
+  if (rec && d->reset != SNN_RESET_SUBTRACT) return SNN_ERR_UNSUPPORTED;
   if (n > 0 && (!I || !spk)) return SNN_ERR_INVALID_ARG;
   if (n > 0 && !recompute && !mem) return SNN_ERR_INVALID_ARG;
   if (recompute && snn_scan_ckpt_elems(d, syn) > 0 && !ckpt) return SNN_ERR_INVALID_ARG;
@@ -168,7 +173,8 @@ snn_status_t scan_fwd(const snn_scan_desc* d, bool syn, const void* I, const flo
   ScanArgs a = base_args(d, ws);
   a.beta = beta;
   a.thr = thr;
-  a.alpha = syn ? alpha : nullptr;
+  a.alpha = (syn || rec) ? alpha : nullptr;
+  a.rec = rec ? 1 : 0;
   a.mem0 = mem0;
   a.syn0 = syn ? syn0 : nullptr;
   a.I = I;
@@ -186,7 +192,7 @@ snn_status_t scan_fwd(const snn_scan_desc* d, bool syn, const void* I, const flo
   return cuda_status(launch_scan_fwd(a, syn, d->in_dtype, d->io_dtype, staged, stream));
 }
 
-snn_status_t scan_bwd(const snn_scan_desc* d, bool syn, const void* I, const float* ckpt,
+snn_status_t scan_bwd(const snn_scan_desc* d, int neuron, const void* I, const float* ckpt,
                       const void* mem, const void* spk, const void* synin, const float* alpha,
                       const float* beta, const float* thr, const float* mem0, const float* syn0,
                       const void* grad_spk, const void* grad_mem, const float* grad_mem_final,
@@ -195,9 +201,11 @@ snn_status_t scan_bwd(const snn_scan_desc* d, bool syn, const void* I, const flo
                       void* ws, size_t ws_bytes, cudaStream_t stream) {
   snn_status_t s = check_desc(d);
   if (s != SNN_OK) return s;
+  const bool syn = neuron == kSynaptic, rec = neuron == kRecurrentLeaky;
   const int64_t n = d->T * d->B * d->N;
   const bool recompute = d->save == SNN_SAVE_RECOMPUTE;
-  if (!beta || !thr || (syn && !alpha)) return SNN_ERR_INVALID_ARG;
+  if (!beta || !thr || ((syn || rec) && !alpha)) return SNN_ERR_INVALID_ARG;
+  if (rec && d->reset != SNN_RESET_SUBTRACT) return SNN_ERR_UNSUPPORTED;
   if (n > 0 && (!grad_spk || !grad_I)) return SNN_ERR_INVALID_ARG;
   if (n > 0 && recompute && !I) return SNN_ERR_INVALID_ARG;
   if (recompute && snn_scan_ckpt_elems(d, syn) > 0 && !ckpt) return SNN_ERR_INVALID_ARG;
@@ -214,7 +222,7 @@ snn_status_t scan_bwd(const snn_scan_desc* d, bool syn, const void* I, const flo
     return s;
   if ((s = check_ws(d, ws, ws_bytes)) != SNN_OK) return s;
   const int64_t L = d->B * d->N;
-  float* outs[3] = {grad_beta, grad_thr, syn ? grad_alpha : nullptr};
+  float* outs[3] = {grad_beta, grad_thr, (syn || rec) ? grad_alpha : nullptr};
   const int modes[3] = {d->beta_mode, d->thr_mode, d->alpha_mode};
   if (L == 0) {
     for (int k = 0; k < 3; ++k)
@@ -228,7 +236,8 @@ snn_status_t scan_bwd(const snn_scan_desc* d, bool syn, const void* I, const flo
   ScanArgs a = base_args(d, ws);
   a.beta = beta;
   a.thr = thr;
-  a.alpha = syn ? alpha : nullptr;
+  a.alpha = (syn || rec) ? alpha : nullptr;
+  a.rec = rec ? 1 : 0;
   a.mem0 = mem0;
   a.syn0 = syn ? syn0 : nullptr;
   a.I = recompute ? I : nullptr;
@@ -247,7 +256,7 @@ snn_status_t scan_bwd(const snn_scan_desc* d, bool syn, const void* I, const flo
   a.gI = grad_I;
   a.part_beta = grad_beta ? v.part[0] : nullptr;
   a.part_thr = grad_thr ? v.part[1] : nullptr;
-  a.part_alpha = (syn && grad_alpha) ? v.part[2] : nullptr;
+  a.part_alpha = ((syn || rec) && grad_alpha) ? v.part[2] : nullptr;
   a.gmem0 = grad_mem0;
   a.gsyn0 = syn ? grad_syn0 : nullptr;
   const bool staged = staged_ok(d);
@@ -325,7 +334,7 @@ snn_status_t snn_leaky_fwd(const snn_scan_desc* desc, const void* I, const float
                            const float* thr, const float* mem0, void* spk, void* mem,
                            float* ckpt, float* mem_final, void* ws, size_t ws_bytes,
                            snn_stream_t stream) {
-  return scan_fwd(desc, false, I, nullptr, beta, thr, mem0, nullptr, spk, mem, nullptr, ckpt,
+  return scan_fwd(desc, kLeaky, I, nullptr, beta, thr, mem0, nullptr, spk, mem, nullptr, ckpt,
                   mem_final, nullptr, ws, ws_bytes, (cudaStream_t)stream);
 }
 
@@ -335,7 +344,7 @@ snn_status_t snn_leaky_bwd(const snn_scan_desc* desc, const void* I, const float
                            const void* grad_mem, const float* grad_mem_final, void* grad_I,
                            float* grad_beta, float* grad_thr, float* grad_mem0, void* ws,
                            size_t ws_bytes, snn_stream_t stream) {
-  return scan_bwd(desc, false, I, ckpt, mem, spk, nullptr, nullptr, beta, thr, mem0, nullptr,
+  return scan_bwd(desc, kLeaky, I, ckpt, mem, spk, nullptr, nullptr, beta, thr, mem0, nullptr,
                   grad_spk, grad_mem, grad_mem_final, nullptr, grad_I, nullptr, grad_beta,
                   grad_thr, grad_mem0, nullptr, ws, ws_bytes, (cudaStream_t)stream);
 }
@@ -345,7 +354,7 @@ snn_status_t snn_synaptic_fwd(const snn_scan_desc* desc, const void* I, const fl
                               const float* syn0, void* spk, void* mem, void* syn,
                               float* ckpt, float* mem_final, float* syn_final, void* ws,
                               size_t ws_bytes, snn_stream_t stream) {
-  return scan_fwd(desc, true, I, alpha, beta, thr, mem0, syn0, spk, mem, syn, ckpt, mem_final,
+  return scan_fwd(desc, kSynaptic, I, alpha, beta, thr, mem0, syn0, spk, mem, syn, ckpt, mem_final,
                   syn_final, ws, ws_bytes, (cudaStream_t)stream);
 }
 
@@ -358,9 +367,28 @@ snn_status_t snn_synaptic_bwd(const snn_scan_desc* desc, const void* I, const fl
                               float* grad_beta, float* grad_thr, float* grad_mem0,
                               float* grad_syn0, void* ws, size_t ws_bytes,
                               snn_stream_t stream) {
-  return scan_bwd(desc, true, I, ckpt, mem, spk, syn, alpha, beta, thr, mem0, syn0, grad_spk,
+  return scan_bwd(desc, kSynaptic, I, ckpt, mem, spk, syn, alpha, beta, thr, mem0, syn0, grad_spk,
                   grad_mem, grad_mem_final, grad_syn_final, grad_I, grad_alpha, grad_beta,
                   grad_thr, grad_mem0, grad_syn0, ws, ws_bytes, (cudaStream_t)stream);
+}
+
+snn_status_t snn_rleaky_fwd(const snn_scan_desc* desc, const void* I, const float* v,
+                            const float* beta, const float* thr, const float* mem0, void* spk,
+                            void* mem, float* ckpt, float* mem_final, void* ws, size_t ws_bytes,
+                            snn_stream_t stream) {
+  return scan_fwd(desc, kRecurrentLeaky, I, v, beta, thr, mem0, nullptr, spk, mem, nullptr, ckpt,
+                  mem_final, nullptr, ws, ws_bytes, (cudaStream_t)stream);
+}
+
+snn_status_t snn_rleaky_bwd(const snn_scan_desc* desc, const void* I, const float* ckpt,
+                            const void* mem, const void* spk, const float* v, const float* beta,
+                            const float* thr, const float* mem0, const void* grad_spk,
+                            const void* grad_mem, const float* grad_mem_final, void* grad_I,
+                            float* grad_v, float* grad_beta, float* grad_thr, float* grad_mem0,
+                            void* ws, size_t ws_bytes, snn_stream_t stream) {
+  return scan_bwd(desc, kRecurrentLeaky, I, ckpt, mem, spk, nullptr, v, beta, thr, mem0, nullptr,
+                  grad_spk, grad_mem, grad_mem_final, nullptr, grad_I, grad_v, grad_beta,
+                  grad_thr, grad_mem0, nullptr, ws, ws_bytes, (cudaStream_t)stream);
 }
 
 }  // extern "C"

@@ -70,6 +70,8 @@ _SIGS = {
     "snn_synaptic_fwd": ([ctypes.POINTER(ScanDesc)] + [_P] * 13 + [ctypes.c_size_t, _P], ctypes.c_int),
     "snn_synaptic_bwd": ([ctypes.POINTER(ScanDesc)] + [_P] * 21 + [ctypes.c_size_t, _P], ctypes.c_int),
     "snn_leaky_bwd_noalloc": ([ctypes.POINTER(ScanDesc)] + [_P] * 16, ctypes.c_int),
+    "snn_rleaky_fwd": ([ctypes.POINTER(ScanDesc)] + [_P] * 10 + [ctypes.c_size_t, _P], ctypes.c_int),
+    "snn_rleaky_bwd": ([ctypes.POINTER(ScanDesc)] + [_P] * 17 + [ctypes.c_size_t, _P], ctypes.c_int),
     "snn_dense_layer_fwd": ([ctypes.c_int64] * 3 + [_P] * 4 + [ctypes.c_size_t, _P], ctypes.c_int),
     "snn_dense_workspace_bytes": ([ctypes.c_int64] * 3, ctypes.c_size_t),
     "snn_dense_layer_bwd": ([ctypes.c_int64] * 3 + [_P] * 6 + [ctypes.c_size_t, _P], ctypes.c_int),
@@ -139,7 +141,7 @@ def make_desc(w: W.ScanWorkload, **over) -> ScanDesc:
     d.surrogate = SG_CODE[w.surrogate]
     d.sg_param = w.sg_param
     d.beta_mode, d.thr_mode = PMODE_CODE[w.beta_mode], PMODE_CODE[w.thr_mode]
-    d.alpha_mode = PMODE_CODE[w.alpha_mode]
+    d.alpha_mode = PMODE_CODE[w.v_mode if w.neuron == "rleaky" else w.alpha_mode]
     d.save = SAVE_CODE[w.save]
     d.ckpt_every = w.ckpt_every if w.save == "recompute" else 0
     for k, v in over.items():
@@ -202,6 +204,23 @@ def snn_synaptic_bwd(desc, I, ckpt, mem, spk, syn, alpha, beta, thr, mem0, syn0,
         _ptr(grad_mem_final), _ptr(grad_syn_final), _ptr(grad_I), _ptr(grad_alpha),
         _ptr(grad_beta), _ptr(grad_thr), _ptr(grad_mem0), _ptr(grad_syn0), _ptr(ws),
         ws.numel() * ws.element_size(), _stream(stream)), "snn_synaptic_bwd")
+
+
+def snn_rleaky_fwd(desc, I, v, beta, thr, mem0, spk, mem, ckpt, mem_final, ws, stream=None):
+    _check(load_library().snn_rleaky_fwd(
+        ctypes.byref(desc), _ptr(I), _ptr(v), _ptr(beta), _ptr(thr), _ptr(mem0), _ptr(spk),
+        _ptr(mem), _ptr(ckpt), _ptr(mem_final), _ptr(ws), ws.numel() * ws.element_size(),
+        _stream(stream)), "snn_rleaky_fwd")
+
+
+def snn_rleaky_bwd(desc, I, ckpt, mem, spk, v, beta, thr, mem0, grad_spk, grad_mem,
+                   grad_mem_final, grad_I, grad_v, grad_beta, grad_thr, grad_mem0, ws,
+                   stream=None):
+    _check(load_library().snn_rleaky_bwd(
+        ctypes.byref(desc), _ptr(I), _ptr(ckpt), _ptr(mem), _ptr(spk), _ptr(v), _ptr(beta),
+        _ptr(thr), _ptr(mem0), _ptr(grad_spk), _ptr(grad_mem), _ptr(grad_mem_final),
+        _ptr(grad_I), _ptr(grad_v), _ptr(grad_beta), _ptr(grad_thr), _ptr(grad_mem0), _ptr(ws),
+        ws.numel() * ws.element_size(), _stream(stream)), "snn_rleaky_bwd")
 
 
 def snn_leaky_bwd_noalloc(desc, I, ckpt, mem, spk, beta, thr, mem0, grad_spk, grad_mem,
@@ -277,6 +296,7 @@ class ScanLayer:
     def __init__(self, w: W.ScanWorkload, device="cuda", want_syn: bool = False, **desc_over):
         self.w = w
         self.synaptic = w.neuron == "synaptic"
+        self.recurrent = w.neuron == "rleaky"   # Eq. (7): v in the alpha slot
         self.desc = make_desc(w, **desc_over)
         self.device = torch.device(device)
         io = W.TORCH_DTYPE[w.io_dtype]
@@ -296,6 +316,8 @@ class ScanLayer:
         self.grad_thr = torch.empty(plen[w.thr_mode], dtype=torch.float32, device=dev)
         self.grad_alpha = torch.empty(plen[w.alpha_mode], dtype=torch.float32, device=dev) \
             if self.synaptic else None
+        self.grad_v = torch.empty(plen[w.v_mode], dtype=torch.float32, device=dev) \
+            if self.recurrent else None
         self.grad_mem0 = torch.empty((w.B, w.N), dtype=torch.float32, device=dev)
         self.grad_syn0 = torch.empty((w.B, w.N), dtype=torch.float32, device=dev) \
             if self.synaptic else None
@@ -305,8 +327,11 @@ class ScanLayer:
         self.ws = torch.empty(nws, dtype=torch.uint8, device=dev)
         snn_workspace_init(self.ws)
 
-    def forward(self, I, beta, thr, alpha=None, mem0=None, syn0=None, stream=None):
-        if self.synaptic:
+    def forward(self, I, beta, thr, alpha=None, mem0=None, syn0=None, stream=None, v=None):
+        if self.recurrent:
+            snn_rleaky_fwd(self.desc, I, v, beta, thr, mem0, self.spk, self.mem, self.ckpt,
+                           self.mem_final, self.ws, stream)
+        elif self.synaptic:
             snn_synaptic_fwd(self.desc, I, alpha, beta, thr, mem0, syn0, self.spk, self.mem,
                              self.syn, self.ckpt, self.mem_final, self.syn_final, self.ws, stream)
         else:
@@ -316,12 +341,17 @@ class ScanLayer:
 
     def backward(self, I, beta, thr, grad_spk, alpha=None, mem0=None, syn0=None, grad_mem=None,
                  grad_mem_final=None, grad_syn_final=None, want_param_grads=True,
-                 want_state_grads=True, stream=None):
+                 want_state_grads=True, stream=None, v=None):
         gb = self.grad_beta if want_param_grads else None
         gt = self.grad_thr if want_param_grads else None
         gm0 = self.grad_mem0 if want_state_grads else None
         recompute = self.w.save == "recompute"
-        if self.synaptic:
+        if self.recurrent:
+            snn_rleaky_bwd(self.desc, I if recompute else None, self.ckpt, self.mem, self.spk, v,
+                           beta, thr, mem0, grad_spk, grad_mem, grad_mem_final, self.grad_I,
+                           self.grad_v if want_param_grads else None, gb, gt, gm0, self.ws,
+                           stream)
+        elif self.synaptic:
             ga = self.grad_alpha if (want_param_grads and (recompute or self.syn is not None)) else None
             gs0 = self.grad_syn0 if want_state_grads else None
             snn_synaptic_bwd(self.desc, I if recompute else None, self.ckpt, self.mem, self.spk,

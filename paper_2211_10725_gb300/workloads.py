@@ -15,6 +15,8 @@ in for the datasets, which are not used):
                                 [12,24,24] and [64,8,8], per-channel beta.
 * ``leaky_bf16_T500_B64_N8192`` large Leaky layer, bf16 storage, per-neuron
                                 beta/threshold.
+* ``rleaky_T25_B128_N1000``     recurrent Leaky layer (Eq. 7), fp32, per-neuron v.
+* ``rleaky_bf16_T500_B64_N8192`` large recurrent Leaky layer, bf16 storage.
 """
 from __future__ import annotations
 
@@ -34,7 +36,7 @@ class ScanWorkload:
     """Shape and distribution of one scan layer's synthetic inputs."""
 
     name: str
-    neuron: str                 # "leaky" (Eq. 4) or "synaptic" (Eqs. 5-6)
+    neuron: str                 # "leaky" (Eq. 4), "synaptic" (Eqs. 5-6), "rleaky" (Eq. 7)
     T: int
     B: int
     N: int                      # flattened neurons per sample (C*H*W for conv maps)
@@ -50,6 +52,8 @@ class ScanWorkload:
     beta_mode: str = "scalar"   # scalar | per_neuron | per_channel
     thr_mode: str = "scalar"
     alpha_mode: str = "scalar"
+    v: tuple = ("uniform", -0.5, 0.5)   # recurrent weight (rleaky)
+    v_mode: str = "per_neuron"
     reset: str = "subtract"     # subtract | zero | none
     surrogate: str = "fast_sigmoid"     # fast_sigmoid | atan
     sg_param: float = 25.0
@@ -95,7 +99,14 @@ BIG_C5 = ScanWorkload(
     beta_mode="per_neuron", thr_mode="per_neuron", surrogate="atan", sg_param=2.0,
     save="recompute", ckpt_every=8, want_mem=False, seed_index=4)
 
-SCAN_WORKLOADS = {w.name: w for w in (LEAKY_C1, SYNAPTIC_C2, CONV_C4A, CONV_C4B, BIG_C5)}
+# Recurrent Leaky neuron (Eq. 7; the paper's recurrent SNN of Fig. 6a): the
+# C1 and C5 shapes with a one-to-one recurrent weight v ~ U(-0.5, 0.5) per
+# neuron.
+RLEAKY_C6 = LEAKY_C1.scaled(name="rleaky_T25_B128_N1000", neuron="rleaky", seed_index=6)
+RLEAKY_C7 = BIG_C5.scaled(name="rleaky_bf16_T500_B64_N8192", neuron="rleaky", seed_index=7)
+
+SCAN_WORKLOADS = {w.name: w for w in (LEAKY_C1, SYNAPTIC_C2, CONV_C4A, CONV_C4B, BIG_C5,
+                                      RLEAKY_C6, RLEAKY_C7)}
 
 
 def _gen(seed: int) -> torch.Generator:
@@ -122,7 +133,8 @@ def make_scan_inputs(w: ScanWorkload, seed: Optional[int] = None,
     Returns a dict of CPU tensors: ``I`` [T,B,N] in_dtype, ``grad_spk`` [T,B,N]
     io_dtype ~ N(0,1), ``beta``/``thr``/``alpha`` fp32 of length 1, N or C, and
     optionally ``mem0``/``syn0`` [B,N] fp32, ``grad_mem`` [T,B,N] io_dtype and
-    ``grad_mem_final``/``grad_syn_final`` [B,N] fp32.
+    ``grad_mem_final``/``grad_syn_final`` [B,N] fp32; ``v`` (length 1, N or
+    C) for the recurrent neuron.
     """
     seed = SEED_BASE + w.seed_index if seed is None else seed
     g = _gen(seed)
@@ -133,6 +145,8 @@ def make_scan_inputs(w: ScanWorkload, seed: Optional[int] = None,
     out["thr"] = _param(w.thr, w.thr_mode, w, g)
     if w.neuron == "synaptic":
         out["alpha"] = _param(w.alpha, w.alpha_mode, w, g)
+    if w.neuron == "rleaky":
+        out["v"] = _param(w.v, w.v_mode, w, g)
     out["grad_spk"] = torch.randn(shape, generator=g, dtype=torch.float32).to(
         TORCH_DTYPE[w.io_dtype])
     if with_mem0:

@@ -59,6 +59,7 @@ def oracle_expect(w: W.ScanWorkload, inp: dict, lanes=None, backward=True) -> di
     L = B * N
     idx = np.arange(L) if lanes is None else np.asarray(lanes)
     syn = w.neuron == "synaptic"
+    rec = w.neuron == "rleaky"
 
     def par(name, mode):
         full = O.lane_param(inp[name].numpy(), B, N, mode, C, HW)
@@ -66,6 +67,7 @@ def oracle_expect(w: W.ScanWorkload, inp: dict, lanes=None, backward=True) -> di
 
     beta, thr = par("beta", w.beta_mode), par("thr", w.thr_mode)
     alpha = par("alpha", w.alpha_mode) if syn else None
+    v = par("v", w.v_mode) if rec else None
     I = lanes_2d(inp["I"], idx)
     mem0 = lanes_1d(inp["mem0"], idx) if "mem0" in inp else None
     syn0 = lanes_1d(inp["syn0"], idx) if "syn0" in inp else None
@@ -75,6 +77,10 @@ def oracle_expect(w: W.ScanWorkload, inp: dict, lanes=None, backward=True) -> di
     if syn:
         spk32, mem32, syn32 = O.synaptic_forward(f32(I), f32(alpha), f32(beta), f32(thr), w.reset,
                                                  mem0=f32(mem0), syn0=f32(syn0), dtype=np.float32)
+    elif rec:
+        spk32, mem32 = O.rleaky_forward(f32(I), f32(v), f32(beta), f32(thr), mem0=f32(mem0),
+                                        dtype=np.float32)
+        syn32 = None
     else:
         spk32, mem32 = O.leaky_forward(f32(I), f32(beta), f32(thr), w.reset, mem0=f32(mem0),
                                        dtype=np.float32)
@@ -86,11 +92,14 @@ def oracle_expect(w: W.ScanWorkload, inp: dict, lanes=None, backward=True) -> di
     if syn:
         _, mem64, syn64 = O.synaptic_forward(I, alpha, beta, thr, w.reset, mem0=mem0, syn0=syn0,
                                              z_reset=z_reset)
+    elif rec:
+        _, mem64 = O.rleaky_forward(I, v, beta, thr, mem0=mem0, z_path=z_reset)
+        syn64 = None
     else:
         _, mem64 = O.leaky_forward(I, beta, thr, w.reset, mem0=mem0, z_reset=z_reset)
         syn64 = None
     out = {"lanes": idx, "spk32": spk32.astype(np.float64), "mem32": mem32.astype(np.float64),
-           "mem64": mem64, "thr": thr, "beta": beta, "alpha": alpha, "I": I,
+           "mem64": mem64, "thr": thr, "beta": beta, "alpha": alpha, "v": v, "I": I,
            "mem0": mem0, "syn0": syn0, "reset": w.reset}
     if syn:
         out["syn32"], out["syn64"] = syn32.astype(np.float64), syn64
@@ -109,6 +118,9 @@ def oracle_expect(w: W.ScanWorkload, inp: dict, lanes=None, backward=True) -> di
         syn_b = out["syn32"] if w.save == "recompute" else round_to(w.io_dtype, out["syn32"])
         g = O.synaptic_backward(mem_b, out["spk32"], syn_b, gs, alpha, beta, thr, syn0=syn0,
                                 grad_syn_final=gsf, **kw)
+    elif rec:
+        kr = {k: kw[k] for k in kw if k != "reset"}
+        g = O.rleaky_backward(mem_b, out["spk32"], gs, v, beta, thr, **kr)
     else:
         g = O.leaky_backward(mem_b, out["spk32"], gs, beta, thr, **kw)
     out.update(g)
@@ -121,6 +133,12 @@ def oracle_expect(w: W.ScanWorkload, inp: dict, lanes=None, backward=True) -> di
         ga = O.synaptic_backward(mem_b, out["spk32"], syn_b, np.abs(gs), alpha, beta, thr,
                                  syn0=syn0, grad_syn_final=ab(gsf), **kwa)
         out["grad_syn0_scale"] = np.maximum(ga["grad_syn0"], np.abs(g["grad_syn0"]))
+    elif rec:
+        # |v| (+ thr for a live reset) as the spike's coefficient keeps every
+        # term of the absolute-value pass non-negative
+        va = np.abs(v) + (0.0 if w.detach_reset else np.abs(thr))
+        kra = {k: kwa[k] for k in kwa if k != "reset"}
+        ga = O.rleaky_backward(mem_b, out["spk32"], np.abs(gs), va, beta, thr, **kra)
     else:
         ga = O.leaky_backward(mem_b, out["spk32"], np.abs(gs), beta, thr, **kwa)
     out["grad_I_scale"] = np.maximum(ga["grad_I"], np.abs(g["grad_I"]))
@@ -130,6 +148,8 @@ def oracle_expect(w: W.ScanWorkload, inp: dict, lanes=None, backward=True) -> di
         out["grad_thr"] = O.reduce_lane_grad(g["grad_thr_lane"], B, N, w.thr_mode, C, HW)
         if syn:
             out["grad_alpha"] = O.reduce_lane_grad(g["grad_alpha_lane"], B, N, w.alpha_mode, C, HW)
+        if rec:
+            out["grad_v"] = O.reduce_lane_grad(g["grad_v_lane"], B, N, w.v_mode, C, HW)
     return out
 
 
@@ -162,6 +182,8 @@ def fp32_trace_bound(ref) -> tuple:
         decayed = beta * keep * u_prev
         eu = beta * keep * eu + (ei if syn else 0.0) + EPS32 * (
             np.abs(decayed) + np.abs(decayed + x) + np.abs(u64[t]))
+        if ref.get("v") is not None:  # v - thr is rounded once in fp32
+            eu = eu + z_prev * EPS32 * np.abs(ref["v"] - ref["thr"])
         bu[t] = eu
         u_prev, z_prev = u64[t], z[t]
     return bu, bi
@@ -225,11 +247,12 @@ def run_gpu(w: W.ScanWorkload, inp: dict, device="cuda", **desc_over):
     from paper_2211_10725_gb300 import snn
     d = {k: v.to(device) for k, v in inp.items()}
     layer = snn.ScanLayer(w, device=device, want_syn=True, **desc_over)
-    layer.forward(d["I"], d["beta"], d["thr"], d.get("alpha"), d.get("mem0"), d.get("syn0"))
+    layer.forward(d["I"], d["beta"], d["thr"], d.get("alpha"), d.get("mem0"), d.get("syn0"),
+                  v=d.get("v"))
     layer.backward(d["I"], d["beta"], d["thr"], d["grad_spk"], alpha=d.get("alpha"),
                    mem0=d.get("mem0"), syn0=d.get("syn0"), grad_mem=d.get("grad_mem"),
                    grad_mem_final=d.get("grad_mem_final"),
-                   grad_syn_final=d.get("grad_syn_final"))
+                   grad_syn_final=d.get("grad_syn_final"), v=d.get("v"))
     torch.cuda.synchronize()
     return layer
 
@@ -257,4 +280,7 @@ def check_all(w: W.ScanWorkload, inp: dict, layer, ref: dict, lanes=None):
         if syn:
             check_param_grad("grad_alpha", lanes_1d(layer.grad_alpha), ref["grad_alpha"],
                              ref["grad_alpha_lane"], B, N, w.alpha_mode, C, HW)
+        if w.neuron == "rleaky":
+            check_param_grad("grad_v", lanes_1d(layer.grad_v), ref["grad_v"],
+                             ref["grad_v_lane"], B, N, w.v_mode, C, HW)
     return amb

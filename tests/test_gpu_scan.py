@@ -207,3 +207,76 @@ def test_ring_wraps_with_many_warps(neuron, dt, save, cuda_device):
     rng = np.random.default_rng(9)
     lanes = np.sort(rng.choice(w.B * w.N, 20000, replace=False))
     H.check_all(w, inp, layer, H.oracle_expect(w, inp, lanes=lanes), lanes=lanes)
+
+
+# ---------------------------------------------------------------------------
+# Recurrent Leaky neuron (Eq. 7)
+# ---------------------------------------------------------------------------
+
+def rleaky_case(i):
+    T, B, N = SHAPES[i % len(SHAPES)]
+    C, HW = CHANNELS[N]
+    in_dt, io_dt = DTYPES[(i // 3) % len(DTYPES)]
+    w = W.ScanWorkload(
+        name=f"rleaky{i}", neuron="rleaky", T=T, B=B, N=N, C=C, HW=HW, in_dtype=in_dt,
+        io_dtype=io_dt, i_mean=0.5, i_std=0.6, beta=("uniform", 0.5, 0.95),
+        thr=("uniform", 0.6, 1.4), v=("uniform", -0.6, 0.6),
+        beta_mode=MODES[(i // 5) % 3], thr_mode=MODES[(i // 2) % 3], v_mode=MODES[i % 3],
+        detach_reset=(i % 2 == 0), surrogate=["fast_sigmoid", "atan"][(i // 4) % 2],
+        sg_param=[25.0, 2.0][(i // 4) % 2], save=["mem", "recompute"][(i // 6) % 2],
+        ckpt_every=[8, 3][(i // 12) % 2], want_mem=True, seed_index=300 + i)
+    opts = dict(with_mem0=(i % 4 == 1), with_grad_mem=(i % 5 == 2), with_grad_final=(i % 3 == 1))
+    return w, opts
+
+
+@pytest.mark.parametrize("i", range(24))
+def test_rleaky_small_cases(i, cuda_device):
+    w, opts = rleaky_case(i)
+    inp = W.make_scan_inputs(w, **opts)
+    layer = H.run_gpu(w, inp)
+    assert layer.status() == 0
+    H.check_all(w, inp, layer, H.oracle_expect(w, inp))
+
+
+@pytest.mark.parametrize("i", [2, 3, 8, 9, 15, 20])
+def test_rleaky_staged_and_plain_kernels_agree(i, cuda_device):
+    w, opts = rleaky_case(i)
+    inp = W.make_scan_inputs(w, **opts)
+    a = H.run_gpu(w, inp)
+    b = H.run_gpu(w, inp, debug_flags=snn.DEBUG_FORCE_PLAIN)
+    assert torch.equal(a.spk, b.spk) and torch.equal(a.mem, b.mem)
+    assert torch.equal(a.mem_final, b.mem_final)
+    H.assert_close("grad_I", H.lanes_2d(a.grad_I), H.lanes_2d(b.grad_I), *H.TOL[w.io_dtype])
+
+
+def test_rleaky_zero_reset_is_unsupported(cuda_device):
+    w = W.RLEAKY_C6.scaled(T=2, B=2, N=8, reset="zero")
+    layer = snn.ScanLayer(w, device=cuda_device)
+    inp = {k: t.to(cuda_device) for k, t in W.make_scan_inputs(w).items()}
+    with pytest.raises(snn.SnnError):
+        layer.forward(inp["I"], inp["beta"], inp["thr"], v=inp["v"])
+
+
+def test_rleaky_full_size(cuda_device):
+    w = W.RLEAKY_C6
+    inp = W.make_scan_inputs(w)
+    layer = H.run_gpu(w, inp)
+    assert layer.status() == 0
+    H.check_all(w, inp, layer, H.oracle_expect(w, inp))
+
+
+@pytest.mark.parametrize("save", ["recompute", "mem"])
+def test_rleaky_full_size_large_bf16(save, cuda_device):
+    w = W.RLEAKY_C7.scaled(save=save)
+    inp = W.make_scan_inputs(w)
+    layer = H.run_gpu(w, inp)
+    assert layer.status() == 0
+    rng = np.random.default_rng(6)
+    ns = np.unique(np.concatenate([np.sort(rng.choice(w.N, 24, replace=False)), [0, w.N - 1]]))
+    lanes = (np.arange(w.B)[:, None] * w.N + ns[None, :]).reshape(-1)
+    ref = H.oracle_expect(w, inp, lanes=lanes)
+    H.check_all(w, inp, layer, ref, lanes=lanes)
+    for pname in ("beta", "thr", "v"):
+        part = ref[f"grad_{pname}_lane"].reshape(w.B, len(ns))
+        got = H.lanes_1d(getattr(layer, f"grad_{pname}"))[ns]
+        H.assert_close(f"grad_{pname}", got, part.sum(0), 1e-5, 1e-5 * np.abs(part).sum(0) + 1e-6)

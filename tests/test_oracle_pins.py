@@ -509,6 +509,10 @@ def test_rleaky_special_cases_reduce_to_leaky():
         g1 = O.leaky_backward(m1, s1, gs, beta, thr, "subtract", detach=detach, **kw)
         for k in ("grad_I", "grad_beta_lane", "grad_thr_lane", "grad_mem0"):
             np.testing.assert_allclose(g0[k], g1[k], rtol=1e-13, atol=1e-15)
+    # following the free run's own spike path reproduces it
+    zp = np.vstack([np.zeros((1, L)), s0[:-1]])
+    s4, m4 = O.rleaky_forward(I, np.zeros(L), beta, thr, z_path=zp)
+    assert np.array_equal(s4, s0) and np.array_equal(m4, m0)
     s2, m2 = O.rleaky_forward(I, thr, beta, thr)
     s3, m3 = O.leaky_forward(I, beta, thr, "none")
     assert np.array_equal(s2, s3)
