@@ -100,7 +100,8 @@ def hbm_peak():
 
 
 SCAN_SOURCES = ("scan_kernels.cuh", "scan_dispatch.cuh", "scan_host.cuh", "snn_device.cuh",
-                "scan_fwd.cu", "scan_bwd_leaky.cu", "scan_bwd_synaptic.cu", "snn_api.cu")
+                "scan_fwd.cu", "scan_bwd_leaky.cu", "scan_bwd_leaky_recompute.cu",
+                "scan_bwd_synaptic.cu", "scan_bwd_synaptic_recompute.cu", "snn_api.cu")
 
 
 def kernel_source_hash():
@@ -205,7 +206,8 @@ def oracle_inputs(w, inp):
     T, B, N = w.T, w.B, w.N
     host = {"I": inp["I"].float().numpy().reshape(T, B * N),
             "gs": inp["grad_spk"].float().numpy().reshape(T, B * N)}
-    for name, mode in (("beta", w.beta_mode), ("thr", w.thr_mode), ("alpha", w.alpha_mode)):
+    for name, mode in (("beta", w.beta_mode), ("thr", w.thr_mode), ("alpha", w.alpha_mode),
+                       ("v", w.v_mode)):
         if name in inp:
             host[name] = O.lane_param(inp[name].numpy(), B, N, mode, w.C, w.HW)
     return host
@@ -223,6 +225,10 @@ def oracle_step(w, host, lanes):
         spk, mem, syn = O.synaptic_forward(I, alpha, beta, thr, w.reset)
         O.synaptic_backward(mem, spk, syn, gs, alpha, beta, thr, w.reset, w.detach_reset,
                             w.surrogate, w.sg_param)
+    elif w.neuron == "rleaky":
+        v = host["v"][lanes]
+        spk, mem = O.rleaky_forward(I, v, beta, thr)
+        O.rleaky_backward(mem, spk, gs, v, beta, thr, w.detach_reset, w.surrogate, w.sg_param)
     else:
         spk, mem = O.leaky_forward(I, beta, thr, w.reset)
         O.leaky_backward(mem, spk, gs, beta, thr, w.reset, w.detach_reset, w.surrogate,
@@ -362,9 +368,9 @@ def run_ours(args):
     stream = torch.cuda.current_stream(dev)
 
     def step():
-        layer.forward(d["I"], d["beta"], d["thr"], d.get("alpha"))
+        layer.forward(d["I"], d["beta"], d["thr"], d.get("alpha"), v=d.get("v"))
         layer.backward(d["I"], d["beta"], d["thr"], d["grad_spk"], alpha=d.get("alpha"),
-                       want_state_grads=False)
+                       want_state_grads=False, v=d.get("v"))
 
     for _ in range(args.warmup):
         step()
@@ -385,10 +391,10 @@ def run_ours(args):
     t_wall0 = time.time()
     ev[0].record(stream)
     for k in range(K):
-        layer.forward(d["I"], d["beta"], d["thr"], d.get("alpha"))
+        layer.forward(d["I"], d["beta"], d["thr"], d.get("alpha"), v=d.get("v"))
         ev[3 * k + 1].record(stream)
         layer.backward(d["I"], d["beta"], d["thr"], d["grad_spk"], alpha=d.get("alpha"),
-                       want_state_grads=False)
+                       want_state_grads=False, v=d.get("v"))
         ev[3 * k + 2].record(stream)
         ev[3 * k + 3].record(stream)
     torch.cuda.synchronize()
@@ -429,8 +435,10 @@ def run_ours(args):
     kernel_key = f"scan_bwd_staged[{w.neuron},{w.save}]"  # dominant kernel
     traffic = profiled_traffic(kernel_key, w.name)
     clocks = sampler.summary(t_wall0, t_wall1)
-    # forward scan + backward scan + a two-stage reduction per parameter gradient
-    launches_per_step = 2 + 2 * 2
+    # forward scan + backward scan + a two-stage reduction per parameter
+    # gradient (beta, thr, and alpha or v for the Synaptic / recurrent neuron)
+    n_param_grads = 3 if w.neuron in ("synaptic", "rleaky") else 2
+    launches_per_step = 2 + 2 * n_param_grads
     cpu = None
     if not args.no_cpu_baseline and world == 1:
         v, n, dt = time_oracle(w, inp, args.cpu_seconds)
@@ -742,6 +750,7 @@ def run_e2e(args, w, inp, layer, dev, world):
     dG = torch.empty_like(hG, device=dev)
     beta, thr = inp["beta"].to(dev), inp["thr"].to(dev)
     alpha = inp["alpha"].to(dev) if "alpha" in inp else None
+    v = inp["v"].to(dev) if "v" in inp else None
     out_spk = torch.empty_like(layer.spk, device="cpu").pin_memory()
     out_gI = torch.empty_like(layer.grad_I, device="cpu").pin_memory()
     out_gb = torch.empty_like(layer.grad_beta, device="cpu").pin_memory()
@@ -751,8 +760,8 @@ def run_e2e(args, w, inp, layer, dev, world):
     def step():
         dI.copy_(hI, non_blocking=True)
         dG.copy_(hG, non_blocking=True)
-        layer.forward(dI, beta, thr, alpha)
-        layer.backward(dI, beta, thr, dG, alpha=alpha, want_state_grads=False)
+        layer.forward(dI, beta, thr, alpha, v=v)
+        layer.backward(dI, beta, thr, dG, alpha=alpha, want_state_grads=False, v=v)
         out_spk.copy_(layer.spk, non_blocking=True)
         out_gI.copy_(layer.grad_I, non_blocking=True)
         out_gb.copy_(layer.grad_beta, non_blocking=True)

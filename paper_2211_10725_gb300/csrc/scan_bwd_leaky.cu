@@ -1,11 +1,13 @@
-// BPTT launchers for the Leaky neuron (store and recompute variants).
+// BPTT launchers for the Leaky neuron: the store variant here, the
+// recompute variant in scan_bwd_leaky_recompute.cu (separate translation
+// units compile in parallel).
 #include "scan_dispatch.cuh"
 
 namespace snn {
 
-cudaError_t launch_scan_bwd_leaky(ScanArgs a, bool recompute, int in_dt, int io_dt, bool staged,
-                                  cudaStream_t stream) {
-  if (recompute) SNN_DTYPE_DISPATCH(in_dt, io_dt, return (bwd_t<false, true, TI, TO>(a, staged, stream)));
+cudaError_t launch_scan_bwd_leaky(ScanArgs a, bool recompute, int in_dt, int io_dt,
+                                  bool staged, cudaStream_t stream) {
+  if (recompute) return launch_scan_bwd_leaky_recompute(a, in_dt, io_dt, staged, stream);
   SNN_DTYPE_DISPATCH(in_dt, io_dt, return (bwd_t<false, false, TI, TO>(a, staged, stream)));
 }
 

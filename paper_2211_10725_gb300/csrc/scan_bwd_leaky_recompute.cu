@@ -1,0 +1,12 @@
+// BPTT launchers for the Leaky neuron, recompute variant (checkpointed
+// replay of the forward inside the reverse pass).
+#include "scan_dispatch.cuh"
+
+namespace snn {
+
+cudaError_t launch_scan_bwd_leaky_recompute(ScanArgs a, int in_dt, int io_dt, bool staged,
+                                            cudaStream_t stream) {
+  SNN_DTYPE_DISPATCH(in_dt, io_dt, return (bwd_t<false, true, TI, TO>(a, staged, stream)));
+}
+
+}  // namespace snn

@@ -83,7 +83,15 @@ cudaError_t bwd_t(ScanArgs a, bool staged, cudaStream_t st) {
     cudaError_t e = cudaSuccess;
     bool done = false;
     if (!SYN && a.rec) {  // recurrent Leaky neuron: reset by subtraction (Eq. 7)
-      e = bwd_staged<false, RECOMP, TI, TO, RESET_SUBTRACT, -1, 0, true>(a, st, &launched);
+      if constexpr (kSpecialise<TI, TO>) {
+        if (a.sg == SG_ATAN)
+          e = bwd_staged<false, RECOMP, TI, TO, RESET_SUBTRACT, SG_ATAN, 0, true>(a, st, &launched);
+        else
+          e = bwd_staged<false, RECOMP, TI, TO, RESET_SUBTRACT, SG_FAST_SIGMOID, 0, true>(a, st,
+                                                                                      &launched);
+      } else {
+        e = bwd_staged<false, RECOMP, TI, TO, RESET_SUBTRACT, -1, 0, true>(a, st, &launched);
+      }
       done = true;
     } else if constexpr (kSpecialise<TI, TO>) {
       done = true;

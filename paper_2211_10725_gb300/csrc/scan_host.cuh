@@ -148,6 +148,11 @@ cudaError_t launch_scan_bwd_leaky(ScanArgs a, bool recompute, int in_dt, int io_
                                   cudaStream_t stream);
 cudaError_t launch_scan_bwd_synaptic(ScanArgs a, bool recompute, int in_dt, int io_dt,
                                      bool staged, cudaStream_t stream);
+// the recompute variants, compiled in translation units of their own
+cudaError_t launch_scan_bwd_leaky_recompute(ScanArgs a, int in_dt, int io_dt, bool staged,
+                                            cudaStream_t stream);
+cudaError_t launch_scan_bwd_synaptic_recompute(ScanArgs a, int in_dt, int io_dt, bool staged,
+                                               cudaStream_t stream);
 // fp64 scratch the reduction of one parameter needs (elements)
 inline int64_t param_reduce_scratch(int64_t N, int64_t C) {
   const int64_t a = 1024, b = 8 * N, c = 64 * C;
