@@ -252,7 +252,8 @@ snn_status_t snn_synaptic_bwd(const snn_scan_desc* desc, const void* I, const fl
 snn_status_t snn_dense_layer_fwd(int64_t M, int64_t K, int64_t N, const void* X, const void* W,
                                  float* I, void* ws, size_t ws_bytes, snn_stream_t stream);
 
-/* Workspace bytes of snn_dense_layer_bwd (transposed operand copies). */
+/* Workspace bytes of snn_dense_layer_bwd (a status word; the operands are
+ * read in place, W and X and dI through MN-major tensor-core tiles). */
 size_t snn_dense_workspace_bytes(int64_t M, int64_t K, int64_t N);
 
 /*

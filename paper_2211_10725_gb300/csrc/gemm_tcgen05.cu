@@ -12,9 +12,13 @@
 // is bounded; a kernel that gives up records SNN_ERR_TIMEOUT and still
 // drains its copies and frees its TMEM.
 //
-// The backward products dX = dI*W and dW = dI^T*X use the same kernel on
-// transposed copies (made by a tiled transpose kernel) so both operands stay
-// K-major.
+// Either operand may instead be stored MN-major (its M or N index
+// contiguous, K the row index): the backward products dX = dI*W (W read
+// MN-major) and dW = dI^T*X (dI and X read MN-major) then run on the stored
+// matrices without transposed copies.  An MN-major tile is loaded as
+// 64-element-wide TMA boxes (64 MN x 64 K, 128-byte swizzle) and described
+// to the tensor core as atoms of 8 K-rows of 128 bytes: 1024 bytes apart
+// along K, one box (8 KB) apart along MN.
 #include <cuda.h>
 #include <cudaTypedefs.h>
 #include <cuda_bf16.h>
@@ -78,11 +82,30 @@ __device__ __forceinline__ uint64_t sdesc_sw128(const void* tile) {
   return d;
 }
 
-// Instruction descriptor: bf16 x bf16 -> fp32, both operands K-major.
-__host__ __device__ constexpr uint32_t idesc_bf16(int m, int n) {
+// Descriptor of an MN-major operand tile: 64-element (128-byte) rows along
+// MN for consecutive K; atoms of 8 K-rows (1024 bytes) repeat along K every
+// 1024 bytes and along MN every 64x64 box (8192 bytes).
+constexpr uint32_t kMnBoxBytes = 64 * BK * 2;
+__device__ __forceinline__ uint64_t sdesc_sw128_mn(const void* tile) {
+  const uint32_t addr = smem_u32(tile);
+  uint64_t d = 0;
+  d |= (uint64_t)((addr >> 4) & 0x3FFFu);      // start address
+  d |= (uint64_t)(kMnBoxBytes >> 4) << 16;      // leading byte offset: next 64 along MN
+  d |= (uint64_t)(1024u >> 4) << 32;            // stride byte offset: next 8 along K
+  d |= (uint64_t)1 << 46;                       // descriptor version
+  d |= (uint64_t)2 << 61;                       // 128-byte swizzle
+  return d;
+}
+
+// Instruction descriptor: bf16 x bf16 -> fp32; each operand K-major or
+// (a_mn / b_mn) MN-major.
+__host__ __device__ constexpr uint32_t idesc_bf16(int m, int n, bool a_mn = false,
+                                                  bool b_mn = false) {
   return (1u << 4)                         // D format: f32
          | (1u << 7)                       // A format: bf16
          | (1u << 10)                      // B format: bf16
+         | ((a_mn ? 1u : 0u) << 15)        // A major-ness: MN
+         | ((b_mn ? 1u : 0u) << 16)        // B major-ness: MN
          | ((uint32_t)(n >> 3) << 17)      // N / 8
          | ((uint32_t)(m >> 4) << 24);     // M / 16
 }
@@ -156,11 +179,12 @@ __host__ __device__ constexpr size_t smem_bytes() {
 // Kernel
 // ---------------------------------------------------------------------------
 
-template <int BN, bool OUT_BF16>
+template <int BN, bool OUT_BF16, bool A_MN = false, bool B_MN = false>
 __global__ void __launch_bounds__(kThreads, 1)
     gemm_tn_tcgen05(const __grid_constant__ CUtensorMap ta, const __grid_constant__ CUtensorMap tb,
                     const GemmArgs g) {
   static_assert(BN % 16 == 0 && BN >= 16 && BN <= 256, "UMMA N for M=128");
+  static_assert(!B_MN || BN % 64 == 0, "an MN-major B tile is whole 64-wide boxes");
   constexpr int A_BYTES = BM * BK * 2;
   constexpr int B_BYTES = BN * BK * 2;
   constexpr uint32_t TCOLS = tmem_cols<BN>();
@@ -202,8 +226,20 @@ __global__ void __launch_bounds__(kThreads, 1)
           break;
         }
         mbar_arrive_expect_tx(&full[s], A_BYTES + B_BYTES);
-        tma_load_2d(sA + s * A_BYTES, &ta, kb * BK, m0, &full[s]);
-        tma_load_2d(sB + s * B_BYTES, &tb, kb * BK, n0, &full[s]);
+        if (A_MN) {
+#pragma unroll
+          for (int j = 0; j < BM / 64; ++j)
+            tma_load_2d(sA + s * A_BYTES + j * kMnBoxBytes, &ta, m0 + 64 * j, kb * BK, &full[s]);
+        } else {
+          tma_load_2d(sA + s * A_BYTES, &ta, kb * BK, m0, &full[s]);
+        }
+        if (B_MN) {
+#pragma unroll
+          for (int j = 0; j < BN / 64; ++j)
+            tma_load_2d(sB + s * B_BYTES + j * kMnBoxBytes, &tb, n0 + 64 * j, kb * BK, &full[s]);
+        } else {
+          tma_load_2d(sB + s * B_BYTES, &tb, kb * BK, n0, &full[s]);
+        }
         ++issued;
       }
       // every copy this thread issued has landed before the CTA may exit
@@ -212,7 +248,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
   } else if (warp == 1) {
     if (lid == 0) {
-      constexpr uint32_t idesc = idesc_bf16(BM, BN);
+      constexpr uint32_t idesc = idesc_bf16(BM, BN, A_MN, B_MN);
       for (int kb = 0; kb < nk; ++kb) {
         const int s = kb % kStages;
         if (!mbar_wait_bounded(&full[s], (uint32_t)((kb / kStages) & 1), g.wait_ns)) {
@@ -220,11 +256,15 @@ __global__ void __launch_bounds__(kThreads, 1)
           break;
         }
         tc_fence_after();
-        const uint64_t da = sdesc_sw128(sA + s * A_BYTES);
-        const uint64_t db = sdesc_sw128(sB + s * B_BYTES);
+        const uint64_t da = A_MN ? sdesc_sw128_mn(sA + s * A_BYTES) : sdesc_sw128(sA + s * A_BYTES);
+        const uint64_t db = B_MN ? sdesc_sw128_mn(sB + s * B_BYTES) : sdesc_sw128(sB + s * B_BYTES);
+        // 16 more along K: 32 bytes inside a K-major row, or 16 rows (2048
+        // bytes) of an MN-major tile; the descriptor holds the address >> 4
+        constexpr uint64_t stepA = A_MN ? 2048 >> 4 : 32 >> 4;
+        constexpr uint64_t stepB = B_MN ? 2048 >> 4 : 32 >> 4;
 #pragma unroll
-        for (int kk = 0; kk < BK / 16; ++kk)  // 16 bf16 = 32 bytes further along K
-          tc_mma(tmem, da + 2 * kk, db + 2 * kk, idesc, (kb | kk) != 0 ? 1u : 0u);
+        for (int kk = 0; kk < BK / 16; ++kk)
+          tc_mma(tmem, da + stepA * kk, db + stepB * kk, idesc, (kb | kk) != 0 ? 1u : 0u);
         tc_commit(&empty[s]);  // the stage is free once these MMAs are done
       }
       tc_commit(accum);  // the accumulator is final once every MMA is done
@@ -283,23 +323,6 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
 }
 
-// bf16 [R, C] row-major -> [C, R] row-major, 32x32 tiles through shared memory.
-__global__ void __launch_bounds__(256) transpose_bf16(const __nv_bfloat16* in, __nv_bfloat16* out,
-                                                      int R, int C) {
-  __shared__ __nv_bfloat16 tile[32][34];
-  const int bx = blockIdx.x * 32, by = blockIdx.y * 32;
-  const int tx = threadIdx.x & 31, ty = threadIdx.x >> 5;  // 32 x 8
-  for (int j = ty; j < 32; j += 8) {
-    const int r = by + j, c = bx + tx;
-    if (r < R && c < C) tile[j][tx] = in[(int64_t)r * C + c];
-  }
-  __syncthreads();
-  for (int j = ty; j < 32; j += 8) {
-    const int r = bx + j, c = by + tx;  // output row = input column
-    if (r < C && c < R) out[(int64_t)r * R + c] = tile[tx][j];
-  }
-}
-
 // ---------------------------------------------------------------------------
 // Host side
 // ---------------------------------------------------------------------------
@@ -319,55 +342,66 @@ PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
 }
 
 // Tensor map of a bf16 row-major [rows, cols] matrix read as box_rows x 64
-// tiles with 128-byte swizzle; out-of-range elements read as zero.
+// tiles (box_cols = 64 elements = 128 bytes across a row) with 128-byte
+// swizzle; out-of-range elements read as zero.  A K-major operand is read
+// as rows of its M/N index; an MN-major one as 64 x 64 boxes.
 bool make_map(CUtensorMap* map, const void* base, int64_t rows, int64_t cols, int box_rows) {
   auto fn = encode_fn();
   if (!fn) return false;
   const cuuint64_t dims[2] = {(cuuint64_t)cols, (cuuint64_t)rows};
   const cuuint64_t strides[1] = {(cuuint64_t)cols * 2};
-  const cuuint32_t box[2] = {(cuuint32_t)BK, (cuuint32_t)box_rows};
+  const cuuint32_t box[2] = {64u, (cuuint32_t)box_rows};
   const cuuint32_t estr[2] = {1, 1};
   return fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box,
             estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
             CU_TENSOR_MAP_L2_PROMOTION_L2_128B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-template <int BN, bool OUT_BF16>
+template <int BN, bool OUT_BF16, bool A_MN, bool B_MN>
 cudaError_t launch_bn(const CUtensorMap& ta, const CUtensorMap& tb, const GemmArgs& g,
                       cudaStream_t st) {
-  const void* k = (const void*)gemm_tn_tcgen05<BN, OUT_BF16>;
+  const void* k = (const void*)gemm_tn_tcgen05<BN, OUT_BF16, A_MN, B_MN>;
   const cudaError_t attr = ensure_smem(k, smem_bytes<BN>());  // once per device
   if (attr != cudaSuccess) return attr;
   const dim3 grid((unsigned)((g.N + BN - 1) / BN), (unsigned)((g.M + BM - 1) / BM));
-  gemm_tn_tcgen05<BN, OUT_BF16><<<grid, kThreads, smem_bytes<BN>(), st>>>(ta, tb, g);
+  gemm_tn_tcgen05<BN, OUT_BF16, A_MN, B_MN><<<grid, kThreads, smem_bytes<BN>(), st>>>(ta, tb, g);
   return cudaGetLastError();
 }
 
-// D[M, N] = A[M, K] * B[N, K]^T with the widest N tile that the output needs.
-template <bool OUT_BF16>
+// D[M, N] = A[M, K] * B[N, K]^T.  A is stored [M, K] row-major (K-major) or,
+// with A_MN, [K, M] row-major; B likewise [N, K] or, with B_MN, [K, N].
+// N tile: the widest the output needs (64 or 128 for an MN-major B), and 64
+// rather than 128 when 128-wide tiles would leave most SMs idle.
+template <bool OUT_BF16, bool A_MN = false, bool B_MN = false>
 cudaError_t gemm_tn(const void* A, const void* B, void* D, int M, int N, int K, int* status,
                     cudaStream_t st) {
   int bn = 128;
-  if (N <= 16) bn = 16;
-  else if (N <= 32) bn = 32;
+  if (N <= 16 && !B_MN) bn = 16;
+  else if (N <= 32 && !B_MN) bn = 32;
   else if (N <= 64) bn = 64;
-  CUtensorMap ta, tb;
-  if (!make_map(&ta, A, M, K, BM) || !make_map(&tb, B, N, K, bn)) return cudaErrorInvalidValue;
-  GemmArgs g{M, N, K, D, (int64_t)N, status, kDefaultWaitNs};
-  switch (bn) {
-    case 16: return launch_bn<16, OUT_BF16>(ta, tb, g, st);
-    case 32: return launch_bn<32, OUT_BF16>(ta, tb, g, st);
-    case 64: return launch_bn<64, OUT_BF16>(ta, tb, g, st);
-    default: return launch_bn<128, OUT_BF16>(ta, tb, g, st);
+  else {
+    int dev = 0, sms = 152;
+    if (cudaGetDevice(&dev) == cudaSuccess)
+      cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    const int64_t tiles128 = (int64_t)((N + 127) / 128) * ((M + BM - 1) / BM);
+    if (tiles128 < sms) bn = 64;
   }
-}
-
-cudaError_t transpose(const void* in, void* out, int R, int C, cudaStream_t st) {
-  if (R == 0 || C == 0) return cudaSuccess;
-  const dim3 grid((unsigned)((C + 31) / 32), (unsigned)((R + 31) / 32));
-  transpose_bf16<<<grid, 256, 0, st>>>(static_cast<const __nv_bfloat16*>(in),
-                                       static_cast<__nv_bfloat16*>(out), R, C);
-  return cudaGetLastError();
+  CUtensorMap ta, tb;
+  const bool okA = A_MN ? make_map(&ta, A, K, M, 64) : make_map(&ta, A, M, K, BM);
+  const bool okB = B_MN ? make_map(&tb, B, K, N, 64) : make_map(&tb, B, N, K, bn);
+  if (!okA || !okB) return cudaErrorInvalidValue;
+  GemmArgs g{M, N, K, D, (int64_t)N, status, kDefaultWaitNs};
+  if constexpr (B_MN) {
+    if (bn == 64) return launch_bn<64, OUT_BF16, A_MN, B_MN>(ta, tb, g, st);
+    return launch_bn<128, OUT_BF16, A_MN, B_MN>(ta, tb, g, st);
+  } else {
+    switch (bn) {
+      case 16: return launch_bn<16, OUT_BF16, A_MN, B_MN>(ta, tb, g, st);
+      case 32: return launch_bn<32, OUT_BF16, A_MN, B_MN>(ta, tb, g, st);
+      case 64: return launch_bn<64, OUT_BF16, A_MN, B_MN>(ta, tb, g, st);
+      default: return launch_bn<128, OUT_BF16, A_MN, B_MN>(ta, tb, g, st);
+    }
+  }
 }
 
 bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
@@ -388,8 +422,7 @@ extern "C" {
 
 size_t snn_dense_workspace_bytes(int64_t M, int64_t K, int64_t N) {
   if (check_dims(M, K, N) != SNN_OK) return 0;
-  return 256 + round256((size_t)K * N * 2) + round256((size_t)N * M * 2) +
-         round256((size_t)K * M * 2);
+  return 256;  // the status word: the backward reads its operands in place
 }
 
 snn_status_t snn_dense_layer_fwd(int64_t M, int64_t K, int64_t N, const void* X, const void* W,
@@ -421,29 +454,18 @@ snn_status_t snn_dense_layer_bwd(int64_t M, int64_t K, int64_t N, const void* X,
     if (!aligned16(p)) return SNN_ERR_ALIGNMENT;
   if (!ws || ws_bytes < snn_dense_workspace_bytes(M, K, N)) return SNN_ERR_WORKSPACE;
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
-  unsigned char* w = static_cast<unsigned char*>(ws);
-  int* status = reinterpret_cast<int*>(w);
-  void* Wt = w + 256;                                       // [K, N]
-  void* dIt = w + 256 + round256((size_t)K * N * 2);       // [N, M]
-  void* Xt = static_cast<unsigned char*>(dIt) + round256((size_t)N * M * 2);  // [K, M]
+  int* status = static_cast<int*>(ws);
   cudaError_t e = cudaSuccess;
   if (dX && M > 0 && K > 0) {
-    if (N == 0) {
-      e = cudaMemsetAsync(dX, 0, (size_t)M * K * 2, st);
-    } else {
-      e = transpose(W, Wt, (int)N, (int)K, st);
-      if (e == cudaSuccess) e = gemm_tn<true>(dI, Wt, dX, (int)M, (int)K, (int)N, status, st);
-    }
+    // dX[M, K] = dI[M, N] * W[N, K]: W is the MN-major B operand
+    if (N == 0) e = cudaMemsetAsync(dX, 0, (size_t)M * K * 2, st);
+    else e = gemm_tn<true, false, true>(dI, W, dX, (int)M, (int)K, (int)N, status, st);
     if (e != cudaSuccess) return e == cudaErrorInvalidValue ? SNN_ERR_UNSUPPORTED : SNN_ERR_CUDA;
   }
   if (dW && N > 0 && K > 0) {
-    if (M == 0) {
-      e = cudaMemsetAsync(dW, 0, (size_t)N * K * sizeof(float), st);
-    } else {
-      e = transpose(dI, dIt, (int)M, (int)N, st);
-      if (e == cudaSuccess) e = transpose(X, Xt, (int)M, (int)K, st);
-      if (e == cudaSuccess) e = gemm_tn<false>(dIt, Xt, dW, (int)N, (int)K, (int)M, status, st);
-    }
+    // dW[N, K] = dI[M, N]^T * X[M, K]: both operands MN-major (K = M here)
+    if (M == 0) e = cudaMemsetAsync(dW, 0, (size_t)N * K * sizeof(float), st);
+    else e = gemm_tn<false, true, true>(dI, X, dW, (int)N, (int)K, (int)M, status, st);
     if (e != cudaSuccess) return e == cudaErrorInvalidValue ? SNN_ERR_UNSUPPORTED : SNN_ERR_CUDA;
   }
   return SNN_OK;
