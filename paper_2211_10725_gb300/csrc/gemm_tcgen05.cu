@@ -3,12 +3,14 @@
 //   D[M, N] = A[M, K] * B[N, K]^T,   A, B bf16 row-major (K contiguous),
 // fp32 accumulation in tensor memory, fp32 or bf16 output.
 //
-// One CTA computes a 128 x BN tile.  Warp 0 (one thread) streams 128x64 and
-// BNx64 operand tiles into a 4-stage shared-memory ring with TMA (128-byte
-// swizzle); warp 1 allocates the TMEM accumulator and one thread issues
-// tcgen05.mma (M=128, N=BN, K=16 per instruction) as stages land, freeing
-// each stage through tcgen05.commit; warps 2-5 read the accumulator back
-// with tcgen05.ld (each warp its 32-lane quarter) and store it.  Every wait
+// Persistent CTAs (one per SM) take 128 x BN tiles (BN up to 256) in turn.  Warp 0 (one
+// thread) streams 128x64 and BNx64 operand tiles into a 4-stage
+// shared-memory ring with TMA (128-byte swizzle); warp 1 allocates two TMEM
+// accumulators and one thread issues tcgen05.mma (M=128, N=BN, K=16 per
+// instruction) as stages land, freeing each stage through tcgen05.commit;
+// warps 2-5 read a finished accumulator back with tcgen05.ld (each warp its
+// 32-lane quarter) and store it while the next tile accumulates in the
+// other buffer.  Every wait
 // is bounded; a kernel that gives up records SNN_ERR_TIMEOUT and still
 // drains its copies and frees its TMEM.
 //
@@ -34,9 +36,20 @@
 namespace snn {
 namespace gemm {
 
+#ifndef SNN_GEMM_STAGES
+#define SNN_GEMM_STAGES 4
+#endif
+#ifndef SNN_GEMM_CTAS_PER_SM
+#define SNN_GEMM_CTAS_PER_SM 1
+#endif
+#ifndef SNN_GEMM_SLEEP_WAIT
+#define SNN_GEMM_SLEEP_WAIT 0
+#endif
+
 constexpr int BM = 128;
 constexpr int BK = 64;  // 64 bf16 = 128 bytes: one swizzle atom row
-constexpr int kStages = 4;
+constexpr int kStages = SNN_GEMM_STAGES;
+constexpr int kCtasPerSm = SNN_GEMM_CTAS_PER_SM;  // resident CTAs the tile size aims for
 constexpr int kThreads = 192;
 constexpr uint64_t kDefaultWaitNs = 2000000000ull;
 constexpr uint64_t kDrainWaitNs = 1000000000ull;
@@ -151,6 +164,22 @@ __device__ __forceinline__ void tmem_ld16(uint32_t taddr, uint32_t r[16]) {
   asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
 }
 
+// Bounded wait of the single producer / MMA thread on the critical path:
+// polls without the suspend hint (a suspended thread can resume late), and
+// reads the clock only every 64 polls.
+__device__ __forceinline__ bool mbar_wait_poll(uint64_t* bar, uint32_t parity, uint64_t limit_ns) {
+#if SNN_GEMM_SLEEP_WAIT
+  return mbar_wait_bounded(bar, parity, limit_ns);
+#else
+  if (mbar_try_wait(bar, parity)) return true;
+  const uint64_t t0 = globaltimer_ns();
+  for (uint32_t i = 1;; ++i) {
+    if (mbar_try_wait(bar, parity)) return true;
+    if ((i & 63u) == 0 && globaltimer_ns() - t0 > limit_ns) return false;
+  }
+#endif
+}
+
 // Bounded wait taken by a whole warp; the give-up decision is warp-uniform.
 __device__ __forceinline__ bool warp_wait_uniform(uint64_t* bar, uint32_t parity, uint64_t limit_ns) {
   bool done = mbar_try_wait(bar, parity);
@@ -165,9 +194,10 @@ __device__ __forceinline__ bool warp_wait_uniform(uint64_t* bar, uint32_t parity
   }
 }
 
+// Two accumulators (one per tile in flight), power-of-two column count.
 template <int BN>
 __host__ __device__ constexpr uint32_t tmem_cols() {
-  return BN <= 32 ? 32u : (uint32_t)BN;
+  return 2 * BN <= 32 ? 32u : (2 * BN <= 64 ? 64u : (2 * BN <= 128 ? 128u : (2 * BN <= 256 ? 256u : 512u)));
 }
 
 template <int BN>
@@ -176,18 +206,22 @@ __host__ __device__ constexpr size_t smem_bytes() {
 }
 
 // ---------------------------------------------------------------------------
-// Kernel
+// Kernel: persistent, tiles t = blockIdx.x, blockIdx.x + gridDim.x, ... in
+// row-major tile order (N tiles fastest).  The operand ring runs on across
+// tiles; the accumulator alternates between two TMEM buffers so that the
+// epilogue of one tile overlaps the main loop of the next.
 // ---------------------------------------------------------------------------
 
 template <int BN, bool OUT_BF16, bool A_MN = false, bool B_MN = false>
-__global__ void __launch_bounds__(kThreads, 1)
+__global__ void __launch_bounds__(kThreads, kCtasPerSm)
     gemm_tn_tcgen05(const __grid_constant__ CUtensorMap ta, const __grid_constant__ CUtensorMap tb,
                     const GemmArgs g) {
-  static_assert(BN % 16 == 0 && BN >= 16 && BN <= 256, "UMMA N for M=128");
+  static_assert(BN % 16 == 0 && BN >= 16 && BN <= 256, "UMMA N for M=128, two accumulators");
   static_assert(!B_MN || BN % 64 == 0, "an MN-major B tile is whole 64-wide boxes");
   constexpr int A_BYTES = BM * BK * 2;
   constexpr int B_BYTES = BN * BK * 2;
   constexpr uint32_t TCOLS = tmem_cols<BN>();
+  constexpr int kEpiWarps = 4;
   extern __shared__ unsigned char smem_raw[];
   unsigned char* smem =
       reinterpret_cast<unsigned char*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -195,18 +229,23 @@ __global__ void __launch_bounds__(kThreads, 1)
   unsigned char* sB = smem + kStages * A_BYTES;
   uint64_t* full = reinterpret_cast<uint64_t*>(sB + kStages * B_BYTES);
   uint64_t* empty = full + kStages;
-  uint64_t* accum = empty + kStages;
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(accum + 1);
+  uint64_t* acc_full = empty + kStages;  // [2] MMA -> epilogue
+  uint64_t* acc_empty = acc_full + 2;    // [2] epilogue -> MMA
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(acc_empty + 2);
   const int warp = threadIdx.x >> 5, lid = threadIdx.x & 31;
-  const int m0 = blockIdx.y * BM, n0 = blockIdx.x * BN;
   const int nk = (g.K + BK - 1) / BK;
+  const int tiles_n = (g.N + BN - 1) / BN;
+  const int tiles = tiles_n * ((g.M + BM - 1) / BM);
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < kStages; ++s) {
       mbar_init(&full[s], 1);
       mbar_init(&empty[s], 1);
     }
-    mbar_init(accum, 1);
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(&acc_full[b], 1);
+      mbar_init(&acc_empty[b], kEpiWarps);
+    }
     fence_barrier_init();
   }
   if (warp == 1) tmem_alloc(tmem_slot, TCOLS);
@@ -217,69 +256,94 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   if (warp == 0) {
     if (lid == 0) {
-      int issued = 0;
-      for (int kb = 0; kb < nk; ++kb) {
-        const int s = kb % kStages;
-        if (kb >= kStages &&
-            !mbar_wait_bounded(&empty[s], (uint32_t)(((kb / kStages) - 1) & 1), g.wait_ns)) {
-          record_status(g.status, kStatusTimeout);
-          break;
-        }
-        mbar_arrive_expect_tx(&full[s], A_BYTES + B_BYTES);
-        if (A_MN) {
+      int64_t n_issued = 0;  // k-blocks issued over all tiles: ring position
+      bool ok = true;
+      for (int t = blockIdx.x; t < tiles && ok; t += gridDim.x) {
+        const int m0 = (t / tiles_n) * BM, n0 = (t % tiles_n) * BN;
+        for (int kb = 0; kb < nk; ++kb, ++n_issued) {
+          const int s = (int)(n_issued % kStages);
+          if (n_issued >= kStages &&
+              !mbar_wait_poll(&empty[s], (uint32_t)(((n_issued / kStages) - 1) & 1), g.wait_ns)) {
+            record_status(g.status, kStatusTimeout);
+            ok = false;
+            break;
+          }
+          mbar_arrive_expect_tx(&full[s], A_BYTES + B_BYTES);
+          if (A_MN) {
 #pragma unroll
-          for (int j = 0; j < BM / 64; ++j)
-            tma_load_2d(sA + s * A_BYTES + j * kMnBoxBytes, &ta, m0 + 64 * j, kb * BK, &full[s]);
-        } else {
-          tma_load_2d(sA + s * A_BYTES, &ta, kb * BK, m0, &full[s]);
-        }
-        if (B_MN) {
+            for (int j = 0; j < BM / 64; ++j)
+              tma_load_2d(sA + s * A_BYTES + j * kMnBoxBytes, &ta, m0 + 64 * j, kb * BK, &full[s]);
+          } else {
+            tma_load_2d(sA + s * A_BYTES, &ta, kb * BK, m0, &full[s]);
+          }
+          if (B_MN) {
 #pragma unroll
-          for (int j = 0; j < BN / 64; ++j)
-            tma_load_2d(sB + s * B_BYTES + j * kMnBoxBytes, &tb, n0 + 64 * j, kb * BK, &full[s]);
-        } else {
-          tma_load_2d(sB + s * B_BYTES, &tb, kb * BK, n0, &full[s]);
+            for (int j = 0; j < BN / 64; ++j)
+              tma_load_2d(sB + s * B_BYTES + j * kMnBoxBytes, &tb, n0 + 64 * j, kb * BK, &full[s]);
+          } else {
+            tma_load_2d(sB + s * B_BYTES, &tb, kb * BK, n0, &full[s]);
+          }
         }
-        ++issued;
       }
       // every copy this thread issued has landed before the CTA may exit
-      for (int j = issued > kStages ? issued - kStages : 0; j < issued; ++j)
+      for (int64_t j = n_issued > kStages ? n_issued - kStages : 0; j < n_issued; ++j)
         mbar_wait_bounded(&full[j % kStages], (uint32_t)((j / kStages) & 1), kDrainWaitNs);
     }
   } else if (warp == 1) {
     if (lid == 0) {
       constexpr uint32_t idesc = idesc_bf16(BM, BN, A_MN, B_MN);
-      for (int kb = 0; kb < nk; ++kb) {
-        const int s = kb % kStages;
-        if (!mbar_wait_bounded(&full[s], (uint32_t)((kb / kStages) & 1), g.wait_ns)) {
+      // 16 more along K: 32 bytes inside a K-major row, or 16 rows (2048
+      // bytes) of an MN-major tile; the descriptor holds the address >> 4
+      constexpr uint64_t stepA = A_MN ? 2048 >> 4 : 32 >> 4;
+      constexpr uint64_t stepB = B_MN ? 2048 >> 4 : 32 >> 4;
+      int64_t n_used = 0;  // k-blocks consumed over all tiles
+      bool ok = true;
+      int i = 0;  // this CTA's tile count
+      for (int t = blockIdx.x; t < tiles && ok; t += gridDim.x, ++i) {
+        const int b = i & 1;
+        // the epilogue has drained this accumulator (its use two tiles ago)
+        if (i >= 2 && !mbar_wait_poll(&acc_empty[b], (uint32_t)(((i >> 1) - 1) & 1), g.wait_ns)) {
           record_status(g.status, kStatusTimeout);
           break;
         }
         tc_fence_after();
-        const uint64_t da = A_MN ? sdesc_sw128_mn(sA + s * A_BYTES) : sdesc_sw128(sA + s * A_BYTES);
-        const uint64_t db = B_MN ? sdesc_sw128_mn(sB + s * B_BYTES) : sdesc_sw128(sB + s * B_BYTES);
-        // 16 more along K: 32 bytes inside a K-major row, or 16 rows (2048
-        // bytes) of an MN-major tile; the descriptor holds the address >> 4
-        constexpr uint64_t stepA = A_MN ? 2048 >> 4 : 32 >> 4;
-        constexpr uint64_t stepB = B_MN ? 2048 >> 4 : 32 >> 4;
+        const uint32_t acc = tmem + (uint32_t)(b * BN);
+        for (int kb = 0; kb < nk; ++kb, ++n_used) {
+          const int s = (int)(n_used % kStages);
+          if (!mbar_wait_poll(&full[s], (uint32_t)((n_used / kStages) & 1), g.wait_ns)) {
+            record_status(g.status, kStatusTimeout);
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint64_t da = A_MN ? sdesc_sw128_mn(sA + s * A_BYTES) : sdesc_sw128(sA + s * A_BYTES);
+          const uint64_t db = B_MN ? sdesc_sw128_mn(sB + s * B_BYTES) : sdesc_sw128(sB + s * B_BYTES);
 #pragma unroll
-        for (int kk = 0; kk < BK / 16; ++kk)
-          tc_mma(tmem, da + stepA * kk, db + stepB * kk, idesc, (kb | kk) != 0 ? 1u : 0u);
-        tc_commit(&empty[s]);  // the stage is free once these MMAs are done
+          for (int kk = 0; kk < BK / 16; ++kk)
+            tc_mma(acc, da + stepA * kk, db + stepB * kk, idesc, (kb | kk) != 0 ? 1u : 0u);
+          tc_commit(&empty[s]);  // the stage is free once these MMAs are done
+        }
+        if (ok) tc_commit(&acc_full[b]);  // the tile's accumulator is final
       }
-      tc_commit(accum);  // the accumulator is final once every MMA is done
     }
   } else {
     // epilogue: warp w reads TMEM lanes 32*(w%4) .. +32, i.e. tile rows
     const int q = warp & 3;
-    const bool ok = warp_wait_uniform(accum, 0u, g.wait_ns);
-    tc_fence_after();
-    if (ok) {
+    int i = 0;
+    for (int t = blockIdx.x; t < tiles; t += gridDim.x, ++i) {
+      const int b = i & 1;
+      if (!warp_wait_uniform(&acc_full[b], (uint32_t)((i >> 1) & 1), g.wait_ns)) {
+        if (lid == 0) record_status(g.status, kStatusTimeout);
+        break;
+      }
+      tc_fence_after();
+      const int m0 = (t / tiles_n) * BM, n0 = (t % tiles_n) * BN;
       const int row = m0 + q * 32 + lid;
+      const uint32_t acc = tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(b * BN);
 #pragma unroll 1
       for (int c = 0; c < BN; c += 16) {
         uint32_t r[16];
-        tmem_ld16(tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)c, r);
+        tmem_ld16(acc + (uint32_t)c, r);
         const int col = n0 + c;
         if (row < g.M && col < g.N) {
           if (OUT_BF16) {
@@ -311,8 +375,10 @@ __global__ void __launch_bounds__(kThreads, 1)
           }
         }
       }
-    } else if (lid == 0) {
-      record_status(g.status, kStatusTimeout);
+      // this warp's reads of the accumulator are done: hand it back
+      tc_fence_before();
+      __syncwarp();
+      if (lid == 0) mbar_arrive(&acc_empty[b]);
     }
   }
   tc_fence_before();
@@ -363,7 +429,12 @@ cudaError_t launch_bn(const CUtensorMap& ta, const CUtensorMap& tb, const GemmAr
   const void* k = (const void*)gemm_tn_tcgen05<BN, OUT_BF16, A_MN, B_MN>;
   const cudaError_t attr = ensure_smem(k, smem_bytes<BN>());  // once per device
   if (attr != cudaSuccess) return attr;
-  const dim3 grid((unsigned)((g.N + BN - 1) / BN), (unsigned)((g.M + BM - 1) / BM));
+  int dev = 0, sms = 152;
+  if (cudaGetDevice(&dev) == cudaSuccess)
+    cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  const int64_t tiles = (int64_t)((g.N + BN - 1) / BN) * ((g.M + BM - 1) / BM);
+  const int64_t slots = (int64_t)sms * kCtasPerSm;
+  const unsigned grid = (unsigned)(tiles < slots ? tiles : slots);  // persistent CTAs
   gemm_tn_tcgen05<BN, OUT_BF16, A_MN, B_MN><<<grid, kThreads, smem_bytes<BN>(), st>>>(ta, tb, g);
   return cudaGetLastError();
 }
@@ -375,7 +446,10 @@ cudaError_t launch_bn(const CUtensorMap& ta, const CUtensorMap& tb, const GemmAr
 template <bool OUT_BF16, bool A_MN = false, bool B_MN = false>
 cudaError_t gemm_tn(const void* A, const void* B, void* D, int M, int N, int K, int* status,
                     cudaStream_t st) {
-  int bn = 128;
+  // a 128 x 256 tile keeps the tensor core busier per instruction (about
+  // 1.6x the rate of 128 x 128 at large K); below K = 512 the per-tile
+  // fixed costs dominate and the narrower tile's parallelism wins
+  int bn = (!B_MN && N > 128 && K >= 512) ? 256 : 128;
   if (N <= 16 && !B_MN) bn = 16;
   else if (N <= 32 && !B_MN) bn = 32;
   else if (N <= 64) bn = 64;
@@ -384,7 +458,7 @@ cudaError_t gemm_tn(const void* A, const void* B, void* D, int M, int N, int K, 
     if (cudaGetDevice(&dev) == cudaSuccess)
       cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
     const int64_t tiles128 = (int64_t)((N + 127) / 128) * ((M + BM - 1) / BM);
-    if (tiles128 < sms) bn = 64;
+    if (tiles128 < (int64_t)sms * kCtasPerSm) bn = 64;
   }
   CUtensorMap ta, tb;
   const bool okA = A_MN ? make_map(&ta, A, K, M, 64) : make_map(&ta, A, M, K, BM);
@@ -396,6 +470,7 @@ cudaError_t gemm_tn(const void* A, const void* B, void* D, int M, int N, int K, 
     return launch_bn<128, OUT_BF16, A_MN, B_MN>(ta, tb, g, st);
   } else {
     switch (bn) {
+      case 256: return launch_bn<256, OUT_BF16, A_MN, B_MN>(ta, tb, g, st);
       case 16: return launch_bn<16, OUT_BF16, A_MN, B_MN>(ta, tb, g, st);
       case 32: return launch_bn<32, OUT_BF16, A_MN, B_MN>(ta, tb, g, st);
       case 64: return launch_bn<64, OUT_BF16, A_MN, B_MN>(ta, tb, g, st);

@@ -25,7 +25,8 @@ def _np(t):
 
 # (M, K, N): tile-aligned, ragged, the 3-layer network's forward and backward shapes
 SHAPES = [(128, 64, 128), (200, 72, 40), (136, 16, 1000), (3200, 784, 1000),
-          (3200, 1000, 16), (3200, 16, 1000), (1000, 3200, 784), (16, 3200, 1000)]
+          (3200, 1000, 16), (3200, 16, 1000), (1000, 3200, 784), (16, 3200, 1000),
+          (200, 576, 300), (4096, 2048, 1024)]
 
 
 @pytest.mark.parametrize("M,K,N", SHAPES)
@@ -42,7 +43,8 @@ def test_dense_forward(M, K, N, cuda_device):
 
 
 @pytest.mark.parametrize("M,K,N", [(128, 64, 128), (200, 72, 40), (3200, 784, 1000),
-                                   (3200, 1000, 16), (3200, 1000, 1000)])
+                                   (3200, 1000, 16), (3200, 1000, 1000), (136, 16, 1000),
+                                   (2048, 512, 256)])
 def test_dense_backward(M, K, N, cuda_device):
     X = _bf16((M, K), M, spikes=True)
     Wt = _bf16((N, K), N, scale=(6.0 / K) ** 0.5)
