@@ -435,10 +435,14 @@ def run_ours(args):
     kernel_key = f"scan_bwd_staged[{w.neuron},{w.save}]"  # dominant kernel
     traffic = profiled_traffic(kernel_key, w.name)
     clocks = sampler.summary(t_wall0, t_wall1)
-    # forward scan + backward scan + a two-stage reduction per parameter
-    # gradient (beta, thr, and alpha or v for the Synaptic / recurrent neuron)
-    n_param_grads = 3 if w.neuron in ("synaptic", "rleaky") else 2
-    launches_per_step = 2 + 2 * n_param_grads
+    # forward scan + backward scan + one reduction launch per layout among
+    # the parameter gradients (beta, thr, and alpha or v)
+    modes = {w.beta_mode, w.thr_mode}
+    if w.neuron == "synaptic":
+        modes.add(w.alpha_mode)
+    if w.neuron == "rleaky":
+        modes.add(w.v_mode)
+    launches_per_step = 2 + len(modes)
     cpu = None
     if not args.no_cpu_baseline and world == 1:
         v, n, dt = time_oracle(w, inp, args.cpu_seconds)

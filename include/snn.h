@@ -120,8 +120,12 @@ int snn_version(void);
 /* sizeof(snn_scan_desc) as compiled into the library (ABI check). */
 size_t snn_scan_desc_size(void);
 
-/* Bytes of device workspace every scan call of `desc` needs (a status word
- * plus per-lane parameter-gradient partials).  0 if desc is invalid. */
+/* Bytes of device workspace every scan call of `desc` needs (a status word,
+ * per-lane parameter-gradient partials, fp64 reduction scratch and the
+ * reductions' completion tickets).  0 if desc is invalid.  The tickets must
+ * start at zero (snn_workspace_init) and each reduction leaves them at zero;
+ * after a call that reported SNN_ERR_TIMEOUT, initialise the workspace
+ * again. */
 size_t snn_scan_workspace_bytes(const snn_scan_desc* desc);
 
 /* Number of fp32 elements of the ckpt buffer passed to the forward and the

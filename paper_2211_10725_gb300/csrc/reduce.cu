@@ -3,6 +3,13 @@
 // scalar, per neuron [N] (sum over b) or per channel [C] (sum over b and the
 // channel's H*W positions).  Cross-lane sums run in fp64 in a fixed order, so
 // repeated calls give identical bits.
+//
+// One launch reduces every parameter that shares a layout (blockIdx.z picks
+// the parameter).  Block (x, y) of a parameter sums split y of output group
+// x into fp64 scratch; the last of a group's splits to finish (a ticket
+// taken after its partial is published) adds the group's partials in split
+// order and writes the result, then resets the group's ticket to zero for
+// the next call.
 #include "scan_host.cuh"
 
 namespace snn {
@@ -19,108 +26,132 @@ __device__ __forceinline__ double block_sum(double v, double* sh) {
     if ((int)threadIdx.x < s) sh[threadIdx.x] += sh[threadIdx.x + s];
     __syncthreads();
   }
-  return sh[0];
+  const double r = sh[0];
+  __syncthreads();
+  return r;
 }
 
-// Stage 1 of the scalar sum: block b sums lanes [b*chunk, (b+1)*chunk).
-__global__ void __launch_bounds__(kRedThreads) reduce_scalar_blocks(const float* part, int64_t L,
-                                                                     int64_t chunk, double* out) {
+struct ReduceJob {
+  const float* part;  // per-lane partials [B*N]
+  float* out;         // reduced gradient
+  double* scratch;    // fp64 partials
+  int* tickets;       // one per output group, zero between calls
+};
+
+struct ReduceJobs {
+  ReduceJob job[3];
+};
+
+// True in every thread of the block that finished a group last.
+__device__ __forceinline__ bool last_of_group(int* ticket, int splits) {
+  __shared__ int last;
+  __threadfence();  // this block's partial is visible before its ticket
+  __syncthreads();
+  if (threadIdx.x == 0) last = atomicAdd(ticket, 1) == splits - 1;
+  __syncthreads();
+  if (last) __threadfence();  // and the other blocks' partials before the sum
+  return last;
+}
+
+// Scalar: group 0, split y sums lanes [y*chunk, (y+1)*chunk).
+__global__ void __launch_bounds__(kRedThreads) reduce_scalar(ReduceJobs js, int64_t L,
+                                                              int64_t chunk) {
   __shared__ double sh[kRedThreads];
-  const int64_t lo = (int64_t)blockIdx.x * chunk;
+  const ReduceJob& j = js.job[blockIdx.z];
+  const int S = gridDim.y;
+  const int64_t lo = (int64_t)blockIdx.y * chunk;
   const int64_t hi = min(L, lo + chunk);
   double acc = 0.0;
-  for (int64_t l = lo + threadIdx.x; l < hi; l += blockDim.x) acc += (double)part[l];
+  for (int64_t l = lo + threadIdx.x; l < hi; l += blockDim.x) acc += (double)j.part[l];
   const double s = block_sum(acc, sh);
-  if (threadIdx.x == 0) out[blockIdx.x] = s;
+  if (threadIdx.x == 0) j.scratch[blockIdx.y] = s;
+  if (!last_of_group(&j.tickets[0], S)) return;
+  double t = 0.0;
+  for (int i = threadIdx.x; i < S; i += blockDim.x) t += j.scratch[i];
+  const double total = block_sum(t, sh);
+  if (threadIdx.x == 0) {
+    j.out[0] = (float)total;
+    j.tickets[0] = 0;
+  }
 }
 
-__global__ void __launch_bounds__(kRedThreads) reduce_scalar_final(const double* in, int n,
-                                                                    float* out) {
-  __shared__ double sh[kRedThreads];
-  double acc = 0.0;
-  for (int i = threadIdx.x; i < n; i += blockDim.x) acc += in[i];
-  const double s = block_sum(acc, sh);
-  if (threadIdx.x == 0) out[0] = (float)s;
-}
-
-// Per-neuron sum, stage 1: block (x, s) sums samples b in [b0, b1) of
-// split s for 256 neurons; stage 2 adds the splits of each neuron in order.
-__global__ void __launch_bounds__(kRedThreads) reduce_per_neuron_blocks(const float* part,
-                                                                         int64_t B, int64_t N,
-                                                                         double* out) {
+// Per neuron: group x = neurons [256x, 256x + 256), split y = samples
+// [B*y/S, B*(y+1)/S); the last split adds the S partials of each neuron.
+__global__ void __launch_bounds__(kRedThreads) reduce_per_neuron(ReduceJobs js, int64_t B,
+                                                                  int64_t N) {
+  const ReduceJob& j = js.job[blockIdx.z];
   const int64_t n = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
-  if (n >= N) return;
   const int64_t S = gridDim.y, s = blockIdx.y;
-  const int64_t b0 = B * s / S, b1 = B * (s + 1) / S;
-  double acc = 0.0;
-  for (int64_t b = b0; b < b1; ++b) acc += (double)part[b * N + n];
-  out[s * N + n] = acc;
+  if (n < N) {
+    const int64_t b0 = B * s / S, b1 = B * (s + 1) / S;
+    double acc = 0.0;
+    for (int64_t b = b0; b < b1; ++b) acc += (double)j.part[b * N + n];
+    j.scratch[s * N + n] = acc;
+  }
+  if (!last_of_group(&j.tickets[blockIdx.x], (int)S)) return;
+  if (n < N) {
+    double acc = 0.0;
+    for (int64_t q = 0; q < S; ++q) acc += j.scratch[q * N + n];
+    j.out[n] = (float)acc;
+  }
+  if (threadIdx.x == 0) j.tickets[blockIdx.x] = 0;
 }
 
-__global__ void __launch_bounds__(kRedThreads) reduce_per_neuron_final(const double* in, int64_t N,
-                                                                        int S, float* out) {
-  const int64_t n = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
-  if (n >= N) return;
-  double acc = 0.0;
-  for (int s = 0; s < S; ++s) acc += in[s * N + n];
-  out[n] = (float)acc;
-}
-
-// Per-channel sum, stage 1: block (c, s) sums the runs j = s, s + S, ... of
-// channel c, where run j = (b, r) is the HW contiguous lanes of neurons
+// Per channel: group x = channel c, split y sums the runs j = y, y + S, ...
+// of channel c, where run j = (b, r) is the HW contiguous lanes of neurons
 // (r*C + c)*HW .. +HW of sample b (r < N/(C*HW)).  The block's runs are
 // flattened so that short runs still keep every thread busy.
-__global__ void __launch_bounds__(kRedThreads) reduce_per_channel_blocks(
-    const float* part, int64_t B, int64_t N, int64_t C, int64_t HW, double* out) {
+__global__ void __launch_bounds__(kRedThreads) reduce_per_channel(ReduceJobs js, int64_t B,
+                                                                   int64_t N, int64_t C,
+                                                                   int64_t HW) {
   __shared__ double sh[kRedThreads];
+  const ReduceJob& j = js.job[blockIdx.z];
   const int64_t c = blockIdx.x, s = blockIdx.y, S = gridDim.y;
   const int64_t R = N / (C * HW);
   const int64_t runs = (B * R - s + S - 1) / S;  // runs j = s + q*S, q < runs
   double acc = 0.0;
   for (int64_t e = threadIdx.x; e < runs * HW; e += blockDim.x) {
     const int64_t q = e / HW, h = e - q * HW;
-    const int64_t j = s + q * S;
-    const int64_t b = j / R, r = j - b * R;
-    acc += (double)part[b * N + (r * C + c) * HW + h];
+    const int64_t jr = s + q * S;
+    const int64_t b = jr / R, r = jr - b * R;
+    acc += (double)j.part[b * N + (r * C + c) * HW + h];
   }
   const double v = block_sum(acc, sh);
-  if (threadIdx.x == 0) out[c * S + s] = v;
-}
-
-// Stage 2: channel c adds its S partials in order.
-__global__ void __launch_bounds__(kRedThreads) reduce_per_channel_final(const double* in, int64_t C,
-                                                                         int S, float* out) {
-  const int64_t c = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
-  if (c >= C) return;
-  double acc = 0.0;
-  for (int s = 0; s < S; ++s) acc += in[c * S + s];
-  out[c] = (float)acc;
+  if (threadIdx.x == 0) j.scratch[c * S + s] = v;
+  if (!last_of_group(&j.tickets[c], (int)S)) return;
+  if (threadIdx.x == 0) {
+    double t = 0.0;
+    for (int64_t q = 0; q < S; ++q) t += j.scratch[c * S + q];
+    j.out[c] = (float)t;
+    j.tickets[c] = 0;
+  }
 }
 
 }  // namespace
 
-cudaError_t launch_param_reduce(const float* part, int64_t B, int64_t N, int64_t C, int64_t HW,
-                                int mode, double* scratch, int64_t scratch_len, float* out,
-                                cudaStream_t stream) {
+cudaError_t launch_param_reduce(const ParamReduce* p, int n, int64_t B, int64_t N, int64_t C,
+                                int64_t HW, int mode, int64_t scratch_len, cudaStream_t stream) {
+  if (n <= 0) return cudaSuccess;
+  if (n > 3) return cudaErrorInvalidValue;
+  ReduceJobs js;
+  for (int k = 0; k < n; ++k) js.job[k] = ReduceJob{p[k].part, p[k].out, p[k].scratch, p[k].tickets};
   const int64_t L = B * N;
   if (mode == PM_SCALAR) {
     const int64_t chunk_min = 4096;
     int64_t nb = ceil_div(L, chunk_min);
     if (nb > scratch_len) nb = scratch_len;
+    if (nb > 65535) nb = 65535;
     if (nb < 1) nb = 1;
     const int64_t chunk = ceil_div(L > 0 ? L : 1, nb);
     nb = ceil_div(L > 0 ? L : 1, chunk);
-    reduce_scalar_blocks<<<(unsigned)nb, kRedThreads, 0, stream>>>(part, L, chunk, scratch);
-    reduce_scalar_final<<<1, kRedThreads, 0, stream>>>(scratch, (int)nb, out);
+    reduce_scalar<<<dim3(1, (unsigned)nb, (unsigned)n), kRedThreads, 0, stream>>>(js, L, chunk);
   } else if (mode == PM_PER_NEURON) {
     if (N > 0) {
       int64_t S = B < kNeuronSplit ? B : kNeuronSplit;
       if (S * N > scratch_len) S = scratch_len / N;
       if (S < 1) return cudaErrorInvalidValue;  // the workspace is sized for S >= 1
-      reduce_per_neuron_blocks<<<dim3((unsigned)ceil_div(N, kRedThreads), (unsigned)S), kRedThreads,
-                                 0, stream>>>(part, B, N, scratch);
-      reduce_per_neuron_final<<<(unsigned)ceil_div(N, kRedThreads), kRedThreads, 0, stream>>>(
-          scratch, N, (int)S, out);
+      reduce_per_neuron<<<dim3((unsigned)ceil_div(N, kRedThreads), (unsigned)S, (unsigned)n),
+                          kRedThreads, 0, stream>>>(js, B, N);
     }
   } else if (C > 0) {
     const int64_t R = N / (C * HW);
@@ -131,10 +162,8 @@ cudaError_t launch_param_reduce(const float* part, int64_t B, int64_t N, int64_t
     if (S > B * R) S = B * R;
     if (S > scratch_len / C) S = scratch_len / C;
     if (S < 1) return cudaErrorInvalidValue;  // the workspace is sized for S >= 1
-    reduce_per_channel_blocks<<<dim3((unsigned)C, (unsigned)S), kRedThreads, 0, stream>>>(
-        part, B, N, C, HW, scratch);
-    reduce_per_channel_final<<<(unsigned)ceil_div(C, kRedThreads), kRedThreads, 0, stream>>>(
-        scratch, C, (int)S, out);
+    reduce_per_channel<<<dim3((unsigned)C, (unsigned)S, (unsigned)n), kRedThreads, 0, stream>>>(
+        js, B, N, C, HW);
   }
   return cudaGetLastError();
 }

@@ -158,8 +158,21 @@ inline int64_t param_reduce_scratch(int64_t N, int64_t C) {
   const int64_t a = 1024, b = 8 * N, c = 64 * C;
   return a > b ? (a > c ? a : c) : (b > c ? b : c);
 }
-cudaError_t launch_param_reduce(const float* part, int64_t B, int64_t N, int64_t C, int64_t HW,
-                                int mode, double* scratch, int64_t scratch_len, float* out,
-                                cudaStream_t stream);
+// One parameter's reduction: per-lane partials in, gradient out, fp64
+// scratch and zero-initialised tickets (one per output group: 1 for a
+// scalar, ceil(N/256) per neuron, C per channel) from the workspace.
+struct ParamReduce {
+  const float* part;
+  float* out;
+  double* scratch;
+  int* tickets;
+};
+inline int64_t param_reduce_groups(int64_t N, int64_t C) {
+  const int64_t a = (N + 255) / 256;
+  return a > C ? (a > 1 ? a : 1) : (C > 1 ? C : 1);
+}
+// Reduce n (<= 3) parameters that share `mode` in one launch.
+cudaError_t launch_param_reduce(const ParamReduce* p, int n, int64_t B, int64_t N, int64_t C,
+                                int64_t HW, int mode, int64_t scratch_len, cudaStream_t stream);
 
 }  // namespace snn

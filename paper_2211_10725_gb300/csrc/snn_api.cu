@@ -64,14 +64,20 @@ size_t lane_bytes(const snn_scan_desc* d) {
 // fp64 partials of one parameter's cross-lane reduction
 int64_t red_scratch(const snn_scan_desc* d) { return param_reduce_scratch(d->N, d->C); }
 
+size_t ticket_bytes(const snn_scan_desc* d) {
+  return (size_t)round_up(param_reduce_groups(d->N, d->C) * (int64_t)sizeof(int), 256);
+}
+
 size_t workspace_bytes(const snn_scan_desc* d) {
-  return kStatusBytes + 3 * lane_bytes(d) + 3 * (size_t)red_scratch(d) * sizeof(double);
+  return kStatusBytes + 3 * lane_bytes(d) + 3 * (size_t)red_scratch(d) * sizeof(double) +
+         3 * ticket_bytes(d);
 }
 
 struct WsView {
   int* status;
-  float* part[3];  // beta, thr, alpha
+  float* part[3];  // beta, thr, alpha (or v)
   double* scratch[3];
+  int* tickets[3];
 };
 
 WsView ws_view(void* ws, const snn_scan_desc* d) {
@@ -82,6 +88,8 @@ WsView ws_view(void* ws, const snn_scan_desc* d) {
   for (int k = 0; k < 3; ++k) v.part[k] = reinterpret_cast<float*>(p + kStatusBytes + k * lb);
   for (int k = 0; k < 3; ++k)
     v.scratch[k] = reinterpret_cast<double*>(p + kStatusBytes + 3 * lb + k * red_scratch(d) * sizeof(double));
+  unsigned char* t = p + kStatusBytes + 3 * lb + 3 * red_scratch(d) * sizeof(double);
+  for (int k = 0; k < 3; ++k) v.tickets[k] = reinterpret_cast<int*>(t + k * ticket_bytes(d));
   return v;
 }
 
@@ -263,11 +271,15 @@ snn_status_t scan_bwd(const snn_scan_desc* d, int neuron, const void* I, const f
   cudaError_t e = syn ? launch_scan_bwd_synaptic(a, recompute, d->in_dtype, d->io_dtype, staged, stream)
                       : launch_scan_bwd_leaky(a, recompute, d->in_dtype, d->io_dtype, staged, stream);
   if (e != cudaSuccess) return cuda_status(e);
+  // one launch per parameter layout in use
   float* parts[3] = {a.part_beta, a.part_thr, a.part_alpha};
-  for (int k = 0; k < 3; ++k) {
-    if (!outs[k]) continue;
-    e = launch_param_reduce(parts[k], d->B, d->N, d->C, d->HW, modes[k], v.scratch[k], red_scratch(d),
-                            outs[k], stream);
+  for (int mode = SNN_P_SCALAR; mode <= SNN_P_PER_CHANNEL; ++mode) {
+    ParamReduce jobs[3];
+    int n = 0;
+    for (int k = 0; k < 3; ++k)
+      if (outs[k] && modes[k] == mode) jobs[n++] = ParamReduce{parts[k], outs[k], v.scratch[k], v.tickets[k]};
+    if (n == 0) continue;
+    e = launch_param_reduce(jobs, n, d->B, d->N, d->C, d->HW, mode, red_scratch(d), stream);
     if (e != cudaSuccess) return SNN_ERR_CUDA;
   }
   return SNN_OK;
