@@ -431,15 +431,20 @@ def dense_backward(X, W, dI):
     return np.matmul(dI, W), np.matmul(dI.T, X)
 
 
-def rate_ce_loss(spk_out, labels):
+def rate_ce_loss(spk_out, labels, pop: int = 1):
     """Cross-entropy on output spike counts (rate-coded readout, Sec. V-A).
 
-    spk_out: [T, B, C] spikes; labels: [B].  Loss = mean_b CE(sum_t spk, y_b).
-    Returns (loss, grad_spk [T, B, C]) with grad = (softmax - onehot)/B at every t.
+    spk_out: [T, B, C*pop] spikes; labels: [B].  With a population code
+    (Sec. VII: pop output neurons per class, class c owning neurons
+    c*pop .. c*pop + pop - 1), a class's count is the spikes of its whole
+    population over all t.  Loss = mean_b CE(counts_b, y_b).
+    Returns (loss, grad_spk [T, B, C*pop]) with grad = (softmax - onehot)/B
+    of the neuron's class, at every t.
     """
     s = np.asarray(spk_out, dtype=np.float64)
-    T, B, C = s.shape
-    counts = s.sum(axis=0)
+    T, B, CP = s.shape
+    C = CP // pop
+    counts = s.sum(axis=0).reshape(B, C, pop).sum(axis=2)
     m = counts.max(axis=1, keepdims=True)
     lse = m[:, 0] + np.log(np.exp(counts - m).sum(axis=1))
     y = np.asarray(labels).astype(np.int64)
@@ -447,8 +452,8 @@ def rate_ce_loss(spk_out, labels):
     p = np.exp(counts - lse[:, None])
     onehot = np.zeros((B, C))
     onehot[np.arange(B), y] = 1.0
-    g = (p - onehot) / B
-    return loss, np.broadcast_to(g, (T, B, C)).copy()
+    g = np.repeat((p - onehot) / B, pop, axis=1)
+    return loss, np.broadcast_to(g, (T, B, CP)).copy()
 
 
 # ---------------------------------------------------------------------------
@@ -486,10 +491,11 @@ def dsnn_forward(X, Ws, T: int, B: int, beta: float, thr: float, dtype=np.float3
 
 
 def dsnn_backward(fwd, Ws, labels, T: int, B: int, beta: float, thr: float,
-                  sg_param: float, store=None):
+                  sg_param: float, store=None, pop: int = 1):
     """Loss and BPTT of ``dsnn_forward``.
 
-    The loss is ``rate_ce_loss`` on the last layer's spikes.  Then, from the
+    The loss is ``rate_ce_loss`` on the last layer's spikes (``pop`` output
+    neurons per class).  Then, from the
     top layer down: ``leaky_backward`` (detached reset, fast-sigmoid
     surrogate of slope ``sg_param``) on the layer's saved trace turns the
     spike gradient into dL/dI_l; ``dense_backward`` turns that into dL/dW_l
@@ -504,8 +510,8 @@ def dsnn_backward(fwd, Ws, labels, T: int, B: int, beta: float, thr: float,
     """
     keep = (lambda a: a) if store is None else store
     nl = len(Ws)
-    C = Ws[-1].shape[0]
-    loss, g_out = rate_ce_loss(fwd["spk"][-1].reshape(T, B, C), labels)
+    C = Ws[-1].shape[0]   # output neurons (classes * pop)
+    loss, g_out = rate_ce_loss(fwd["spk"][-1].reshape(T, B, C), labels, pop)
     g_out = keep(g_out)
     gs = g_out.reshape(T, B * C)
     res = {"loss": loss, "grad_out": g_out, "grad_spk": [None] * nl,

@@ -565,3 +565,23 @@ def test_rleaky_bptt_matches_finite_differences(detach, sg, k):
                          ("mem0", "grad_mem0"), ("v", "grad_v_lane")]:
         for l in range(L):
             np.testing.assert_allclose(g[gname][l], fd(pname, l), rtol=1e-6, atol=1e-8)
+
+
+def test_population_ce_matches_torch_autograd():
+    """Population code (pop neurons per class, class-contiguous): the loss
+    and spike gradient against torch's cross-entropy on population sums;
+    pop = 1 is the plain readout."""
+    rng = np.random.default_rng(15)
+    T, B, C, pop = 1, 7, 10, 5
+    spk = (rng.uniform(0, 1, (T, B, C * pop)) < 0.3).astype(np.float64)
+    y = rng.integers(0, C, B)
+    loss, g = O.rate_ce_loss(spk, y, pop)
+    ts = torch.tensor(spk, requires_grad=True)
+    counts = ts.sum(0).reshape(B, C, pop).sum(-1)
+    ref = torch.nn.functional.cross_entropy(counts, torch.tensor(y))
+    ref.backward()
+    assert abs(loss - ref.item()) < 1e-12
+    np.testing.assert_allclose(g, ts.grad.numpy(), rtol=1e-12, atol=1e-14)
+    l1, g1 = O.rate_ce_loss(spk[:, :, :C], y, 1)
+    l2, g2 = O.rate_ce_loss(spk[:, :, :C], y)
+    assert l1 == l2 and np.array_equal(g1, g2)
