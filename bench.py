@@ -59,7 +59,7 @@ def workload(args):
 
 def is_dense(args):
     from paper_2211_10725_gb300 import workloads as W
-    return args.workload == W.DSNN_C3.name
+    return args.workload in W.DENSE_WORKLOADS
 
 
 # ---------------------------------------------------------------------------
@@ -259,7 +259,7 @@ def run_dense_reference(args):
     import numpy as np
     from oracle import snn_oracle as O
     from paper_2211_10725_gb300 import workloads as W
-    w = W.DSNN_C3
+    w = W.DENSE_WORKLOADS[args.workload]
     inp = W.make_dense_inputs(w)
     Ws = [x.float().numpy().astype(np.float64) for x in inp["W"]]
     X = inp["X"].float().numpy().astype(np.float64)          # [T, B, K0]
@@ -268,7 +268,7 @@ def run_dense_reference(args):
     def one(bs):
         xb = X[:, bs].reshape(w.T * len(bs), -1)
         fwd = O.dsnn_forward(xb, Ws, w.T, len(bs), w.beta, w.thr)
-        O.dsnn_backward(fwd, Ws, y[bs], w.T, len(bs), w.beta, w.thr, w.sg_param)
+        O.dsnn_backward(fwd, Ws, y[bs], w.T, len(bs), w.beta, w.thr, w.sg_param, pop=w.pop)
 
     t0 = time.perf_counter()
     one(np.arange(8))
@@ -524,7 +524,7 @@ def run_dense(args):
         dist.init_process_group("nccl")
     torch.cuda.set_device(local)
     dev = torch.device("cuda", local)
-    w = W.DSNN_C3
+    w = W.DENSE_WORKLOADS[args.workload]
     save = args.save or "recompute"
     inp = W.make_dense_inputs(w, seed=W.SEED_BASE + w.seed_index + 1000 * rank)
     net = DenseSNN(w, inp["W"], device=dev, save=save)
@@ -556,25 +556,36 @@ def run_dense(args):
         if layer.status() != 0:
             raise RuntimeError("kernel status after warm-up")
 
-    # one step as a CUDA graph, with a timing event between consecutive ops
-    graph, evs = None, None
-    if not args.no_graph and world == 1:
-        try:
-            evs = [_timing_events(True) for _ in range(len(names) + 1)]
-            graph = torch.cuda.CUDAGraph()
-            with torch.cuda.graph(graph, stream=stream):
+    # one step as a CUDA graph; a second graph of the same step has a timing
+    # event between consecutive ops (event nodes), for the per-op times
+    def capture(with_events):
+        evs = [_timing_events(True) for _ in range(len(names) + 1)] if with_events else None
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=stream):
+            if evs:
                 evs[0].record()
-                for i, (_, call) in enumerate(step_ops()):
-                    call()
+            for i, (_, call) in enumerate(step_ops()):
+                call()
+                if evs:
                     evs[i + 1].record()
+        return g, evs
+
+    graph = graph_ev = None
+    evs = None
+    if not args.no_graph and world == 1:
+        graph, _ = capture(False)
+        try:
+            graph_ev, evs = capture(True)
         except TypeError:
-            graph, evs = None, None   # no graph-capturable timing events in this torch
-    if graph is None:
+            graph_ev, evs = None, None   # no graph-capturable timing events in this torch
+    if graph_ev is None:
         evs = [_timing_events(False) for _ in range(len(names) + 1)]
 
-    def launch():
-        if graph is not None:
+    def launch(with_events):
+        if graph is not None and not with_events:
             graph.replay()
+        elif graph_ev is not None:
+            graph_ev.replay()
         else:
             evs[0].record(stream)
             for i, (_, call) in enumerate(step_ops(stream)):
@@ -583,7 +594,8 @@ def run_dense(args):
 
     with torch.cuda.stream(stream):
         for _ in range(3):
-            launch()
+            launch(False)
+            launch(True)
     stream.synchronize()
 
     sampler = ClockSampler(local)
@@ -592,7 +604,6 @@ def run_dense(args):
         time.sleep(0.3)
     K = args.steps
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    per_op = [0.0] * len(names)
     if world > 1:
         dist.barrier()
     torch.cuda.synchronize()
@@ -600,14 +611,26 @@ def run_dense(args):
     with torch.cuda.stream(stream):
         e0.record(stream)
         for _ in range(K):
-            launch()
+            launch(graph is None)
         e1.record(stream)
     torch.cuda.synchronize()
     t_wall1 = time.time()
-    # per-op durations of the last step of the timed region
-    per_op = [evs[i].elapsed_time(evs[i + 1]) for i in range(len(names))]
     if world > 1:
         dist.barrier()
+    # per-op durations: a timed region of the graph with event nodes (K2
+    # steps), each op averaged over the steps
+    K2 = max(1, min(K, 100))
+    per_op = [0.0] * len(names)
+    ev_total = 0.0
+    with torch.cuda.stream(stream):
+        for _ in range(K2):
+            s0 = torch.cuda.Event(enable_timing=True)
+            s0.record(stream)
+            launch(True)
+            torch.cuda.synchronize()
+            per_op = [acc + evs[i].elapsed_time(evs[i + 1]) for i, acc in enumerate(per_op)]
+            ev_total += evs[0].elapsed_time(evs[-1])
+    per_op = [x / K2 for x in per_op]
     if rank == 0:
         time.sleep(0.2)
         sampler.stop()
@@ -650,6 +673,7 @@ def run_dense(args):
         "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
         "config": {"workload": w.name, "sizes": list(w.sizes), "T": w.T, "B": w.B,
+                   "classes": w.n_classes, "neurons_per_class": w.pop,
                    "step": "forward GEMMs + Leaky scans, rate-coded CE loss, BPTT scans, "
                            "dense backward (dX, dW), AdamW",
                    "neuron_steps_per_step": ns_per_step, "save": save,
@@ -662,9 +686,10 @@ def run_dense(args):
                      "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
                      "frac": achieved / peak, "peak_kind": f"{peak_kind} sustained bf16",
                      "traffic": None, "flops_per_step": {"fwd": fwd_f, "dW": dw_f, "dX": dx_f},
-                     "op_ms_last_step": op_ms,
-                     "timing": "timing events between the ops of the step, read after the "
-                               "last step of the timed region"},
+                     "op_ms": op_ms,
+                     "op_timed_step_ms": ev_total / K2,
+                     "timing": "per-op: a second timed region of the same step graph with "
+                               "event nodes between the ops, averaged over its steps"},
         "clocks": clocks,
         "gpu_launches": launches * K,
         "cpu_baseline": cpu,
@@ -687,7 +712,7 @@ def time_dense_oracle(w, inp, seconds):
     while t_total < seconds or n == 0:
         t0 = time.perf_counter()
         fwd = O.dsnn_forward(X, Ws, w.T, w.B, w.beta, w.thr)
-        O.dsnn_backward(fwd, Ws, y, w.T, w.B, w.beta, w.thr, w.sg_param)
+        O.dsnn_backward(fwd, Ws, y, w.T, w.B, w.beta, w.thr, w.sg_param, pop=w.pop)
         t_total += time.perf_counter() - t0
         n += 1
     ns = w.T * w.B * sum(w.sizes[1:])

@@ -303,21 +303,30 @@ snn_status_t snn_rleaky_bwd(const snn_scan_desc* desc, const void* I, const floa
 
 /*
  * Rate-coded readout loss (Sec. V-A: the predicted class is the output
- * neuron that fires most): cross-entropy of the spike counts over T.
- *   spk   [T, B, ld] in `dtype` (snn_dtype_t); the first C of ld neurons are
- *         the classes (C <= 1024)
+ * neuron, or with a population code (Sec. VII) the population of pop
+ * neurons, that fires most): cross-entropy of the spike counts over T.
+ *   spk   [T, B, ld] in `dtype` (snn_dtype_t); the first C*pop of ld
+ *         neurons are the classes' populations, class c owning neurons
+ *         c*pop .. c*pop + pop - 1 (C <= 1024, pop >= 1, C*pop <= 32768)
  *   labels int32 [B]
  *   batch_total  the batch the mean is taken over: 0 for B; the global batch
  *         (>= B) when these B samples are one data-parallel shard, so that
  *         the shards' losses and gradients add up to the global ones
- *   loss  fp32 [1] (out) = sum_b CE(sum_t spk[:, b, :C], y_b) / batch_total
- *   grad_spk [T, B, ld] (out) = (softmax - onehot) / batch_total for every
- *         t; 0 for neurons C..ld-1
- * Deterministic (fixed summation order).
+ *   loss  fp32 [1] (out) = sum_b CE(counts_b, y_b) / batch_total, with
+ *         counts_b[c] = sum_t sum_j spk[t, b, c*pop + j]
+ *   grad_spk [T, B, ld] (out) = (softmax - onehot)[class of the neuron] /
+ *         batch_total for every t; 0 for neurons C*pop .. ld-1
+ *   ws    device workspace of snn_rate_ce_workspace_bytes(B) bytes, 16-byte
+ *         aligned, zeroed once before the first call (every call leaves its
+ *         completion ticket at zero; re-zero after an error)
+ * One block per sample; the loss terms are added in sample order
+ * (deterministic).
  */
-snn_status_t snn_rate_ce_loss(int64_t T, int64_t B, int64_t C, int64_t ld, int64_t batch_total,
-                              int32_t dtype, const void* spk, const int32_t* labels, float* loss,
-                              void* grad_spk, snn_stream_t stream);
+size_t snn_rate_ce_workspace_bytes(int64_t B);
+snn_status_t snn_rate_ce_loss(int64_t T, int64_t B, int64_t C, int64_t pop, int64_t ld,
+                              int64_t batch_total, int32_t dtype, const void* spk,
+                              const int32_t* labels, float* loss, void* grad_spk, void* ws,
+                              size_t ws_bytes, snn_stream_t stream);
 
 /*
  * AdamW update of n fp32 master weights (the optimiser of the paper's

@@ -84,6 +84,8 @@ class DenseSNN:
             nb = snn.snn_dense_workspace_bytes(self.M, self.padded[l], self.padded[l + 1])
             self.ws_bwd.append(torch.zeros(nb, dtype=torch.uint8, device=dev))
         self.loss = torch.zeros(1, dtype=torch.float32, device=dev)
+        self.ws_loss = torch.zeros(snn.snn_rate_ce_workspace_bytes(B), dtype=torch.uint8,
+                                   device=dev)
         self.grad_out = torch.empty((T, B, self.padded[-1]), dtype=torch.bfloat16, device=dev)
         self.grad_in = [torch.empty((self.M, self.padded[l]), dtype=torch.bfloat16, device=dev)
                         for l in range(1, len(weights))]
@@ -124,8 +126,8 @@ class DenseSNN:
             out.append((f"scan_fwd{l}", lambda l=l, layer=layer: layer.forward(
                 self.I[l].view(T, B, -1), self.beta, self.thr, stream=stream)))
         out.append(("ce_loss", lambda: snn.snn_rate_ce_loss(
-            self.layers[-1].spk, labels, self.sizes[-1], self.loss, self.grad_out, stream,
-            batch_total=self.batch_total)))
+            self.layers[-1].spk, labels, self.w.n_classes, self.loss, self.grad_out,
+            self.ws_loss, stream, batch_total=self.batch_total, pop=self.w.pop)))
         for l in range(len(self.layers) - 1, -1, -1):
             grad = self.grad_out if l == len(self.layers) - 1 else \
                 self.grad_in[l].view(T, B, -1)

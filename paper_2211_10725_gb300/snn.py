@@ -75,7 +75,9 @@ _SIGS = {
     "snn_dense_layer_fwd": ([ctypes.c_int64] * 3 + [_P] * 4 + [ctypes.c_size_t, _P], ctypes.c_int),
     "snn_dense_workspace_bytes": ([ctypes.c_int64] * 3, ctypes.c_size_t),
     "snn_dense_layer_bwd": ([ctypes.c_int64] * 3 + [_P] * 6 + [ctypes.c_size_t, _P], ctypes.c_int),
-    "snn_rate_ce_loss": ([ctypes.c_int64] * 5 + [ctypes.c_int32] + [_P] * 4 + [_P], ctypes.c_int),
+    "snn_rate_ce_workspace_bytes": ([ctypes.c_int64], ctypes.c_size_t),
+    "snn_rate_ce_loss": ([ctypes.c_int64] * 6 + [ctypes.c_int32] + [_P] * 5 + [ctypes.c_size_t, _P],
+                         ctypes.c_int),
     "snn_adamw_step": ([ctypes.c_int64] + [_P] * 5 + [ctypes.c_float] * 5 + [ctypes.c_int64] +
                        [_P, _P], ctypes.c_int),
 }
@@ -257,14 +259,24 @@ def snn_dense_layer_bwd(X, W, dI, dX, dW, ws, stream=None):
                                               _stream(stream)), "snn_dense_layer_bwd")
 
 
-def snn_rate_ce_loss(spk, labels, C, loss, grad_spk, stream=None, batch_total=None):
-    """Cross-entropy on output spike counts; spk/grad_spk [T, B, ld].  The
-    mean is over batch_total samples (default B: this batch)."""
+def snn_rate_ce_workspace_bytes(B: int) -> int:
+    return load_library().snn_rate_ce_workspace_bytes(B)
+
+
+def snn_rate_ce_loss(spk, labels, C, loss, grad_spk, ws=None, stream=None, batch_total=None,
+                     pop=1):
+    """Cross-entropy on output spike counts; spk/grad_spk [T, B, ld], C
+    classes of pop neurons each.  The mean is over batch_total samples
+    (default B: this batch).  ws: a zeroed uint8 device tensor of
+    snn_rate_ce_workspace_bytes(B) bytes (a fresh one when None)."""
     T, B, ld = spk.shape
     dt = {torch.float32: 0, torch.bfloat16: 1, torch.float16: 2}[spk.dtype]
-    _check(load_library().snn_rate_ce_loss(T, B, C, ld, batch_total or 0, dt, _ptr(spk),
-                                           _ptr(labels), _ptr(loss), _ptr(grad_spk),
-                                           _stream(stream)), "snn_rate_ce_loss")
+    if ws is None:
+        ws = torch.zeros(snn_rate_ce_workspace_bytes(B), dtype=torch.uint8, device=spk.device)
+    _check(load_library().snn_rate_ce_loss(T, B, C, pop, ld, batch_total or 0, dt, _ptr(spk),
+                                           _ptr(labels), _ptr(loss), _ptr(grad_spk), _ptr(ws),
+                                           ws.numel() * ws.element_size(), _stream(stream)),
+           "snn_rate_ce_loss")
 
 
 def snn_adamw_step(w, w_bf16, grad, m, v, lr, beta1=0.9, beta2=0.999, eps=1e-8,

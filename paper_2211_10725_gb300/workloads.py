@@ -11,6 +11,8 @@ in for the datasets, which are not used):
 * ``leaky_T25_B128_N1000``      Leaky LIF layer (Eq. 4), fp32.
 * ``synaptic_T100_B128_N4096``  current-based LIF layer (Eqs. 5-6), fp32.
 * ``dsnn_784_1000_1000_10``     3-layer dense SNN, bf16 GEMMs, T=25, B=128.
+* ``dsnn_pop_3072_1000_500_T1``  2-layer dense SNN with a population-coded
+                                output (50 neurons per class), T=1.
 * ``conv_lif_T25_B128``         LIF on the conv-SNN activation shapes
                                 [12,24,24] and [64,8,8], per-channel beta.
 * ``leaky_bf16_T500_B64_N8192`` large Leaky layer, bf16 storage, per-neuron
@@ -178,6 +180,7 @@ class DenseWorkload:
     thr: float = 1.0
     sg_param: float = 25.0      # fast-sigmoid slope
     n_classes: int = 10
+    pop: int = 1                # output neurons per class (population code, Sec. VII)
     seed_index: int = 2
 
     def scaled(self, **kw) -> "DenseWorkload":
@@ -185,6 +188,13 @@ class DenseWorkload:
 
 
 DSNN_C3 = DenseWorkload()
+
+# Population-coded output (Sec. VII): one time step, a CIFAR-10-sized input
+# (32x32x3, synthetic spikes as for C3), 50 output neurons per class.
+DSNN_POP = DenseWorkload(name="dsnn_pop_3072_1000_500_T1_B128", T=1, B=128,
+                         sizes=(3072, 1000, 500), pop=50, seed_index=8)
+
+DENSE_WORKLOADS = {w.name: w for w in (DSNN_C3, DSNN_POP)}
 
 
 def make_dense_inputs(w: DenseWorkload, seed: Optional[int] = None) -> dict:

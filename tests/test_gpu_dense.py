@@ -109,5 +109,29 @@ def test_rate_ce_loss_shard_normalisation(cuda_device):
     assert abs(loss.item() - rl * k) <= 1e-6 * max(1.0, abs(rl))
     np.testing.assert_allclose(_np(grad.cpu())[:, :, :C], rg * k, rtol=1e-5, atol=1e-8)
     lib = snn.load_library()
-    assert lib.snn_rate_ce_loss(T, B, C, ld, B - 1, 0, grad.data_ptr(), labels.data_ptr(),
-                                loss.data_ptr(), grad.data_ptr(), None) == 1
+    ws = torch.zeros(snn.snn_rate_ce_workspace_bytes(B), dtype=torch.uint8, device=cuda_device)
+    args = (grad.data_ptr(), labels.data_ptr(), loss.data_ptr(), grad.data_ptr(), ws.data_ptr())
+    assert lib.snn_rate_ce_loss(T, B, C, 1, ld, B - 1, 0, *args, ws.numel(), None) == 1
+    assert lib.snn_rate_ce_loss(T, B, C, 2, ld, 0, 0, *args, ws.numel(), None) == 1  # C*pop > ld
+    assert lib.snn_rate_ce_loss(T, B, C, 1, ld, 0, 0, *args, 64, None) == 4         # workspace
+
+
+# (T, B, C, pop, ld): the population-coded output layer (500 = 10 x 50,
+# padded to 504), several time steps with a ragged population
+@pytest.mark.parametrize("T,B,C,pop,ld", [(1, 128, 10, 50, 504), (3, 37, 13, 7, 96)])
+@pytest.mark.parametrize("dtype", [torch.float32, torch.bfloat16])
+def test_rate_ce_loss_population(T, B, C, pop, ld, dtype, cuda_device):
+    g = torch.Generator().manual_seed(7 + pop)
+    spk = (torch.rand((T, B, ld), generator=g) < 0.2).to(dtype)
+    labels = torch.randint(0, C, (B,), generator=g, dtype=torch.int32)
+    loss = torch.zeros(1, dtype=torch.float32, device=cuda_device)
+    grad = torch.full((T, B, ld), float("nan"), dtype=dtype, device=cuda_device)
+    snn.snn_rate_ce_loss(spk.to(cuda_device), labels.to(cuda_device), C, loss, grad, pop=pop)
+    torch.cuda.synchronize()
+    rl, rg = O.rate_ce_loss(_np(spk[:, :, :C * pop]), labels.numpy(), pop)
+    assert abs(loss.item() - rl) <= 1e-6 * max(1.0, abs(rl))
+    got = _np(grad.cpu())
+    tol = 1e-7 if dtype == torch.float32 else 2 ** -8 * np.abs(rg).max()
+    np.testing.assert_allclose(got[:, :, :C * pop], rg,
+                               rtol=1e-5 if dtype == torch.float32 else 2e-2, atol=tol)
+    assert np.all(got[:, :, C * pop:] == 0)

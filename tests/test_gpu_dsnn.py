@@ -44,6 +44,8 @@ GRAD_RTOL = 6 * 2.0 ** -7
 MARGIN = 1e-4   # spike decisions / bf16 midpoints closer than this may differ
 
 SMALL = W.DSNN_C3.scaled(name="dsnn_784_128_64_10_T6_B16", T=6, B=16, sizes=(784, 128, 64, 10))
+SMALL_POP = W.DSNN_POP.scaled(name="dsnn_pop_784_128_60_T2_B16", T=2, B=16, sizes=(784, 128, 60),
+                              pop=6)
 
 
 def _np(t):
@@ -143,24 +145,24 @@ def _gpu_layer(net, l):
     }
 
 
-def _small_seed():
+def _small_seed(w):
     """First seed whose oracle run has every spike decision of every layer
     at least MARGIN from the threshold, with every layer spiking."""
     for s in range(200):
         seed = W.SEED_BASE + 1000 + s
-        inp = W.make_dense_inputs(SMALL, seed)
-        Ws, X, fwd = _oracle(SMALL, inp)
+        inp = W.make_dense_inputs(w, seed)
+        Ws, X, fwd = _oracle(w, inp)
         ok = all(0.0 < f.mean() for f in fwd["spk"])
-        ok = ok and all(bool(np.all(np.abs(m - SMALL.thr) > MARGIN)) for m in fwd["mem"])
+        ok = ok and all(bool(np.all(np.abs(m - w.thr) > MARGIN)) for m in fwd["mem"])
         if ok:
             return seed
     raise AssertionError("no seed with clear spike decisions")
 
 
-@pytest.mark.parametrize("save", ["recompute", "mem"])
-def test_dsnn_step_small_matches_oracle(save, cuda_device):
-    w = SMALL
-    seed = _small_seed()
+@pytest.mark.parametrize("w,save", [(SMALL, "recompute"), (SMALL, "mem"),
+                                    (SMALL_POP, "recompute")])
+def test_dsnn_step_small_matches_oracle(w, save, cuda_device):
+    seed = _small_seed(w)
     inp = W.make_dense_inputs(w, seed)
     Ws, X, fwd = _oracle(w, inp)
     net = _run(w, inp, cuda_device, save)
@@ -171,7 +173,7 @@ def test_dsnn_step_small_matches_oracle(save, cuda_device):
         # the backward reads the bf16 trace the forward stored
         fwd = dict(fwd, mem=[store(m) for m in fwd["mem"]])
     res = O.dsnn_backward(fwd, Ws, _np(inp["labels"]).astype(np.int64), T, B, w.beta, w.thr,
-                          w.sg_param, store=store)
+                          w.sg_param, store=store, pop=w.pop)
     mag = _magnitudes(w, Ws, fwd, res)
     unc = _storage_uncertainty(w, Ws, fwd32, res, mag) if save == "mem" else None
 
@@ -202,11 +204,12 @@ def test_dsnn_step_small_matches_oracle(save, cuda_device):
             assert not p.any(), f"layer {l} padding not zero"
 
 
-def test_dsnn_step_full_size(cuda_device):
-    """784-1000-1000-10, T = 25, B = 128 (the configuration timed by the
+@pytest.mark.parametrize("w", [W.DSNN_C3, W.DSNN_POP], ids=lambda w: w.name)
+def test_dsnn_step_full_size(w, cuda_device):
+    """784-1000-1000-10, T = 25, B = 128, and the population-coded
+    3072-1000-500 network at T = 1 (the configurations timed by the
     benchmark): per-sample parity for every sample whose spikes match in all
     layers, ambiguity-only differences elsewhere, and dW close overall."""
-    w = W.DSNN_C3
     inp = W.make_dense_inputs(w)
     Ws, X, fwd = _oracle(w, inp)
     net = _run(w, inp, cuda_device)
@@ -231,7 +234,7 @@ def test_dsnn_step_full_size(cuda_device):
     assert clean.sum() >= B // 2, f"only {clean.sum()} samples agree in every layer"
 
     res = O.dsnn_backward(fwd, Ws, _np(inp["labels"]).astype(np.int64), T, B, w.beta, w.thr,
-                          w.sg_param, store=O.bf16_round)
+                          w.sg_param, store=O.bf16_round, pop=w.pop)
     mag = _magnitudes(w, Ws, fwd, res)
     for l in range(len(Ws)):
         g = _gpu_layer(net, l)
