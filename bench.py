@@ -47,6 +47,8 @@ def parse():
                    help="dense-SNN workload: launch the step eagerly, not as a CUDA graph")
     p.add_argument("--no-e2e", action="store_true")
     p.add_argument("--no-cpu-baseline", action="store_true")
+    p.add_argument("--no-torch-eager", action="store_true",
+                   help="skip the PyTorch-eager per-timestep context measurement")
     p.add_argument("--cpu-seconds", type=float, default=15.0)
     return p.parse_args()
 
@@ -443,6 +445,9 @@ def run_ours(args):
     if w.neuron == "rleaky":
         modes.add(w.v_mode)
     launches_per_step = 2 + len(modes)
+    eager = None
+    if not args.no_torch_eager and world == 1:
+        eager = time_torch_eager(w, inp, dev)
     cpu = None
     if not args.no_cpu_baseline and world == 1:
         v, n, dt = time_oracle(w, inp, args.cpu_seconds)
@@ -473,6 +478,7 @@ def run_ours(args):
         "clocks": clocks,
         "gpu_launches": launches_per_step * K,
         "cpu_baseline": cpu,
+        "torch_eager_context": eager,
         "e2e": e2e,
     }
     print(json.dumps(line), flush=True)
@@ -766,6 +772,85 @@ def run_dense_e2e(args, w, inp, net, dev, world):
     return {"value": world * w.T * w.B * sum(w.sizes[1:]) * K / (ms * 1e-3), "unit": UNIT,
             "h2d_bytes_per_step": nb(hX) + nb(hy), "d2h_bytes_per_step": nb(out), "steps": K,
             "launch": "eager"}
+
+
+def time_torch_eager(w, inp, dev, steps=2):
+    """Context only: the same fwd + BPTT as a PyTorch-eager per-timestep loop
+    with autograd on the same GPU (the shape of the paper's GPU path),
+    written from Eqs. (3)-(7): fp32 state, the surrogate as a custom
+    backward, the reset detached as the workload says.  Returns NS/s."""
+    import math
+    import torch
+
+    fast = w.surrogate == "fast_sigmoid"
+    k, a_half, b_arg = w.sg_param, 0.5 * w.sg_param, math.pi * 0.5 * w.sg_param
+
+    class Spike(torch.autograd.Function):
+        @staticmethod
+        def forward(ctx, x):
+            ctx.save_for_backward(x)
+            return (x > 0).float()
+
+        @staticmethod
+        def backward(ctx, g):
+            (x,) = ctx.saved_tensors
+            if fast:
+                return g / (1.0 + k * x.abs()) ** 2
+            return g * a_half / (1.0 + (b_arg * x) ** 2)
+
+    def lane(p, mode):
+        t = p.to(dev).float()
+        if mode == "per_channel":
+            t = t.repeat_interleave(w.HW).repeat(w.N // (w.C * w.HW))
+        return t.reshape(1, -1).expand(w.B, w.N)
+
+    I = inp["I"].to(dev)
+    gs = inp["grad_spk"].to(dev).float()
+
+    def one():
+        beta = lane(inp["beta"], w.beta_mode).clone().requires_grad_(True)
+        thr = lane(inp["thr"], w.thr_mode).clone().requires_grad_(True)
+        x = I.float().requires_grad_(True)
+        third = None
+        if w.neuron == "synaptic":
+            third = lane(inp["alpha"], w.alpha_mode).clone().requires_grad_(True)
+        elif w.neuron == "rleaky":
+            third = lane(inp["v"], w.v_mode).clone().requires_grad_(True)
+        u = torch.zeros(w.B, w.N, device=dev)
+        i = torch.zeros_like(u)
+        z = torch.zeros_like(u)
+        loss = 0.0
+        for t in range(w.T):
+            zr = z.detach() if w.detach_reset else z
+            inp_t = x[t]
+            if w.neuron == "synaptic":
+                i = third * i + x[t]
+                inp_t = i
+            if w.reset == "zero":
+                u = beta * ((1 - zr) * u) + inp_t
+            elif w.reset == "none":
+                u = beta * u + inp_t
+            else:
+                u = beta * u + inp_t - zr * thr
+            if w.neuron == "rleaky":
+                u = u + z * third
+            z = Spike.apply(u - thr)
+            loss = loss + (z * gs[t]).sum()
+        loss.backward()
+
+    one()
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record()
+    for _ in range(steps):
+        one()
+    e1.record()
+    torch.cuda.synchronize()
+    ms = e0.elapsed_time(e1) / steps
+    return {"value": w.T * w.B * w.N / (ms * 1e-3), "unit": UNIT, "ms_per_step": ms,
+            "steps": steps, "kind": "context",
+            "note": "PyTorch eager per-timestep loop with autograd on the same GPU, fp32 "
+                    "state; context for the paper's GPU path, not a baseline of this build"}
 
 
 def run_e2e(args, w, inp, layer, dev, world):
