@@ -17,6 +17,7 @@
 #include <cmath>
 #include <cstdint>
 
+#include "launch.cuh"
 #include "snn.h"
 
 namespace snn {
@@ -65,6 +66,7 @@ __global__ void __launch_bounds__(kAdamThreads) adamw_kernel(int64_t n, float* _
                                                              float* __restrict__ v, AdamCoef c,
                                                              AdamHyper h,
                                                              unsigned long long* counter) {
+  grid_dep_wait();
   if (counter) {
     // counter[0]: updates done so far; counter[1]: blocks finished reading
     __shared__ AdamCoef sc;
@@ -145,8 +147,9 @@ extern "C" snn_status_t snn_adamw_step(int64_t n, float* w, void* w_bf16, const 
     cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
   const int64_t want = (n / 4 + snn::kAdamThreads - 1) / snn::kAdamThreads;
   const int blocks = (int)std::max<int64_t>(1, std::min<int64_t>(want, (int64_t)sms * 8));
-  snn::adamw_kernel<<<blocks, snn::kAdamThreads, 0, reinterpret_cast<cudaStream_t>(stream)>>>(
-      n, w, static_cast<__nv_bfloat16*>(w_bf16), grad, m, v, c, h,
-      reinterpret_cast<unsigned long long*>(step_counter));
-  return cudaGetLastError() == cudaSuccess ? SNN_OK : SNN_ERR_CUDA;
+  const cudaError_t e = snn::launch_pdl(
+      snn::adamw_kernel, dim3(blocks), dim3(snn::kAdamThreads), 0,
+      reinterpret_cast<cudaStream_t>(stream), n, w, static_cast<__nv_bfloat16*>(w_bf16), grad, m,
+      v, c, h, reinterpret_cast<unsigned long long*>(step_counter));
+  return e == cudaSuccess ? SNN_OK : SNN_ERR_CUDA;
 }

@@ -59,6 +59,7 @@ __global__ void __launch_bounds__(kCeThreads) rate_ce_kernel(int64_t Tn, int64_t
   float* ncnt = ce_smem;       // [CP] neuron counts
   float* ccnt = ce_smem + CP;  // [C] class counts, then class gradients
   __shared__ int last;
+  grid_dep_wait();
   const int64_t b = blockIdx.x;
   const int64_t step = B * ld;
   const T* row = spk + b * ld;
@@ -133,10 +134,9 @@ cudaError_t launch_ce(int64_t Tn, int64_t B, int C, int pop, int64_t ld, int64_t
   const void* k = (const void*)rate_ce_kernel<T>;
   const cudaError_t e = ensure_smem(k, smem);
   if (e != cudaSuccess) return e;
-  rate_ce_kernel<T><<<(unsigned)B, kCeThreads, smem, st>>>(
-      Tn, B, C, pop, ld, Bn, static_cast<const T*>(spk), labels, loss, static_cast<T*>(grad),
-      terms, ticket);
-  return cudaGetLastError();
+  return launch_pdl(rate_ce_kernel<T>, dim3((unsigned)B), dim3(kCeThreads), smem, st, Tn, B, C,
+                    pop, ld, Bn, static_cast<const T*>(spk), labels, loss, static_cast<T*>(grad),
+                    terms, ticket);
 }
 
 }  // namespace

@@ -253,6 +253,7 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm)
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
+  grid_dep_wait();  // the previous kernel on the stream is complete
 
   if (warp == 0) {
     if (lid == 0) {
@@ -435,8 +436,8 @@ cudaError_t launch_bn(const CUtensorMap& ta, const CUtensorMap& tb, const GemmAr
   const int64_t tiles = (int64_t)((g.N + BN - 1) / BN) * ((g.M + BM - 1) / BM);
   const int64_t slots = (int64_t)sms * kCtasPerSm;
   const unsigned grid = (unsigned)(tiles < slots ? tiles : slots);  // persistent CTAs
-  gemm_tn_tcgen05<BN, OUT_BF16, A_MN, B_MN><<<grid, kThreads, smem_bytes<BN>(), st>>>(ta, tb, g);
-  return cudaGetLastError();
+  return launch_pdl(gemm_tn_tcgen05<BN, OUT_BF16, A_MN, B_MN>, dim3(grid), dim3(kThreads),
+                    smem_bytes<BN>(), st, ta, tb, g);
 }
 
 // D[M, N] = A[M, K] * B[N, K]^T.  A is stored [M, K] row-major (K-major) or,

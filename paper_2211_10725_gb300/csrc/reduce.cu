@@ -57,6 +57,7 @@ __device__ __forceinline__ bool last_of_group(int* ticket, int splits) {
 __global__ void __launch_bounds__(kRedThreads) reduce_scalar(ReduceJobs js, int64_t L,
                                                               int64_t chunk) {
   __shared__ double sh[kRedThreads];
+  grid_dep_wait();
   const ReduceJob& j = js.job[blockIdx.z];
   const int S = gridDim.y;
   const int64_t lo = (int64_t)blockIdx.y * chunk;
@@ -79,6 +80,7 @@ __global__ void __launch_bounds__(kRedThreads) reduce_scalar(ReduceJobs js, int6
 // [B*y/S, B*(y+1)/S); the last split adds the S partials of each neuron.
 __global__ void __launch_bounds__(kRedThreads) reduce_per_neuron(ReduceJobs js, int64_t B,
                                                                   int64_t N) {
+  grid_dep_wait();
   const ReduceJob& j = js.job[blockIdx.z];
   const int64_t n = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
   const int64_t S = gridDim.y, s = blockIdx.y;
@@ -105,6 +107,7 @@ __global__ void __launch_bounds__(kRedThreads) reduce_per_channel(ReduceJobs js,
                                                                    int64_t N, int64_t C,
                                                                    int64_t HW) {
   __shared__ double sh[kRedThreads];
+  grid_dep_wait();
   const ReduceJob& j = js.job[blockIdx.z];
   const int64_t c = blockIdx.x, s = blockIdx.y, S = gridDim.y;
   const int64_t R = N / (C * HW);
@@ -144,14 +147,19 @@ cudaError_t launch_param_reduce(const ParamReduce* p, int n, int64_t B, int64_t 
     if (nb < 1) nb = 1;
     const int64_t chunk = ceil_div(L > 0 ? L : 1, nb);
     nb = ceil_div(L > 0 ? L : 1, chunk);
-    reduce_scalar<<<dim3(1, (unsigned)nb, (unsigned)n), kRedThreads, 0, stream>>>(js, L, chunk);
+    const cudaError_t e = launch_pdl(reduce_scalar, dim3(1, (unsigned)nb, (unsigned)n),
+                                     dim3(kRedThreads), 0, stream, js, L, chunk);
+    if (e != cudaSuccess) return e;
   } else if (mode == PM_PER_NEURON) {
     if (N > 0) {
       int64_t S = B < kNeuronSplit ? B : kNeuronSplit;
       if (S * N > scratch_len) S = scratch_len / N;
       if (S < 1) return cudaErrorInvalidValue;  // the workspace is sized for S >= 1
-      reduce_per_neuron<<<dim3((unsigned)ceil_div(N, kRedThreads), (unsigned)S, (unsigned)n),
-                          kRedThreads, 0, stream>>>(js, B, N);
+      const cudaError_t e =
+          launch_pdl(reduce_per_neuron, dim3((unsigned)ceil_div(N, kRedThreads), (unsigned)S,
+                                             (unsigned)n),
+                     dim3(kRedThreads), 0, stream, js, B, N);
+      if (e != cudaSuccess) return e;
     }
   } else if (C > 0) {
     const int64_t R = N / (C * HW);
@@ -162,8 +170,9 @@ cudaError_t launch_param_reduce(const ParamReduce* p, int n, int64_t B, int64_t 
     if (S > B * R) S = B * R;
     if (S > scratch_len / C) S = scratch_len / C;
     if (S < 1) return cudaErrorInvalidValue;  // the workspace is sized for S >= 1
-    reduce_per_channel<<<dim3((unsigned)C, (unsigned)S, (unsigned)n), kRedThreads, 0, stream>>>(
-        js, B, N, C, HW);
+    const cudaError_t e = launch_pdl(reduce_per_channel, dim3((unsigned)C, (unsigned)S, (unsigned)n),
+                                     dim3(kRedThreads), 0, stream, js, B, N, C, HW);
+    if (e != cudaSuccess) return e;
   }
   return cudaGetLastError();
 }

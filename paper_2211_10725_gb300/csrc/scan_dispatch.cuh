@@ -24,9 +24,9 @@ cudaError_t fwd_staged(ScanArgs a, cudaStream_t st, bool* launched) {
   a.lanes_per_cta = p.lanes_per_cta;
   a.stages = p.stages;
   a.stage_bytes = p.stage_bytes;
-  scan_fwd_staged<SYN, TI, TO, RESET, REC><<<(unsigned)p.grid, p.threads, p.smem, st>>>(a);
   *launched = true;
-  return cudaGetLastError();
+  return launch_pdl(scan_fwd_staged<SYN, TI, TO, RESET, REC>, dim3((unsigned)p.grid),
+                    dim3(p.threads), p.smem, st, a);
 }
 
 template <bool SYN, typename TI, typename TO>
@@ -41,8 +41,8 @@ cudaError_t fwd_t(ScanArgs a, bool staged, cudaStream_t st) {
     if (launched || e != cudaSuccess) return e;
   }
   if (a.L == 0) return cudaSuccess;
-  scan_fwd_plain<SYN, TI, TO><<<(unsigned)ceil_div(a.L, 256), 256, 0, st>>>(a);
-  return cudaGetLastError();
+  return launch_pdl(scan_fwd_plain<SYN, TI, TO>, dim3((unsigned)ceil_div(a.L, 256)), dim3(256), 0,
+                    st, a);
 }
 
 template <bool SYN, bool RECOMP, typename TI, typename TO, int RESET, int SG, int KC = 0,
@@ -70,10 +70,9 @@ cudaError_t bwd_staged(ScanArgs a, cudaStream_t st, bool* launched) {
   a.lanes_per_cta = p.lanes_per_cta;
   a.stages = p.stages;
   a.stage_bytes = p.stage_bytes;
-  scan_bwd_staged<SYN, RECOMP, TI, TO, RESET, SG, KC, REC><<<(unsigned)p.grid, p.threads, p.smem,
-                                                             st>>>(a);
   *launched = true;
-  return cudaGetLastError();
+  return launch_pdl(scan_bwd_staged<SYN, RECOMP, TI, TO, RESET, SG, KC, REC>,
+                    dim3((unsigned)p.grid), dim3(p.threads), p.smem, st, a);
 }
 
 template <bool SYN, bool RECOMP, typename TI, typename TO>
@@ -124,8 +123,8 @@ cudaError_t bwd_t(ScanArgs a, bool staged, cudaStream_t st) {
   const void* k = (const void*)scan_bwd_plain<SYN, RECOMP, TI, TO>;
   cudaError_t e = ensure_smem(k, smem);
   if (e != cudaSuccess) return e;
-  scan_bwd_plain<SYN, RECOMP, TI, TO><<<(unsigned)ceil_div(a.L, threads), threads, smem, st>>>(a);
-  return cudaGetLastError();
+  return launch_pdl(scan_bwd_plain<SYN, RECOMP, TI, TO>, dim3((unsigned)ceil_div(a.L, threads)),
+                    dim3(threads), smem, st, a);
 }
 
 // dtype codes (snn_dtype_t): 0 f32, 1 bf16, 2 f16.  Instantiated pairs

@@ -22,6 +22,7 @@
 // they give bit-identical forward results.
 #pragma once
 
+#include "launch.cuh"
 #include "snn_device.cuh"
 
 namespace snn {
@@ -505,6 +506,7 @@ __global__ void __launch_bounds__(kMaxStagedThreads) scan_fwd_staged(const ScanA
   const int64_t lane0 = (int64_t)blockIdx.x * a.lanes_per_cta;
   const int cta_lanes = (int)min((int64_t)a.lanes_per_cta, a.L - lane0);
   init_ring_barriers(full, empty, S, cwarps);
+  grid_dep_wait();  // the previous kernel on the stream is complete
 
   if (warp == cwarps) {  // producer warp
     if (lid == 0 && !(a.debug & DEBUG_PRODUCER_IDLE)) {
@@ -648,6 +650,7 @@ __global__ void __launch_bounds__(kMaxStagedThreads) scan_bwd_staged(const ScanA
   unsigned char* ck_base = ring + (size_t)S * a.stage_bytes +
                            (RECOMP ? (size_t)nthr * V * 4 * a.K * (SYN ? 2 : 1) : 0);
   init_ring_barriers(full, empty, S, cwarps);
+  grid_dep_wait();  // the previous kernel on the stream is complete
 
   if (warp == cwarps) {
     if (lid == 0 && !(a.debug & DEBUG_PRODUCER_IDLE)) {
@@ -1010,6 +1013,7 @@ __global__ void __launch_bounds__(kMaxStagedThreads) scan_bwd_staged(const ScanA
 
 template <bool SYN, typename TI, typename TO>
 __global__ void __launch_bounds__(256) scan_fwd_plain(const ScanArgs a) {
+  grid_dep_wait();
   const int64_t l = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
   if (l >= a.L) return;
   const float beta = lane_param(a.beta, a.beta_mode, l, a);
@@ -1048,6 +1052,7 @@ __global__ void __launch_bounds__(256) scan_fwd_plain(const ScanArgs a) {
 template <bool SYN, bool RECOMP, typename TI, typename TO>
 __global__ void __launch_bounds__(128) scan_bwd_plain(const ScanArgs a) {
   extern __shared__ __align__(16) float segbuf[];  // [K][blockDim] u, then i
+  grid_dep_wait();
   const int64_t l = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
   if (l >= a.L) return;
   const float beta = lane_param(a.beta, a.beta_mode, l, a);
