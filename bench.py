@@ -50,6 +50,8 @@ def parse():
     p.add_argument("--no-torch-eager", action="store_true",
                    help="skip the PyTorch-eager per-timestep context measurement")
     p.add_argument("--cpu-seconds", type=float, default=15.0)
+    p.add_argument("--reference-seconds", type=float, default=120.0,
+                   help="--impl reference: about how long the whole run takes")
     return p.parse_args()
 
 
@@ -276,7 +278,7 @@ def run_dense_reference(args):
     one(np.arange(8))
     per_sample = (time.perf_counter() - t0) / 8
     total = max(1, args.steps + args.warmup)
-    n = int(max(1, min(w.B, 120.0 / total / per_sample)))
+    n = int(max(1, min(w.B, args.reference_seconds / total / per_sample)))
     rng = np.random.default_rng(0)
     samples = [np.sort(rng.choice(w.B, n, replace=False)) for _ in range(total)]
     for i in range(args.warmup):
@@ -319,7 +321,7 @@ def run_reference(args):
     oracle_step(w, inp, np.arange(probe))
     per_lane = (time.perf_counter() - t0) / probe
     total = max(1, args.steps + args.warmup)
-    n = int(max(64, min(L, 120.0 / total / per_lane)))
+    n = int(max(64, min(L, args.reference_seconds / total / per_lane)))
     rng = np.random.default_rng(0)
     samples = [np.sort(rng.choice(L, n, replace=False)) for _ in range(total)]
     for i in range(args.warmup):
