@@ -546,3 +546,140 @@ def adamw_step(w, g, m, v, lr, beta1, beta2, eps, weight_decay, step):
     v_hat = v / (1.0 - beta2 ** step)
     w = w - lr * weight_decay * w - lr * m_hat / (np.sqrt(v_hat) + eps)
     return w, m, v
+
+
+# ---------------------------------------------------------------------------
+# The convolutional SNN of Tab. I (CSNN): 5x5 convolutions and 2x2 max
+# pooling around Leaky layers, channel-last activations [M, H, W, C]
+# ---------------------------------------------------------------------------
+
+def conv2d_nhwc(X, Wc):
+    """Valid 2-D convolution (stride 1) of X [M, H, W, Cin] with filters
+    Wc [Cout, KH, KW, Cin]: Y[m, y, x, o] = sum_{ky,kx,c} X[m, y+ky, x+kx, c]
+    * Wc[o, ky, kx, c] (float64).  Returns [M, H-KH+1, W-KW+1, Cout]."""
+    X = np.asarray(X, np.float64)
+    Wc = np.asarray(Wc, np.float64)
+    KH, KW = Wc.shape[1], Wc.shape[2]
+    win = np.lib.stride_tricks.sliding_window_view(X, (KH, KW), axis=(1, 2))
+    # win: [M, Ho, Wo, Cin, KH, KW]
+    return np.einsum("mhwcij,oijc->mhwo", win, Wc)
+
+
+def conv2d_nhwc_backward(X, Wc, dY):
+    """Gradients of conv2d_nhwc: dX [M, H, W, Cin] (each output gradient
+    spread back over the input window it read) and dW [Cout, KH, KW, Cin]."""
+    X = np.asarray(X, np.float64)
+    Wc = np.asarray(Wc, np.float64)
+    dY = np.asarray(dY, np.float64)
+    KH, KW = Wc.shape[1], Wc.shape[2]
+    Ho, Wo = dY.shape[1], dY.shape[2]
+    win = np.lib.stride_tricks.sliding_window_view(X, (KH, KW), axis=(1, 2))
+    dW = np.einsum("mhwo,mhwcij->oijc", dY, win)
+    dX = np.zeros_like(X)
+    for ky in range(KH):
+        for kx in range(KW):
+            dX[:, ky:ky + Ho, kx:kx + Wo, :] += np.einsum("mhwo,oc->mhwc", dY, Wc[:, ky, kx, :])
+    return dX, dW
+
+
+def maxpool2_nhwc(X):
+    """2x2 max pooling with stride 2 of X [M, H, W, C] (H, W even).  Returns
+    (Y [M, H/2, W/2, C], idx) where idx is the window position (0..3, row
+    major) of the first maximum, which the backward routes the gradient to."""
+    X = np.asarray(X, np.float64)
+    M, H, W, C = X.shape
+    w = X.reshape(M, H // 2, 2, W // 2, 2, C).transpose(0, 1, 3, 5, 2, 4).reshape(
+        M, H // 2, W // 2, C, 4)
+    idx = np.argmax(w, axis=-1)   # first maximum in window order
+    return np.take_along_axis(w, idx[..., None], -1)[..., 0], idx
+
+
+def maxpool2_nhwc_backward(dY, idx, shape):
+    """Gradient of maxpool2_nhwc: dY to the window position idx, 0 elsewhere."""
+    M, H, W, C = shape
+    d = np.zeros((M, H // 2, W // 2, C, 4))
+    np.put_along_axis(d, np.asarray(idx)[..., None], np.asarray(dY, np.float64)[..., None], -1)
+    return d.reshape(M, H // 2, W // 2, C, 2, 2).transpose(0, 1, 4, 2, 5, 3).reshape(M, H, W, C)
+
+
+def csnn_forward(X, convs, Wfc, T: int, B: int, beta_convs, beta_fc: float, thr: float,
+                 reset: str = "zero", dtype=np.float32):
+    """Forward pass of the CSNN: per conv layer conv2d_nhwc, a Leaky layer
+    (Eq. 4 with the given reset, per-channel beta) over t, maxpool2_nhwc;
+    then a dense layer (the flattened [H, W, C] map) and a Leaky output
+    layer.  X: [T*B, H, W, Cin] input spikes; convs: list of [Cout, KH, KW,
+    Cin] filters; Wfc [Nout, H*W*C]; beta_convs: per-channel betas (one
+    array per conv layer).  Spike decisions in ``dtype``.
+
+    Returns a dict of per-layer lists: ``ins`` (layer input), ``I`` (input
+    current, float64), ``spk``/``mem`` ([T, B*N], N = H*W*C), ``pool`` (the
+    pooled spikes) and ``idx`` (pooling positions)."""
+    x = np.asarray(X, np.float64)
+    out = {"ins": [], "I": [], "spk": [], "mem": [], "pool": [], "idx": []}
+    for Wc, bc in zip(convs, beta_convs):
+        I = conv2d_nhwc(x, Wc)
+        Mq, Ho, Wo, Co = I.shape
+        L = B * Ho * Wo * Co
+        beta = np.tile(np.asarray(bc, np.float64), B * Ho * Wo)  # channel-last lanes
+        spk, mem = leaky_forward(I.astype(dtype).reshape(T, L), beta.astype(dtype),
+                                 np.full(L, thr, dtype), reset, dtype=dtype)
+        s = spk.astype(np.float64).reshape(T * B, Ho, Wo, Co)
+        p, idx = maxpool2_nhwc(s)
+        for k, v in (("ins", x), ("I", I), ("spk", spk.astype(np.float64)),
+                     ("mem", mem.astype(np.float64)), ("pool", p), ("idx", idx)):
+            out[k].append(v)
+        x = p
+    flat = x.reshape(T * B, -1)
+    I = dense_forward(flat, Wfc)
+    n = Wfc.shape[0]
+    spk, mem = leaky_forward(I.astype(dtype).reshape(T, B * n), np.full(B * n, beta_fc, dtype),
+                             np.full(B * n, thr, dtype), reset, dtype=dtype)
+    out["fc_in"], out["fc_I"] = flat, I
+    out["fc_spk"], out["fc_mem"] = spk.astype(np.float64), mem.astype(np.float64)
+    return out
+
+
+def csnn_backward(fwd, convs, Wfc, labels, T: int, B: int, beta_convs, beta_fc: float,
+                  thr: float, sg_param: float, reset: str = "zero", store=None):
+    """Loss and BPTT of ``csnn_forward``: rate_ce_loss on the output spikes;
+    the output layer's BPTT and dense backward; then per conv layer from
+    the top the max-pool backward, the Leaky BPTT (detached reset,
+    fast-sigmoid slope ``sg_param``; per-channel beta gradients) and the
+    convolution backward.  ``store`` rounds where the path keeps a value in
+    a storage format (as in dsnn_backward).
+
+    Returns dict: loss, dW_fc, dW (per conv layer), dbeta (per conv layer,
+    per channel), and the gradients of every stage (grad_out, grad_I_fc,
+    grad_pool, grad_I)."""
+    keep = (lambda a: a) if store is None else store
+    n = Wfc.shape[0]
+    loss, g_out = rate_ce_loss(fwd["fc_spk"].reshape(T, B, n), labels)
+    g_out = keep(g_out)
+    g = leaky_backward(fwd["fc_mem"], fwd["fc_spk"], g_out.reshape(T, B * n),
+                       np.full(B * n, beta_fc), np.full(B * n, thr), reset=reset, detach=True,
+                       sg="fast_sigmoid", sg_param=sg_param)
+    dI_fc = keep(g["grad_I"]).reshape(T * B, n)
+    d_flat, dW_fc = dense_backward(fwd["fc_in"], Wfc, dI_fc)
+    res = {"loss": loss, "grad_out": g_out, "grad_I_fc": dI_fc, "dW_fc": dW_fc,
+           "dW": [None] * len(convs), "dbeta": [None] * len(convs),
+           "grad_pool": [None] * len(convs), "grad_I": [None] * len(convs)}
+    d_pool = keep(d_flat).reshape(fwd["pool"][-1].shape)
+    for l in range(len(convs) - 1, -1, -1):
+        res["grad_pool"][l] = d_pool
+        s_shape = fwd["I"][l].shape
+        Mq, Ho, Wo, Co = s_shape
+        d_spk = maxpool2_nhwc_backward(d_pool, fwd["idx"][l], s_shape)
+        L = B * Ho * Wo * Co
+        beta = np.tile(np.asarray(beta_convs[l], np.float64), B * Ho * Wo)
+        g = leaky_backward(fwd["mem"][l], fwd["spk"][l], d_spk.reshape(T, L), beta,
+                           np.full(L, thr), reset=reset, detach=True, sg="fast_sigmoid",
+                           sg_param=sg_param)
+        dI = keep(g["grad_I"]).reshape(T * B, Ho, Wo, Co)
+        res["grad_I"][l] = dI
+        res["dbeta"][l] = reduce_lane_grad(g["grad_beta_lane"], B, Ho * Wo * Co, "per_channel",
+                                           C=Co, HW=1)
+        dX, dW = conv2d_nhwc_backward(fwd["ins"][l], convs[l], dI)
+        res["dW"][l] = dW
+        if l > 0:
+            d_pool = keep(dX)
+    return res

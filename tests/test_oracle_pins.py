@@ -585,3 +585,99 @@ def test_population_ce_matches_torch_autograd():
     l1, g1 = O.rate_ce_loss(spk[:, :, :C], y, 1)
     l2, g2 = O.rate_ce_loss(spk[:, :, :C], y)
     assert l1 == l2 and np.array_equal(g1, g2)
+
+
+# ---------------------------------------------------------------------------
+# Convolutional SNN pieces (channel-last) against torch's NCHW operators
+# ---------------------------------------------------------------------------
+
+def test_conv2d_nhwc_matches_torch():
+    rng = np.random.default_rng(16)
+    X = rng.normal(0, 1, (3, 9, 11, 4))
+    Wc = rng.normal(0, 1, (5, 3, 2, 4))
+    tX = torch.tensor(X.transpose(0, 3, 1, 2), requires_grad=True)
+    tW = torch.tensor(Wc.transpose(0, 3, 1, 2), requires_grad=True)
+    y = torch.nn.functional.conv2d(tX, tW)
+    dY = rng.normal(0, 1, y.shape)
+    y.backward(torch.tensor(dY))
+    np.testing.assert_allclose(O.conv2d_nhwc(X, Wc), y.detach().numpy().transpose(0, 2, 3, 1),
+                               rtol=1e-12, atol=1e-12)
+    dX, dW = O.conv2d_nhwc_backward(X, Wc, dY.transpose(0, 2, 3, 1))
+    np.testing.assert_allclose(dX, tX.grad.numpy().transpose(0, 2, 3, 1), rtol=1e-12, atol=1e-12)
+    np.testing.assert_allclose(dW, tW.grad.numpy().transpose(0, 2, 3, 1), rtol=1e-12, atol=1e-12)
+
+
+def test_maxpool2_nhwc_matches_torch_including_ties():
+    rng = np.random.default_rng(17)
+    X = (rng.uniform(0, 1, (4, 6, 8, 3)) < 0.3).astype(np.float64)   # binary: many ties
+    tX = torch.tensor(X.transpose(0, 3, 1, 2), requires_grad=True)
+    y = torch.nn.functional.max_pool2d(tX, 2)
+    dY = rng.normal(0, 1, y.shape)
+    y.backward(torch.tensor(dY))
+    Y, idx = O.maxpool2_nhwc(X)
+    np.testing.assert_array_equal(Y, y.detach().numpy().transpose(0, 2, 3, 1))
+    dX = O.maxpool2_nhwc_backward(dY.transpose(0, 2, 3, 1), idx, X.shape)
+    np.testing.assert_array_equal(dX, tX.grad.numpy().transpose(0, 2, 3, 1))
+
+
+def test_csnn_matches_torch_autograd():
+    """The CSNN (conv -> Leaky with per-channel beta and reset to zero ->
+    max pool, twice, then dense -> Leaky, rate-coded CE) against a torch
+    float64 NCHW network differentiated by autograd with the reset
+    detached: spikes, loss, every filter, the dense weights and the
+    per-channel beta gradients agree."""
+    rng = np.random.default_rng(18)
+    T, B, k = 3, 2, 5.0
+    X = (rng.uniform(0, 1, (T * B, 16, 16, 1)) < 0.4).astype(np.float64)
+    convs = [rng.uniform(-1, 1, (3, 5, 5, 1)) * 0.6, rng.uniform(-1, 1, (4, 5, 5, 3)) * 0.5]
+    # 16x16 -conv5-> 12x12 -pool-> 6x6 -conv5-> 2x2 -pool-> 1x1: 4 features
+    Wfc = rng.uniform(-1, 1, (5, 4)) * 1.5
+    betas = [rng.uniform(0.7, 0.95, 3), rng.uniform(0.7, 0.95, 4)]
+    beta_fc, thr = 0.9, 1.0
+    y = rng.integers(0, 5, B)
+    fwd = O.csnn_forward(X, convs, Wfc, T, B, betas, beta_fc, thr, dtype=np.float64)
+    res = O.csnn_backward(fwd, convs, Wfc, y, T, B, betas, beta_fc, thr, k)
+
+    tconv = [torch.tensor(c.transpose(0, 3, 1, 2), requires_grad=True) for c in convs]
+    tbeta = [torch.tensor(b, requires_grad=True) for b in betas]
+    tfc = torch.tensor(Wfc, requires_grad=True)
+    x = torch.tensor(X.transpose(0, 3, 1, 2))            # [T*B, C, H, W]
+    spikes = []
+    for wc, bc in zip(tconv, tbeta):
+        cur = torch.nn.functional.conv2d(x, wc)
+        C_, H_, W_ = cur.shape[1:]
+        cur = cur.reshape(T, B, C_, H_, W_)
+        u = torch.zeros(B, C_, H_, W_, dtype=torch.float64)
+        z = torch.zeros_like(u)
+        zs = []
+        for t in range(T):
+            u = bc.view(1, -1, 1, 1) * ((1 - z.detach()) * u) + cur[t]
+            z = _SpikeFastSigmoid.apply(u - thr, k)
+            zs.append(z)
+        s = torch.stack(zs).reshape(T * B, C_, H_, W_)
+        spikes.append(s)
+        x = torch.nn.functional.max_pool2d(s, 2)
+    flat = x.permute(0, 2, 3, 1).reshape(T * B, -1)      # channel-last flattening
+    cur = (flat @ tfc.T).reshape(T, B, -1)
+    u = torch.zeros(B, Wfc.shape[0], dtype=torch.float64)
+    z = torch.zeros_like(u)
+    zs = []
+    for t in range(T):
+        u = beta_fc * ((1 - z.detach()) * u) + cur[t]
+        z = _SpikeFastSigmoid.apply(u - thr, k)
+        zs.append(z)
+    out = torch.stack(zs)
+    loss = torch.nn.functional.cross_entropy(out.sum(0), torch.tensor(y))
+    loss.backward()
+
+    for l, s in enumerate(spikes):
+        assert np.array_equal(fwd["spk"][l].reshape(-1), s.detach().numpy().transpose(0, 2, 3, 1).reshape(-1))
+    assert np.array_equal(fwd["fc_spk"], out.detach().numpy().reshape(T, -1))
+    assert all(0 < s.mean() < 1 for s in fwd["spk"])
+    assert abs(res["loss"] - loss.item()) < 1e-12
+    np.testing.assert_allclose(res["dW_fc"], tfc.grad.numpy(), rtol=1e-10, atol=1e-14)
+    for l in range(2):
+        assert np.abs(tconv[l].grad.numpy()).max() > 1e-6
+        np.testing.assert_allclose(res["dW"][l], tconv[l].grad.numpy().transpose(0, 2, 3, 1),
+                                   rtol=1e-10, atol=1e-14)
+        np.testing.assert_allclose(res["dbeta"][l], tbeta[l].grad.numpy(), rtol=1e-10, atol=1e-14)
