@@ -61,9 +61,75 @@ def workload(args):
     return w.scaled(save=args.save or "mem")
 
 
-def is_dense(args):
+def is_net(args):
+    """A whole-network training step (dense or convolutional SNN)."""
     from paper_2211_10725_gb300 import workloads as W
-    return args.workload in W.DENSE_WORKLOADS
+    return args.workload in W.DENSE_WORKLOADS or args.workload in W.CONV_WORKLOADS
+
+
+def net_workload(name):
+    from paper_2211_10725_gb300 import workloads as W
+    return W.DENSE_WORKLOADS.get(name) or W.CONV_WORKLOADS[name]
+
+
+def is_conv(w):
+    return hasattr(w, "convs")
+
+
+def net_inputs(w, seed=None):
+    from paper_2211_10725_gb300 import workloads as W
+    return W.make_conv_inputs(w, seed) if is_conv(w) else W.make_dense_inputs(w, seed)
+
+
+def net_neurons(w):
+    """Spiking neurons per sample (unpadded): every layer's neurons."""
+    if is_conv(w):
+        shapes, _ = w.shapes()
+        return sum(ho * wo * cout for (_, _, _, cout, _, ho, wo, _, _) in shapes) + w.n_classes
+    return sum(w.sizes[1:])
+
+
+def net_config(w):
+    if is_conv(w):
+        return {"workload": w.name, "input": [w.H, w.W, w.Cin],
+                "convs": [list(c) for c in w.convs], "pool": "2x2 max", "T": w.T, "B": w.B,
+                "classes": w.n_classes, "reset": w.reset,
+                "beta": "per channel, learnable (conv layers)"}
+    return {"workload": w.name, "sizes": list(w.sizes), "T": w.T, "B": w.B,
+            "classes": w.n_classes, "neurons_per_class": w.pop}
+
+
+def net_oracle_pass(w, host, bs):
+    """The oracle's forward + loss + BPTT over samples bs of the batch."""
+    from oracle import snn_oracle as O
+    import numpy as np
+    n = len(bs)
+    if is_conv(w):
+        X = host["X"][:, bs].reshape(w.T * n, w.H, w.W, w.Cin)
+        betas = [np.full(c, w.beta) for c, _ in w.convs]
+        fwd = O.csnn_forward(X, host["convs"], host["Wfc"], w.T, n, betas, w.beta_fc, w.thr,
+                             reset=w.reset)
+        O.csnn_backward(fwd, host["convs"], host["Wfc"], host["y"][bs], w.T, n, betas,
+                        w.beta_fc, w.thr, w.sg_param, reset=w.reset)
+    else:
+        xb = host["X"][:, bs].reshape(w.T * n, -1)
+        fwd = O.dsnn_forward(xb, host["W"], w.T, n, w.beta, w.thr)
+        O.dsnn_backward(fwd, host["W"], host["y"][bs], w.T, n, w.beta, w.thr, w.sg_param,
+                        pop=w.pop)
+
+
+def net_oracle_host(w, inp):
+    import numpy as np
+    f64 = lambda t: t.float().numpy().astype(np.float64)
+    host = {"y": inp["labels"].numpy().astype(np.int64)}
+    if is_conv(w):
+        host["X"] = f64(inp["X"])                                  # [T, B, H, W, Cin]
+        host["convs"] = [f64(c) for c in inp["convs"]]
+        host["Wfc"] = f64(inp["Wfc"])
+    else:
+        host["X"] = f64(inp["X"])                                  # [T, B, K0]
+        host["W"] = [f64(x) for x in inp["W"]]
+    return host
 
 
 # ---------------------------------------------------------------------------
@@ -257,44 +323,34 @@ def time_oracle(w, inp, seconds):
     return w.T * done / t_total, done, t_total
 
 
-def run_dense_reference(args):
-    """The oracle's dense-SNN forward + loss + BPTT on a bounded sample of
-    the batch per step (samples are independent until the dW sums)."""
+def run_net_reference(args):
+    """The oracle's network forward + loss + BPTT on a bounded sample of the
+    batch per step (samples are independent until the dW sums)."""
     import numpy as np
-    from oracle import snn_oracle as O
-    from paper_2211_10725_gb300 import workloads as W
-    w = W.DENSE_WORKLOADS[args.workload]
-    inp = W.make_dense_inputs(w)
-    Ws = [x.float().numpy().astype(np.float64) for x in inp["W"]]
-    X = inp["X"].float().numpy().astype(np.float64)          # [T, B, K0]
-    y = inp["labels"].numpy().astype(np.int64)
-
-    def one(bs):
-        xb = X[:, bs].reshape(w.T * len(bs), -1)
-        fwd = O.dsnn_forward(xb, Ws, w.T, len(bs), w.beta, w.thr)
-        O.dsnn_backward(fwd, Ws, y[bs], w.T, len(bs), w.beta, w.thr, w.sg_param, pop=w.pop)
-
+    w = net_workload(args.workload)
+    host = net_oracle_host(w, net_inputs(w))
     t0 = time.perf_counter()
-    one(np.arange(8))
-    per_sample = (time.perf_counter() - t0) / 8
+    probe = min(w.B, 4)
+    net_oracle_pass(w, host, np.arange(probe))
+    per_sample = (time.perf_counter() - t0) / probe
     total = max(1, args.steps + args.warmup)
     n = int(max(1, min(w.B, args.reference_seconds / total / per_sample)))
     rng = np.random.default_rng(0)
     samples = [np.sort(rng.choice(w.B, n, replace=False)) for _ in range(total)]
     for i in range(args.warmup):
-        one(samples[i])
+        net_oracle_pass(w, host, samples[i])
     t0 = time.perf_counter()
     for i in range(args.steps):
-        one(samples[args.warmup + i])
+        net_oracle_pass(w, host, samples[args.warmup + i])
     dt = time.perf_counter() - t0
-    value = w.T * n * sum(w.sizes[1:]) * args.steps / dt
+    value = w.T * n * net_neurons(w) * args.steps / dt
     line = {
         "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT,
         "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
         "ms_per_step": 1e3 * dt / args.steps, "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-        "config": {"workload": w.name, "sizes": list(w.sizes), "T": w.T, "B": w.B,
-                   "sample_batch_per_step": n},
+        "config": dict(net_config(w), sample_batch_per_step=n),
+        "images_per_s": n * args.steps / dt,
         "cpu_baseline": {"value": value, "unit": UNIT, "cores": 1, "kind": "oracle",
                          "sample": f"{n} random samples of {w.B} per step, all T={w.T} steps, "
                                    f"float64 oracle forward+loss+BPTT (no optimiser)"},
@@ -307,8 +363,8 @@ def run_reference(args):
     rank = int(os.environ.get("RANK", "0"))
     if rank != 0:
         return
-    if is_dense(args):
-        run_dense_reference(args)
+    if is_net(args):
+        run_net_reference(args)
         return
     import numpy as np
     from paper_2211_10725_gb300 import workloads as W
@@ -376,9 +432,12 @@ def run_ours(args):
         layer.backward(d["I"], d["beta"], d["thr"], d["grad_spk"], alpha=d.get("alpha"),
                        want_state_grads=False, v=d.get("v"))
 
-    for _ in range(args.warmup):
+    c0 = snn.snn_kernel_launches()
+    warm = max(1, args.warmup)
+    for _ in range(warm):
         step()
     torch.cuda.synchronize()
+    launches_per_step = (snn.snn_kernel_launches() - c0) // warm
     status = layer.status()
     if status != 0:
         raise RuntimeError(f"kernel status {status} after warm-up")
@@ -439,14 +498,6 @@ def run_ours(args):
     kernel_key = f"scan_bwd_staged[{w.neuron},{w.save}]"  # dominant kernel
     traffic = profiled_traffic(kernel_key, w.name)
     clocks = sampler.summary(t_wall0, t_wall1)
-    # forward scan + backward scan + one reduction launch per layout among
-    # the parameter gradients (beta, thr, and alpha or v)
-    modes = {w.beta_mode, w.thr_mode}
-    if w.neuron == "synaptic":
-        modes.add(w.alpha_mode)
-    if w.neuron == "rleaky":
-        modes.add(w.v_mode)
-    launches_per_step = 2 + len(modes)
     eager = None
     if not args.no_torch_eager and world == 1:
         eager = time_torch_eager(w, inp, dev)
@@ -478,7 +529,10 @@ def run_ours(args):
                      "minimal_achieved": minimal_b * ns_per_step / (total_ms / K * 1e-3) / 1e9,
                      "minimal_frac": minimal_b * ns_per_step / (total_ms / K * 1e-3) / 1e9 / peak},
         "clocks": clocks,
+        # counted by the library over the warm-up steps: forward scan,
+        # backward scan, one reduction per parameter layout
         "gpu_launches": launches_per_step * K,
+        "gpu_launches_per_step": launches_per_step,
         "cpu_baseline": cpu,
         "torch_eager_context": eager,
         "e2e": e2e,
@@ -501,14 +555,58 @@ def tensor_peak(sustained):
         return (1700.0 if sustained else 1900.0), "fallback"
 
 
-def dense_flops(w):
-    """Algorithmic GEMM flops of one training step (unpadded layer sizes):
-    forward I = X W^T per layer, dW per layer, dX for every layer but the
-    first."""
+def net_flops(w):
+    """Algorithmic GEMM flops of one training step (unpadded sizes): the
+    forward currents of every layer, every dW, and dX of every layer but the
+    first (a convolution as its patch-row product)."""
     M = w.T * w.B
+    if is_conv(w):
+        shapes, n_flat = w.shapes()
+        conv = [2 * M * ho * wo * k * k * cin * cout
+                for (_, _, cin, cout, k, ho, wo, _, _) in shapes]
+        fc = 2 * M * n_flat * w.n_classes
+        fwd = sum(conv) + fc
+        return fwd, fwd, sum(conv[1:]) + fc
     fwd = sum(2 * M * k * n for k, n in zip(w.sizes[:-1], w.sizes[1:]))
     dx = sum(2 * M * k * n for k, n in zip(w.sizes[1:-1], w.sizes[2:]))
     return fwd, fwd, dx
+
+
+def conv_op_bytes(net):
+    """Bytes each op of the CSNN step must read and write as designed (the
+    sizes of its operands and results, each once), for the per-op HBM
+    roofline; the scans by the scan byte model (I, spk, grad_spk, grad_I;
+    checkpoints excluded)."""
+    nb = lambda t: 0 if t is None else t.numel() * t.element_size()
+    T, B, M = net.w.T, net.w.B, net.M
+    out = {}
+    for l, g in enumerate(net.geo):
+        x_bytes = M * g[0] * g[1] * g[2] * 2
+        layer = net.layers[l]
+        ns = T * B * layer.w.N
+        f, b = algorithmic_bytes(layer.w)
+        out[f"im2col{l}"] = x_bytes + nb(net.cols[l])
+        out[f"conv_fwd{l}"] = nb(net.cols[l]) + nb(net.W[l]) + nb(net.I[l])
+        out[f"scan_fwd{l}"] = f * ns
+        out[f"pool_fwd{l}"] = nb(layer.spk) + nb(net.pool[l]) + nb(net.idx[l])
+        out[f"pool_bwd{l}"] = nb(net.grad_pool[l]) + nb(net.idx[l]) + nb(net.grad_spk[l])
+        out[f"scan_bwd{l}"] = b * ns
+        out[f"conv_bwd{l}"] = (nb(net.cols[l]) + nb(layer.grad_I) + nb(net.W[l])
+                               + nb(net.dcols[l]) + nb(net.dW[l]))
+        if l > 0:
+            out[f"col2im{l}"] = nb(net.dcols[l]) + nb(net.grad_pool[l - 1])
+    o = net.out_layer
+    f, b = algorithmic_bytes(o.w)
+    ns = T * B * o.w.N
+    flat = nb(net.pool[-1])
+    out["fc_fwd"] = flat + nb(net.W[-1]) + nb(net.I_fc)
+    out["scan_fwd_out"] = f * ns
+    out["ce_loss"] = nb(o.spk) + nb(net.grad_out)
+    out["scan_bwd_out"] = b * ns
+    out["fc_bwd"] = flat + nb(net.W[-1]) + nb(o.grad_I) + nb(net.grad_pool[-1]) + nb(net.dW[-1])
+    out["adamw"] = (4 * 2 * nb(net.W32_flat) + nb(net.W_flat)
+                    + 4 * 2 * nb(net.beta_flat))
+    return out
 
 
 def _timing_events(external):
@@ -518,12 +616,13 @@ def _timing_events(external):
     return torch.cuda.Event(enable_timing=True)
 
 
-def run_dense(args):
+def run_net(args):
+    """The training step of a whole network (the dense SNN of Tab. I, its
+    population-coded variant, or the convolutional SNN) as one CUDA graph."""
     import torch
     import torch.distributed as dist
 
-    from paper_2211_10725_gb300 import workloads as W
-    from paper_2211_10725_gb300.dsnn import DenseSNN
+    from paper_2211_10725_gb300 import snn
 
     world = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
@@ -532,35 +631,48 @@ def run_dense(args):
         dist.init_process_group("nccl")
     torch.cuda.set_device(local)
     dev = torch.device("cuda", local)
-    w = W.DENSE_WORKLOADS[args.workload]
+    w = net_workload(args.workload)
     save = args.save or "recompute"
-    inp = W.make_dense_inputs(w, seed=W.SEED_BASE + w.seed_index + 1000 * rank)
-    net = DenseSNN(w, inp["W"], device=dev, save=save)
-    X = inp["X"].reshape(w.T * w.B, -1).to(dev)
+    from paper_2211_10725_gb300 import workloads as W
+    inp = net_inputs(w, seed=W.SEED_BASE + w.seed_index + 1000 * rank)
+    if is_conv(w):
+        from paper_2211_10725_gb300.csnn import ConvSNN
+        net = ConvSNN(w, inp["convs"], inp["Wfc"], device=dev, save=save)
+        X = inp["X"].reshape(w.T * w.B, w.H, w.W, w.Cin).to(dev)
+        scans = net.layers + [net.out_layer]
+    else:
+        from paper_2211_10725_gb300.dsnn import DenseSNN
+        net = DenseSNN(w, inp["W"], device=dev, save=save)
+        X = inp["X"].reshape(w.T * w.B, -1).to(dev)
+        scans = net.layers
     labels = inp["labels"].to(dev)
     stream = torch.cuda.Stream(dev)
     if world > 1:
-        # data parallel: this rank's 128 samples are its shard of a global
-        # batch of world * 128; dW and the loss are summed over the ranks
+        # data parallel: this rank's samples are its shard of a global batch
+        # of world * B; dW (and dbeta) and the loss are summed over the ranks
         # (NCCL) before the AdamW update
         from paper_2211_10725_gb300.data_parallel import allreduce_sum_
         net.batch_total = world * w.B
+        from paper_2211_10725_gb300.data_parallel import grad_buffers
+        grads = grad_buffers(net)
 
     def step_ops(st=None):
         ops = net.ops(X, labels, st)
         if world > 1:
-            ops.insert(len(ops) - 1, ("allreduce_dW", lambda: allreduce_sum_([net.dW_flat,
-                                                                             net.loss])))
+            ops.insert(len(ops) - 1, ("allreduce_grads", lambda: allreduce_sum_(grads)))
         return ops
 
     names = [n for n, _ in step_ops()]
 
+    c0 = snn.snn_kernel_launches()
+    warm = max(1, args.warmup)
     with torch.cuda.stream(stream):
-        for _ in range(args.warmup):
+        for _ in range(warm):
             for _, call in step_ops():
                 call()
     stream.synchronize()
-    for layer in net.layers:
+    launches = (snn.snn_kernel_launches() - c0) // warm
+    for layer in scans:
         if layer.status() != 0:
             raise RuntimeError("kernel status after warm-up")
 
@@ -632,8 +744,6 @@ def run_dense(args):
     ev_total = 0.0
     with torch.cuda.stream(stream):
         for _ in range(K2):
-            s0 = torch.cuda.Event(enable_timing=True)
-            s0.record(stream)
             launch(True)
             torch.cuda.synchronize()
             per_op = [acc + evs[i].elapsed_time(evs[i + 1]) for i, acc in enumerate(per_op)]
@@ -647,59 +757,75 @@ def run_dense(args):
         t = torch.tensor([total_ms], device=dev)
         dist.all_reduce(t, op=dist.ReduceOp.MAX)
         total_ms = float(t.item())
-    for layer in net.layers:
+    for layer in scans:
         if layer.status() != 0:
             raise RuntimeError("kernel status in the timed region")
     loss = float(net.loss.item())
     if not (loss == loss):
         raise RuntimeError("loss is NaN")
 
-    ns_per_step = w.T * w.B * sum(w.sizes[1:])
+    ns_per_step = w.T * w.B * net_neurons(w)
     ms = total_ms / K
     value = world * ns_per_step / (ms * 1e-3)
-    e2e = None if args.no_e2e else run_dense_e2e(args, w, inp, net, dev, world)
+    e2e = None if args.no_e2e else run_net_e2e(args, w, inp, net, dev, world)
     if rank != 0:
         if world > 1:
             dist.destroy_process_group()
         return
-    fwd_f, dw_f, dx_f = dense_flops(w)
+    fwd_f, dw_f, dx_f = net_flops(w)
     op_ms = dict(zip(names, per_op))
-    gemm_fwd_ms = sum(v for k, v in op_ms.items() if k.startswith("dense_fwd"))
-    peak, peak_kind = tensor_peak(sustained=True)
-    achieved = fwd_f / (gemm_fwd_ms * 1e-3) / 1e12
     clocks = sampler.summary(t_wall0, t_wall1)
     cpu = None
     if not args.no_cpu_baseline and world == 1:
-        cpu = time_dense_oracle(w, inp, args.cpu_seconds)
-    # launches of our kernels per step: per forward GEMM 1, per forward scan
-    # 1, the loss 1, per scan BPTT 1, per dense backward 3 transposes + 2
-    # GEMMs (the first layer: 2 + 1), AdamW 1
-    nl = len(w.sizes) - 1
-    launches = nl + nl + 1 + nl + (5 * (nl - 1) + 3) + 1
+        cpu = time_net_oracle(w, inp, args.cpu_seconds)
+    if is_conv(w):
+        # every op is memory-bound (the GEMMs' K is 32 or 400, N 16 or 64):
+        # the HBM roofline of the op that takes longest
+        ob = conv_op_bytes(net)
+        top = max(ob, key=lambda k: op_ms.get(k, 0.0))
+        peak, peak_kind = hbm_peak()
+        achieved = ob[top] / (op_ms[top] * 1e-3) / 1e9
+        roofline = {"bound": "hbm", "kernel": top, "achieved": achieved, "peak": peak,
+                    "unit": "GB/s", "frac": achieved / peak, "peak_kind": peak_kind,
+                    "traffic": None, "bytes_per_launch": ob[top],
+                    "op_bytes": ob,
+                    "op_gbs": {k: ob[k] / (op_ms[k] * 1e-3) / 1e9 for k in ob if op_ms.get(k)},
+                    "flops_per_step": {"fwd": fwd_f, "dW": dw_f, "dX": dx_f}}
+        step_desc = ("per conv layer im2col, tcgen05 GEMM, Leaky scan, 2x2 max pool; dense "
+                     "readout GEMM + scan; rate-coded CE loss; BPTT (max-pool routing, scans "
+                     "with per-channel dbeta, GEMM dX/dW, col2im); AdamW on weights and betas")
+        l2 = "working set ~1.2 GB, larger than L2; no flush"
+    else:
+        gemm_fwd_ms = sum(v for k, v in op_ms.items() if k.startswith("dense_fwd"))
+        peak, peak_kind = tensor_peak(sustained=True)
+        achieved = fwd_f / (gemm_fwd_ms * 1e-3) / 1e12
+        roofline = {"bound": "tensor", "kernel": "gemm_tn_tcgen05 (forward GEMMs)",
+                    "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
+                    "frac": achieved / peak, "peak_kind": f"{peak_kind} sustained bf16",
+                    "traffic": None, "flops_per_step": {"fwd": fwd_f, "dW": dw_f, "dX": dx_f}}
+        step_desc = ("forward GEMMs + Leaky scans, rate-coded CE loss, BPTT scans, dense "
+                     "backward (dX, dW), AdamW")
+        l2 = "working set (~70 MB) fits in L2; no flush between steps"
+    roofline.update({"op_ms": op_ms, "op_timed_step_ms": ev_total / K2,
+                     "timing": "per-op: a second timed region of the same step graph with "
+                               "event nodes between the ops, averaged over its steps"})
+    cfg = net_config(w)
+    cfg.update({"step": step_desc, "neuron_steps_per_step": ns_per_step, "save": save,
+                "launch": "CUDA graph replay" if graph is not None else "eager", "l2": l2,
+                "parallelism": (f"data parallel x{world} (global batch {world * w.B}, "
+                                "gradients all-reduced over NCCL)") if world > 1
+                else "single GPU"})
     line = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": K,
         "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
-        "config": {"workload": w.name, "sizes": list(w.sizes), "T": w.T, "B": w.B,
-                   "classes": w.n_classes, "neurons_per_class": w.pop,
-                   "step": "forward GEMMs + Leaky scans, rate-coded CE loss, BPTT scans, "
-                           "dense backward (dX, dW), AdamW",
-                   "neuron_steps_per_step": ns_per_step, "save": save,
-                   "launch": "CUDA graph replay" if graph is not None else "eager",
-                   "l2": "working set (~70 MB) fits in L2; no flush between steps",
-                   "parallelism": (f"data parallel x{world} (global batch {world * w.B}, "
-                                   "dW all-reduced over NCCL)") if world > 1 else "single GPU"},
+        "config": cfg,
         "images_per_s": world * w.B / (ms * 1e-3),
-        "roofline": {"bound": "tensor", "kernel": "gemm_tn_tcgen05 (forward GEMMs)",
-                     "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
-                     "frac": achieved / peak, "peak_kind": f"{peak_kind} sustained bf16",
-                     "traffic": None, "flops_per_step": {"fwd": fwd_f, "dW": dw_f, "dX": dx_f},
-                     "op_ms": op_ms,
-                     "op_timed_step_ms": ev_total / K2,
-                     "timing": "per-op: a second timed region of the same step graph with "
-                               "event nodes between the ops, averaged over its steps"},
+        "roofline": roofline,
         "clocks": clocks,
+        # counted by the library over the eager warm-up steps
         "gpu_launches": launches * K,
+        "gpu_launches_per_step": launches,
         "cpu_baseline": cpu,
         "e2e": e2e,
     }
@@ -708,42 +834,50 @@ def run_dense(args):
         dist.destroy_process_group()
 
 
-def time_dense_oracle(w, inp, seconds):
-    """The oracle's forward + loss + BPTT of the dense SNN (float64 GEMMs,
-    float32 spike decisions) on the full batch, repeated for about `seconds`."""
+def time_net_oracle(w, inp, seconds):
+    """The oracle's forward + loss + BPTT of the network on consecutive
+    sample batches (at most the whole batch), repeated for about `seconds`."""
     import numpy as np
-    from oracle import snn_oracle as O
-    Ws = [x.float().numpy().astype(np.float64) for x in inp["W"]]
-    X = inp["X"].float().numpy().astype(np.float64).reshape(w.T * w.B, -1)
-    y = inp["labels"].numpy().astype(np.int64)
-    n, t_total = 0, 0.0
-    while t_total < seconds or n == 0:
+    host = net_oracle_host(w, inp)
+    t0 = time.perf_counter()
+    probe = min(w.B, 4)
+    net_oracle_pass(w, host, np.arange(probe))
+    per_sample = (time.perf_counter() - t0) / probe
+    n = int(max(1, min(w.B, seconds / 3 / per_sample)))
+    done, t_total, start = 0, 0.0, 0
+    while t_total < seconds or done == 0:
+        bs = (start + np.arange(n)) % w.B
         t0 = time.perf_counter()
-        fwd = O.dsnn_forward(X, Ws, w.T, w.B, w.beta, w.thr)
-        O.dsnn_backward(fwd, Ws, y, w.T, w.B, w.beta, w.thr, w.sg_param, pop=w.pop)
+        net_oracle_pass(w, host, np.sort(bs))
         t_total += time.perf_counter() - t0
-        n += 1
-    ns = w.T * w.B * sum(w.sizes[1:])
-    return {"value": ns * n / t_total, "unit": UNIT, "cores": 1, "kind": "oracle",
-            "sample": f"{n} full forward+loss+BPTT passes of the oracle (no optimiser), "
-                      f"{t_total:.1f} s, BLAS on one thread"}
+        done += n
+        start = (start + n) % w.B
+    ns = w.T * done * net_neurons(w)
+    return {"value": ns / t_total, "unit": UNIT, "cores": 1, "kind": "oracle",
+            "sample": f"{done} samples in batches of {n} (of {w.B}), all T={w.T} steps, "
+                      f"oracle forward+loss+BPTT (no optimiser), {t_total:.1f} s, BLAS on "
+                      f"one thread"}
 
 
-def run_dense_e2e(args, w, inp, net, dev, world):
+def run_net_e2e(args, w, inp, net, dev, world):
     """Training steps through the public API with the batch copied from
     pinned host memory each step and the loss read back."""
     import torch
     import torch.distributed as dist
-    hX = inp["X"].reshape(w.T * w.B, -1).pin_memory()
+    shape = (w.T * w.B, w.H, w.W, w.Cin) if is_conv(w) else (w.T * w.B, -1)
+    hX = inp["X"].reshape(shape).pin_memory()
     hy = inp["labels"].pin_memory()
     dX = torch.empty_like(hX, device=dev)
     dy = torch.empty_like(hy, device=dev)
     out = torch.empty(1, dtype=torch.float32).pin_memory()
     stream = torch.cuda.current_stream(dev)
 
-    if world > 1:
+    if world > 1 and not is_conv(w):
         from paper_2211_10725_gb300.data_parallel import DataParallelDenseSNN
         train = DataParallelDenseSNN(net, world * w.B).train_step
+    elif world > 1:
+        from paper_2211_10725_gb300.data_parallel import DataParallelConvSNN
+        train = DataParallelConvSNN(net, world * w.B).train_step
     else:
         train = net.train_step
 
@@ -771,7 +905,7 @@ def run_dense_e2e(args, w, inp, net, dev, world):
         dist.all_reduce(t, op=dist.ReduceOp.MAX)
         ms = float(t.item())
     nb = lambda t: t.numel() * t.element_size()
-    return {"value": world * w.T * w.B * sum(w.sizes[1:]) * K / (ms * 1e-3), "unit": UNIT,
+    return {"value": world * w.T * w.B * net_neurons(w) * K / (ms * 1e-3), "unit": UNIT,
             "h2d_bytes_per_step": nb(hX) + nb(hy), "d2h_bytes_per_step": nb(out), "steps": K,
             "launch": "eager"}
 
@@ -934,8 +1068,8 @@ def main():
     args = parse()
     if args.impl == "reference":
         run_reference(args)
-    elif is_dense(args):
-        run_dense(args)
+    elif is_net(args):
+        run_net(args)
     else:
         run_ours(args)
 

@@ -114,6 +114,11 @@ typedef struct snn_scan_desc {
 /* Human-readable name of a status code (static string, never NULL). */
 const char* snn_status_string(snn_status_t status);
 
+/* Number of kernels this library has launched in this process (a launch
+ * captured into a CUDA graph counts once, at capture): the difference over
+ * one eagerly issued step is that step's launch count. */
+uint64_t snn_kernel_launches(void);
+
 /* Library version, as 10000*major + 100*minor + patch. */
 int snn_version(void);
 
@@ -256,8 +261,12 @@ snn_status_t snn_synaptic_bwd(const snn_scan_desc* desc, const void* I, const fl
 snn_status_t snn_dense_layer_fwd(int64_t M, int64_t K, int64_t N, const void* X, const void* W,
                                  float* I, void* ws, size_t ws_bytes, snn_stream_t stream);
 
-/* Workspace bytes of snn_dense_layer_bwd (a status word; the operands are
- * read in place, W and X and dI through MN-major tensor-core tiles). */
+/* Workspace bytes of snn_dense_layer_bwd: a status word (the operands are
+ * read in place, W and X and dI through MN-major tensor-core tiles), plus,
+ * when dW's few output tiles would each sum a long M (a convolution's
+ * weight gradient sums over every patch row), S fp32 partial copies of dW
+ * [N, K]: the rows are split S ways, S a function of (M, K, N) alone, and
+ * the partials are added in split order (the same bits on every call). */
 size_t snn_dense_workspace_bytes(int64_t M, int64_t K, int64_t N);
 
 /*
@@ -327,6 +336,36 @@ snn_status_t snn_rate_ce_loss(int64_t T, int64_t B, int64_t C, int64_t pop, int6
                               int64_t batch_total, int32_t dtype, const void* spk,
                               const int32_t* labels, float* loss, void* grad_spk, void* ws,
                               size_t ws_bytes, snn_stream_t stream);
+
+/*
+ * Convolutional SNN layout kernels (Tab. I CSNN: 5x5 convolutions, 2x2 max
+ * pooling) on channel-last bf16 activations [M, H, W, C], M = T*B.  A
+ * convolution is a snn_dense_layer_fwd/bwd over the patch rows:
+ *   snn_im2col_nhwc: cols [M*Ho*Wo, Kpad] (out), Ho = H-KH+1, Wo = W-KW+1,
+ *     cols[(m, oy, ox), (ky*KW + kx)*Cin + c] = X[m, oy+ky, ox+kx, c], zero
+ *     for columns KH*KW*Cin .. Kpad-1 (Kpad a multiple of 8, >= KH*KW*Cin;
+ *     cols 16-byte aligned).  With filters W [Cout, Kpad] (same column
+ *     order), snn_dense_layer_fwd(cols, W) is the valid, stride-1
+ *     convolution.
+ *   snn_col2im_nhwc: dX [M, H, W, Cin] (out) = the patch-row gradient dcols
+ *     [M*Ho*Wo, Kpad] summed back onto the input pixels each column read
+ *     (fp32 sums in (ky, kx) order, rounded to bf16).
+ *   snn_maxpool2_fwd_nhwc: Y [M, H/2, W/2, C] (out) = the maximum of each
+ *     2x2 window (H, W even); idx uint8 [M, H/2, W/2, C] (out) = the
+ *     window position (0..3, row major) of its first maximum.
+ *   snn_maxpool2_bwd_nhwc: dX [M, H, W, C] (out) = dY at the recorded
+ *     position of each window, 0 at the other three.
+ * Asynchronous on stream; SNN_ERR_INVALID_ARG / SNN_ERR_ALIGNMENT for bad
+ * shapes or pointers.
+ */
+snn_status_t snn_im2col_nhwc(int64_t M, int64_t H, int64_t W, int64_t Cin, int64_t KH, int64_t KW,
+                             int64_t Kpad, const void* X, void* cols, snn_stream_t stream);
+snn_status_t snn_col2im_nhwc(int64_t M, int64_t H, int64_t W, int64_t Cin, int64_t KH, int64_t KW,
+                             int64_t Kpad, const void* dcols, void* dX, snn_stream_t stream);
+snn_status_t snn_maxpool2_fwd_nhwc(int64_t M, int64_t H, int64_t W, int64_t C, const void* X,
+                                   void* Y, uint8_t* idx, snn_stream_t stream);
+snn_status_t snn_maxpool2_bwd_nhwc(int64_t M, int64_t H, int64_t W, int64_t C, const void* dY,
+                                   const uint8_t* idx, void* dX, snn_stream_t stream);
 
 /*
  * AdamW update of n fp32 master weights (the optimiser of the paper's

@@ -1,0 +1,220 @@
+// The convolutional SNN's layout kernels (Tab. I CSNN: 5x5 convolutions and
+// 2x2 max pooling), for channel-last bf16 activations [M, H, W, C] with
+// M = T*B.  A convolution runs as a tensor-core GEMM over patch rows:
+//   im2col   cols[(m, oy, ox), (ky, kx, c)] = X[m, oy+ky, ox+kx, c]
+//            (columns past KH*KW*Cin up to Kpad are zero), so the layer's
+//            input current is cols * W^T with W [Cout, KH, KW, Cin];
+//   col2im   dX[m, y, x, c] = sum over the (ky, kx) with a valid output
+//            pixel (y-ky, x-kx) of dcols[(m, y-ky, x-kx), (ky, kx, c)],
+//            added in (ky, kx) order in fp32 (deterministic);
+//   max pool 2x2 windows, stride 2; the first maximum in window order
+//            (row major) is kept and its position recorded, and the
+//            backward routes the gradient there (every input element
+//            belongs to one window, so no two threads write one element).
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+
+#include <climits>
+#include <cstdint>
+
+#include "launch.cuh"
+#include "snn.h"
+
+namespace snn {
+namespace {
+
+constexpr int kThreads = 256;
+
+// Eight consecutive columns of one patch row per thread (one 16-byte store).
+__global__ void __launch_bounds__(kThreads) im2col_kernel(const __nv_bfloat16* __restrict__ X,
+                                                          __nv_bfloat16* __restrict__ cols,
+                                                          int64_t rows, int H, int W, int Cin,
+                                                          int KH, int KW, int Kpad) {
+  grid_dep_wait();
+  const int Ho = H - KH + 1, Wo = W - KW + 1;
+  const int K = KH * KW * Cin;
+  const int vec_per_row = Kpad / 8;
+  const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (i >= rows * vec_per_row) return;
+  const int64_t r = i / vec_per_row;
+  const int k0 = (int)(i - r * vec_per_row) * 8;
+  const int64_t m = r / (Ho * Wo);
+  const int p = (int)(r - m * (Ho * Wo));
+  const int oy = p / Wo, ox = p - oy * Wo;
+  const __nv_bfloat16* xm = X + m * H * W * Cin;
+  __align__(16) __nv_bfloat16 v[8];
+#pragma unroll
+  for (int j = 0; j < 8; ++j) {
+    const int k = k0 + j;
+    __nv_bfloat16 e = __float2bfloat16_rn(0.0f);
+    if (k < K) {
+      const int ky = k / (KW * Cin);
+      const int rem = k - ky * KW * Cin;
+      const int kx = rem / Cin, c = rem - kx * Cin;
+      e = xm[((oy + ky) * W + (ox + kx)) * Cin + c];
+    }
+    v[j] = e;
+  }
+  *reinterpret_cast<uint4*>(cols + r * Kpad + k0) = *reinterpret_cast<const uint4*>(v);
+}
+
+__global__ void __launch_bounds__(kThreads) col2im_kernel(const __nv_bfloat16* __restrict__ dcols,
+                                                          __nv_bfloat16* __restrict__ dX,
+                                                          int64_t total, int H, int W, int Cin,
+                                                          int KH, int KW, int Kpad) {
+  grid_dep_wait();
+  const int Ho = H - KH + 1, Wo = W - KW + 1;
+  const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (i >= total) return;
+  const int c = (int)(i % Cin);
+  const int64_t q = i / Cin;
+  const int x = (int)(q % W);
+  const int64_t q2 = q / W;
+  const int y = (int)(q2 % H);
+  const int64_t m = q2 / H;
+  float s = 0.0f;
+  for (int ky = 0; ky < KH; ++ky) {
+    const int oy = y - ky;
+    if (oy < 0 || oy >= Ho) continue;
+    for (int kx = 0; kx < KW; ++kx) {
+      const int ox = x - kx;
+      if (ox < 0 || ox >= Wo) continue;
+      const int64_t r = (m * Ho + oy) * Wo + ox;
+      s += __bfloat162float(dcols[r * Kpad + (ky * KW + kx) * Cin + c]);
+    }
+  }
+  dX[i] = __float2bfloat16_rn(s);
+}
+
+__global__ void __launch_bounds__(kThreads) maxpool_fwd_kernel(const __nv_bfloat16* __restrict__ X,
+                                                               __nv_bfloat16* __restrict__ Y,
+                                                               uint8_t* __restrict__ idx,
+                                                               int64_t total, int H, int W,
+                                                               int C) {
+  grid_dep_wait();
+  const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (i >= total) return;
+  const int Hp = H / 2, Wp = W / 2;
+  const int c = (int)(i % C);
+  const int64_t q = i / C;
+  const int px = (int)(q % Wp);
+  const int64_t q2 = q / Wp;
+  const int py = (int)(q2 % Hp);
+  const int64_t m = q2 / Hp;
+  const __nv_bfloat16* base = X + ((m * H + 2 * py) * W + 2 * px) * C + c;
+  const int64_t off[4] = {0, (int64_t)C, (int64_t)W * C, (int64_t)W * C + C};
+  float best = __bfloat162float(base[0]);
+  int arg = 0;
+#pragma unroll
+  for (int j = 1; j < 4; ++j) {
+    const float v = __bfloat162float(base[off[j]]);
+    if (v > best) {  // strict: the first maximum is kept
+      best = v;
+      arg = j;
+    }
+  }
+  Y[i] = __float2bfloat16_rn(best);
+  idx[i] = (uint8_t)arg;
+}
+
+__global__ void __launch_bounds__(kThreads) maxpool_bwd_kernel(const __nv_bfloat16* __restrict__ dY,
+                                                               const uint8_t* __restrict__ idx,
+                                                               __nv_bfloat16* __restrict__ dX,
+                                                               int64_t total, int H, int W,
+                                                               int C) {
+  grid_dep_wait();
+  const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (i >= total) return;
+  const int Hp = H / 2, Wp = W / 2;
+  const int c = (int)(i % C);
+  const int64_t q = i / C;
+  const int x = (int)(q % W);
+  const int64_t q2 = q / W;
+  const int y = (int)(q2 % H);
+  const int64_t m = q2 / H;
+  const int64_t o = ((m * Hp + y / 2) * Wp + x / 2) * C + c;
+  const int pos = (y & 1) * 2 + (x & 1);
+  dX[i] = idx[o] == pos ? dY[o] : __float2bfloat16_rn(0.0f);
+}
+
+bool aligned(const void* p, uintptr_t a) { return (reinterpret_cast<uintptr_t>(p) & (a - 1)) == 0; }
+
+unsigned blocks_for(int64_t n) { return (unsigned)((n + kThreads - 1) / kThreads); }
+
+}  // namespace
+}  // namespace snn
+
+using namespace snn;
+
+extern "C" snn_status_t snn_im2col_nhwc(int64_t M, int64_t H, int64_t W, int64_t Cin, int64_t KH,
+                                        int64_t KW, int64_t Kpad, const void* X, void* cols,
+                                        snn_stream_t stream) {
+  if (M < 0 || KH < 1 || KW < 1 || H < KH || W < KW || Cin < 1) return SNN_ERR_INVALID_ARG;
+  if (H * W * Cin > INT_MAX / 2 || Kpad > INT_MAX / 2) return SNN_ERR_INVALID_ARG;
+  if (Kpad < KH * KW * Cin || Kpad % 8 != 0) return SNN_ERR_INVALID_ARG;
+  if (M == 0) return SNN_OK;
+  if (!X || !cols) return SNN_ERR_INVALID_ARG;
+  if (!aligned(cols, 16) || !aligned(X, 2)) return SNN_ERR_ALIGNMENT;
+  const int64_t rows = M * (H - KH + 1) * (W - KW + 1);
+  const int64_t n = rows * (Kpad / 8);
+  if (n / kThreads >= INT_MAX) return SNN_ERR_INVALID_ARG;
+  const cudaError_t e = launch_pdl(im2col_kernel, dim3(blocks_for(n)), dim3(kThreads), 0,
+                                   reinterpret_cast<cudaStream_t>(stream),
+                                   static_cast<const __nv_bfloat16*>(X),
+                                   static_cast<__nv_bfloat16*>(cols), rows, (int)H, (int)W, (int)Cin,
+                                   (int)KH, (int)KW, (int)Kpad);
+  return e == cudaSuccess ? SNN_OK : SNN_ERR_CUDA;
+}
+
+extern "C" snn_status_t snn_col2im_nhwc(int64_t M, int64_t H, int64_t W, int64_t Cin, int64_t KH,
+                                        int64_t KW, int64_t Kpad, const void* dcols, void* dX,
+                                        snn_stream_t stream) {
+  if (M < 0 || KH < 1 || KW < 1 || H < KH || W < KW || Cin < 1) return SNN_ERR_INVALID_ARG;
+  if (H * W * Cin > INT_MAX / 2 || Kpad > INT_MAX / 2) return SNN_ERR_INVALID_ARG;
+  if (Kpad < KH * KW * Cin) return SNN_ERR_INVALID_ARG;
+  if (M == 0) return SNN_OK;
+  if (!dcols || !dX) return SNN_ERR_INVALID_ARG;
+  if (!aligned(dcols, 2) || !aligned(dX, 2)) return SNN_ERR_ALIGNMENT;
+  const int64_t n = M * H * W * Cin;
+  if (n / kThreads >= INT_MAX) return SNN_ERR_INVALID_ARG;
+  const cudaError_t e = launch_pdl(col2im_kernel, dim3(blocks_for(n)), dim3(kThreads), 0,
+                                   reinterpret_cast<cudaStream_t>(stream),
+                                   static_cast<const __nv_bfloat16*>(dcols),
+                                   static_cast<__nv_bfloat16*>(dX), n, (int)H, (int)W, (int)Cin,
+                                   (int)KH, (int)KW, (int)Kpad);
+  return e == cudaSuccess ? SNN_OK : SNN_ERR_CUDA;
+}
+
+extern "C" snn_status_t snn_maxpool2_fwd_nhwc(int64_t M, int64_t H, int64_t W, int64_t C,
+                                              const void* X, void* Y, uint8_t* idx,
+                                              snn_stream_t stream) {
+  if (M < 0 || H < 2 || W < 2 || C < 1 || H % 2 || W % 2) return SNN_ERR_INVALID_ARG;
+  if (H * W * C > INT_MAX / 2) return SNN_ERR_INVALID_ARG;
+  if (M == 0) return SNN_OK;
+  if (!X || !Y || !idx) return SNN_ERR_INVALID_ARG;
+  if (!aligned(X, 2) || !aligned(Y, 2)) return SNN_ERR_ALIGNMENT;
+  const int64_t n = M * (H / 2) * (W / 2) * C;
+  if (n / kThreads >= INT_MAX) return SNN_ERR_INVALID_ARG;
+  const cudaError_t e = launch_pdl(maxpool_fwd_kernel, dim3(blocks_for(n)), dim3(kThreads), 0,
+                                   reinterpret_cast<cudaStream_t>(stream),
+                                   static_cast<const __nv_bfloat16*>(X),
+                                   static_cast<__nv_bfloat16*>(Y), idx, n, (int)H, (int)W, (int)C);
+  return e == cudaSuccess ? SNN_OK : SNN_ERR_CUDA;
+}
+
+extern "C" snn_status_t snn_maxpool2_bwd_nhwc(int64_t M, int64_t H, int64_t W, int64_t C,
+                                              const void* dY, const uint8_t* idx, void* dX,
+                                              snn_stream_t stream) {
+  if (M < 0 || H < 2 || W < 2 || C < 1 || H % 2 || W % 2) return SNN_ERR_INVALID_ARG;
+  if (H * W * C > INT_MAX / 2) return SNN_ERR_INVALID_ARG;
+  if (M == 0) return SNN_OK;
+  if (!dY || !idx || !dX) return SNN_ERR_INVALID_ARG;
+  if (!aligned(dY, 2) || !aligned(dX, 2)) return SNN_ERR_ALIGNMENT;
+  const int64_t n = M * H * W * C;
+  if (n / kThreads >= INT_MAX) return SNN_ERR_INVALID_ARG;
+  const cudaError_t e = launch_pdl(maxpool_bwd_kernel, dim3(blocks_for(n)), dim3(kThreads), 0,
+                                   reinterpret_cast<cudaStream_t>(stream),
+                                   static_cast<const __nv_bfloat16*>(dY), idx,
+                                   static_cast<__nv_bfloat16*>(dX), n, (int)H, (int)W, (int)C);
+  return e == cudaSuccess ? SNN_OK : SNN_ERR_CUDA;
+}

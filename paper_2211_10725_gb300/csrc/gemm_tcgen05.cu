@@ -21,6 +21,12 @@
 // 64-element-wide TMA boxes (64 MN x 64 K, 128-byte swizzle) and described
 // to the tensor core as atoms of 8 K-rows of 128 bytes: 1024 bytes apart
 // along K, one box (8 KB) apart along MN.
+//
+// Split K: a product whose few output tiles each sum a long K (the weight
+// gradient of a convolution sums over every patch row) runs as tiles x S
+// work items, item (tile, s) summing k-blocks [s*nk/S, (s+1)*nk/S) into
+// partial output s; a second kernel adds the S partials in split order, so
+// the result does not depend on which CTA ran which item.
 #include <cuda.h>
 #include <cudaTypedefs.h>
 #include <cuda_bf16.h>
@@ -60,6 +66,8 @@ struct GemmArgs {
   int64_t ldd;  // row stride of D in elements
   int* status;
   uint64_t wait_ns;
+  int ksplit;            // K splits per tile (1: D is the result)
+  int64_t split_stride;  // elements between the partial outputs of two splits
 };
 
 // ---------------------------------------------------------------------------
@@ -206,8 +214,9 @@ __host__ __device__ constexpr size_t smem_bytes() {
 }
 
 // ---------------------------------------------------------------------------
-// Kernel: persistent, tiles t = blockIdx.x, blockIdx.x + gridDim.x, ... in
-// row-major tile order (N tiles fastest).  The operand ring runs on across
+// Kernel: persistent, work items blockIdx.x, blockIdx.x + gridDim.x, ...;
+// item i is split i % S of tile i / S, tiles in row-major order (N tiles
+// fastest).  The operand ring runs on across
 // tiles; the accumulator alternates between two TMEM buffers so that the
 // epilogue of one tile overlaps the main loop of the next.
 // ---------------------------------------------------------------------------
@@ -235,7 +244,8 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm)
   const int warp = threadIdx.x >> 5, lid = threadIdx.x & 31;
   const int nk = (g.K + BK - 1) / BK;
   const int tiles_n = (g.N + BN - 1) / BN;
-  const int tiles = tiles_n * ((g.M + BM - 1) / BM);
+  const int S = g.ksplit;
+  const int items = tiles_n * ((g.M + BM - 1) / BM) * S;  // (tile, split), split fastest
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < kStages; ++s) {
@@ -259,9 +269,11 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm)
     if (lid == 0) {
       int64_t n_issued = 0;  // k-blocks issued over all tiles: ring position
       bool ok = true;
-      for (int t = blockIdx.x; t < tiles && ok; t += gridDim.x) {
+      for (int it = blockIdx.x; it < items && ok; it += gridDim.x) {
+        const int t = it / S, sp = it - t * S;
         const int m0 = (t / tiles_n) * BM, n0 = (t % tiles_n) * BN;
-        for (int kb = 0; kb < nk; ++kb, ++n_issued) {
+        const int kb1 = (int)((int64_t)nk * (sp + 1) / S);
+        for (int kb = (int)((int64_t)nk * sp / S); kb < kb1; ++kb, ++n_issued) {
           const int s = (int)(n_issued % kStages);
           if (n_issued >= kStages &&
               !mbar_wait_poll(&empty[s], (uint32_t)(((n_issued / kStages) - 1) & 1), g.wait_ns)) {
@@ -300,7 +312,9 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm)
       int64_t n_used = 0;  // k-blocks consumed over all tiles
       bool ok = true;
       int i = 0;  // this CTA's tile count
-      for (int t = blockIdx.x; t < tiles && ok; t += gridDim.x, ++i) {
+      for (int it = blockIdx.x; it < items && ok; it += gridDim.x, ++i) {
+        const int sp = it % S;
+        const int kb0 = (int)((int64_t)nk * sp / S), kb1 = (int)((int64_t)nk * (sp + 1) / S);
         const int b = i & 1;
         // the epilogue has drained this accumulator (its use two tiles ago)
         if (i >= 2 && !mbar_wait_poll(&acc_empty[b], (uint32_t)(((i >> 1) - 1) & 1), g.wait_ns)) {
@@ -309,7 +323,7 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm)
         }
         tc_fence_after();
         const uint32_t acc = tmem + (uint32_t)(b * BN);
-        for (int kb = 0; kb < nk; ++kb, ++n_used) {
+        for (int kb = kb0; kb < kb1; ++kb, ++n_used) {
           const int s = (int)(n_used % kStages);
           if (!mbar_wait_poll(&full[s], (uint32_t)((n_used / kStages) & 1), g.wait_ns)) {
             record_status(g.status, kStatusTimeout);
@@ -321,7 +335,7 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm)
           const uint64_t db = B_MN ? sdesc_sw128_mn(sB + s * B_BYTES) : sdesc_sw128(sB + s * B_BYTES);
 #pragma unroll
           for (int kk = 0; kk < BK / 16; ++kk)
-            tc_mma(acc, da + stepA * kk, db + stepB * kk, idesc, (kb | kk) != 0 ? 1u : 0u);
+            tc_mma(acc, da + stepA * kk, db + stepB * kk, idesc, (kb != kb0 || kk != 0) ? 1u : 0u);
           tc_commit(&empty[s]);  // the stage is free once these MMAs are done
         }
         if (ok) tc_commit(&acc_full[b]);  // the tile's accumulator is final
@@ -331,7 +345,8 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm)
     // epilogue: warp w reads TMEM lanes 32*(w%4) .. +32, i.e. tile rows
     const int q = warp & 3;
     int i = 0;
-    for (int t = blockIdx.x; t < tiles; t += gridDim.x, ++i) {
+    for (int it = blockIdx.x; it < items; it += gridDim.x, ++i) {
+      const int t = it / S, sp = it - t * S;
       const int b = i & 1;
       if (!warp_wait_uniform(&acc_full[b], (uint32_t)((i >> 1) & 1), g.wait_ns)) {
         if (lid == 0) record_status(g.status, kStatusTimeout);
@@ -340,6 +355,8 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm)
       tc_fence_after();
       const int m0 = (t / tiles_n) * BM, n0 = (t % tiles_n) * BN;
       const int row = m0 + q * 32 + lid;
+      void* const Dout = OUT_BF16 ? (void*)(static_cast<__nv_bfloat16*>(g.D) + sp * g.split_stride)
+                                  : (void*)(static_cast<float*>(g.D) + sp * g.split_stride);
       const uint32_t acc = tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(b * BN);
 #pragma unroll 1
       for (int c = 0; c < BN; c += 16) {
@@ -348,7 +365,7 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm)
         const int col = n0 + c;
         if (row < g.M && col < g.N) {
           if (OUT_BF16) {
-            __nv_bfloat16* d = static_cast<__nv_bfloat16*>(g.D) + (int64_t)row * g.ldd + col;
+            __nv_bfloat16* d = static_cast<__nv_bfloat16*>(Dout) + (int64_t)row * g.ldd + col;
             if (col + 16 <= g.N && (((int64_t)row * g.ldd + col) & 7) == 0) {
               uint4 v[2];
               uint32_t* w = reinterpret_cast<uint32_t*>(v);
@@ -363,7 +380,7 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm)
               for (int j = 0; j < 16 && col + j < g.N; ++j) d[j] = __float2bfloat16_rn(__uint_as_float(r[j]));
             }
           } else {
-            float* d = static_cast<float*>(g.D) + (int64_t)row * g.ldd + col;
+            float* d = static_cast<float*>(Dout) + (int64_t)row * g.ldd + col;
             if (col + 16 <= g.N && (((int64_t)row * g.ldd + col) & 3) == 0) {
 #pragma unroll
               for (int j = 0; j < 4; ++j)
@@ -433,9 +450,9 @@ cudaError_t launch_bn(const CUtensorMap& ta, const CUtensorMap& tb, const GemmAr
   int dev = 0, sms = 152;
   if (cudaGetDevice(&dev) == cudaSuccess)
     cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-  const int64_t tiles = (int64_t)((g.N + BN - 1) / BN) * ((g.M + BM - 1) / BM);
+  const int64_t items = (int64_t)((g.N + BN - 1) / BN) * ((g.M + BM - 1) / BM) * g.ksplit;
   const int64_t slots = (int64_t)sms * kCtasPerSm;
-  const unsigned grid = (unsigned)(tiles < slots ? tiles : slots);  // persistent CTAs
+  const unsigned grid = (unsigned)(items < slots ? items : slots);  // persistent CTAs
   return launch_pdl(gemm_tn_tcgen05<BN, OUT_BF16, A_MN, B_MN>, dim3(grid), dim3(kThreads),
                     smem_bytes<BN>(), st, ta, tb, g);
 }
@@ -446,7 +463,7 @@ cudaError_t launch_bn(const CUtensorMap& ta, const CUtensorMap& tb, const GemmAr
 // rather than 128 when 128-wide tiles would leave most SMs idle.
 template <bool OUT_BF16, bool A_MN = false, bool B_MN = false>
 cudaError_t gemm_tn(const void* A, const void* B, void* D, int M, int N, int K, int* status,
-                    cudaStream_t st) {
+                    cudaStream_t st, int ksplit = 1) {
   // a 128 x 256 tile keeps the tensor core busier per instruction (about
   // 1.6x the rate of 128 x 128 at large K); below K = 512 the per-tile
   // fixed costs dominate and the narrower tile's parallelism wins
@@ -465,7 +482,7 @@ cudaError_t gemm_tn(const void* A, const void* B, void* D, int M, int N, int K, 
   const bool okA = A_MN ? make_map(&ta, A, K, M, 64) : make_map(&ta, A, M, K, BM);
   const bool okB = B_MN ? make_map(&tb, B, K, N, 64) : make_map(&tb, B, N, K, bn);
   if (!okA || !okB) return cudaErrorInvalidValue;
-  GemmArgs g{M, N, K, D, (int64_t)N, status, kDefaultWaitNs};
+  GemmArgs g{M, N, K, D, (int64_t)N, status, kDefaultWaitNs, ksplit, (int64_t)M * N};
   if constexpr (B_MN) {
     if (bn == 64) return launch_bn<64, OUT_BF16, A_MN, B_MN>(ta, tb, g, st);
     return launch_bn<128, OUT_BF16, A_MN, B_MN>(ta, tb, g, st);
@@ -483,6 +500,37 @@ cudaError_t gemm_tn(const void* A, const void* B, void* D, int M, int N, int K, 
 bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 size_t round256(size_t b) { return (b + 255) & ~size_t(255); }
 
+// K splits of the weight-gradient product dW[N, K] = dI^T X (reduction over
+// the M rows), from the shapes alone so that a shape always sums in the same
+// order: enough (tile, split) items to give each of about one GPU's worth of
+// SMs (kSplitSlots) one, with at least kMinSplitKBlocks k-blocks per split.
+constexpr int64_t kSplitSlots = 152;
+constexpr int64_t kMinSplitKBlocks = 8;
+int dw_splits(int64_t M, int64_t K, int64_t N) {
+  const int64_t tiles = ((N + BM - 1) / BM) * ((K + 63) / 64);
+  const int64_t nk = (M + BK - 1) / BK;
+  int64_t s = kSplitSlots / (tiles > 0 ? tiles : 1);
+  if (s > nk / kMinSplitKBlocks) s = nk / kMinSplitKBlocks;
+  return s < 1 ? 1 : (int)s;
+}
+
+// out[i] = sum over s = 0 .. S-1 of part[s * n + i], in split order.
+__global__ void __launch_bounds__(256) sum_splits(const float4* __restrict__ part,
+                                                  float4* __restrict__ out, int64_t n4, int S) {
+  grid_dep_wait();
+  const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (i >= n4) return;
+  float4 a = part[i];
+  for (int s = 1; s < S; ++s) {
+    const float4 b = part[(int64_t)s * n4 + i];
+    a.x += b.x;
+    a.y += b.y;
+    a.z += b.z;
+    a.w += b.w;
+  }
+  out[i] = a;
+}
+
 snn_status_t check_dims(int64_t M, int64_t K, int64_t N) {
   if (M < 0 || K < 0 || N < 0) return SNN_ERR_INVALID_ARG;
   if (M > INT_MAX / 2 || K > INT_MAX / 2 || N > INT_MAX / 2) return SNN_ERR_INVALID_ARG;
@@ -498,7 +546,10 @@ extern "C" {
 
 size_t snn_dense_workspace_bytes(int64_t M, int64_t K, int64_t N) {
   if (check_dims(M, K, N) != SNN_OK) return 0;
-  return 256;  // the status word: the backward reads its operands in place
+  // the status word (the backward reads its operands in place), then the
+  // split-K partials of dW when the weight gradient is split
+  const int S = dw_splits(M, K, N);
+  return 256 + (S > 1 ? round256((size_t)S * N * K * sizeof(float)) : 0);
 }
 
 snn_status_t snn_dense_layer_fwd(int64_t M, int64_t K, int64_t N, const void* X, const void* W,
@@ -540,8 +591,19 @@ snn_status_t snn_dense_layer_bwd(int64_t M, int64_t K, int64_t N, const void* X,
   }
   if (dW && N > 0 && K > 0) {
     // dW[N, K] = dI[M, N]^T * X[M, K]: both operands MN-major (K = M here)
-    if (M == 0) e = cudaMemsetAsync(dW, 0, (size_t)N * K * sizeof(float), st);
-    else e = gemm_tn<false, true, true>(dI, X, dW, (int)N, (int)K, (int)M, status, st);
+    const int S = dw_splits(M, K, N);
+    if (M == 0) {
+      e = cudaMemsetAsync(dW, 0, (size_t)N * K * sizeof(float), st);
+    } else if (S == 1) {
+      e = gemm_tn<false, true, true>(dI, X, dW, (int)N, (int)K, (int)M, status, st);
+    } else {
+      float* part = reinterpret_cast<float*>(static_cast<unsigned char*>(ws) + 256);
+      e = gemm_tn<false, true, true>(dI, X, part, (int)N, (int)K, (int)M, status, st, S);
+      const int64_t n4 = N * K / 4;  // K is a multiple of 8
+      if (e == cudaSuccess)
+        e = snn::launch_pdl(sum_splits, dim3((unsigned)((n4 + 255) / 256)), dim3(256), 0, st,
+                       reinterpret_cast<const float4*>(part), reinterpret_cast<float4*>(dW), n4, S);
+    }
     if (e != cudaSuccess) return e == cudaErrorInvalidValue ? SNN_ERR_UNSUPPORTED : SNN_ERR_CUDA;
   }
   return SNN_OK;

@@ -8,7 +8,13 @@
 
 #include <cuda_runtime.h>
 
+#include <atomic>
+
 namespace snn {
+
+// Kernels launched (or captured into a graph) through launch_pdl in this
+// process; read through snn_kernel_launches().
+extern std::atomic<unsigned long long> g_kernel_launches;
 
 __device__ __forceinline__ void grid_dep_wait() {
   asm volatile("griddepcontrol.wait;" ::: "memory");
@@ -27,7 +33,9 @@ cudaError_t launch_pdl(void (*kernel)(Params...), dim3 grid, dim3 block, size_t 
   attr[0].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
-  return cudaLaunchKernelEx(&cfg, kernel, static_cast<Params>(args)...);
+  const cudaError_t e = cudaLaunchKernelEx(&cfg, kernel, static_cast<Params>(args)...);
+  if (e == cudaSuccess) g_kernel_launches.fetch_add(1, std::memory_order_relaxed);
+  return e;
 }
 
 }  // namespace snn

@@ -286,11 +286,16 @@ snn_status_t scan_bwd(const snn_scan_desc* d, int neuron, const void* I, const f
 }
 
 }  // namespace
+
+std::atomic<unsigned long long> g_kernel_launches{0};
+
 }  // namespace snn
 
 using namespace snn;
 
 extern "C" {
+
+uint64_t snn_kernel_launches(void) { return g_kernel_launches.load(std::memory_order_relaxed); }
 
 const char* snn_status_string(snn_status_t status) {
   switch (status) {

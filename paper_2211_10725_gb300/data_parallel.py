@@ -39,11 +39,19 @@ def allreduce_sum_(tensors: Iterable[torch.Tensor], group: Optional[dist.Process
             dist.all_reduce(t, op=dist.ReduceOp.SUM, group=group)
 
 
+def grad_buffers(net):
+    """The buffers a replica's gradients and loss live in: dW of every layer
+    (one flat buffer), the learnable betas' gradients if the net has them
+    (the convolutional SNN), and the loss."""
+    return [net.dW_flat, getattr(net, "dbeta_flat", None), net.loss]
+
+
 class DataParallelDenseSNN:
-    """A DenseSNN replica per rank training on its shard of each global
-    batch: forward and BPTT on the shard (loss normalised by the global
-    batch), SUM all-reduce of dW (one flat buffer), then the same AdamW
-    update on every rank, so the replicas stay identical."""
+    """A network replica (DenseSNN or ConvSNN) per rank training on its
+    shard of each global batch: forward and BPTT on the shard (loss
+    normalised by the global batch), SUM all-reduce of the gradients (one
+    flat buffer per kind), then the same AdamW update on every rank, so the
+    replicas stay identical."""
 
     def __init__(self, net, global_batch: int, group: Optional[dist.ProcessGroup] = None):
         self.net = net
@@ -55,6 +63,9 @@ class DataParallelDenseSNN:
         net = self.net
         net.forward(X_shard, labels_shard, stream)
         net.backward(X_shard, stream)
-        allreduce_sum_([net.dW_flat, net.loss], self.group)
+        allreduce_sum_(grad_buffers(net), self.group)
         net.update(stream)
         return net.loss
+
+
+DataParallelConvSNN = DataParallelDenseSNN

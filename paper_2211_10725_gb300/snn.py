@@ -76,6 +76,11 @@ _SIGS = {
     "snn_dense_workspace_bytes": ([ctypes.c_int64] * 3, ctypes.c_size_t),
     "snn_dense_layer_bwd": ([ctypes.c_int64] * 3 + [_P] * 6 + [ctypes.c_size_t, _P], ctypes.c_int),
     "snn_rate_ce_workspace_bytes": ([ctypes.c_int64], ctypes.c_size_t),
+    "snn_kernel_launches": ([], ctypes.c_uint64),
+    "snn_im2col_nhwc": ([ctypes.c_int64] * 7 + [_P] * 3, ctypes.c_int),
+    "snn_col2im_nhwc": ([ctypes.c_int64] * 7 + [_P] * 3, ctypes.c_int),
+    "snn_maxpool2_fwd_nhwc": ([ctypes.c_int64] * 4 + [_P] * 4, ctypes.c_int),
+    "snn_maxpool2_bwd_nhwc": ([ctypes.c_int64] * 4 + [_P] * 4, ctypes.c_int),
     "snn_rate_ce_loss": ([ctypes.c_int64] * 6 + [ctypes.c_int32] + [_P] * 5 + [ctypes.c_size_t, _P],
                          ctypes.c_int),
     "snn_adamw_step": ([ctypes.c_int64] + [_P] * 5 + [ctypes.c_float] * 5 + [ctypes.c_int64] +
@@ -292,6 +297,37 @@ def snn_adamw_step(w, w_bf16, grad, m, v, lr, beta1=0.9, beta2=0.999, eps=1e-8,
     _check(load_library().snn_adamw_step(n, _ptr(w), _ptr(w_bf16), _ptr(grad), _ptr(m), _ptr(v),
                                          lr, beta1, beta2, eps, weight_decay, step,
                                          _ptr(step_counter), _stream(stream)), "snn_adamw_step")
+
+
+def snn_kernel_launches() -> int:
+    """Kernels the library has launched (or captured) in this process."""
+    return int(load_library().snn_kernel_launches())
+
+
+def snn_im2col_nhwc(X, cols, KH, KW, stream=None):
+    """Patch rows of channel-last X [M, H, W, Cin] into cols [M*Ho*Wo, Kpad]."""
+    M, H, W_, Cin = X.shape
+    _check(load_library().snn_im2col_nhwc(M, H, W_, Cin, KH, KW, cols.shape[-1], _ptr(X),
+                                          _ptr(cols), _stream(stream)), "snn_im2col_nhwc")
+
+
+def snn_col2im_nhwc(dcols, dX, KH, KW, stream=None):
+    """Patch-row gradient dcols [M*Ho*Wo, Kpad] summed onto dX [M, H, W, Cin]."""
+    M, H, W_, Cin = dX.shape
+    _check(load_library().snn_col2im_nhwc(M, H, W_, Cin, KH, KW, dcols.shape[-1], _ptr(dcols),
+                                          _ptr(dX), _stream(stream)), "snn_col2im_nhwc")
+
+
+def snn_maxpool2_fwd_nhwc(X, Y, idx, stream=None):
+    M, H, W_, C = X.shape
+    _check(load_library().snn_maxpool2_fwd_nhwc(M, H, W_, C, _ptr(X), _ptr(Y), _ptr(idx),
+                                                _stream(stream)), "snn_maxpool2_fwd_nhwc")
+
+
+def snn_maxpool2_bwd_nhwc(dY, idx, dX, stream=None):
+    M, H, W_, C = dX.shape
+    _check(load_library().snn_maxpool2_bwd_nhwc(M, H, W_, C, _ptr(dY), _ptr(idx), _ptr(dX),
+                                                _stream(stream)), "snn_maxpool2_bwd_nhwc")
 
 
 # ---------------------------------------------------------------------------

@@ -19,6 +19,8 @@ in for the datasets, which are not used):
                                 beta/threshold.
 * ``rleaky_T25_B128_N1000``     recurrent Leaky layer (Eq. 7), fp32, per-neuron v.
 * ``rleaky_bf16_T500_B64_N8192`` large recurrent Leaky layer, bf16 storage.
+* ``csnn_12c5_mp2_64c5_mp2_10_T25_B128`` convolutional SNN on 28x28 input
+                                (Tab. I CSNN), per-channel learnable beta.
 """
 from __future__ import annotations
 
@@ -214,3 +216,66 @@ def make_dense_inputs(w: DenseWorkload, seed: Optional[int] = None) -> dict:
         Ws.append(Wl.to(torch.bfloat16))
     labels = torch.randint(0, w.n_classes, (w.B,), generator=g, dtype=torch.int64).to(torch.int32)
     return {"X": X, "W": Ws, "labels": labels}
+
+
+# ---------------------------------------------------------------------------
+# Convolutional SNN (Tab. I CSNN: 12C5-MP2-64C5-MP2-10 on 28x28, T=25, B=128)
+# ---------------------------------------------------------------------------
+
+@dataclasses.dataclass(frozen=True)
+class ConvWorkload:
+    name: str = "csnn_12c5_mp2_64c5_mp2_10_T25_B128"
+    T: int = 25
+    B: int = 128
+    H: int = 28
+    W: int = 28
+    Cin: int = 1
+    convs: tuple = ((12, 5), (64, 5))   # (output channels, square kernel) per layer
+    n_classes: int = 10
+    rate_max: float = 0.3
+    beta: float = 0.95          # initial per-channel beta of the conv layers
+    beta_fc: float = 0.95       # output layer's beta (scalar, fixed)
+    thr: float = 1.0
+    sg_param: float = 25.0      # fast-sigmoid slope
+    reset: str = "zero"
+    seed_index: int = 9
+
+    def scaled(self, **kw) -> "ConvWorkload":
+        return dataclasses.replace(self, **kw)
+
+    def shapes(self):
+        """Per conv layer (H, W, Cin, Cout, k, Ho, Wo, Hp, Wp); then the
+        flattened size of the last pooled map."""
+        out, h, wd, c = [], self.H, self.W, self.Cin
+        for cout, k in self.convs:
+            ho, wo = h - k + 1, wd - k + 1
+            out.append((h, wd, c, cout, k, ho, wo, ho // 2, wo // 2))
+            h, wd, c = ho // 2, wo // 2, cout
+        return out, h * wd * c
+
+
+CSNN_C4 = ConvWorkload()
+
+CONV_WORKLOADS = {w.name: w for w in (CSNN_C4,)}
+
+
+def make_conv_inputs(w: ConvWorkload, seed: Optional[int] = None) -> dict:
+    """Bernoulli input spikes [T, B, H, W, Cin] (channel-last) with a
+    per-(sample, pixel) rate ~ U(0, rate_max) drawn once and independent over
+    t; He-uniform bf16 filters [Cout, k, k, Cin] and readout weights [10,
+    flattened pooled map (y, x, c order)] without bias; uniform labels."""
+    seed = SEED_BASE + w.seed_index if seed is None else seed
+    g = _gen(seed)
+    rate = w.rate_max * torch.rand((w.B, w.H, w.W, w.Cin), generator=g, dtype=torch.float32)
+    u = torch.rand((w.T, w.B, w.H, w.W, w.Cin), generator=g, dtype=torch.float32)
+    X = (u < rate.unsqueeze(0)).to(torch.bfloat16)
+    layers, n_flat = w.shapes()
+    convs = []
+    for (_, _, cin, cout, k, *_rest) in layers:
+        bound = (6.0 / (k * k * cin)) ** 0.5
+        Wc = (2.0 * torch.rand((cout, k, k, cin), generator=g, dtype=torch.float32) - 1.0) * bound
+        convs.append(Wc.to(torch.bfloat16))
+    bound = (6.0 / n_flat) ** 0.5
+    Wfc = (2.0 * torch.rand((w.n_classes, n_flat), generator=g, dtype=torch.float32) - 1.0) * bound
+    labels = torch.randint(0, w.n_classes, (w.B,), generator=g, dtype=torch.int64).to(torch.int32)
+    return {"X": X, "convs": convs, "Wfc": Wfc.to(torch.bfloat16), "labels": labels}

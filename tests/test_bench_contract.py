@@ -23,7 +23,8 @@ def _run(*args, env=None):
 
 
 @pytest.mark.parametrize("workload", [None, "dsnn_784_1000_1000_10_T25_B128",
-                                      "rleaky_T25_B128_N1000"])
+                                      "rleaky_T25_B128_N1000",
+                                      "csnn_12c5_mp2_64c5_mp2_10_T25_B128"])
 def test_reference_leg_prints_one_contract_line(workload):
     args = ["--impl", "reference", "--steps", "2", "--warmup", "1", "--reference-seconds", "3"]
     if workload:
