@@ -585,14 +585,18 @@ def conv_op_bytes(net):
         layer = net.layers[l]
         ns = T * B * layer.w.N
         f, b = algorithmic_bytes(layer.w)
-        out[f"im2col{l}"] = x_bytes + nb(net.cols[l])
-        out[f"conv_fwd{l}"] = nb(net.cols[l]) + nb(net.W[l]) + nb(net.I[l])
+        if net.cols[l] is None:   # direct convolution: reads the input map itself
+            out[f"conv_fwd{l}"] = x_bytes + nb(net.W[l]) + nb(net.I[l])
+        else:
+            out[f"im2col{l}"] = x_bytes + nb(net.cols[l])
+            out[f"conv_fwd{l}"] = nb(net.cols[l]) + nb(net.W[l]) + nb(net.I[l])
         out[f"scan_fwd{l}"] = f * ns
         out[f"pool_fwd{l}"] = nb(layer.spk) + nb(net.pool[l]) + nb(net.idx[l])
         out[f"pool_bwd{l}"] = nb(net.grad_pool[l]) + nb(net.idx[l]) + nb(net.grad_spk[l])
         out[f"scan_bwd{l}"] = b * ns
-        out[f"conv_bwd{l}"] = (nb(net.cols[l]) + nb(layer.grad_I) + nb(net.W[l])
-                               + nb(net.dcols[l]) + nb(net.dW[l]))
+        src = x_bytes if net.cols[l] is None else nb(net.cols[l])
+        out[f"conv_bwd{l}"] = (src + nb(layer.grad_I) + nb(net.W[l]) + nb(net.dcols[l])
+                               + nb(net.dW[l]))
         if l > 0:
             out[f"col2im{l}"] = nb(net.dcols[l]) + nb(net.grad_pool[l - 1])
     o = net.out_layer

@@ -368,6 +368,34 @@ snn_status_t snn_maxpool2_bwd_nhwc(int64_t M, int64_t H, int64_t W, int64_t C, c
                                    const uint8_t* idx, void* dX, snn_stream_t stream);
 
 /*
+ * Convolution with few input channels on the CUDA cores (the CSNN's first
+ * layer, Tab. I: 5x5 filters over the 1-channel input map), where the patch
+ * rows of a GEMM would be mostly padding: KH*KW*Cin <= 32, Cout <= 16 and a
+ * multiple of 4, H*W*Cin <= 8192 (else SNN_ERR_UNSUPPORTED).
+ *   X  bf16 [M, H, W, Cin] channel-last;  Wt bf16 [Cout, ldw] filters with
+ *      column k = (ky*KW + kx)*Cin + c (the im2col order), ldw >= KH*KW*Cin
+ *   snn_conv2d_small_fwd_nhwc: I fp32 [M, Ho, Wo, Cout] (out, 16-byte
+ *      aligned) = the valid stride-1 convolution, fp32 fused multiply-adds
+ *      in k order
+ *   snn_conv2d_small_dw_nhwc: dW fp32 [Cout, ldw] (out; 0 past column K) =
+ *      sum over (m, oy, ox) of dI[m, oy, ox, o] * X[m, oy+ky, ox+kx, c] for
+ *      dI bf16 [M, Ho, Wo, Cout]; a fixed number of blocks each sum a fixed
+ *      set of images, the block partials (ws, at least
+ *      snn_conv2d_small_dw_workspace_bytes, 16-byte aligned) are added in
+ *      block order: the same bits on every call
+ * Asynchronous on stream.
+ */
+snn_status_t snn_conv2d_small_fwd_nhwc(int64_t M, int64_t H, int64_t W, int64_t Cin, int64_t Cout,
+                                       int64_t KH, int64_t KW, int64_t ldw, const void* X,
+                                       const void* Wt, float* I, snn_stream_t stream);
+size_t snn_conv2d_small_dw_workspace_bytes(int64_t M, int64_t H, int64_t W, int64_t Cin,
+                                           int64_t Cout, int64_t KH, int64_t KW);
+snn_status_t snn_conv2d_small_dw_nhwc(int64_t M, int64_t H, int64_t W, int64_t Cin, int64_t Cout,
+                                      int64_t KH, int64_t KW, int64_t ldw, const void* X,
+                                      const void* dI, float* dW, void* ws, size_t ws_bytes,
+                                      snn_stream_t stream);
+
+/*
  * AdamW update of n fp32 master weights (the optimiser of the paper's
  * training runs, Sec. V; decoupled weight decay):
  *   m <- beta1 m + (1 - beta1) g ;  v <- beta2 v + (1 - beta2) g^2

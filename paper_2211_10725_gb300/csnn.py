@@ -18,8 +18,14 @@ kernels.
 Channel counts are padded to a multiple of 8 (12 -> 16, the 10 outputs ->
 16) because the GEMM's TMA tiles need 16-byte row strides.  A padded
 channel has zero filters: its current is 0, it never fires, no later
-filter reads it, and its gradients are exactly 0.  The first layer's
-5x5x1 patch (25 columns) is padded to 32 zero columns.
+filter reads it, and its gradients are exactly 0.
+
+The first layer (a 5x5 filter over one input channel: 25 products per
+output) runs as a direct convolution on the CUDA cores, with its image
+staged in shared memory, and so does its weight gradient; a patch-row GEMM
+would write and read 32 padded columns per output pixel for that
+(``direct_first=False`` keeps the im2col + GEMM path, whose 25 columns are
+padded to 32).
 """
 from __future__ import annotations
 
@@ -39,7 +45,8 @@ class ConvSNN:
 
     def __init__(self, w: W.ConvWorkload, convs, Wfc, device="cuda", save: str = "recompute",
                  lr: float = 1e-3, betas=(0.9, 0.999), eps: float = 1e-8,
-                 weight_decay: float = 1e-2, learn_beta: bool = True):
+                 weight_decay: float = 1e-2, learn_beta: bool = True,
+                 direct_first: bool = True):
         self.w = w
         self.save = save
         self.lr, self.betas, self.eps, self.weight_decay = lr, betas, eps, weight_decay
@@ -59,6 +66,11 @@ class ConvSNN:
             cin_p = cout_p
         hf, wf, cf = self.geo[-1][7], self.geo[-1][8], self.geo[-1][3]
         self.n_flat = hf * wf * cf
+        # layers that run as a direct convolution (only the first: it needs
+        # no input gradient)
+        g0 = self.geo[0]
+        self.direct = [direct_first and g0[4] * g0[4] * g0[2] <= 32 and g0[3] <= 16
+                       and g0[0] * g0[1] * g0[2] <= 8192] + [False] * (len(self.geo) - 1)
         self.n_out = _pad8(w.n_classes)
 
         # weights: one flat buffer per quantity, each block on a 64-element
@@ -114,7 +126,7 @@ class ConvSNN:
         self.grad_spk, self.grad_pool, self.dcols, self.ws_bwd = [], [], [], []
         for l, (h, wd, cin, cout, k, ho, wo, hp, wp, kpad) in enumerate(self.geo):
             rows = M * ho * wo
-            self.cols.append(torch.empty((rows, kpad), **bf))
+            self.cols.append(None if self.direct[l] else torch.empty((rows, kpad), **bf))
             self.I.append(torch.empty((rows, cout), dtype=torch.float32, device=dev))
             lw = W.ScanWorkload(name=f"csnn_conv{l}", neuron="leaky", T=T, B=B,
                                 N=ho * wo * cout, C=cout, HW=1, in_dtype=W.F32, io_dtype=W.BF16,
@@ -127,8 +139,11 @@ class ConvSNN:
             self.grad_spk.append(torch.empty((M, ho, wo, cout), **bf))
             self.grad_pool.append(torch.empty((M, hp, wp, cout), **bf))
             self.dcols.append(torch.empty((rows, kpad), **bf) if l > 0 else None)
-            nb = snn.snn_dense_workspace_bytes(rows, kpad, cout)
-            self.ws_bwd.append(torch.zeros(nb, dtype=torch.uint8, device=dev))
+            if self.direct[l]:
+                nb = snn.snn_conv2d_small_dw_workspace_bytes(M, h, wd, cin, cout, k, k)
+            else:
+                nb = snn.snn_dense_workspace_bytes(rows, kpad, cout)
+            self.ws_bwd.append(torch.zeros(max(nb, 256), dtype=torch.uint8, device=dev))
         self.I_fc = torch.empty((M, self.n_out), dtype=torch.float32, device=dev)
         fw = W.ScanWorkload(name="csnn_out", neuron="leaky", T=T, B=B, N=self.n_out,
                             in_dtype=W.F32, io_dtype=W.BF16, beta=("const", w.beta_fc),
@@ -157,10 +172,15 @@ class ConvSNN:
         out = []
         for l, (h, wd, cin, cout, k, ho, wo, hp, wp, kpad) in enumerate(self.geo):
             layer = self.layers[l]
-            out.append((f"im2col{l}", lambda l=l, k=k: snn.snn_im2col_nhwc(
-                self.layer_input(l, X), self.cols[l], k, k, stream)))
-            out.append((f"conv_fwd{l}", lambda l=l: snn.snn_dense_layer_fwd(
-                self.cols[l], self.W[l], self.I[l], self.ws_fwd, stream)))
+            if self.direct[l]:
+                out.append((f"conv_fwd{l}", lambda l=l, k=k, s=(M, ho, wo, cout):
+                            snn.snn_conv2d_small_fwd_nhwc(self.layer_input(l, X), self.W[l],
+                                                          self.I[l].view(s), k, k, stream)))
+            else:
+                out.append((f"im2col{l}", lambda l=l, k=k: snn.snn_im2col_nhwc(
+                    self.layer_input(l, X), self.cols[l], k, k, stream)))
+                out.append((f"conv_fwd{l}", lambda l=l: snn.snn_dense_layer_fwd(
+                    self.cols[l], self.W[l], self.I[l], self.ws_fwd, stream)))
             out.append((f"scan_fwd{l}", lambda l=l, layer=layer: layer.forward(
                 self.I[l].view(T, B, -1), self.beta[l], self.thr, stream=stream)))
             out.append((f"pool_fwd{l}", lambda l=l, layer=layer, s=(M, ho, wo, cout):
@@ -187,10 +207,16 @@ class ConvSNN:
             out.append((f"pool_bwd{l}", lambda l=l: snn.snn_maxpool2_bwd_nhwc(
                 self.grad_pool[l], self.idx[l], self.grad_spk[l], stream)))
             out.append((f"scan_bwd{l}", lambda l=l, layer=layer: self._scan_bwd(l, stream)))
-            out.append((f"conv_bwd{l}", lambda l=l, layer=layer, rows=M * ho * wo, c=cout:
-                        snn.snn_dense_layer_bwd(self.cols[l], self.W[l],
-                                                layer.grad_I.view(rows, c), self.dcols[l],
-                                                self.dW[l], self.ws_bwd[l], stream)))
+            if self.direct[l]:
+                out.append((f"conv_bwd{l}", lambda l=l, layer=layer, k=k, s=(M, ho, wo, cout):
+                            snn.snn_conv2d_small_dw_nhwc(self.layer_input(l, X),
+                                                         layer.grad_I.view(s), self.dW[l], k, k,
+                                                         self.ws_bwd[l], stream)))
+            else:
+                out.append((f"conv_bwd{l}", lambda l=l, layer=layer, rows=M * ho * wo, c=cout:
+                            snn.snn_dense_layer_bwd(self.cols[l], self.W[l],
+                                                    layer.grad_I.view(rows, c), self.dcols[l],
+                                                    self.dW[l], self.ws_bwd[l], stream)))
             if l > 0:
                 out.append((f"col2im{l}", lambda l=l, k=k: snn.snn_col2im_nhwc(
                     self.dcols[l], self.grad_pool[l - 1], k, k, stream)))
@@ -218,7 +244,7 @@ class ConvSNN:
                                step_counter=self.beta_counter, stream=stream)
 
     def _n_fwd(self):
-        return 4 * len(self.geo) + 3
+        return 3 * len(self.geo) + sum(not d for d in self.direct) + 3
 
     def forward(self, X, labels, stream=None):
         """X: bf16 [T*B, H, W, Cin] spikes on the device; labels int32 [B]."""

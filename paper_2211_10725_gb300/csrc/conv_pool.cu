@@ -11,6 +11,8 @@
 //            (row major) is kept and its position recorded, and the
 //            backward routes the gradient there (every input element
 //            belongs to one window, so no two threads write one element).
+// With a channel count that is a multiple of 8 every kernel moves 8
+// channels (16 bytes) per thread; otherwise one element per thread.
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
 
@@ -26,19 +28,20 @@ namespace {
 constexpr int kThreads = 256;
 
 // Eight consecutive columns of one patch row per thread (one 16-byte store).
+template <typename Ix>
 __global__ void __launch_bounds__(kThreads) im2col_kernel(const __nv_bfloat16* __restrict__ X,
                                                           __nv_bfloat16* __restrict__ cols,
-                                                          int64_t rows, int H, int W, int Cin,
+                                                          Ix rows, int H, int W, int Cin,
                                                           int KH, int KW, int Kpad) {
   grid_dep_wait();
   const int Ho = H - KH + 1, Wo = W - KW + 1;
   const int K = KH * KW * Cin;
   const int vec_per_row = Kpad / 8;
-  const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  const Ix i = (Ix)blockIdx.x * blockDim.x + threadIdx.x;
   if (i >= rows * vec_per_row) return;
-  const int64_t r = i / vec_per_row;
+  const Ix r = i / vec_per_row;
   const int k0 = (int)(i - r * vec_per_row) * 8;
-  const int64_t m = r / (Ho * Wo);
+  const Ix m = r / (Ho * Wo);
   const int p = (int)(r - m * (Ho * Wo));
   const int oy = p / Wo, ox = p - oy * Wo;
   const __nv_bfloat16* xm = X + m * H * W * Cin;
@@ -58,20 +61,21 @@ __global__ void __launch_bounds__(kThreads) im2col_kernel(const __nv_bfloat16* _
   *reinterpret_cast<uint4*>(cols + r * Kpad + k0) = *reinterpret_cast<const uint4*>(v);
 }
 
+template <typename Ix>
 __global__ void __launch_bounds__(kThreads) col2im_kernel(const __nv_bfloat16* __restrict__ dcols,
                                                           __nv_bfloat16* __restrict__ dX,
-                                                          int64_t total, int H, int W, int Cin,
+                                                          Ix total, int H, int W, int Cin,
                                                           int KH, int KW, int Kpad) {
   grid_dep_wait();
   const int Ho = H - KH + 1, Wo = W - KW + 1;
-  const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  const Ix i = (Ix)blockIdx.x * blockDim.x + threadIdx.x;
   if (i >= total) return;
   const int c = (int)(i % Cin);
-  const int64_t q = i / Cin;
+  const Ix q = i / Cin;
   const int x = (int)(q % W);
-  const int64_t q2 = q / W;
+  const Ix q2 = q / W;
   const int y = (int)(q2 % H);
-  const int64_t m = q2 / H;
+  const Ix m = q2 / H;
   float s = 0.0f;
   for (int ky = 0; ky < KH; ++ky) {
     const int oy = y - ky;
@@ -79,30 +83,31 @@ __global__ void __launch_bounds__(kThreads) col2im_kernel(const __nv_bfloat16* _
     for (int kx = 0; kx < KW; ++kx) {
       const int ox = x - kx;
       if (ox < 0 || ox >= Wo) continue;
-      const int64_t r = (m * Ho + oy) * Wo + ox;
+      const Ix r = (m * Ho + oy) * Wo + ox;
       s += __bfloat162float(dcols[r * Kpad + (ky * KW + kx) * Cin + c]);
     }
   }
   dX[i] = __float2bfloat16_rn(s);
 }
 
+template <typename Ix>
 __global__ void __launch_bounds__(kThreads) maxpool_fwd_kernel(const __nv_bfloat16* __restrict__ X,
                                                                __nv_bfloat16* __restrict__ Y,
                                                                uint8_t* __restrict__ idx,
-                                                               int64_t total, int H, int W,
+                                                               Ix total, int H, int W,
                                                                int C) {
   grid_dep_wait();
-  const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  const Ix i = (Ix)blockIdx.x * blockDim.x + threadIdx.x;
   if (i >= total) return;
   const int Hp = H / 2, Wp = W / 2;
   const int c = (int)(i % C);
-  const int64_t q = i / C;
+  const Ix q = i / C;
   const int px = (int)(q % Wp);
-  const int64_t q2 = q / Wp;
+  const Ix q2 = q / Wp;
   const int py = (int)(q2 % Hp);
-  const int64_t m = q2 / Hp;
+  const Ix m = q2 / Hp;
   const __nv_bfloat16* base = X + ((m * H + 2 * py) * W + 2 * px) * C + c;
-  const int64_t off[4] = {0, (int64_t)C, (int64_t)W * C, (int64_t)W * C + C};
+  const Ix off[4] = {0, (Ix)C, (Ix)W * C, (Ix)W * C + C};
   float best = __bfloat162float(base[0]);
   int arg = 0;
 #pragma unroll
@@ -117,24 +122,177 @@ __global__ void __launch_bounds__(kThreads) maxpool_fwd_kernel(const __nv_bfloat
   idx[i] = (uint8_t)arg;
 }
 
+template <typename Ix>
 __global__ void __launch_bounds__(kThreads) maxpool_bwd_kernel(const __nv_bfloat16* __restrict__ dY,
                                                                const uint8_t* __restrict__ idx,
                                                                __nv_bfloat16* __restrict__ dX,
-                                                               int64_t total, int H, int W,
+                                                               Ix total, int H, int W,
                                                                int C) {
   grid_dep_wait();
-  const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  const Ix i = (Ix)blockIdx.x * blockDim.x + threadIdx.x;
   if (i >= total) return;
   const int Hp = H / 2, Wp = W / 2;
   const int c = (int)(i % C);
-  const int64_t q = i / C;
+  const Ix q = i / C;
   const int x = (int)(q % W);
-  const int64_t q2 = q / W;
+  const Ix q2 = q / W;
   const int y = (int)(q2 % H);
-  const int64_t m = q2 / H;
-  const int64_t o = ((m * Hp + y / 2) * Wp + x / 2) * C + c;
+  const Ix m = q2 / H;
+  const Ix o = ((m * Hp + y / 2) * Wp + x / 2) * C + c;
   const int pos = (y & 1) * 2 + (x & 1);
   dX[i] = idx[o] == pos ? dY[o] : __float2bfloat16_rn(0.0f);
+}
+
+// ---- 8 channels per thread (C % 8 == 0, 16-byte aligned tensors) --------
+
+union Pack8 {
+  uint4 u;
+  __nv_bfloat16 h[8];
+};
+
+// Thread i copies column group j = i % (Kpad/8) of patch row i / (Kpad/8):
+// the 8 channels of one tap (groups past K are zero).
+template <typename Ix>
+__global__ void __launch_bounds__(kThreads) im2col_vec8_kernel(const uint4* __restrict__ X,
+                                                               uint4* __restrict__ cols,
+                                                               Ix rows, int H, int W, int Cin,
+                                                               int KH, int KW, int Kpad) {
+  grid_dep_wait();
+  const int Ho = H - KH + 1, Wo = W - KW + 1;
+  const int G = Cin / 8;  // channel groups per tap
+  const int vpr = Kpad / 8;
+  const Ix i = (Ix)blockIdx.x * blockDim.x + threadIdx.x;
+  if (i >= rows * vpr) return;
+  const Ix r = i / vpr;
+  const int j = (int)(i - r * vpr);
+  uint4 v = make_uint4(0u, 0u, 0u, 0u);
+  if (j < KH * KW * G) {
+    const Ix m = r / (Ho * Wo);
+    const int p = (int)(r - m * (Ho * Wo));
+    const int oy = p / Wo, ox = p - oy * Wo;
+    const int tap = j / G, g = j - tap * G;
+    const int ky = tap / KW, kx = tap - ky * KW;
+    v = X[((m * H + oy + ky) * W + ox + kx) * G + g];
+  }
+  cols[i] = v;
+}
+
+// Thread i sums the 8 channels of group i % G of pixel i / G over the taps
+// that read it, in (ky, kx) order.
+template <typename Ix>
+__global__ void __launch_bounds__(kThreads) col2im_vec8_kernel(const uint4* __restrict__ dcols,
+                                                               uint4* __restrict__ dX,
+                                                               Ix total, int H, int W, int Cin,
+                                                               int KH, int KW, int Kpad) {
+  grid_dep_wait();
+  const int Ho = H - KH + 1, Wo = W - KW + 1;
+  const int G = Cin / 8, vpr = Kpad / 8;
+  const Ix i = (Ix)blockIdx.x * blockDim.x + threadIdx.x;
+  if (i >= total) return;
+  const Ix q = i / G;
+  const int g = (int)(i - q * G);
+  const int x = (int)(q % W);
+  const Ix q2 = q / W;
+  const int y = (int)(q2 % H);
+  const Ix m = q2 / H;
+  float s[8];
+#pragma unroll
+  for (int e = 0; e < 8; ++e) s[e] = 0.0f;
+  for (int ky = 0; ky < KH; ++ky) {
+    const int oy = y - ky;
+    if (oy < 0 || oy >= Ho) continue;
+    for (int kx = 0; kx < KW; ++kx) {
+      const int ox = x - kx;
+      if (ox < 0 || ox >= Wo) continue;
+      const Ix r = (m * Ho + oy) * Wo + ox;
+      Pack8 v;
+      v.u = dcols[r * vpr + (ky * KW + kx) * G + g];
+#pragma unroll
+      for (int e = 0; e < 8; ++e) s[e] += __bfloat162float(v.h[e]);
+    }
+  }
+  Pack8 o;
+#pragma unroll
+  for (int e = 0; e < 8; ++e) o.h[e] = __float2bfloat16_rn(s[e]);
+  dX[i] = o.u;
+}
+
+// Thread i pools the 8 channels of group i % G of output pixel i / G.
+template <typename Ix>
+__global__ void __launch_bounds__(kThreads) maxpool_fwd_vec8_kernel(const uint4* __restrict__ X,
+                                                                    uint4* __restrict__ Y,
+                                                                    uint2* __restrict__ idx,
+                                                                    Ix total, int H, int W,
+                                                                    int C) {
+  grid_dep_wait();
+  const Ix i = (Ix)blockIdx.x * blockDim.x + threadIdx.x;
+  if (i >= total) return;
+  const int G = C / 8, Hp = H / 2, Wp = W / 2;
+  const Ix q = i / G;
+  const int g = (int)(i - q * G);
+  const int px = (int)(q % Wp);
+  const Ix q2 = q / Wp;
+  const int py = (int)(q2 % Hp);
+  const Ix m = q2 / Hp;
+  const Ix base = ((m * H + 2 * py) * W + 2 * px) * G + g;
+  Pack8 w[4];
+  w[0].u = X[base];
+  w[1].u = X[base + G];
+  w[2].u = X[base + (Ix)W * G];
+  w[3].u = X[base + (Ix)W * G + G];
+  Pack8 best = w[0];
+  uint8_t arg[8] = {0, 0, 0, 0, 0, 0, 0, 0};
+#pragma unroll
+  for (int j = 1; j < 4; ++j) {
+#pragma unroll
+    for (int e = 0; e < 8; ++e) {
+      if (__bfloat162float(w[j].h[e]) > __bfloat162float(best.h[e])) {  // first maximum kept
+        best.h[e] = w[j].h[e];
+        arg[e] = (uint8_t)j;
+      }
+    }
+  }
+  Y[i] = best.u;
+  uint2 a;
+  a.x = (uint32_t)arg[0] | ((uint32_t)arg[1] << 8) | ((uint32_t)arg[2] << 16) | ((uint32_t)arg[3] << 24);
+  a.y = (uint32_t)arg[4] | ((uint32_t)arg[5] << 8) | ((uint32_t)arg[6] << 16) | ((uint32_t)arg[7] << 24);
+  idx[i] = a;
+}
+
+// Thread i routes the 8 channels of group i % G of output pixel i / G back
+// to its window, writing all four positions (zero where not the maximum).
+template <typename Ix>
+__global__ void __launch_bounds__(kThreads) maxpool_bwd_vec8_kernel(const uint4* __restrict__ dY,
+                                                                    const uint2* __restrict__ idx,
+                                                                    uint4* __restrict__ dX,
+                                                                    Ix total, int H, int W,
+                                                                    int C) {
+  grid_dep_wait();
+  const Ix i = (Ix)blockIdx.x * blockDim.x + threadIdx.x;
+  if (i >= total) return;
+  const int G = C / 8, Hp = H / 2, Wp = W / 2;
+  const Ix q = i / G;
+  const int g = (int)(i - q * G);
+  const int px = (int)(q % Wp);
+  const Ix q2 = q / Wp;
+  const int py = (int)(q2 % Hp);
+  const Ix m = q2 / Hp;
+  Pack8 d;
+  d.u = dY[i];
+  const uint2 a = idx[i];
+  const __nv_bfloat16 zero = __float2bfloat16_rn(0.0f);
+  Pack8 o[4];
+#pragma unroll
+  for (int e = 0; e < 8; ++e) {
+    const int pos = (int)(((e < 4 ? a.x : a.y) >> (8 * (e & 3))) & 0xFFu);
+#pragma unroll
+    for (int j = 0; j < 4; ++j) o[j].h[e] = pos == j ? d.h[e] : zero;
+  }
+  const Ix base = ((m * H + 2 * py) * W + 2 * px) * G + g;
+  dX[base] = o[0].u;
+  dX[base + G] = o[1].u;
+  dX[base + (Ix)W * G] = o[2].u;
+  dX[base + (Ix)W * G + G] = o[3].u;
 }
 
 bool aligned(const void* p, uintptr_t a) { return (reinterpret_cast<uintptr_t>(p) & (a - 1)) == 0; }
@@ -158,7 +316,24 @@ extern "C" snn_status_t snn_im2col_nhwc(int64_t M, int64_t H, int64_t W, int64_t
   const int64_t rows = M * (H - KH + 1) * (W - KW + 1);
   const int64_t n = rows * (Kpad / 8);
   if (n / kThreads >= INT_MAX) return SNN_ERR_INVALID_ARG;
-  const cudaError_t e = launch_pdl(im2col_kernel, dim3(blocks_for(n)), dim3(kThreads), 0,
+  const bool i32 = rows * Kpad < INT_MAX && M * H * W * Cin < INT_MAX;  // 32-bit index math
+  if (Cin % 8 == 0 && aligned(X, 16)) {
+    const cudaError_t e = i32 ? launch_pdl(im2col_vec8_kernel<int>, dim3(blocks_for(n)), dim3(kThreads), 0,
+                                     reinterpret_cast<cudaStream_t>(stream),
+                                     static_cast<const uint4*>(X), static_cast<uint4*>(cols), rows,
+                                     (int)H, (int)W, (int)Cin, (int)KH, (int)KW, (int)Kpad)
+                                   : launch_pdl(im2col_vec8_kernel<int64_t>, dim3(blocks_for(n)), dim3(kThreads), 0,
+                                     reinterpret_cast<cudaStream_t>(stream),
+                                     static_cast<const uint4*>(X), static_cast<uint4*>(cols), rows,
+                                     (int)H, (int)W, (int)Cin, (int)KH, (int)KW, (int)Kpad);
+    return e == cudaSuccess ? SNN_OK : SNN_ERR_CUDA;
+  }
+  const cudaError_t e = i32 ? launch_pdl(im2col_kernel<int>, dim3(blocks_for(n)), dim3(kThreads), 0,
+                                   reinterpret_cast<cudaStream_t>(stream),
+                                   static_cast<const __nv_bfloat16*>(X),
+                                   static_cast<__nv_bfloat16*>(cols), rows, (int)H, (int)W, (int)Cin,
+                                   (int)KH, (int)KW, (int)Kpad)
+                                   : launch_pdl(im2col_kernel<int64_t>, dim3(blocks_for(n)), dim3(kThreads), 0,
                                    reinterpret_cast<cudaStream_t>(stream),
                                    static_cast<const __nv_bfloat16*>(X),
                                    static_cast<__nv_bfloat16*>(cols), rows, (int)H, (int)W, (int)Cin,
@@ -177,7 +352,24 @@ extern "C" snn_status_t snn_col2im_nhwc(int64_t M, int64_t H, int64_t W, int64_t
   if (!aligned(dcols, 2) || !aligned(dX, 2)) return SNN_ERR_ALIGNMENT;
   const int64_t n = M * H * W * Cin;
   if (n / kThreads >= INT_MAX) return SNN_ERR_INVALID_ARG;
-  const cudaError_t e = launch_pdl(col2im_kernel, dim3(blocks_for(n)), dim3(kThreads), 0,
+  const bool i32 = M * (H - KH + 1) * (W - KW + 1) * Kpad < INT_MAX && n < INT_MAX;
+  if (Cin % 8 == 0 && Kpad % 8 == 0 && aligned(dcols, 16) && aligned(dX, 16)) {
+    const cudaError_t e = i32 ? launch_pdl(col2im_vec8_kernel<int>, dim3(blocks_for(n / 8)), dim3(kThreads), 0,
+                                     reinterpret_cast<cudaStream_t>(stream),
+                                     static_cast<const uint4*>(dcols), static_cast<uint4*>(dX),
+                                     n / 8, (int)H, (int)W, (int)Cin, (int)KH, (int)KW, (int)Kpad)
+                                   : launch_pdl(col2im_vec8_kernel<int64_t>, dim3(blocks_for(n / 8)), dim3(kThreads), 0,
+                                     reinterpret_cast<cudaStream_t>(stream),
+                                     static_cast<const uint4*>(dcols), static_cast<uint4*>(dX),
+                                     n / 8, (int)H, (int)W, (int)Cin, (int)KH, (int)KW, (int)Kpad);
+    return e == cudaSuccess ? SNN_OK : SNN_ERR_CUDA;
+  }
+  const cudaError_t e = i32 ? launch_pdl(col2im_kernel<int>, dim3(blocks_for(n)), dim3(kThreads), 0,
+                                   reinterpret_cast<cudaStream_t>(stream),
+                                   static_cast<const __nv_bfloat16*>(dcols),
+                                   static_cast<__nv_bfloat16*>(dX), n, (int)H, (int)W, (int)Cin,
+                                   (int)KH, (int)KW, (int)Kpad)
+                                   : launch_pdl(col2im_kernel<int64_t>, dim3(blocks_for(n)), dim3(kThreads), 0,
                                    reinterpret_cast<cudaStream_t>(stream),
                                    static_cast<const __nv_bfloat16*>(dcols),
                                    static_cast<__nv_bfloat16*>(dX), n, (int)H, (int)W, (int)Cin,
@@ -195,7 +387,23 @@ extern "C" snn_status_t snn_maxpool2_fwd_nhwc(int64_t M, int64_t H, int64_t W, i
   if (!aligned(X, 2) || !aligned(Y, 2)) return SNN_ERR_ALIGNMENT;
   const int64_t n = M * (H / 2) * (W / 2) * C;
   if (n / kThreads >= INT_MAX) return SNN_ERR_INVALID_ARG;
-  const cudaError_t e = launch_pdl(maxpool_fwd_kernel, dim3(blocks_for(n)), dim3(kThreads), 0,
+  const bool i32 = M * H * W * C < INT_MAX;
+  if (C % 8 == 0 && aligned(X, 16) && aligned(Y, 16) && aligned(idx, 8)) {
+    const cudaError_t e = i32 ? launch_pdl(maxpool_fwd_vec8_kernel<int>, dim3(blocks_for(n / 8)),
+                                     dim3(kThreads), 0, reinterpret_cast<cudaStream_t>(stream),
+                                     static_cast<const uint4*>(X), static_cast<uint4*>(Y),
+                                     reinterpret_cast<uint2*>(idx), n / 8, (int)H, (int)W, (int)C)
+                                   : launch_pdl(maxpool_fwd_vec8_kernel<int64_t>, dim3(blocks_for(n / 8)),
+                                     dim3(kThreads), 0, reinterpret_cast<cudaStream_t>(stream),
+                                     static_cast<const uint4*>(X), static_cast<uint4*>(Y),
+                                     reinterpret_cast<uint2*>(idx), n / 8, (int)H, (int)W, (int)C);
+    return e == cudaSuccess ? SNN_OK : SNN_ERR_CUDA;
+  }
+  const cudaError_t e = i32 ? launch_pdl(maxpool_fwd_kernel<int>, dim3(blocks_for(n)), dim3(kThreads), 0,
+                                   reinterpret_cast<cudaStream_t>(stream),
+                                   static_cast<const __nv_bfloat16*>(X),
+                                   static_cast<__nv_bfloat16*>(Y), idx, n, (int)H, (int)W, (int)C)
+                                   : launch_pdl(maxpool_fwd_kernel<int64_t>, dim3(blocks_for(n)), dim3(kThreads), 0,
                                    reinterpret_cast<cudaStream_t>(stream),
                                    static_cast<const __nv_bfloat16*>(X),
                                    static_cast<__nv_bfloat16*>(Y), idx, n, (int)H, (int)W, (int)C);
@@ -212,7 +420,26 @@ extern "C" snn_status_t snn_maxpool2_bwd_nhwc(int64_t M, int64_t H, int64_t W, i
   if (!aligned(dY, 2) || !aligned(dX, 2)) return SNN_ERR_ALIGNMENT;
   const int64_t n = M * H * W * C;
   if (n / kThreads >= INT_MAX) return SNN_ERR_INVALID_ARG;
-  const cudaError_t e = launch_pdl(maxpool_bwd_kernel, dim3(blocks_for(n)), dim3(kThreads), 0,
+  const bool i32 = n < INT_MAX;
+  if (C % 8 == 0 && aligned(dY, 16) && aligned(dX, 16) && aligned(idx, 8)) {
+    const int64_t np = n / 32;  // output pixels x channel groups
+    const cudaError_t e = i32 ? launch_pdl(maxpool_bwd_vec8_kernel<int>, dim3(blocks_for(np)),
+                                     dim3(kThreads), 0, reinterpret_cast<cudaStream_t>(stream),
+                                     static_cast<const uint4*>(dY),
+                                     reinterpret_cast<const uint2*>(idx), static_cast<uint4*>(dX),
+                                     np, (int)H, (int)W, (int)C)
+                                   : launch_pdl(maxpool_bwd_vec8_kernel<int64_t>, dim3(blocks_for(np)),
+                                     dim3(kThreads), 0, reinterpret_cast<cudaStream_t>(stream),
+                                     static_cast<const uint4*>(dY),
+                                     reinterpret_cast<const uint2*>(idx), static_cast<uint4*>(dX),
+                                     np, (int)H, (int)W, (int)C);
+    return e == cudaSuccess ? SNN_OK : SNN_ERR_CUDA;
+  }
+  const cudaError_t e = i32 ? launch_pdl(maxpool_bwd_kernel<int>, dim3(blocks_for(n)), dim3(kThreads), 0,
+                                   reinterpret_cast<cudaStream_t>(stream),
+                                   static_cast<const __nv_bfloat16*>(dY), idx,
+                                   static_cast<__nv_bfloat16*>(dX), n, (int)H, (int)W, (int)C)
+                                   : launch_pdl(maxpool_bwd_kernel<int64_t>, dim3(blocks_for(n)), dim3(kThreads), 0,
                                    reinterpret_cast<cudaStream_t>(stream),
                                    static_cast<const __nv_bfloat16*>(dY), idx,
                                    static_cast<__nv_bfloat16*>(dX), n, (int)H, (int)W, (int)C);

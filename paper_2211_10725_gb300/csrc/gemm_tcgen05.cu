@@ -22,6 +22,12 @@
 // to the tensor core as atoms of 8 K-rows of 128 bytes: 1024 bytes apart
 // along K, one box (8 KB) apart along MN.
 //
+// Output: with 16-byte output rows each epilogue warp stages its 32 rows
+// of a 128-byte-wide column chunk in shared memory (128-byte swizzle, two
+// buffers per warp) and one lane writes the chunk with a TMA tensor store,
+// so every warp write is whole 128-byte lines; otherwise the threads store
+// their rows directly.
+//
 // Split K: a product whose few output tiles each sum a long K (the weight
 // gradient of a convolution sums over every patch row) runs as tiles x S
 // work items, item (tile, s) summing k-blocks [s*nk/S, (s+1)*nk/S) into
@@ -34,6 +40,7 @@
 
 #include <climits>
 #include <cstdint>
+#include <cstring>
 #include <mutex>
 
 #include "scan_host.cuh"
@@ -202,15 +209,41 @@ __device__ __forceinline__ bool warp_wait_uniform(uint64_t* bar, uint32_t parity
   }
 }
 
+// TMA tensor store of a 3-D box (x = column, y = row, z = split) from
+// shared memory, as one bulk async-group of the issuing thread.
+__device__ __forceinline__ void tma_store_3d(const CUtensorMap* map, const void* src, int x, int y,
+                                             int z) {
+  asm volatile(
+      "cp.async.bulk.tensor.3d.global.shared::cta.bulk_group [%0, {%2, %3, %4}], [%1];" ::"l"(
+          reinterpret_cast<uint64_t>(map)),
+      "r"(smem_u32(src)), "r"(x), "r"(y), "r"(z)
+      : "memory");
+}
+__device__ __forceinline__ void bulk_commit() { asm volatile("cp.async.bulk.commit_group;" ::: "memory"); }
+// this thread's bulk groups but the newest have finished reading shared memory
+__device__ __forceinline__ void bulk_wait_read_all_but_one() {
+  asm volatile("cp.async.bulk.wait_group.read 1;" ::: "memory");
+}
+__device__ __forceinline__ void bulk_wait_all() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }
+// generic-proxy writes to shared memory are visible to the async proxy (TMA)
+__device__ __forceinline__ void fence_async_smem() {
+  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
+
+constexpr int kOutRows = 32;                     // rows per epilogue warp (its TMEM lanes)
+constexpr int kOutChunkBytes = kOutRows * 128;   // one staged chunk: 32 rows x 128 bytes
+constexpr int kOutStaging = 4 * 2 * kOutChunkBytes;  // 4 warps x 2 buffers
+
 // Two accumulators (one per tile in flight), power-of-two column count.
 template <int BN>
 __host__ __device__ constexpr uint32_t tmem_cols() {
   return 2 * BN <= 32 ? 32u : (2 * BN <= 64 ? 64u : (2 * BN <= 128 ? 128u : (2 * BN <= 256 ? 256u : 512u)));
 }
 
-template <int BN>
+template <int BN, bool TMA_OUT = false>
 __host__ __device__ constexpr size_t smem_bytes() {
-  return 1024 /* alignment slack */ + (size_t)kStages * (BM * BK * 2 + BN * BK * 2) + 256;
+  return 1024 /* alignment slack */ + (size_t)kStages * (BM * BK * 2 + BN * BK * 2) +
+         (TMA_OUT ? kOutStaging : 0) + 256;
 }
 
 // ---------------------------------------------------------------------------
@@ -221,12 +254,14 @@ __host__ __device__ constexpr size_t smem_bytes() {
 // epilogue of one tile overlaps the main loop of the next.
 // ---------------------------------------------------------------------------
 
-template <int BN, bool OUT_BF16, bool A_MN = false, bool B_MN = false>
+template <int BN, bool OUT_BF16, bool A_MN = false, bool B_MN = false, bool TMA_OUT = false>
 __global__ void __launch_bounds__(kThreads, kCtasPerSm)
     gemm_tn_tcgen05(const __grid_constant__ CUtensorMap ta, const __grid_constant__ CUtensorMap tb,
-                    const GemmArgs g) {
+                    const __grid_constant__ CUtensorMap td, const GemmArgs g) {
   static_assert(BN % 16 == 0 && BN >= 16 && BN <= 256, "UMMA N for M=128, two accumulators");
   static_assert(!B_MN || BN % 64 == 0, "an MN-major B tile is whole 64-wide boxes");
+  constexpr int OUT_CW = OUT_BF16 ? 64 : 32;  // columns of one 128-byte output chunk
+  static_assert(!TMA_OUT || BN % OUT_CW == 0, "the tile is whole output chunks");
   constexpr int A_BYTES = BM * BK * 2;
   constexpr int B_BYTES = BN * BK * 2;
   constexpr uint32_t TCOLS = tmem_cols<BN>();
@@ -236,7 +271,8 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm)
       reinterpret_cast<unsigned char*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   unsigned char* sA = smem;
   unsigned char* sB = smem + kStages * A_BYTES;
-  uint64_t* full = reinterpret_cast<uint64_t*>(sB + kStages * B_BYTES);
+  unsigned char* sOut = sB + kStages * B_BYTES;  // output staging (TMA_OUT), 1024-aligned
+  uint64_t* full = reinterpret_cast<uint64_t*>(sOut + (TMA_OUT ? kOutStaging : 0));
   uint64_t* empty = full + kStages;
   uint64_t* acc_full = empty + kStages;  // [2] MMA -> epilogue
   uint64_t* acc_empty = acc_full + 2;    // [2] epilogue -> MMA
@@ -344,6 +380,8 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm)
   } else {
     // epilogue: warp w reads TMEM lanes 32*(w%4) .. +32, i.e. tile rows
     const int q = warp & 3;
+    unsigned char* stage_out = sOut + q * 2 * kOutChunkBytes;
+    int nchunk = 0;  // chunks this warp has staged (buffer parity)
     int i = 0;
     for (int it = blockIdx.x; it < items; it += gridDim.x, ++i) {
       const int t = it / S, sp = it - t * S;
@@ -358,6 +396,46 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm)
       void* const Dout = OUT_BF16 ? (void*)(static_cast<__nv_bfloat16*>(g.D) + sp * g.split_stride)
                                   : (void*)(static_cast<float*>(g.D) + sp * g.split_stride);
       const uint32_t acc = tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(b * BN);
+      if constexpr (TMA_OUT) {
+        // 128-byte column chunks: TMEM -> registers -> swizzled staging ->
+        // TMA store (rows and columns past M and N are clipped by the map)
+#pragma unroll 1
+        for (int c = 0; c < BN && n0 + c < g.N; c += OUT_CW) {
+          unsigned char* buf = stage_out + (nchunk & 1) * kOutChunkBytes;
+          if (lid == 0) bulk_wait_read_all_but_one();  // this buffer's last store has read it
+          __syncwarp();
+          unsigned char* rowp = buf + lid * 128;
+#pragma unroll
+          for (int cc = 0; cc < OUT_CW; cc += 16) {
+            uint32_t r[16];
+            tmem_ld16(acc + (uint32_t)(c + cc), r);
+            if (OUT_BF16) {
+              uint32_t w[8];
+#pragma unroll
+              for (int j = 0; j < 8; ++j) {
+                __nv_bfloat162 h = __floats2bfloat162_rn(__uint_as_float(r[2 * j]), __uint_as_float(r[2 * j + 1]));
+                w[j] = *reinterpret_cast<uint32_t*>(&h);
+              }
+              const int j0 = cc / 8;  // 16-byte chunk index of column cc within the row
+              *reinterpret_cast<uint4*>(rowp + (((j0) ^ (lid & 7)) << 4)) = make_uint4(w[0], w[1], w[2], w[3]);
+              *reinterpret_cast<uint4*>(rowp + (((j0 + 1) ^ (lid & 7)) << 4)) = make_uint4(w[4], w[5], w[6], w[7]);
+            } else {
+              const int j0 = cc / 4;
+#pragma unroll
+              for (int j = 0; j < 4; ++j)
+                *reinterpret_cast<uint4*>(rowp + (((j0 + j) ^ (lid & 7)) << 4)) =
+                    make_uint4(r[4 * j], r[4 * j + 1], r[4 * j + 2], r[4 * j + 3]);
+            }
+          }
+          fence_async_smem();
+          __syncwarp();
+          if (lid == 0) {
+            tma_store_3d(&td, buf, n0 + c, m0 + q * 32, sp);
+            bulk_commit();
+          }
+          ++nchunk;
+        }
+      } else {
 #pragma unroll 1
       for (int c = 0; c < BN; c += 16) {
         uint32_t r[16];
@@ -393,11 +471,13 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm)
           }
         }
       }
+      }
       // this warp's reads of the accumulator are done: hand it back
       tc_fence_before();
       __syncwarp();
       if (lid == 0) mbar_arrive(&acc_empty[b]);
     }
+    if (TMA_OUT && lid == 0) bulk_wait_all();  // the staged chunks are written out
   }
   tc_fence_before();
   __syncthreads();
@@ -441,11 +521,26 @@ bool make_map(CUtensorMap* map, const void* base, int64_t rows, int64_t cols, in
             CU_TENSOR_MAP_L2_PROMOTION_L2_128B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-template <int BN, bool OUT_BF16, bool A_MN, bool B_MN>
-cudaError_t launch_bn(const CUtensorMap& ta, const CUtensorMap& tb, const GemmArgs& g,
-                      cudaStream_t st) {
-  const void* k = (const void*)gemm_tn_tcgen05<BN, OUT_BF16, A_MN, B_MN>;
-  const cudaError_t attr = ensure_smem(k, smem_bytes<BN>());  // once per device
+// Tensor map of the output D [S, M, N] (S split partials, N contiguous;
+// bf16 or fp32) written as 32-row x 128-byte boxes with 128-byte swizzle.
+bool make_out_map(CUtensorMap* map, void* D, int64_t S, int64_t M, int64_t N, bool bf16) {
+  auto fn = encode_fn();
+  if (!fn) return false;
+  const int64_t es = bf16 ? 2 : 4;
+  const cuuint64_t dims[3] = {(cuuint64_t)N, (cuuint64_t)M, (cuuint64_t)S};
+  const cuuint64_t strides[2] = {(cuuint64_t)(N * es), (cuuint64_t)(M * N * es)};
+  const cuuint32_t box[3] = {(cuuint32_t)(128 / es), (cuuint32_t)kOutRows, 1u};
+  const cuuint32_t estr[3] = {1, 1, 1};
+  return fn(map, bf16 ? CU_TENSOR_MAP_DATA_TYPE_BFLOAT16 : CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 3, D,
+            dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+            CU_TENSOR_MAP_L2_PROMOTION_NONE, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+template <int BN, bool OUT_BF16, bool A_MN, bool B_MN, bool TMA_OUT>
+cudaError_t launch_bn(const CUtensorMap& ta, const CUtensorMap& tb, const CUtensorMap& td,
+                      const GemmArgs& g, cudaStream_t st) {
+  const void* k = (const void*)gemm_tn_tcgen05<BN, OUT_BF16, A_MN, B_MN, TMA_OUT>;
+  const cudaError_t attr = ensure_smem(k, smem_bytes<BN, TMA_OUT>());  // once per device
   if (attr != cudaSuccess) return attr;
   int dev = 0, sms = 152;
   if (cudaGetDevice(&dev) == cudaSuccess)
@@ -453,8 +548,25 @@ cudaError_t launch_bn(const CUtensorMap& ta, const CUtensorMap& tb, const GemmAr
   const int64_t items = (int64_t)((g.N + BN - 1) / BN) * ((g.M + BM - 1) / BM) * g.ksplit;
   const int64_t slots = (int64_t)sms * kCtasPerSm;
   const unsigned grid = (unsigned)(items < slots ? items : slots);  // persistent CTAs
-  return launch_pdl(gemm_tn_tcgen05<BN, OUT_BF16, A_MN, B_MN>, dim3(grid), dim3(kThreads),
-                    smem_bytes<BN>(), st, ta, tb, g);
+  return launch_pdl(gemm_tn_tcgen05<BN, OUT_BF16, A_MN, B_MN, TMA_OUT>, dim3(grid),
+                    dim3(kThreads), smem_bytes<BN, TMA_OUT>(), st, ta, tb, td, g);
+}
+
+// The TMA-store epilogue when the output rows are 16-byte multiples and
+// the tile is whole 128-byte chunks; else direct stores.
+template <int BN, bool OUT_BF16, bool A_MN, bool B_MN>
+cudaError_t launch_out(const CUtensorMap& ta, const CUtensorMap& tb, const GemmArgs& g,
+                       cudaStream_t st) {
+  constexpr int cw = OUT_BF16 ? 64 : 32;
+  CUtensorMap td;
+  if constexpr (BN % cw == 0) {
+    const int64_t es = OUT_BF16 ? 2 : 4;
+    if (((int64_t)g.N * es) % 16 == 0 && (reinterpret_cast<uintptr_t>(g.D) & 15u) == 0 &&
+        make_out_map(&td, g.D, g.ksplit, g.M, g.N, OUT_BF16))
+      return launch_bn<BN, OUT_BF16, A_MN, B_MN, true>(ta, tb, td, g, st);
+  }
+  memset(&td, 0, sizeof(td));
+  return launch_bn<BN, OUT_BF16, A_MN, B_MN, false>(ta, tb, td, g, st);
 }
 
 // D[M, N] = A[M, K] * B[N, K]^T.  A is stored [M, K] row-major (K-major) or,
@@ -484,15 +596,15 @@ cudaError_t gemm_tn(const void* A, const void* B, void* D, int M, int N, int K, 
   if (!okA || !okB) return cudaErrorInvalidValue;
   GemmArgs g{M, N, K, D, (int64_t)N, status, kDefaultWaitNs, ksplit, (int64_t)M * N};
   if constexpr (B_MN) {
-    if (bn == 64) return launch_bn<64, OUT_BF16, A_MN, B_MN>(ta, tb, g, st);
-    return launch_bn<128, OUT_BF16, A_MN, B_MN>(ta, tb, g, st);
+    if (bn == 64) return launch_out<64, OUT_BF16, A_MN, B_MN>(ta, tb, g, st);
+    return launch_out<128, OUT_BF16, A_MN, B_MN>(ta, tb, g, st);
   } else {
     switch (bn) {
-      case 256: return launch_bn<256, OUT_BF16, A_MN, B_MN>(ta, tb, g, st);
-      case 16: return launch_bn<16, OUT_BF16, A_MN, B_MN>(ta, tb, g, st);
-      case 32: return launch_bn<32, OUT_BF16, A_MN, B_MN>(ta, tb, g, st);
-      case 64: return launch_bn<64, OUT_BF16, A_MN, B_MN>(ta, tb, g, st);
-      default: return launch_bn<128, OUT_BF16, A_MN, B_MN>(ta, tb, g, st);
+      case 256: return launch_out<256, OUT_BF16, A_MN, B_MN>(ta, tb, g, st);
+      case 16: return launch_out<16, OUT_BF16, A_MN, B_MN>(ta, tb, g, st);
+      case 32: return launch_out<32, OUT_BF16, A_MN, B_MN>(ta, tb, g, st);
+      case 64: return launch_out<64, OUT_BF16, A_MN, B_MN>(ta, tb, g, st);
+      default: return launch_out<128, OUT_BF16, A_MN, B_MN>(ta, tb, g, st);
     }
   }
 }

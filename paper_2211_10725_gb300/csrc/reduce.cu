@@ -122,12 +122,54 @@ __global__ void __launch_bounds__(kRedThreads) reduce_per_channel(ReduceJobs js,
   const double v = block_sum(acc, sh);
   if (threadIdx.x == 0) j.scratch[c * S + s] = v;
   if (!last_of_group(&j.tickets[c], (int)S)) return;
-  if (threadIdx.x == 0) {
+  if (threadIdx.x < 32) {  // lane l adds splits l, l + 32, ... in order, then a fixed tree
     double t = 0.0;
-    for (int64_t q = 0; q < S; ++q) t += j.scratch[c * S + q];
-    j.out[c] = (float)t;
-    j.tickets[c] = 0;
+    for (int64_t q = threadIdx.x; q < S; q += 32) t += j.scratch[c * S + q];
+#pragma unroll
+    for (int d = 16; d > 0; d >>= 1) t += __shfl_xor_sync(0xffffffffu, t, d);
+    if (threadIdx.x == 0) {
+      j.out[c] = (float)t;
+      j.tickets[c] = 0;
+    }
   }
+}
+
+// Per channel with one position per channel run (HW = 1: channel-last
+// lanes, the channel of lane l is l % C) and C dividing the block size:
+// block x sums lanes [x*chunk, (x+1)*chunk), chunk a multiple of the block
+// size, so thread t only meets channel t % C and its loads are coalesced.
+// The threads of a channel are added in thread order; the last block adds
+// the block partials of each channel with one warp (strided lane sums, then
+// a fixed shuffle tree).
+__global__ void __launch_bounds__(kRedThreads) reduce_channel_last(ReduceJobs js, int64_t L,
+                                                                    int64_t chunk, int C) {
+  __shared__ double sh[kRedThreads];
+  grid_dep_wait();
+  const ReduceJob& j = js.job[blockIdx.z];
+  const int64_t lo = (int64_t)blockIdx.x * chunk;
+  const int64_t hi = min(L, lo + chunk);
+  double acc = 0.0;
+#pragma unroll 4
+  for (int64_t l = lo + threadIdx.x; l < hi; l += kRedThreads) acc += (double)j.part[l];
+  sh[threadIdx.x] = acc;
+  __syncthreads();
+  if ((int)threadIdx.x < C) {
+    double t = 0.0;
+    for (int q = threadIdx.x; q < kRedThreads; q += C) t += sh[q];
+    j.scratch[(int64_t)blockIdx.x * C + threadIdx.x] = t;
+  }
+  if (!last_of_group(&j.tickets[0], (int)gridDim.x)) return;
+  // warp w adds channels w, w + 8, ...: lane l the partials l, l + 32, ...
+  // in order, then a fixed shuffle tree
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  for (int c = warp; c < C; c += kRedThreads / 32) {
+    double t = 0.0;
+    for (int q = lane; q < (int)gridDim.x; q += 32) t += j.scratch[(int64_t)q * C + c];
+#pragma unroll
+    for (int d = 16; d > 0; d >>= 1) t += __shfl_xor_sync(0xffffffffu, t, d);
+    if (lane == 0) j.out[c] = (float)t;
+  }
+  if (threadIdx.x == 0) j.tickets[0] = 0;
 }
 
 }  // namespace
@@ -161,6 +203,16 @@ cudaError_t launch_param_reduce(const ParamReduce* p, int n, int64_t B, int64_t 
                      dim3(kRedThreads), 0, stream, js, B, N);
       if (e != cudaSuccess) return e;
     }
+  } else if (C > 0 && HW == 1 && kRedThreads % C == 0) {
+    int64_t nb = ceil_div(L, 4096);
+    if (nb > scratch_len / C) nb = scratch_len / C;
+    if (nb > 65535) nb = 65535;
+    if (nb < 1) return cudaErrorInvalidValue;  // the workspace is sized for one block
+    const int64_t chunk = ceil_div(ceil_div(L > 0 ? L : 1, nb), kRedThreads) * kRedThreads;
+    nb = ceil_div(L > 0 ? L : 1, chunk);
+    const cudaError_t e = launch_pdl(reduce_channel_last, dim3((unsigned)nb, 1, (unsigned)n),
+                                     dim3(kRedThreads), 0, stream, js, L, chunk, (int)C);
+    if (e != cudaSuccess) return e;
   } else if (C > 0) {
     const int64_t R = N / (C * HW);
     // about four blocks per SM in total, at least ~1k elements per block

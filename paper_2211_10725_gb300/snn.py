@@ -77,6 +77,10 @@ _SIGS = {
     "snn_dense_layer_bwd": ([ctypes.c_int64] * 3 + [_P] * 6 + [ctypes.c_size_t, _P], ctypes.c_int),
     "snn_rate_ce_workspace_bytes": ([ctypes.c_int64], ctypes.c_size_t),
     "snn_kernel_launches": ([], ctypes.c_uint64),
+    "snn_conv2d_small_fwd_nhwc": ([ctypes.c_int64] * 8 + [_P] * 4, ctypes.c_int),
+    "snn_conv2d_small_dw_workspace_bytes": ([ctypes.c_int64] * 7, ctypes.c_size_t),
+    "snn_conv2d_small_dw_nhwc": ([ctypes.c_int64] * 8 + [_P] * 4 + [ctypes.c_size_t, _P],
+                                 ctypes.c_int),
     "snn_im2col_nhwc": ([ctypes.c_int64] * 7 + [_P] * 3, ctypes.c_int),
     "snn_col2im_nhwc": ([ctypes.c_int64] * 7 + [_P] * 3, ctypes.c_int),
     "snn_maxpool2_fwd_nhwc": ([ctypes.c_int64] * 4 + [_P] * 4, ctypes.c_int),
@@ -302,6 +306,30 @@ def snn_adamw_step(w, w_bf16, grad, m, v, lr, beta1=0.9, beta2=0.999, eps=1e-8,
 def snn_kernel_launches() -> int:
     """Kernels the library has launched (or captured) in this process."""
     return int(load_library().snn_kernel_launches())
+
+
+def snn_conv2d_small_fwd_nhwc(X, Wt, I, KH, KW, stream=None):
+    """I [M, Ho, Wo, Cout] fp32 = X [M, H, W, Cin] (*) filters Wt [Cout, ldw]
+    on the CUDA cores (few input channels)."""
+    M, H, W_, Cin = X.shape
+    Cout, ldw = Wt.shape
+    _check(load_library().snn_conv2d_small_fwd_nhwc(M, H, W_, Cin, Cout, KH, KW, ldw, _ptr(X),
+                                                    _ptr(Wt), _ptr(I), _stream(stream)),
+           "snn_conv2d_small_fwd_nhwc")
+
+
+def snn_conv2d_small_dw_workspace_bytes(M, H, W_, Cin, Cout, KH, KW) -> int:
+    return load_library().snn_conv2d_small_dw_workspace_bytes(M, H, W_, Cin, Cout, KH, KW)
+
+
+def snn_conv2d_small_dw_nhwc(X, dI, dW, KH, KW, ws, stream=None):
+    """dW [Cout, ldw] fp32 of snn_conv2d_small_fwd_nhwc from dI [M, Ho, Wo, Cout] bf16."""
+    M, H, W_, Cin = X.shape
+    Cout, ldw = dW.shape
+    _check(load_library().snn_conv2d_small_dw_nhwc(M, H, W_, Cin, Cout, KH, KW, ldw, _ptr(X),
+                                                   _ptr(dI), _ptr(dW), _ptr(ws),
+                                                   ws.numel() * ws.element_size(),
+                                                   _stream(stream)), "snn_conv2d_small_dw_nhwc")
 
 
 def snn_im2col_nhwc(X, cols, KH, KW, stream=None):

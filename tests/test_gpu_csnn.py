@@ -171,6 +171,60 @@ def test_layout_argument_checks(cuda_device):
 
 
 # ---------------------------------------------------------------------------
+# Direct convolution with few input channels
+# ---------------------------------------------------------------------------
+
+@pytest.mark.parametrize("M,Hh,Ww,C,Cout,k,ldw", [(5, 28, 28, 1, 16, 5, 32), (3, 9, 11, 2, 8, 3, 24),
+                                                  (2, 7, 7, 1, 4, 1, 8), (700, 28, 28, 1, 16, 5, 32),
+                                                  (4, 10, 13, 1, 8, 3, 16), (3, 70, 9, 1, 16, 5, 32)])
+def test_small_conv_matches_oracle(M, Hh, Ww, C, Cout, k, ldw, cuda_device):
+    """Forward currents and the weight gradient of the direct convolution
+    against the oracle's convolution and its backward; the weight gradient
+    is the same bits on every call (more images than blocks in the last
+    case, so blocks sum several images)."""
+    g = torch.Generator().manual_seed(M + 31 * Cout + k)
+    X = (torch.rand((M, Hh, Ww, C), generator=g) < 0.3).to(torch.bfloat16)
+    Wc = torch.randn((Cout, k, k, C), generator=g).to(torch.bfloat16)
+    K = k * k * C
+    Wt = torch.zeros((Cout, ldw), dtype=torch.bfloat16)
+    Wt[:, :K] = Wc.reshape(Cout, K)
+    Wt[:, K:] = 3.0   # columns past K must not be read
+    Ho, Wo = Hh - k + 1, Ww - k + 1
+    I = torch.empty((M, Ho, Wo, Cout), dtype=torch.float32, device=cuda_device)
+    Xd = X.to(cuda_device)
+    snn.snn_conv2d_small_fwd_nhwc(Xd, Wt.to(cuda_device), I, k, k)
+    dI = torch.randn((M, Ho, Wo, Cout), generator=g).to(torch.bfloat16)
+    dW = torch.full((Cout, ldw), 9.0, dtype=torch.float32, device=cuda_device)
+    ws = torch.empty(snn.snn_conv2d_small_dw_workspace_bytes(M, Hh, Ww, C, Cout, k, k),
+                     dtype=torch.uint8, device=cuda_device)
+    snn.snn_conv2d_small_dw_nhwc(Xd, dI.to(cuda_device), dW, k, k, ws)
+    first = dW.clone()
+    snn.snn_conv2d_small_dw_nhwc(Xd, dI.to(cuda_device), dW, k, k, ws)
+    torch.cuda.synchronize()
+    assert torch.equal(first, dW)
+    x, wc, di = _np(X), _np(Wc), _np(dI)
+    ref = O.conv2d_nhwc(x, wc)
+    H.assert_close("I", _np(I), ref, 1e-5, 1e-6, O.conv2d_nhwc(x, np.abs(wc)))
+    _, ref_dW = O.conv2d_nhwc_backward(x, wc, di)
+    _, mag = O.conv2d_nhwc_backward(x, wc, np.abs(di))
+    got = _np(dW)
+    H.assert_close("dW", got[:, :K].reshape(Cout, k, k, C), ref_dW, 1e-5, 1e-6, mag)
+    assert not got[:, K:].any()
+
+
+def test_small_conv_argument_checks(cuda_device):
+    lib = snn.load_library()
+    buf = torch.zeros(1 << 16, dtype=torch.float32, device=cuda_device)
+    p = buf.data_ptr()
+    assert lib.snn_conv2d_small_fwd_nhwc(0, 28, 28, 1, 16, 5, 5, 32, None, None, None, None) == 0
+    assert lib.snn_conv2d_small_fwd_nhwc(1, 28, 28, 2, 16, 5, 5, 64, p, p, p, None) == 3  # K > 32
+    assert lib.snn_conv2d_small_fwd_nhwc(1, 28, 28, 1, 20, 5, 5, 32, p, p, p, None) == 3  # Cout
+    assert lib.snn_conv2d_small_fwd_nhwc(1, 28, 28, 1, 16, 5, 5, 24, p, p, p, None) == 1  # ldw < K
+    assert lib.snn_conv2d_small_fwd_nhwc(1, 28, 28, 1, 16, 5, 5, 32, p, p, p + 4, None) == 2
+    assert lib.snn_conv2d_small_dw_nhwc(4, 28, 28, 1, 16, 5, 5, 32, p, p, p, p, 16, None) == 4
+
+
+# ---------------------------------------------------------------------------
 # Split-K weight gradient
 # ---------------------------------------------------------------------------
 
@@ -327,12 +381,16 @@ def _check_step(w, net, convs, Wfc, betas, fwd, res):
     return mag
 
 
-def test_csnn_step_small_matches_oracle(cuda_device):
+@pytest.mark.parametrize("direct_first", [True, False])
+def test_csnn_step_small_matches_oracle(direct_first, cuda_device):
+    """The step at T = 4, B = 8, with the first layer as a direct
+    convolution or as im2col + tensor-core GEMM."""
     w = SMALL
     inp = _exact_inputs(w)
     convs, Wfc, betas, fwd, res = _oracle(w, inp)
     assert all(s.mean() > 0 for s in fwd["spk"]) and fwd["fc_spk"].mean() > 0
-    net, X, labels = _run(w, inp, cuda_device)
+    net, X, labels = _run(w, inp, cuda_device, direct_first=direct_first)
+    assert net.direct[0] == direct_first
     net.step(X, labels)
     torch.cuda.synchronize()
     for layer in net.layers + [net.out_layer]:

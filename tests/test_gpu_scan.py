@@ -159,6 +159,27 @@ def test_wait_timeout_reports_status_and_context_survives(cuda_device):
     H.check_all(w, inp, ok, H.oracle_expect(w, inp))
 
 
+@pytest.mark.parametrize("T,B,N,C", [(5, 3, 9216, 16), (4, 7, 4096, 64), (3, 5, 48, 16),
+                                     (6, 2, 8, 2), (2, 1, 256, 256), (25, 128, 9216, 16)])
+@pytest.mark.parametrize("neuron", ["leaky", "synaptic"])
+def test_channel_last_parameter_gradients(T, B, N, C, neuron, cuda_device):
+    """Per-channel parameters on channel-last lanes (one position per
+    channel run, the channel of lane l is l % C, as in a convolutional
+    layer's [H, W, C] map): the coalesced reduction path, up to the CSNN's
+    first-layer shape."""
+    w = W.ScanWorkload(name=f"chlast_{neuron}_{T}_{B}_{N}_{C}", neuron=neuron, T=T, B=B, N=N, C=C,
+                       HW=1, i_mean=0.5, i_std=0.6, beta=("uniform", 0.5, 0.95),
+                       thr=("uniform", 0.6, 1.4), alpha=("uniform", 0.3, 0.9),
+                       beta_mode="per_channel", thr_mode="per_channel", alpha_mode="per_channel",
+                       reset="zero", save="recompute", want_mem=True, seed_index=400 + C + T)
+    inp = W.make_scan_inputs(w)
+    layer = H.run_gpu(w, inp)
+    assert layer.status() == 0
+    H.check_all(w, inp, layer, H.oracle_expect(w, inp))
+    again = H.run_gpu(w, inp)
+    assert torch.equal(layer.grad_beta, again.grad_beta)   # fixed summation order
+
+
 # ---------------------------------------------------------------------------
 # Full-size workloads
 # ---------------------------------------------------------------------------
