@@ -338,6 +338,29 @@ snn_status_t snn_rate_ce_loss(int64_t T, int64_t B, int64_t C, int64_t pop, int6
                               size_t ws_bytes, snn_stream_t stream);
 
 /*
+ * Dense layer fused with its Leaky scan (Fig. 3's synaptic operation w.x
+ * feeding Eqs. 3-4): the currents of all T steps come out of one tcgen05
+ * GEMM and are scanned in its epilogue, so they never reach HBM.
+ *   desc     the Leaky layer: T <= 128, B, N = P*Nout neurons per sample
+ *            (channel-last: neuron p*Nout + n is output column n at row p),
+ *            io_dtype SNN_BF16, save SNN_SAVE_MEM (the BPTT reads the stored
+ *            trace: snn_leaky_bwd in store mode), any reset; beta_mode and
+ *            thr_mode scalar, per neuron (P = 1) or per channel with
+ *            C = Nout, HW = 1.  Nout and K multiples of 8.
+ *   X        bf16 [T, B*P, K]: row (t, r) of the layer input (r = b*P + p)
+ *   W        bf16 [Nout, K]
+ *   spk, mem bf16 [T, B, N] (out): z_t and u_t, as snn_leaky_fwd writes them
+ *   ckpt     the spike bits of store mode (see snn_scan_ckpt_elems), or NULL
+ *   ws       at least 256 bytes (status word)
+ * Initial state zero (no mem0); mem_final is not produced.  Returns
+ * SNN_ERR_UNSUPPORTED for other modes or shapes.
+ */
+snn_status_t snn_dense_leaky_fwd(const snn_scan_desc* desc, int64_t P, int64_t K, const void* X,
+                                 const void* W, const float* beta, const float* thr, void* spk,
+                                 void* mem, float* ckpt, void* ws, size_t ws_bytes,
+                                 snn_stream_t stream);
+
+/*
  * Convolutional SNN layout kernels (Tab. I CSNN: 5x5 convolutions, 2x2 max
  * pooling) on channel-last bf16 activations [M, H, W, C], M = T*B.  A
  * convolution is a snn_dense_layer_fwd/bwd over the patch rows:

@@ -22,7 +22,7 @@ LIB_PATH = os.path.join(OUT_DIR, "libsnn.so")
 
 SOURCES = ["snn_api.cu", "scan_fwd.cu", "scan_bwd_leaky.cu", "scan_bwd_leaky_recompute.cu",
            "scan_bwd_synaptic.cu", "scan_bwd_synaptic_recompute.cu", "reduce.cu", "snn_noalloc.cu",
-           "gemm_tcgen05.cu", "ce_loss.cu", "adamw.cu", "conv_pool.cu", "conv_small.cu"]
+           "gemm_tcgen05.cu", "gemm_scan.cu", "ce_loss.cu", "adamw.cu", "conv_pool.cu", "conv_small.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 NVCC_FLAGS = ARCH + ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC",
                      "-Xcompiler", "-fvisibility=hidden", "--expt-relaxed-constexpr",

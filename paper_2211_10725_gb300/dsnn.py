@@ -14,7 +14,9 @@ never fires, and its gradients are exactly 0.
 
 The backward recomputes each layer's membrane trace from its input current
 and checkpoints (``save="recompute"``) unless ``save="mem"`` asks for the
-bf16 trace to be stored by the forward.
+bf16 trace to be stored by the forward.  ``save="fused"`` stores the trace
+too, but runs each layer's forward as one kernel: the GEMM with the Leaky
+scan in its epilogue (the currents never reach HBM).
 """
 from __future__ import annotations
 
@@ -37,6 +39,8 @@ class DenseSNN:
                  weight_decay: float = 1e-2):
         self.w = w
         self.save = save
+        self.fused = save == "fused"
+        scan_save = "mem" if self.fused else save
         self.lr, self.betas, self.eps, self.weight_decay = lr, betas, eps, weight_decay
         # batch the loss is averaged over (the global batch under data
         # parallelism; None: this replica's batch)
@@ -73,9 +77,11 @@ class DenseSNN:
             lw = W.ScanWorkload(name=f"dsnn_layer{l}", neuron="leaky", T=T, B=B, N=n,
                                 in_dtype=W.F32, io_dtype=W.BF16, beta=("const", w.beta),
                                 thr=("const", w.thr), surrogate="fast_sigmoid",
-                                sg_param=w.sg_param, save=save, want_mem=save == "mem")
+                                sg_param=w.sg_param, save=scan_save,
+                                want_mem=scan_save == "mem")
             self.layers.append(snn.ScanLayer(lw, device=dev))
-            self.I.append(torch.empty((self.M, n), dtype=torch.float32, device=dev))
+            self.I.append(None if self.fused else
+                          torch.empty((self.M, n), dtype=torch.float32, device=dev))
         self.beta = torch.full((1,), w.beta, dtype=torch.float32, device=dev)
         self.thr = torch.full((1,), w.thr, dtype=torch.float32, device=dev)
         self.ws_fwd = torch.zeros(256, dtype=torch.uint8, device=dev)
@@ -95,15 +101,18 @@ class DenseSNN:
         of layer l - 1."""
         return X if l == 0 else self.layers[l - 1].spk.view(self.M, self.padded[l])
 
+    def _n_fwd(self):
+        return (1 if self.fused else 2) * len(self.layers) + 1
+
     def forward(self, X, labels, stream=None):
         """X: bf16 [T*B, 784] spikes on the device; labels int32 [B]."""
-        for _, call in self.ops(X, labels, stream)[: 2 * len(self.layers) + 1]:
+        for _, call in self.ops(X, labels, stream)[: self._n_fwd()]:
             call()
         return self.loss
 
     def backward(self, X, stream=None):
         """BPTT from the loss gradient of the last forward; returns dW."""
-        for _, call in self.ops(X, None, stream)[2 * len(self.layers) + 1: -1]:
+        for _, call in self.ops(X, None, stream)[self._n_fwd(): -1]:
             call()
         return self.dW
 
@@ -121,6 +130,11 @@ class DenseSNN:
         T, B = self.w.T, self.w.B
         out = []
         for l, layer in enumerate(self.layers):
+            if self.fused:
+                out.append((f"dense_scan_fwd{l}", lambda l=l, layer=layer: snn.snn_dense_leaky_fwd(
+                    layer.desc, self.layer_input(l, X), self.W[l], self.beta, self.thr,
+                    layer.spk, layer.mem, layer.ckpt, self.ws_fwd, stream=stream)))
+                continue
             out.append((f"dense_fwd{l}", lambda l=l: snn.snn_dense_layer_fwd(
                 self.layer_input(l, X), self.W[l], self.I[l], self.ws_fwd, stream)))
             out.append((f"scan_fwd{l}", lambda l=l, layer=layer: layer.forward(
@@ -133,8 +147,8 @@ class DenseSNN:
                 self.grad_in[l].view(T, B, -1)
             dX = self.grad_in[l - 1] if l > 0 else None
             out.append((f"scan_bwd{l}", lambda l=l, grad=grad: self.layers[l].backward(
-                self.I[l].view(T, B, -1), self.beta, self.thr, grad, want_param_grads=False,
-                want_state_grads=False, stream=stream)))
+                None if self.I[l] is None else self.I[l].view(T, B, -1), self.beta, self.thr,
+                grad, want_param_grads=False, want_state_grads=False, stream=stream)))
             out.append((f"dense_bwd{l}", lambda l=l, dX=dX: snn.snn_dense_layer_bwd(
                 self.layer_input(l, X), self.W[l], self.layers[l].grad_I.view(self.M, -1), dX,
                 self.dW[l], self.ws_bwd[l], stream)))

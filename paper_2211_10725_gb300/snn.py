@@ -77,6 +77,8 @@ _SIGS = {
     "snn_dense_layer_bwd": ([ctypes.c_int64] * 3 + [_P] * 6 + [ctypes.c_size_t, _P], ctypes.c_int),
     "snn_rate_ce_workspace_bytes": ([ctypes.c_int64], ctypes.c_size_t),
     "snn_kernel_launches": ([], ctypes.c_uint64),
+    "snn_dense_leaky_fwd": ([ctypes.POINTER(ScanDesc), ctypes.c_int64, ctypes.c_int64] + [_P] * 8
+                            + [ctypes.c_size_t, _P], ctypes.c_int),
     "snn_conv2d_small_fwd_nhwc": ([ctypes.c_int64] * 8 + [_P] * 4, ctypes.c_int),
     "snn_conv2d_small_dw_workspace_bytes": ([ctypes.c_int64] * 7, ctypes.c_size_t),
     "snn_conv2d_small_dw_nhwc": ([ctypes.c_int64] * 8 + [_P] * 4 + [ctypes.c_size_t, _P],
@@ -301,6 +303,16 @@ def snn_adamw_step(w, w_bf16, grad, m, v, lr, beta1=0.9, beta2=0.999, eps=1e-8,
     _check(load_library().snn_adamw_step(n, _ptr(w), _ptr(w_bf16), _ptr(grad), _ptr(m), _ptr(v),
                                          lr, beta1, beta2, eps, weight_decay, step,
                                          _ptr(step_counter), _stream(stream)), "snn_adamw_step")
+
+
+def snn_dense_leaky_fwd(desc, X, W, beta, thr, spk, mem, ckpt, ws, P=1, stream=None):
+    """GEMM of X [T*B*P, K] with W [Nout, K] and the Leaky scan of its
+    currents in one kernel; writes spk, mem (and the spike bits to ckpt)."""
+    K = X.shape[-1]
+    _check(load_library().snn_dense_leaky_fwd(ctypes.byref(desc), P, K, _ptr(X), _ptr(W),
+                                              _ptr(beta), _ptr(thr), _ptr(spk), _ptr(mem),
+                                              _ptr(ckpt), _ptr(ws), ws.numel() * ws.element_size(),
+                                              _stream(stream)), "snn_dense_leaky_fwd")
 
 
 def snn_kernel_launches() -> int:
