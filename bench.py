@@ -42,8 +42,8 @@ def parse():
     p.add_argument("--workload", default=DEFAULT_WORKLOAD)
     # scan workloads: store (mem + spk saved, the default) is the faster
     # variant on GB300; recompute moves fewer bytes but its reverse pass is
-    # instruction-bound.  Dense networks: "fused" (the default) runs each
-    # layer's GEMM with its scan in the epilogue and stores the trace.
+    # instruction-bound.  Networks: "fused" (the default) runs each GEMM
+    # layer with its scan in the epilogue and stores every trace.
     p.add_argument("--save", default=None, choices=["mem", "recompute", "fused"])
     p.add_argument("--no-graph", action="store_true",
                    help="dense-SNN workload: launch the step eagerly, not as a CUDA graph")
@@ -591,8 +591,13 @@ def conv_op_bytes(net):
             out[f"conv_fwd{l}"] = x_bytes + nb(net.W[l]) + nb(net.I[l])
         else:
             out[f"im2col{l}"] = x_bytes + nb(net.cols[l])
-            out[f"conv_fwd{l}"] = nb(net.cols[l]) + nb(net.W[l]) + nb(net.I[l])
-        out[f"scan_fwd{l}"] = f * ns
+            if net.I[l] is None:  # GEMM with the scan in its epilogue
+                out[f"conv_scan_fwd{l}"] = (nb(net.cols[l]) + nb(net.W[l]) + nb(layer.spk)
+                                            + nb(layer.mem) + nb(layer.ckpt))
+            else:
+                out[f"conv_fwd{l}"] = nb(net.cols[l]) + nb(net.W[l]) + nb(net.I[l])
+        if net.I[l] is not None:
+            out[f"scan_fwd{l}"] = f * ns
         out[f"pool_fwd{l}"] = nb(layer.spk) + nb(net.pool[l]) + nb(net.idx[l])
         out[f"pool_bwd{l}"] = nb(net.grad_pool[l]) + nb(net.idx[l]) + nb(net.grad_spk[l])
         out[f"scan_bwd{l}"] = b * ns
@@ -605,8 +610,11 @@ def conv_op_bytes(net):
     f, b = algorithmic_bytes(o.w)
     ns = T * B * o.w.N
     flat = nb(net.pool[-1])
-    out["fc_fwd"] = flat + nb(net.W[-1]) + nb(net.I_fc)
-    out["scan_fwd_out"] = f * ns
+    if net.I_fc is None:
+        out["fc_scan_fwd"] = flat + nb(net.W[-1]) + nb(o.spk) + nb(o.mem) + nb(o.ckpt)
+    else:
+        out["fc_fwd"] = flat + nb(net.W[-1]) + nb(net.I_fc)
+        out["scan_fwd_out"] = f * ns
     out["ce_loss"] = nb(o.spk) + nb(net.grad_out)
     out["scan_bwd_out"] = b * ns
     out["fc_bwd"] = flat + nb(net.W[-1]) + nb(o.grad_I) + nb(net.grad_pool[-1]) + nb(net.dW[-1])
@@ -638,10 +646,9 @@ def run_net(args):
     torch.cuda.set_device(local)
     dev = torch.device("cuda", local)
     w = net_workload(args.workload)
-    # the fastest parity-tested variant: the dense networks' forward fused
-    # with their scans (store mode), the CSNN's BPTT recomputing from its
-    # currents
-    save = args.save or ("recompute" if is_conv(w) else "fused")
+    # the fastest parity-tested variant: every GEMM layer's forward fused
+    # with its scan, every scan storing its bf16 trace for the BPTT
+    save = args.save or "fused"
     from paper_2211_10725_gb300 import workloads as W
     inp = net_inputs(w, seed=W.SEED_BASE + w.seed_index + 1000 * rank)
     if is_conv(w):

@@ -26,6 +26,12 @@ staged in shared memory, and so does its weight gradient; a patch-row GEMM
 would write and read 32 padded columns per output pixel for that
 (``direct_first=False`` keeps the im2col + GEMM path, whose 25 columns are
 padded to 32).
+
+``save="fused"`` stores every scan's bf16 membrane trace (the BPTT reads
+it instead of recomputing from the currents) and runs the GEMM layers (the
+second convolution over its patch rows, the readout) as one kernel each:
+the GEMM with the Leaky scan in its epilogue, so their currents never
+reach HBM.
 """
 from __future__ import annotations
 
@@ -49,6 +55,8 @@ class ConvSNN:
                  direct_first: bool = True):
         self.w = w
         self.save = save
+        self.fused = save == "fused"
+        scan_save = "mem" if self.fused else save
         self.lr, self.betas, self.eps, self.weight_decay = lr, betas, eps, weight_decay
         self.learn_beta = learn_beta
         self.batch_total = None
@@ -127,12 +135,15 @@ class ConvSNN:
         for l, (h, wd, cin, cout, k, ho, wo, hp, wp, kpad) in enumerate(self.geo):
             rows = M * ho * wo
             self.cols.append(None if self.direct[l] else torch.empty((rows, kpad), **bf))
-            self.I.append(torch.empty((rows, cout), dtype=torch.float32, device=dev))
+            fuse = self.fused and not self.direct[l]  # GEMM and scan in one kernel
+            self.I.append(None if fuse else
+                          torch.empty((rows, cout), dtype=torch.float32, device=dev))
             lw = W.ScanWorkload(name=f"csnn_conv{l}", neuron="leaky", T=T, B=B,
                                 N=ho * wo * cout, C=cout, HW=1, in_dtype=W.F32, io_dtype=W.BF16,
                                 beta=("const", w.beta), beta_mode="per_channel",
                                 thr=("const", w.thr), reset=w.reset, surrogate="fast_sigmoid",
-                                sg_param=w.sg_param, save=save, want_mem=save == "mem")
+                                sg_param=w.sg_param, save=scan_save,
+                                want_mem=scan_save == "mem")
             self.layers.append(snn.ScanLayer(lw, device=dev))
             self.pool.append(torch.empty((M, hp, wp, cout), **bf))
             self.idx.append(torch.empty((M, hp, wp, cout), dtype=torch.uint8, device=dev))
@@ -144,11 +155,12 @@ class ConvSNN:
             else:
                 nb = snn.snn_dense_workspace_bytes(rows, kpad, cout)
             self.ws_bwd.append(torch.zeros(max(nb, 256), dtype=torch.uint8, device=dev))
-        self.I_fc = torch.empty((M, self.n_out), dtype=torch.float32, device=dev)
+        self.I_fc = None if self.fused else \
+            torch.empty((M, self.n_out), dtype=torch.float32, device=dev)
         fw = W.ScanWorkload(name="csnn_out", neuron="leaky", T=T, B=B, N=self.n_out,
                             in_dtype=W.F32, io_dtype=W.BF16, beta=("const", w.beta_fc),
                             thr=("const", w.thr), reset=w.reset, surrogate="fast_sigmoid",
-                            sg_param=w.sg_param, save=save, want_mem=save == "mem")
+                            sg_param=w.sg_param, save=scan_save, want_mem=scan_save == "mem")
         self.out_layer = snn.ScanLayer(fw, device=dev)
         self.ws_fwd = torch.zeros(256, dtype=torch.uint8, device=dev)
         self.ws_bwd.append(torch.zeros(snn.snn_dense_workspace_bytes(M, self.n_flat, self.n_out),
@@ -179,25 +191,39 @@ class ConvSNN:
             else:
                 out.append((f"im2col{l}", lambda l=l, k=k: snn.snn_im2col_nhwc(
                     self.layer_input(l, X), self.cols[l], k, k, stream)))
-                out.append((f"conv_fwd{l}", lambda l=l: snn.snn_dense_layer_fwd(
-                    self.cols[l], self.W[l], self.I[l], self.ws_fwd, stream)))
-            out.append((f"scan_fwd{l}", lambda l=l, layer=layer: layer.forward(
-                self.I[l].view(T, B, -1), self.beta[l], self.thr, stream=stream)))
+                if self.I[l] is None:  # fused: the GEMM's epilogue runs the scan
+                    out.append((f"conv_scan_fwd{l}", lambda l=l, layer=layer, p=ho * wo:
+                                snn.snn_dense_leaky_fwd(layer.desc, self.cols[l], self.W[l],
+                                                        self.beta[l], self.thr, layer.spk,
+                                                        layer.mem, layer.ckpt, self.ws_fwd, P=p,
+                                                        stream=stream)))
+                else:
+                    out.append((f"conv_fwd{l}", lambda l=l: snn.snn_dense_layer_fwd(
+                        self.cols[l], self.W[l], self.I[l], self.ws_fwd, stream)))
+            if self.I[l] is not None:
+                out.append((f"scan_fwd{l}", lambda l=l, layer=layer: layer.forward(
+                    self.I[l].view(T, B, -1), self.beta[l], self.thr, stream=stream)))
             out.append((f"pool_fwd{l}", lambda l=l, layer=layer, s=(M, ho, wo, cout):
                         snn.snn_maxpool2_fwd_nhwc(layer.spk.view(s), self.pool[l], self.idx[l],
                                                   stream)))
         L = len(self.geo)
         flat = self.pool[-1].view(M, -1)
-        out.append(("fc_fwd", lambda: snn.snn_dense_layer_fwd(flat, self.W[L], self.I_fc,
-                                                               self.ws_fwd, stream)))
-        out.append(("scan_fwd_out", lambda: self.out_layer.forward(
-            self.I_fc.view(T, B, -1), self.beta_fc, self.thr, stream=stream)))
+        if self.fused:
+            o = self.out_layer
+            out.append(("fc_scan_fwd", lambda: snn.snn_dense_leaky_fwd(
+                o.desc, flat, self.W[L], self.beta_fc, self.thr, o.spk, o.mem, o.ckpt,
+                self.ws_fwd, stream=stream)))
+        else:
+            out.append(("fc_fwd", lambda: snn.snn_dense_layer_fwd(flat, self.W[L], self.I_fc,
+                                                                   self.ws_fwd, stream)))
+            out.append(("scan_fwd_out", lambda: self.out_layer.forward(
+                self.I_fc.view(T, B, -1), self.beta_fc, self.thr, stream=stream)))
         out.append(("ce_loss", lambda: snn.snn_rate_ce_loss(
             self.out_layer.spk, labels, self.w.n_classes, self.loss, self.grad_out,
             self.ws_loss, stream, batch_total=self.batch_total)))
         out.append(("scan_bwd_out", lambda: self.out_layer.backward(
-            self.I_fc.view(T, B, -1), self.beta_fc, self.thr, self.grad_out,
-            want_param_grads=False, want_state_grads=False, stream=stream)))
+            None if self.I_fc is None else self.I_fc.view(T, B, -1), self.beta_fc, self.thr,
+            self.grad_out, want_param_grads=False, want_state_grads=False, stream=stream)))
         out.append(("fc_bwd", lambda: snn.snn_dense_layer_bwd(
             flat, self.W[L], self.out_layer.grad_I.view(M, -1),
             self.grad_pool[-1].view(M, -1), self.dW[L], self.ws_bwd[L], stream)))
@@ -227,7 +253,7 @@ class ConvSNN:
         T, B = self.w.T, self.w.B
         layer = self.layers[l]
         recompute = layer.w.save == "recompute"
-        I = self.I[l].view(T, B, -1)
+        I = self.I[l].view(T, B, -1) if recompute else None
         snn.snn_leaky_bwd(layer.desc, I if recompute else None, layer.ckpt, layer.mem, layer.spk,
                           self.beta[l], self.thr, None, self.grad_spk[l].view(T, B, -1), None,
                           None, layer.grad_I, self.dbeta[l], None, None, layer.ws, stream)
@@ -244,7 +270,8 @@ class ConvSNN:
                                step_counter=self.beta_counter, stream=stream)
 
     def _n_fwd(self):
-        return 3 * len(self.geo) + sum(not d for d in self.direct) + 3
+        names = [n for n, _ in self.ops(None, None)]
+        return names.index("ce_loss") + 1
 
     def forward(self, X, labels, stream=None):
         """X: bf16 [T*B, H, W, Cin] spikes on the device; labels int32 [B]."""

@@ -30,7 +30,7 @@ namespace snn {
 namespace gemm {
 namespace {
 
-constexpr int kFusedStages = 4;
+constexpr int kFusedStages = 3;  // with BN <= 64, two CTAs fit on an SM
 constexpr int kScanWarps = 10;  // warps 2..11 scan; 2..5 also drain the accumulator
 constexpr int kScanThreads = 32 * kScanWarps;
 constexpr int kFusedThreads = 64 + kScanThreads;
@@ -65,7 +65,7 @@ __device__ __forceinline__ void epi_barrier() {
 }
 
 template <int BN, int RESET>
-__global__ void __launch_bounds__(kFusedThreads, 1)
+__global__ void __launch_bounds__(kFusedThreads, 2)
     gemm_leaky_tcgen05(const __grid_constant__ CUtensorMap ta, const __grid_constant__ CUtensorMap tb,
                        const FusedArgs f) {
   static_assert(BN % 16 == 0 && BN >= 16 && BN <= 128, "UMMA N for M=128");
@@ -200,45 +200,56 @@ __global__ void __launch_bounds__(kFusedThreads, 1)
         if (e == 0) record_status(f.status, kStatusTimeout);
         break;
       }
-      // the scan: thread e steps lanes j = e + 128*(g*kScanLanes + v)
+      // the scan: thread e steps lanes j = g0 + kScanThreads*v + e together
+      // (independent chains); groups wholly past the tile are skipped
+      const int64_t RN = (int64_t)f.R * f.N;  // elements per step of spk / mem
       for (int g0 = 0; g0 < lanes; g0 += kScanThreads * kScanLanes) {
+        const int nv = (lanes - g0 + kScanThreads - 1) / kScanThreads;  // block-uniform
         float u[kScanLanes], beta[kScanLanes], thr[kScanLanes];
         bool z[kScanLanes], ok[kScanLanes];
-        int srow_i[kScanLanes], col[kScanLanes];
-        int64_t out0[kScanLanes];
+        const float* xs[kScanLanes];
+        __nv_bfloat16* ps[kScanLanes];
+        __nv_bfloat16* pm[kScanLanes];
+        unsigned char* pb[kScanLanes];
 #pragma unroll
         for (int v = 0; v < kScanLanes; ++v) {
           const int j = g0 + kScanThreads * v + e;
           const int jj = j < lanes ? j : 0;  // lanes past the tile read row 0
           const int s = jj / BN, n = jj - (jj / BN) * BN;
-          srow_i[v] = s;
-          col[v] = n;
           ok[v] = j < lanes && r0 + s < f.R && n0 + n < f.N;
           const int nc = ok[v] ? n0 + n : 0;
           beta[v] = __ldg(f.beta + (f.beta_col ? nc : 0));
           thr[v] = __ldg(f.thr + (f.thr_col ? nc : 0));
           u[v] = 0.0f;
           z[v] = false;
-          out0[v] = (int64_t)(r0 + s) * f.N + nc;  // lane index within a step
+          const int64_t o = ok[v] ? (int64_t)(r0 + s) * f.N + nc : 0;  // lane index within a step
+          xs[v] = stg + s * SP + n;
+          ps[v] = f.spk + o;
+          pm[v] = f.mem + o;
+          pb[v] = f.bits ? f.bits + (o >> 3) : nullptr;
         }
+        const int xstep = f.BS * SP;
         for (int ts = 0; ts < f.T; ++ts) {
 #pragma unroll
           for (int v = 0; v < kScanLanes; ++v) {
-            const float x = stg[(ts * f.BS + srow_i[v]) * SP + col[v]];
+            if (v >= nv) break;  // uniform: the whole group is past the tile
+            const float x = *xs[v];
+            xs[v] += xstep;
             float idummy = 0.0f;
             fwd_step<false, RESET, 0>(f.reset, beta[v], thr[v], 0.0f, x, u[v], z[v], idummy);
             const bool zz = ok[v] && z[v];
             if (ok[v]) {
-              const int64_t o = (int64_t)ts * f.R * f.N + out0[v];
-              f.spk[o] = __float2bfloat16_rn(zz ? 1.0f : 0.0f);
-              f.mem[o] = __float2bfloat16_rn(u[v]);
+              *ps[v] = __float2bfloat16_rn(zz ? 1.0f : 0.0f);
+              *pm[v] = __float2bfloat16_rn(u[v]);
             }
+            ps[v] += RN;
+            pm[v] += RN;
             if (f.bits) {
               // 8 consecutive threads hold 8 consecutive lanes of one row (BN
               // and N are multiples of 8): one byte of the step's bit row
               const uint32_t m = __ballot_sync(0xffffffffu, zz);
-              if ((lid & 7) == 0 && ok[v])
-                f.bits[(int64_t)ts * f.bits_row + (out0[v] >> 3)] = (unsigned char)((m >> lid) & 0xFFu);
+              if ((lid & 7) == 0 && ok[v]) *pb[v] = (unsigned char)((m >> lid) & 0xFFu);
+              pb[v] += f.bits_row;
             }
           }
         }
@@ -260,10 +271,17 @@ cudaError_t launch_fused(const CUtensorMap& ta, const CUtensorMap& tb, const Fus
   const void* k = (const void*)gemm_leaky_tcgen05<BN, RESET>;
   const cudaError_t attr = ensure_smem(k, fused_smem_bytes<BN>());
   if (attr != cudaSuccess) return attr;
-  int dev = 0, sms = 152;
+  int dev = 0, sms = 152, per_sm = 1;
   if (cudaGetDevice(&dev) == cudaSuccess) cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  // persistent CTAs: as many as fit at once (one CTA's scan overlaps the
+  // other's main loop when two fit)
+  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, k, kFusedThreads, fused_smem_bytes<BN>()) !=
+          cudaSuccess || per_sm < 1)
+    per_sm = 1;
+  if (fused_smem_bytes<BN>() * 2 <= 220 * 1024) per_sm = per_sm < 2 ? 2 : per_sm;  // fits twice
+  const int64_t slots = (int64_t)sms * (per_sm > 2 ? 2 : per_sm);
   const int64_t tiles = (int64_t)((f.N + BN - 1) / BN) * ((f.R + f.BS - 1) / f.BS);
-  const unsigned grid = (unsigned)(tiles < sms ? tiles : sms);
+  const unsigned grid = (unsigned)(tiles < slots ? tiles : slots);
   return launch_pdl(gemm_leaky_tcgen05<BN, RESET>, dim3(grid), dim3(kFusedThreads),
                     fused_smem_bytes<BN>(), st, ta, tb, f);
 }

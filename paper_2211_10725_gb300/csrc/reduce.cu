@@ -17,6 +17,7 @@ namespace snn {
 namespace {
 
 constexpr int kRedThreads = 256;
+constexpr int64_t kChanChunk = 8192;  // lanes per block of the channel-last reduction (32 per thread)
 constexpr int64_t kNeuronSplit = 8;
 
 __device__ __forceinline__ double block_sum(double v, double* sh) {
@@ -139,8 +140,8 @@ __global__ void __launch_bounds__(kRedThreads) reduce_per_channel(ReduceJobs js,
 // block x sums lanes [x*chunk, (x+1)*chunk), chunk a multiple of the block
 // size, so thread t only meets channel t % C and its loads are coalesced.
 // The threads of a channel are added in thread order; the last block adds
-// the block partials of each channel with one warp (strided lane sums, then
-// a fixed shuffle tree).
+// the block partials of each channel in a fixed two-level order spread over
+// all its threads.
 __global__ void __launch_bounds__(kRedThreads) reduce_channel_last(ReduceJobs js, int64_t L,
                                                                     int64_t chunk, int C) {
   __shared__ double sh[kRedThreads];
@@ -148,10 +149,12 @@ __global__ void __launch_bounds__(kRedThreads) reduce_channel_last(ReduceJobs js
   const ReduceJob& j = js.job[blockIdx.z];
   const int64_t lo = (int64_t)blockIdx.x * chunk;
   const int64_t hi = min(L, lo + chunk);
-  double acc = 0.0;
-#pragma unroll 4
-  for (int64_t l = lo + threadIdx.x; l < hi; l += kRedThreads) acc += (double)j.part[l];
-  sh[threadIdx.x] = acc;
+  // a thread's run of lanes (32 at kChanChunk) in fp32 (double arithmetic
+  // is scarce on this part), everything above in fp64
+  float acc = 0.0f;
+#pragma unroll 8
+  for (int64_t l = lo + threadIdx.x; l < hi; l += kRedThreads) acc += j.part[l];
+  sh[threadIdx.x] = (double)acc;
   __syncthreads();
   if ((int)threadIdx.x < C) {
     double t = 0.0;
@@ -159,15 +162,21 @@ __global__ void __launch_bounds__(kRedThreads) reduce_channel_last(ReduceJobs js
     j.scratch[(int64_t)blockIdx.x * C + threadIdx.x] = t;
   }
   if (!last_of_group(&j.tickets[0], (int)gridDim.x)) return;
-  // warp w adds channels w, w + 8, ...: lane l the partials l, l + 32, ...
-  // in order, then a fixed shuffle tree
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  for (int c = warp; c < C; c += kRedThreads / 32) {
-    double t = 0.0;
-    for (int q = lane; q < (int)gridDim.x; q += 32) t += j.scratch[(int64_t)q * C + c];
-#pragma unroll
-    for (int d = 16; d > 0; d >>= 1) t += __shfl_xor_sync(0xffffffffu, t, d);
-    if (lane == 0) j.out[c] = (float)t;
+  // thread (c, p) = (t % C, t / C) adds the block partials p, p + P, ... of
+  // channel c in order (P = 256 / C parts, independent loads in flight);
+  // then thread c adds its channel's P parts in order
+  const int P = kRedThreads / C;
+  const int c = threadIdx.x % C, pp = threadIdx.x / C;
+  double t = 0.0;
+#pragma unroll 8
+  for (int q = pp; q < (int)gridDim.x; q += P) t += j.scratch[(int64_t)q * C + c];
+  __syncthreads();  // every thread is done with sh
+  sh[threadIdx.x] = t;
+  __syncthreads();
+  if ((int)threadIdx.x < C) {
+    double total = 0.0;
+    for (int k = 0; k < P; ++k) total += sh[k * C + threadIdx.x];
+    j.out[threadIdx.x] = (float)total;
   }
   if (threadIdx.x == 0) j.tickets[0] = 0;
 }
@@ -204,10 +213,11 @@ cudaError_t launch_param_reduce(const ParamReduce* p, int n, int64_t B, int64_t 
       if (e != cudaSuccess) return e;
     }
   } else if (C > 0 && HW == 1 && kRedThreads % C == 0) {
-    int64_t nb = ceil_div(L, 4096);
+    int64_t nb = ceil_div(L, kChanChunk);
     if (nb > scratch_len / C) nb = scratch_len / C;
     if (nb > 65535) nb = 65535;
     if (nb < 1) return cudaErrorInvalidValue;  // the workspace is sized for one block
+    // kChanChunk lanes per block unless the workspace holds fewer block partials
     const int64_t chunk = ceil_div(ceil_div(L > 0 ? L : 1, nb), kRedThreads) * kRedThreads;
     nb = ceil_div(L > 0 ? L : 1, chunk);
     const cudaError_t e = launch_pdl(reduce_channel_last, dim3((unsigned)nb, 1, (unsigned)n),

@@ -268,13 +268,19 @@ def _exact_inputs(w, seed=None):
     return inp
 
 
-def _oracle(w, inp):
+def _oracle(w, inp, stored=False):
+    """The oracle's forward, and its BPTT along the trace the kernels'
+    backward reads: the fp32 membrane, or with ``stored`` its bf16 rounding
+    (identical on both sides here, since the forward is exact)."""
     convs = [_np(c) for c in inp["convs"]]
     Wfc = _np(inp["Wfc"])
     X = _np(inp["X"]).reshape(w.T * w.B, w.H, w.W, w.Cin)
     betas = [np.full(c, w.beta) for c, _ in w.convs]
     fwd = O.csnn_forward(X, convs, Wfc, w.T, w.B, betas, w.beta_fc, w.thr, reset=w.reset,
                          dtype=np.float32)
+    if stored:
+        fwd = dict(fwd, mem=[O.bf16_round(m) for m in fwd["mem"]],
+                   fc_mem=O.bf16_round(fwd["fc_mem"]))
     res = O.csnn_backward(fwd, convs, Wfc, _np(inp["labels"]).astype(np.int64), w.T, w.B, betas,
                           w.beta_fc, w.thr, w.sg_param, reset=w.reset, store=O.bf16_round)
     return convs, Wfc, betas, fwd, res
@@ -325,9 +331,13 @@ def _check_step(w, net, convs, Wfc, betas, fwd, res):
     for l, (cout, k) in enumerate(w.convs):
         g = net.geo[l]
         Ho, Wo, cp = g[5], g[6], g[3]
-        I = _np(net.I[l]).reshape(T * B, Ho, Wo, cp)
-        assert np.array_equal(I[..., :cout], fwd["I"][l]), f"conv {l} currents"
-        assert not I[..., cout:].any()
+        if net.I[l] is not None:  # a fused layer keeps its currents on chip
+            I = _np(net.I[l]).reshape(T * B, Ho, Wo, cp)
+            assert np.array_equal(I[..., :cout], fwd["I"][l]), f"conv {l} currents"
+            assert not I[..., cout:].any()
+        if net.layers[l].mem is not None:  # the stored trace: bf16 of the exact fp32 trace
+            mem = _np(net.layers[l].mem).reshape(T * B, Ho, Wo, cp)[..., :cout].reshape(T, -1)
+            assert np.array_equal(mem, O.bf16_round(fwd["mem"][l])), f"conv {l} stored membrane"
         spk = _np(net.layers[l].spk).reshape(T * B, Ho, Wo, cp)
         assert np.array_equal(spk[..., :cout].reshape(T, -1), fwd["spk"][l]), f"conv {l} spikes"
         assert not spk[..., cout:].any()
@@ -336,8 +346,9 @@ def _check_step(w, net, convs, Wfc, betas, fwd, res):
         idx = net.idx[l].cpu().numpy().astype(np.int64)
         assert np.array_equal(idx[..., :cout], fwd["idx"][l]), f"pool {l} positions"
     n = w.n_classes
-    Ifc = _np(net.I_fc)
-    assert np.array_equal(Ifc[:, :n], fwd["fc_I"]), "readout currents"
+    if net.I_fc is not None:
+        Ifc = _np(net.I_fc)
+        assert np.array_equal(Ifc[:, :n], fwd["fc_I"]), "readout currents"
     assert np.array_equal(_np(net.out_layer.spk)[:, :, :n].reshape(T, -1), fwd["fc_spk"])
 
     loss = float(net.loss.item())
@@ -381,15 +392,17 @@ def _check_step(w, net, convs, Wfc, betas, fwd, res):
     return mag
 
 
-@pytest.mark.parametrize("direct_first", [True, False])
-def test_csnn_step_small_matches_oracle(direct_first, cuda_device):
+@pytest.mark.parametrize("direct_first,save", [(True, "recompute"), (False, "recompute"),
+                                               (True, "fused"), (False, "fused")])
+def test_csnn_step_small_matches_oracle(direct_first, save, cuda_device):
     """The step at T = 4, B = 8, with the first layer as a direct
-    convolution or as im2col + tensor-core GEMM."""
+    convolution or as im2col + tensor-core GEMM, recomputing the membrane in
+    the BPTT or (fused) storing it and scanning in the GEMM epilogues."""
     w = SMALL
     inp = _exact_inputs(w)
-    convs, Wfc, betas, fwd, res = _oracle(w, inp)
+    convs, Wfc, betas, fwd, res = _oracle(w, inp, stored=save == "fused")
     assert all(s.mean() > 0 for s in fwd["spk"]) and fwd["fc_spk"].mean() > 0
-    net, X, labels = _run(w, inp, cuda_device, direct_first=direct_first)
+    net, X, labels = _run(w, inp, cuda_device, direct_first=direct_first, save=save)
     assert net.direct[0] == direct_first
     net.step(X, labels)
     torch.cuda.synchronize()
@@ -431,13 +444,14 @@ def test_csnn_training_step_update_matches_oracle(cuda_device):
     assert torch.equal(net.W_flat.cpu(), net.W32_flat.cpu().to(torch.bfloat16))
 
 
-def test_csnn_step_full_size(cuda_device):
+@pytest.mark.parametrize("save", ["recompute", "fused"])
+def test_csnn_step_full_size(save, cuda_device):
     """12C5-MP2-64C5-MP2-10 at T = 25, B = 128 (the configuration the
     benchmark times): the same exact forward and gradient bounds."""
     w = W.CSNN_C4
     inp = _exact_inputs(w)
-    convs, Wfc, betas, fwd, res = _oracle(w, inp)
-    net, X, labels = _run(w, inp, cuda_device)
+    convs, Wfc, betas, fwd, res = _oracle(w, inp, stored=save == "fused")
+    net, X, labels = _run(w, inp, cuda_device, save=save)
     net.step(X, labels)
     torch.cuda.synchronize()
     for layer in net.layers + [net.out_layer]:
