@@ -177,9 +177,62 @@ __global__ void __launch_bounds__(kThreads) im2col_vec8_kernel(const uint4* __re
   cols[i] = v;
 }
 
+// As im2col_vec8_kernel, kIm2colPer vectors per thread (a block's threads
+// stride over consecutive vectors, so stores stay coalesced and each thread
+// has several loads in flight), the tap of each column group read from a
+// shared-memory table instead of being divided out per element.
+constexpr int kIm2colPer = 4;
+constexpr int kIm2colMaxGroups = 4096;  // column groups (Kpad / 8) the table holds
+
+template <typename Ix>
+__global__ void __launch_bounds__(kThreads) im2col_vec8_multi_kernel(const uint4* __restrict__ X,
+                                                                     uint4* __restrict__ cols,
+                                                                     Ix rows, int H, int W,
+                                                                     int Cin, int KH, int KW,
+                                                                     int Kpad) {
+  __shared__ int toff[kIm2colMaxGroups];  // input offset (16-byte units) of group j's tap, or -1
+  const int Ho = H - KH + 1, Wo = W - KW + 1;
+  const int G = Cin / 8;
+  const int vpr = Kpad / 8;
+  for (int j = threadIdx.x; j < vpr; j += blockDim.x) {
+    int t = -1;
+    if (j < KH * KW * G) {
+      const int tap = j / G, g = j - tap * G;
+      const int ky = tap / KW, kx = tap - ky * KW;
+      t = (ky * W + kx) * G + g;
+    }
+    toff[j] = t;
+  }
+  __syncthreads();
+  grid_dep_wait();
+  const Ix total = rows * vpr;
+  const Ix base = (Ix)blockIdx.x * blockDim.x * kIm2colPer + threadIdx.x;
+  uint4 v[kIm2colPer];
+#pragma unroll
+  for (int u = 0; u < kIm2colPer; ++u) {
+    const Ix i = base + (Ix)u * blockDim.x;
+    v[u] = make_uint4(0u, 0u, 0u, 0u);
+    if (i < total) {
+      const Ix r = i / vpr;
+      const int t = toff[(int)(i - r * vpr)];
+      if (t >= 0) {
+        const Ix m = r / (Ho * Wo);
+        const int p = (int)(r - m * (Ho * Wo));
+        const int oy = p / Wo, ox = p - oy * Wo;
+        v[u] = X[((m * H + oy) * W + ox) * G + t];
+      }
+    }
+  }
+#pragma unroll
+  for (int u = 0; u < kIm2colPer; ++u) {
+    const Ix i = base + (Ix)u * blockDim.x;
+    if (i < total) cols[i] = v[u];
+  }
+}
+
 // Thread i sums the 8 channels of group i % G of pixel i / G over the taps
 // that read it, in (ky, kx) order.
-template <typename Ix>
+template <typename Ix, int KH_ = 0, int KW_ = 0>
 __global__ void __launch_bounds__(kThreads) col2im_vec8_kernel(const uint4* __restrict__ dcols,
                                                                uint4* __restrict__ dX,
                                                                Ix total, int H, int W, int Cin,
@@ -198,17 +251,42 @@ __global__ void __launch_bounds__(kThreads) col2im_vec8_kernel(const uint4* __re
   float s[8];
 #pragma unroll
   for (int e = 0; e < 8; ++e) s[e] = 0.0f;
-  for (int ky = 0; ky < KH; ++ky) {
-    const int oy = y - ky;
-    if (oy < 0 || oy >= Ho) continue;
-    for (int kx = 0; kx < KW; ++kx) {
-      const int ox = x - kx;
-      if (ox < 0 || ox >= Wo) continue;
-      const Ix r = (m * Ho + oy) * Wo + ox;
-      Pack8 v;
-      v.u = dcols[r * vpr + (ky * KW + kx) * G + g];
+  if constexpr (KH_ > 0) {
+    // fixed taps: one filter row's KW_ loads issued before its adds, which
+    // still run in (ky, kx) order
+#pragma unroll 1
+    for (int ky = 0; ky < KH_; ++ky) {
+      const int oy = y - ky;
+      if (oy < 0 || oy >= Ho) continue;
+      Pack8 v[KW_];
 #pragma unroll
-      for (int e = 0; e < 8; ++e) s[e] += __bfloat162float(v.h[e]);
+      for (int kx = 0; kx < KW_; ++kx) {
+        const int ox = x - kx;
+        v[kx].u = (ox >= 0 && ox < Wo) ? dcols[((m * Ho + oy) * Wo + ox) * vpr + (ky * KW_ + kx) * G + g]
+                                       : make_uint4(0u, 0u, 0u, 0u);
+      }
+#pragma unroll
+      for (int kx = 0; kx < KW_; ++kx) {
+        const int ox = x - kx;
+        if (ox >= 0 && ox < Wo) {
+#pragma unroll
+          for (int e = 0; e < 8; ++e) s[e] += __bfloat162float(v[kx].h[e]);
+        }
+      }
+    }
+  } else {
+    for (int ky = 0; ky < KH; ++ky) {
+      const int oy = y - ky;
+      if (oy < 0 || oy >= Ho) continue;
+      for (int kx = 0; kx < KW; ++kx) {
+        const int ox = x - kx;
+        if (ox < 0 || ox >= Wo) continue;
+        const Ix r = (m * Ho + oy) * Wo + ox;
+        Pack8 v;
+        v.u = dcols[r * vpr + (ky * KW + kx) * G + g];
+#pragma unroll
+        for (int e = 0; e < 8; ++e) s[e] += __bfloat162float(v.h[e]);
+      }
     }
   }
   Pack8 o;
@@ -317,6 +395,19 @@ extern "C" snn_status_t snn_im2col_nhwc(int64_t M, int64_t H, int64_t W, int64_t
   const int64_t n = rows * (Kpad / 8);
   if (n / kThreads >= INT_MAX) return SNN_ERR_INVALID_ARG;
   const bool i32 = rows * Kpad < INT_MAX && M * H * W * Cin < INT_MAX;  // 32-bit index math
+  if (Cin % 8 == 0 && aligned(X, 16) && Kpad / 8 <= kIm2colMaxGroups) {
+    const unsigned nb = (unsigned)((n + (int64_t)kThreads * kIm2colPer - 1) / ((int64_t)kThreads * kIm2colPer));
+    const cudaError_t e =
+        i32 ? launch_pdl(im2col_vec8_multi_kernel<int>, dim3(nb), dim3(kThreads), 0,
+                         reinterpret_cast<cudaStream_t>(stream), static_cast<const uint4*>(X),
+                         static_cast<uint4*>(cols), rows, (int)H, (int)W, (int)Cin, (int)KH,
+                         (int)KW, (int)Kpad)
+            : launch_pdl(im2col_vec8_multi_kernel<int64_t>, dim3(nb), dim3(kThreads), 0,
+                         reinterpret_cast<cudaStream_t>(stream), static_cast<const uint4*>(X),
+                         static_cast<uint4*>(cols), rows, (int)H, (int)W, (int)Cin, (int)KH,
+                         (int)KW, (int)Kpad);
+    return e == cudaSuccess ? SNN_OK : SNN_ERR_CUDA;
+  }
   if (Cin % 8 == 0 && aligned(X, 16)) {
     const cudaError_t e = i32 ? launch_pdl(im2col_vec8_kernel<int>, dim3(blocks_for(n)), dim3(kThreads), 0,
                                      reinterpret_cast<cudaStream_t>(stream),
@@ -354,7 +445,14 @@ extern "C" snn_status_t snn_col2im_nhwc(int64_t M, int64_t H, int64_t W, int64_t
   if (n / kThreads >= INT_MAX) return SNN_ERR_INVALID_ARG;
   const bool i32 = M * (H - KH + 1) * (W - KW + 1) * Kpad < INT_MAX && n < INT_MAX;
   if (Cin % 8 == 0 && Kpad % 8 == 0 && aligned(dcols, 16) && aligned(dX, 16)) {
-    const cudaError_t e = i32 ? launch_pdl(col2im_vec8_kernel<int>, dim3(blocks_for(n / 8)), dim3(kThreads), 0,
+    cudaError_t e;
+    if (KH == 5 && KW == 5 && i32)
+      e = launch_pdl(col2im_vec8_kernel<int, 5, 5>, dim3(blocks_for(n / 8)), dim3(kThreads), 0,
+                     reinterpret_cast<cudaStream_t>(stream), static_cast<const uint4*>(dcols),
+                     static_cast<uint4*>(dX), n / 8, (int)H, (int)W, (int)Cin, (int)KH, (int)KW,
+                     (int)Kpad);
+    else
+      e = i32 ? launch_pdl(col2im_vec8_kernel<int>, dim3(blocks_for(n / 8)), dim3(kThreads), 0,
                                      reinterpret_cast<cudaStream_t>(stream),
                                      static_cast<const uint4*>(dcols), static_cast<uint4*>(dX),
                                      n / 8, (int)H, (int)W, (int)Cin, (int)KH, (int)KW, (int)Kpad)
