@@ -159,3 +159,95 @@ def test_data_parallel_step_order(tmp_path):
         assert calls[0] == ("forward", 128)
         assert calls[1] == ("backward",)
         assert calls[2] == ("update", [3.0] * 4, 1.5)
+
+
+# ---------------------------------------------------------------------------
+# The convolutional SNN: weight gradients, per-channel beta gradients, loss
+# ---------------------------------------------------------------------------
+
+def _csnn_problem():
+    w = W.CSNN_C4.scaled(T=3, B=4, H=12, W=12, convs=((4, 5), (8, 3)), n_classes=5)
+    inp = W.make_conv_inputs(w, seed=W.SEED_BASE + 78)
+    convs = [c.float().numpy().astype(np.float64) * 3.0 for c in inp["convs"]]  # enough spikes
+    Wfc = inp["Wfc"].float().numpy().astype(np.float64) * 3.0
+    X = inp["X"].float().numpy().astype(np.float64)                             # [T, B, H, W, 1]
+    y = inp["labels"].numpy().astype(np.int64)
+    return w, convs, Wfc, X, y
+
+
+def _csnn_grads(w, convs, Wfc, X, y, b0, b1, batch_total):
+    """Oracle gradients (conv filters, readout, per-channel betas) and loss of
+    samples [b0, b1), the loss averaged over batch_total samples."""
+    nb = b1 - b0
+    xb = X[:, b0:b1].reshape(w.T * nb, w.H, w.W, w.Cin)
+    betas = [np.full(c, w.beta) for c, _ in w.convs]
+    fwd = O.csnn_forward(xb, convs, Wfc, w.T, nb, betas, w.beta_fc, w.thr, reset=w.reset)
+    res = O.csnn_backward(fwd, convs, Wfc, y[b0:b1], w.T, nb, betas, w.beta_fc, w.thr,
+                          w.sg_param, reset=w.reset)
+    k = nb / batch_total
+    parts = [d.ravel() for d in res["dW"]] + [res["dW_fc"].ravel()] + \
+        [d.ravel() for d in res["dbeta"]] + [[res["loss"]]]
+    return np.concatenate(parts) * k
+
+
+def _csnn_rank_main(rank, world, port, out_dir):
+    os.environ.update(MASTER_ADDR="127.0.0.1", MASTER_PORT=str(port))
+    dist.init_process_group("gloo", rank=rank, world_size=world)
+    try:
+        w, convs, Wfc, X, y = _csnn_problem()
+        b0, b1 = shard_range(w.B, world, rank)
+        flat = torch.tensor(_csnn_grads(w, convs, Wfc, X, y, b0, b1, w.B))
+        allreduce_sum_([flat])
+        np.save(os.path.join(out_dir, f"csnn{rank}.npy"), flat.numpy())
+    finally:
+        dist.destroy_process_group()
+
+
+def test_csnn_sharded_gradients_sum_to_the_full_batch(tmp_path):
+    """Two gloo ranks on halves of the batch: the summed filter, readout and
+    per-channel beta gradients and the loss equal the full batch's."""
+    world = 2
+    mp.spawn(_csnn_rank_main, args=(world, _free_port(), str(tmp_path)), nprocs=world,
+             join=True)
+    w, convs, Wfc, X, y = _csnn_problem()
+    full = _csnn_grads(w, convs, Wfc, X, y, 0, w.B, w.B)
+    assert np.abs(full[:-1]).max() > 1e-6
+    for r in range(world):
+        np.testing.assert_allclose(np.load(tmp_path / f"csnn{r}.npy"), full, rtol=1e-12,
+                                   atol=1e-15)
+
+
+class _FakeConvNet(_FakeNet):
+    """Stands in for ConvSNN: also holds the betas' gradients."""
+
+    def __init__(self, rank):
+        super().__init__(rank)
+        self.dbeta_flat = torch.full((2,), 10.0 * (rank + 1))
+
+    def update(self, stream=None):
+        self.calls.append(("update", self.dW_flat.tolist(), self.dbeta_flat.tolist(),
+                           float(self.loss)))
+
+
+def _dp_conv_rank_main(rank, world, port, out_dir):
+    os.environ.update(MASTER_ADDR="127.0.0.1", MASTER_PORT=str(port))
+    dist.init_process_group("gloo", rank=rank, world_size=world)
+    try:
+        from paper_2211_10725_gb300.data_parallel import DataParallelConvSNN
+        net = _FakeConvNet(rank)
+        DataParallelConvSNN(net, global_batch=256).train_step(None, None)
+        torch.save(net.calls, os.path.join(out_dir, f"conv_calls{rank}.pt"))
+    finally:
+        dist.destroy_process_group()
+
+
+def test_data_parallel_conv_step_sums_beta_gradients(tmp_path):
+    """The convolutional network's step also sums the betas' gradients
+    before the update."""
+    world = 2
+    mp.spawn(_dp_conv_rank_main, args=(world, _free_port(), str(tmp_path)), nprocs=world,
+             join=True)
+    for r in range(world):
+        calls = torch.load(tmp_path / f"conv_calls{r}.pt")
+        assert calls[0] == ("forward", 256)
+        assert calls[2] == ("update", [3.0] * 4, [30.0] * 2, 1.5)
