@@ -6,6 +6,13 @@ threshold gradients reduced over the batch.  Default workload: I[T=500,
 B=64, N=8192] bf16 storage with fp32 state; BPTT from the stored mem/spk
 traces (--save recompute: from fp32 checkpoints every 8 steps).
 
+Other scan workloads (`--workload`, the names in workloads.SCAN_WORKLOADS)
+time the same step on their shapes.  The network workloads time a whole
+training step as one CUDA graph: the dense SNN (Tab. I DSNN) and its
+population-coded variant, and the convolutional SNN (Tab. I CSNN) --
+forward (by default each GEMM layer fused with its scan), loss, BPTT and
+AdamW -- in the same metric, with images/s and per-op times beside it.
+
 Prints one JSON line (rank 0).  `--impl reference` times the CPU oracle (the
 only other implementation of this path) on a bounded sample of the same
 workload instead.
