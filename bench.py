@@ -832,6 +832,10 @@ def run_net(args):
                     "traffic": None, "flops_per_step": {"fwd": fwd_f, "dW": dw_f, "dX": dx_f}}
         step_desc = ("forward GEMMs + Leaky scans, rate-coded CE loss, BPTT scans, dense "
                      "backward (dX, dW), AdamW")
+        if fused:
+            step_desc = ("forward GEMMs with the Leaky scan in their epilogue, rate-coded CE "
+                         "loss, the readout's BPTT scan, dW GEMMs, dX GEMMs with the lower "
+                         "layer's BPTT scan in their epilogue, AdamW")
         l2 = "working set (~70 MB) fits in L2; no flush between steps"
     roofline.update({"op_ms": op_ms, "op_timed_step_ms": ev_total / K2,
                      "timing": "per-op: a second timed region of the same step graph with "

@@ -361,6 +361,30 @@ snn_status_t snn_dense_leaky_fwd(const snn_scan_desc* desc, int64_t P, int64_t K
                                  snn_stream_t stream);
 
 /*
+ * The dense backward fused with the BPTT of the layer below (the converse of
+ * snn_dense_leaky_fwd): the product dX = dI_up * W of the layer above, whose
+ * rows are the spike gradients dL/dz_t of this layer, is computed on the
+ * tcgen05 tensor cores and this layer's reverse scan (Sec. III-B, the
+ * store-mode arithmetic of snn_leaky_bwd) runs on it in the epilogue; the
+ * spike gradient is neither rounded nor written.
+ *   desc    this (lower) Leaky layer: T <= 128, B, N neurons (multiple of 8),
+ *           io_dtype SNN_BF16, save SNN_SAVE_MEM, any reset, detach and
+ *           surrogate; beta_mode / thr_mode scalar or per neuron
+ *   dI_up   bf16 [T*B, K]: dL/dI of the layer above (K its neurons, multiple
+ *           of 8)
+ *   W       bf16 [K, N]: the layer above's weights (its [N_out, K_in] matrix)
+ *   mem     bf16 [T, B, N] stored trace; ckpt its spike bits, or NULL with
+ *           spk bf16 [T, B, N] instead
+ *   grad_I  bf16 [T, B, N] (out): this layer's dL/dI
+ * No grad_mem, grad_mem_final, mem0 or parameter gradients (use
+ * snn_leaky_bwd for those).  ws: at least 256 bytes.
+ */
+snn_status_t snn_dense_leaky_bwd(const snn_scan_desc* desc, int64_t K, const void* dI_up,
+                                 const void* W, const float* beta, const float* thr,
+                                 const void* mem, const void* spk, const float* ckpt,
+                                 void* grad_I, void* ws, size_t ws_bytes, snn_stream_t stream);
+
+/*
  * Convolutional SNN layout kernels (Tab. I CSNN: 5x5 convolutions, 2x2 max
  * pooling) on channel-last bf16 activations [M, H, W, C], M = T*B.  A
  * convolution is a snn_dense_layer_fwd/bwd over the patch rows:

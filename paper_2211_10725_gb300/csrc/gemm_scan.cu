@@ -17,6 +17,13 @@
 // membrane trace [T, R, N] and, optionally, the spike bits the store-mode
 // BPTT reads (bit k of byte j of row t is z_t of lane 8j + k).  The fp32
 // current is never written.
+//
+// Backward mode (BWD): the same tiles of the product dX = dI_up * W (W read
+// MN-major, as the plain dense backward reads it) are the spike gradients
+// dL/dz of the layer below, and the epilogue runs that layer's BPTT on them
+// in reverse time with the scan kernels' bwd_step, from its stored bf16
+// trace and spike bits, writing its dL/dI.  The spike gradient is never
+// rounded or written.
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
 
@@ -35,6 +42,7 @@ constexpr int kScanWarps = 10;  // warps 2..11 scan; 2..5 also drain the accumul
 constexpr int kScanThreads = 32 * kScanWarps;
 constexpr int kFusedThreads = 64 + kScanThreads;
 constexpr int kScanLanes = 2;  // lanes a scan thread steps together (independent chains)
+constexpr int kBwdChunk = 4;   // steps of stored trace a backward scan thread loads ahead (8 spills)
 
 struct FusedArgs {
   int T, R, K, N;   // steps, rows per step, reduction, output columns (neurons / channels)
@@ -49,6 +57,12 @@ struct FusedArgs {
   int64_t bits_row;
   int* status;
   uint64_t wait_ns;
+  // backward mode: the layer's stored trace, spike bits (or spk) and dL/dI
+  const __nv_bfloat16* mem_in;
+  const unsigned char* bits_in;
+  const __nv_bfloat16* spk_in;
+  __nv_bfloat16* gI;
+  ScanArgs sa;  // reset, detach and surrogate of bwd_step
 };
 
 template <int BN>
@@ -64,11 +78,12 @@ __device__ __forceinline__ void epi_barrier() {
   asm volatile("bar.sync 1, %0;" ::"n"(kScanThreads) : "memory");
 }
 
-template <int BN, int RESET>
+template <int BN, int RESET, bool BWD = false, int SG = 0>
 __global__ void __launch_bounds__(kFusedThreads, 2)
     gemm_leaky_tcgen05(const __grid_constant__ CUtensorMap ta, const __grid_constant__ CUtensorMap tb,
                        const FusedArgs f) {
   static_assert(BN % 16 == 0 && BN >= 16 && BN <= 128, "UMMA N for M=128");
+  static_assert(!BWD || BN % 64 == 0, "an MN-major B tile is whole 64-wide boxes");
   constexpr int A_BYTES = BM * BK * 2;
   constexpr int B_BYTES = BN * BK * 2;
   constexpr int SP = stage_pitch<BN>();
@@ -126,7 +141,13 @@ __global__ void __launch_bounds__(kFusedThreads, 2)
           }
           mbar_arrive_expect_tx(&full[s], a_tx + B_BYTES);
           tma_load_3d(sA + s * A_BYTES, &ta, kb * BK, r0, 0, &full[s]);
-          tma_load_2d(sB + s * B_BYTES, &tb, kb * BK, n0, &full[s]);
+          if constexpr (BWD) {
+#pragma unroll
+            for (int j = 0; j < BN / 64; ++j)
+              tma_load_2d(sB + s * B_BYTES + j * kMnBoxBytes, &tb, n0 + 64 * j, kb * BK, &full[s]);
+          } else {
+            tma_load_2d(sB + s * B_BYTES, &tb, kb * BK, n0, &full[s]);
+          }
         }
       }
       for (int64_t j = n_issued > kFusedStages ? n_issued - kFusedStages : 0; j < n_issued; ++j)
@@ -134,7 +155,10 @@ __global__ void __launch_bounds__(kFusedThreads, 2)
     }
   } else if (warp == 1) {
     if (lid == 0) {
-      constexpr uint32_t idesc = idesc_bf16(BM, BN);
+      constexpr uint32_t idesc = idesc_bf16(BM, BN, false, BWD);
+      // 16 more along K: 32 bytes inside a K-major row, or 16 rows (2048
+      // bytes) of an MN-major tile; the descriptor holds the address >> 4
+      constexpr uint64_t stepB = BWD ? 2048 >> 4 : 32 >> 4;
       int64_t n_used = 0;
       bool ok = true;
       int i = 0;
@@ -155,10 +179,10 @@ __global__ void __launch_bounds__(kFusedThreads, 2)
           }
           tc_fence_after();
           const uint64_t da = sdesc_sw128(sA + s * A_BYTES);
-          const uint64_t db = sdesc_sw128(sB + s * B_BYTES);
+          const uint64_t db = BWD ? sdesc_sw128_mn(sB + s * B_BYTES) : sdesc_sw128(sB + s * B_BYTES);
 #pragma unroll
           for (int kk = 0; kk < BK / 16; ++kk)
-            tc_mma(acc, da + (uint64_t)(2 * kk), db + (uint64_t)(2 * kk), idesc, (kb | kk) != 0 ? 1u : 0u);
+            tc_mma(acc, da + (uint64_t)(2 * kk), db + stepB * kk, idesc, (kb | kk) != 0 ? 1u : 0u);
           tc_commit(&empty[s]);
         }
         if (ok) tc_commit(&acc_full[b]);
@@ -200,6 +224,69 @@ __global__ void __launch_bounds__(kFusedThreads, 2)
         if (e == 0) record_status(f.status, kStatusTimeout);
         break;
       }
+      if constexpr (BWD) {
+      // the reverse scan: thread e steps lanes j = g0 + kScanThreads*v + e
+      // from t = T-1 down to 0; the staged value of (t, lane) is dL/dz_t.
+      // The stored trace of kBwdChunk steps is loaded before they are
+      // stepped, so the loads of a chunk overlap instead of each step
+      // waiting for its own.
+      const int64_t RN = (int64_t)f.R * f.N;
+      for (int g0 = 0; g0 < lanes; g0 += kScanThreads * kScanLanes) {
+        const int nv = (lanes - g0 + kScanThreads - 1) / kScanThreads;  // block-uniform
+        float beta[kScanLanes], thr[kScanLanes];
+        bool ok[kScanLanes];
+        int srow_i[kScanLanes], col[kScanLanes];
+        int64_t o[kScanLanes];
+        BwdLane st[kScanLanes];
+#pragma unroll
+        for (int v = 0; v < kScanLanes; ++v) {
+          const int j = g0 + kScanThreads * v + e;
+          const int jj = j < lanes ? j : 0;  // lanes past the tile read row 0
+          const int sr = jj / BN, n = jj - (jj / BN) * BN;
+          srow_i[v] = sr;
+          col[v] = n;
+          ok[v] = j < lanes && r0 + sr < f.R && n0 + n < f.N;
+          const int nc = ok[v] ? n0 + n : 0;
+          beta[v] = __ldg(f.beta + (f.beta_col ? nc : 0));
+          thr[v] = __ldg(f.thr + (f.thr_col ? nc : 0));
+          o[v] = ok[v] ? (int64_t)(r0 + sr) * f.N + nc : 0;
+          st[v] = BwdLane{0.0f, 0.0f, 0.0f, 0.0f, 0.0f};
+        }
+        for (int tc = f.T - 1; tc >= 0; tc -= kBwdChunk) {
+          static_assert(kScanLanes == 2, "the trace of a step's two lanes is one bf16 pair");
+          __nv_bfloat162 uu[kBwdChunk];  // the bf16 trace as stored (x: lane 0, y: lane 1)
+          uint32_t zz[kScanLanes] = {};  // bit c: z at step tc - c
+#pragma unroll
+          for (int c = 0; c < kBwdChunk; ++c) {
+#pragma unroll
+            for (int v = 0; v < kScanLanes; ++v) {
+              // steps before t = 0 and lanes past the tile load lane 0 of
+              // step 0 (in bounds) and are not stepped
+              const int ts = tc - c >= 0 && v < nv ? tc - c : 0;
+              const int64_t q = (int64_t)ts * RN + o[v];
+              if (v == 0) uu[c].x = f.mem_in[q];
+              else uu[c].y = f.mem_in[q];
+              const uint32_t z = f.bits_in ? (__ldg(f.bits_in + (int64_t)ts * f.bits_row + (o[v] >> 3)) >> (o[v] & 7)) & 1u
+                                           : (__bfloat162float(f.spk_in[q]) != 0.0f ? 1u : 0u);
+              zz[v] |= z << c;
+            }
+          }
+#pragma unroll
+          for (int c = 0; c < kBwdChunk; ++c) {
+            const int ts = tc - c;
+            if (ts < 0) break;  // uniform
+#pragma unroll
+            for (int v = 0; v < kScanLanes; ++v) {
+              if (v >= nv) break;  // uniform: the whole group is past the tile
+              const float gs = stg[(ts * f.BS + srow_i[v]) * SP + col[v]];
+              const float du = bwd_step<false, RESET, SG>(f.sa, beta[v], thr[v], 0.0f, ts + 1 < f.T,
+                                                          __bfloat162float(v == 0 ? uu[c].x : uu[c].y), ((zz[v] >> c) & 1u) != 0, 0.0f, gs, 0.0f, 0.0f, st[v]);
+              if (ok[v]) f.gI[(int64_t)ts * RN + o[v]] = __float2bfloat16_rn(du);
+            }
+          }
+        }
+      }
+      } else {
       // the scan: thread e steps lanes j = g0 + kScanThreads*v + e together
       // (independent chains); groups wholly past the tile are skipped
       const int64_t RN = (int64_t)f.R * f.N;  // elements per step of spk / mem
@@ -254,6 +341,7 @@ __global__ void __launch_bounds__(kFusedThreads, 2)
           }
         }
       }
+      }
       epi_barrier();  // the staged rows are consumed before the next tile's copy
     }
   }
@@ -265,10 +353,10 @@ __global__ void __launch_bounds__(kFusedThreads, 2)
   }
 }
 
-template <int BN, int RESET>
+template <int BN, int RESET, bool BWD = false, int SG = 0>
 cudaError_t launch_fused(const CUtensorMap& ta, const CUtensorMap& tb, const FusedArgs& f,
                          cudaStream_t st) {
-  const void* k = (const void*)gemm_leaky_tcgen05<BN, RESET>;
+  const void* k = (const void*)gemm_leaky_tcgen05<BN, RESET, BWD, SG>;
   const cudaError_t attr = ensure_smem(k, fused_smem_bytes<BN>());
   if (attr != cudaSuccess) return attr;
   int dev = 0, sms = 152, per_sm = 1;
@@ -282,8 +370,25 @@ cudaError_t launch_fused(const CUtensorMap& ta, const CUtensorMap& tb, const Fus
   const int64_t slots = (int64_t)sms * (per_sm > 2 ? 2 : per_sm);
   const int64_t tiles = (int64_t)((f.N + BN - 1) / BN) * ((f.R + f.BS - 1) / f.BS);
   const unsigned grid = (unsigned)(tiles < slots ? tiles : slots);
-  return launch_pdl(gemm_leaky_tcgen05<BN, RESET>, dim3(grid), dim3(kFusedThreads),
+  return launch_pdl(gemm_leaky_tcgen05<BN, RESET, BWD, SG>, dim3(grid), dim3(kFusedThreads),
                     fused_smem_bytes<BN>(), st, ta, tb, f);
+}
+
+template <int BN, int SG>
+cudaError_t launch_fused_bwd_reset(const CUtensorMap& ta, const CUtensorMap& tb, const FusedArgs& f,
+                                   cudaStream_t st) {
+  switch (f.reset) {
+    case RESET_SUBTRACT: return launch_fused<BN, RESET_SUBTRACT, true, SG>(ta, tb, f, st);
+    case RESET_ZERO: return launch_fused<BN, RESET_ZERO, true, SG>(ta, tb, f, st);
+    default: return launch_fused<BN, RESET_NONE, true, SG>(ta, tb, f, st);
+  }
+}
+
+template <int BN>
+cudaError_t launch_fused_bwd(const CUtensorMap& ta, const CUtensorMap& tb, const FusedArgs& f,
+                             cudaStream_t st) {
+  return f.sa.sg == SG_FAST_SIGMOID ? launch_fused_bwd_reset<BN, SG_FAST_SIGMOID>(ta, tb, f, st)
+                                    : launch_fused_bwd_reset<BN, SG_ATAN>(ta, tb, f, st);
 }
 
 template <int BN>
@@ -368,5 +473,77 @@ extern "C" snn_status_t snn_dense_leaky_fwd(const snn_scan_desc* d, int64_t P, i
     case 64: e = launch_fused_reset<64>(ta, tb, f, st); break;
     default: e = launch_fused_reset<128>(ta, tb, f, st);
   }
+  return e == cudaSuccess ? SNN_OK : SNN_ERR_CUDA;
+}
+
+extern "C" snn_status_t snn_dense_leaky_bwd(const snn_scan_desc* d, int64_t K, const void* dI_up,
+                                            const void* W, const float* beta, const float* thr,
+                                            const void* mem, const void* spk, const float* ckpt,
+                                            void* grad_I, void* ws, size_t ws_bytes,
+                                            snn_stream_t stream) {
+  if (!d || K < 0) return SNN_ERR_INVALID_ARG;
+  if (d->T < 1 || d->B < 1 || d->N < 1 || d->reserved0 != 0 || d->reserved1 != 0)
+    return SNN_ERR_INVALID_ARG;
+  if (d->reset < SNN_RESET_SUBTRACT || d->reset > SNN_RESET_NONE) return SNN_ERR_INVALID_ARG;
+  if (d->surrogate != SNN_SG_FAST_SIGMOID && d->surrogate != SNN_SG_ATAN) return SNN_ERR_INVALID_ARG;
+  if (!(d->sg_param > 0.0f)) return SNN_ERR_INVALID_ARG;
+  if (d->io_dtype != SNN_BF16 || d->save != SNN_SAVE_MEM) return SNN_ERR_UNSUPPORTED;
+  if (d->T > 128 || K % 8 != 0 || K == 0 || d->N % 8 != 0) return SNN_ERR_UNSUPPORTED;
+  if (d->B > INT_MAX / 2 || K > INT_MAX / 2 || d->N > INT_MAX / 2 || d->T * d->B * d->N > ((int64_t)1 << 46))
+    return SNN_ERR_INVALID_ARG;
+  auto col_mode = [&](int32_t mode, int* col) {
+    if (mode == SNN_P_SCALAR) { *col = 0; return true; }
+    if (mode == SNN_P_PER_NEURON) { *col = 1; return true; }
+    return false;
+  };
+  int beta_col = 0, thr_col = 0;
+  if (!col_mode(d->beta_mode, &beta_col) || !col_mode(d->thr_mode, &thr_col)) return SNN_ERR_UNSUPPORTED;
+  if (!dI_up || !W || !beta || !thr || !mem || !grad_I || (!ckpt && !spk)) return SNN_ERR_INVALID_ARG;
+  if (!al16(dI_up) || !al16(W) || !al16(mem) || !al16(grad_I) || (spk && !al16(spk)) ||
+      (ckpt && !al16(ckpt)) || !al16(ws))
+    return SNN_ERR_ALIGNMENT;
+  if (!ws || ws_bytes < 256) return SNN_ERR_WORKSPACE;
+  FusedArgs f{};
+  f.T = (int)d->T;
+  f.R = (int)d->B;
+  f.K = (int)K;
+  f.N = (int)d->N;
+  f.BS = (int)(128 / d->T);
+  f.reset = d->reset;
+  f.beta_col = beta_col;
+  f.thr_col = thr_col;
+  f.beta = beta;
+  f.thr = thr;
+  f.bits_row = ((d->B * d->N + 7) / 8 + 15) / 16 * 16;
+  f.status = static_cast<int*>(ws);
+  f.wait_ns = d->wait_limit_ns > 0 ? (uint64_t)d->wait_limit_ns : kDefaultWaitNs;
+  f.mem_in = static_cast<const __nv_bfloat16*>(mem);
+  f.bits_in = reinterpret_cast<const unsigned char*>(ckpt);
+  f.spk_in = static_cast<const __nv_bfloat16*>(spk);
+  f.gI = static_cast<__nv_bfloat16*>(grad_I);
+  f.sa.reset = d->reset;
+  f.sa.detach = d->detach_reset != 0;
+  f.sa.sg = d->surrogate;
+  f.sa.rec = 0;
+  if (d->surrogate == SNN_SG_FAST_SIGMOID) {
+    f.sa.sg_a = d->sg_param;
+    f.sa.sg_b = 0.0f;
+  } else {  // the same constants the scan kernels take
+    f.sa.sg_a = (float)(0.5 * (double)d->sg_param);
+    f.sa.sg_b = (float)(3.14159265358979323846 * 0.5 * (double)d->sg_param);
+  }
+  // 128-wide tiles unless 64-wide ones are needed to give the SMs a second tile
+  int bn = 128;
+  {
+    int dev = 0, sms = 152;
+    if (cudaGetDevice(&dev) == cudaSuccess) cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    const int64_t tiles128 = ((d->N + 127) / 128) * ((d->B + f.BS - 1) / f.BS);
+    if (d->N <= 64 || tiles128 < 2 * (int64_t)sms) bn = 64;
+  }
+  CUtensorMap ta, tb;
+  if (!make_map_3d(&ta, dI_up, d->T, d->B, K, f.BS, (int)d->T) || !make_map(&tb, W, K, d->N, 64))
+    return SNN_ERR_UNSUPPORTED;
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  const cudaError_t e = bn == 64 ? launch_fused_bwd<64>(ta, tb, f, st) : launch_fused_bwd<128>(ta, tb, f, st);
   return e == cudaSuccess ? SNN_OK : SNN_ERR_CUDA;
 }

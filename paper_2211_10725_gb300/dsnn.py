@@ -15,8 +15,10 @@ never fires, and its gradients are exactly 0.
 The backward recomputes each layer's membrane trace from its input current
 and checkpoints (``save="recompute"``) unless ``save="mem"`` asks for the
 bf16 trace to be stored by the forward.  ``save="fused"`` stores the trace
-too, but runs each layer's forward as one kernel: the GEMM with the Leaky
-scan in its epilogue (the currents never reach HBM).
+too, but runs each layer's forward as one kernel, the GEMM with the Leaky
+scan in its epilogue (the currents never reach HBM), and, for T > 1, each
+input-gradient product with the BPTT of the layer below in its epilogue (the
+spike gradients never reach HBM).
 """
 from __future__ import annotations
 
@@ -40,6 +42,9 @@ class DenseSNN:
         self.w = w
         self.save = save
         self.fused = save == "fused"
+        # the input-gradient GEMMs carry the lower layer's BPTT when the scan
+        # has a time chain to hide the GEMM behind (T = 1: separate kernels)
+        self.fused_bwd = self.fused and w.T > 1
         scan_save = "mem" if self.fused else save
         self.lr, self.betas, self.eps, self.weight_decay = lr, betas, eps, weight_decay
         # batch the loss is averaged over (the global batch under data
@@ -142,16 +147,25 @@ class DenseSNN:
         out.append(("ce_loss", lambda: snn.snn_rate_ce_loss(
             self.layers[-1].spk, labels, self.w.n_classes, self.loss, self.grad_out,
             self.ws_loss, stream, batch_total=self.batch_total, pop=self.w.pop)))
-        for l in range(len(self.layers) - 1, -1, -1):
-            grad = self.grad_out if l == len(self.layers) - 1 else \
-                self.grad_in[l].view(T, B, -1)
-            dX = self.grad_in[l - 1] if l > 0 else None
-            out.append((f"scan_bwd{l}", lambda l=l, grad=grad: self.layers[l].backward(
-                None if self.I[l] is None else self.I[l].view(T, B, -1), self.beta, self.thr,
-                grad, want_param_grads=False, want_state_grads=False, stream=stream)))
+        top = len(self.layers) - 1
+        for l in range(top, -1, -1):
+            grad = self.grad_out if l == top else self.grad_in[l].view(T, B, -1)
+            if l == top or not self.fused_bwd:
+                out.append((f"scan_bwd{l}", lambda l=l, grad=grad: self.layers[l].backward(
+                    None if self.I[l] is None else self.I[l].view(T, B, -1), self.beta,
+                    self.thr, grad, want_param_grads=False, want_state_grads=False,
+                    stream=stream)))
+            # fused: layer l's input gradient is the spike gradient of layer
+            # l - 1, whose BPTT runs in the epilogue of that product
+            dX = self.grad_in[l - 1] if (l > 0 and not self.fused_bwd) else None
             out.append((f"dense_bwd{l}", lambda l=l, dX=dX: snn.snn_dense_layer_bwd(
                 self.layer_input(l, X), self.W[l], self.layers[l].grad_I.view(self.M, -1), dX,
                 self.dW[l], self.ws_bwd[l], stream)))
+            if l > 0 and self.fused_bwd:
+                lo = self.layers[l - 1]
+                out.append((f"dense_scan_bwd{l}", lambda l=l, lo=lo: snn.snn_dense_leaky_bwd(
+                    lo.desc, self.layers[l].grad_I.view(self.M, -1), self.W[l], self.beta,
+                    self.thr, lo.mem, lo.spk, lo.ckpt, lo.grad_I, self.ws_fwd, stream)))
         out.append(("adamw", lambda: self.update(stream)))
         return out
 

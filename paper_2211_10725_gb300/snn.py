@@ -77,6 +77,8 @@ _SIGS = {
     "snn_dense_layer_bwd": ([ctypes.c_int64] * 3 + [_P] * 6 + [ctypes.c_size_t, _P], ctypes.c_int),
     "snn_rate_ce_workspace_bytes": ([ctypes.c_int64], ctypes.c_size_t),
     "snn_kernel_launches": ([], ctypes.c_uint64),
+    "snn_dense_leaky_bwd": ([ctypes.POINTER(ScanDesc), ctypes.c_int64] + [_P] * 9
+                            + [ctypes.c_size_t, _P], ctypes.c_int),
     "snn_dense_leaky_fwd": ([ctypes.POINTER(ScanDesc), ctypes.c_int64, ctypes.c_int64] + [_P] * 8
                             + [ctypes.c_size_t, _P], ctypes.c_int),
     "snn_conv2d_small_fwd_nhwc": ([ctypes.c_int64] * 8 + [_P] * 4, ctypes.c_int),
@@ -313,6 +315,17 @@ def snn_dense_leaky_fwd(desc, X, W, beta, thr, spk, mem, ckpt, ws, P=1, stream=N
                                               _ptr(beta), _ptr(thr), _ptr(spk), _ptr(mem),
                                               _ptr(ckpt), _ptr(ws), ws.numel() * ws.element_size(),
                                               _stream(stream)), "snn_dense_leaky_fwd")
+
+
+def snn_dense_leaky_bwd(desc, dI_up, W, beta, thr, mem, spk, ckpt, grad_I, ws, stream=None):
+    """dX = dI_up [T*B, K] @ W [K, N] on the tensor cores, and the Leaky BPTT
+    of the layer below on it in the same kernel; writes that layer's grad_I."""
+    K = dI_up.shape[-1]
+    _check(load_library().snn_dense_leaky_bwd(ctypes.byref(desc), K, _ptr(dI_up), _ptr(W),
+                                              _ptr(beta), _ptr(thr), _ptr(mem), _ptr(spk),
+                                              _ptr(ckpt), _ptr(grad_I), _ptr(ws),
+                                              ws.numel() * ws.element_size(), _stream(stream)),
+           "snn_dense_leaky_bwd")
 
 
 def snn_kernel_launches() -> int:

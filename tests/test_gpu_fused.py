@@ -1,6 +1,8 @@
 """The dense layer with its Leaky scan in the GEMM epilogue
 (snn_dense_leaky_fwd) against the oracle's GEMM followed by its Leaky
-forward, and the dense SNN step built on it.
+forward; the input-gradient GEMM with the lower layer's BPTT in its
+epilogue (snn_dense_leaky_bwd) against the oracle's product followed by its
+Leaky backward.
 
 Comparison protocol: the layer inputs are 0/1 spikes and the weights bf16
 values flushed to zero below 2^-7 in magnitude (and at most 0.25).  Every
@@ -113,4 +115,109 @@ def test_fused_argument_checks(cuda_device):
     assert call(snn.make_desc(w), P=3) == 1                            # N % P
     assert call(snn.make_desc(w.scaled(N=12))) == 3                    # Nout % 8
     assert call(snn.make_desc(w), x=buf[1:].view(-1)[:128].view(8, 16)) == 2  # alignment
+    torch.cuda.synchronize()
+
+
+# The fused backward (snn_dense_leaky_bwd): the spike gradient of the lower
+# layer is dI_up @ W computed on the tensor cores and never stored; its BPTT
+# runs on the stored bf16 trace.  dI_up is k/16 (|k| <= 16) and W is k/1024
+# (|k| < 256): every product is a multiple of 2^-14 and every partial sum of
+# at most 1024 of them stays below 2^8, so the spike gradient is exact in fp32
+# and the oracle's float64 BPTT on the same stored state is the reference,
+# within the bf16 storage tolerance of grad_I.
+# T, B, K (upper neurons), N (lower neurons), reset, parameter mode, surrogate,
+# detached reset, spike source
+BWD_CASES = [
+    (25, 16, 128, 64, "subtract", "scalar", "fast_sigmoid", True, "bits"),
+    (25, 128, 1000, 1000, "subtract", "scalar", "fast_sigmoid", True, "bits"),  # DSNN 1000-1000
+    (25, 128, 16, 1000, "subtract", "scalar", "fast_sigmoid", True, "bits"),    # under the readout
+    (1, 128, 1000, 3072, "subtract", "scalar", "fast_sigmoid", True, "bits"),   # T = 1
+    (3, 7, 40, 64, "zero", "per_neuron", "atan", False, "spk"),
+    (128, 3, 24, 32, "none", "per_neuron", "fast_sigmoid", True, "bits"),       # one row per tile
+    (7, 19, 136, 200, "subtract", "scalar", "atan", False, "bits"),             # ragged tiles
+    (5, 33, 64, 328, "zero", "scalar", "fast_sigmoid", False, "spk"),
+]
+
+
+def _pack_bits(z, T, L):
+    """Spike bits as the store-mode BPTT reads them (bit k of byte j of row t
+    is z_t of lane 8j + k; rows padded to 16 bytes)."""
+    row = ((L + 7) // 8 + 15) // 16 * 16
+    out = np.zeros((T, row), dtype=np.uint8)
+    out[:, : (L + 7) // 8] = np.packbits(z.astype(np.uint8), axis=1, bitorder="little")
+    return torch.from_numpy(out.reshape(-1)).view(torch.float32)
+
+
+@pytest.mark.parametrize("T,B,K,N,reset,mode,sg,detach,src", BWD_CASES)
+def test_fused_backward_matches_oracle(T, B, K, N, reset, mode, sg, detach, src, cuda_device):
+    g = torch.Generator().manual_seed(7 * T + 13 * B + K + 3 * N)
+    L = B * N
+    dI_up = (torch.randint(-16, 17, (T * B, K), generator=g).float() / 16).to(torch.bfloat16)
+    Wt = (torch.randint(-255, 256, (K, N), generator=g).float() / 1024).to(torch.bfloat16)
+    per = mode != "scalar"
+    beta = (0.8 + 0.19 * torch.rand(N if per else 1, generator=g)).float()
+    thr = (0.7 + 0.6 * torch.rand(N if per else 1, generator=g)).float()
+    # a stored trace near the threshold and spikes mostly consistent with it
+    mem = (torch.randn((T, B, N), generator=g) * 0.6 + 0.9).to(torch.bfloat16)
+    lanes_t = O.lane_param(thr.numpy(), B, N, mode, N, 1)
+    lanes_b = O.lane_param(beta.numpy(), B, N, mode, N, 1)
+    z = (_np(mem).reshape(T, L) > lanes_t[None, :]).astype(np.float64)
+    flip = torch.rand((T, L), generator=g).numpy() < 0.02
+    z[flip] = 1 - z[flip]
+    w = W.ScanWorkload(name="fused_bwd", neuron="leaky", T=T, B=B, N=N, C=N, HW=1,
+                       in_dtype=W.F32, io_dtype=W.BF16, beta_mode=mode, thr_mode=mode,
+                       reset=reset, surrogate=sg, sg_param=25.0 if sg == "fast_sigmoid" else 2.0,
+                       detach_reset=detach, save="mem", want_mem=True)
+    desc = snn.make_desc(w)
+    spk = torch.from_numpy(z.reshape(T, B, N)).to(torch.bfloat16)
+    ckpt = _pack_bits(z, T, L).to(cuda_device) if src == "bits" else None
+    gI = torch.full((T, B, N), float("nan"), dtype=torch.bfloat16, device=cuda_device)
+    ws = torch.zeros(256, dtype=torch.uint8, device=cuda_device)
+    snn.snn_dense_leaky_bwd(desc, dI_up.to(cuda_device), Wt.to(cuda_device), beta.to(cuda_device),
+                            thr.to(cuda_device), mem.to(cuda_device),
+                            spk.to(cuda_device) if src == "spk" else None, ckpt, gI, ws)
+    torch.cuda.synchronize()
+    assert snn.snn_workspace_status(ws) == 0
+    gs = (_np(dI_up) @ _np(Wt)).reshape(T, L)
+    assert np.array_equal(gs.astype(np.float32).astype(np.float64), gs)  # exact sums
+    kw = dict(reset=reset, detach=detach, sg=sg, sg_param=w.sg_param)
+    ref = O.leaky_backward(_np(mem).reshape(T, L), z, gs, lanes_b, lanes_t, **kw)["grad_I"]
+    scale = np.maximum(np.abs(ref), O.leaky_backward(_np(mem).reshape(T, L), z, np.abs(gs),
+                                                     lanes_b, lanes_t, **kw)["grad_I"])
+    got = _np(gI).reshape(T, L)
+    assert np.isfinite(got).all()
+    lim = 1e-3 + 2e-2 * scale
+    bad = np.abs(got - ref) > lim
+    assert not bad.any(), f"{bad.sum()} of {bad.size} beyond tolerance"
+    assert np.abs(ref).max() > 0
+
+
+def test_fused_backward_argument_checks(cuda_device):
+    w = W.ScanWorkload(name="fused_bwd", neuron="leaky", T=4, B=2, N=16, in_dtype=W.F32,
+                       io_dtype=W.BF16, save="mem", want_mem=True)
+    buf = torch.zeros(1 << 16, dtype=torch.float32, device=cuda_device)
+    dI = buf[:8 * 16].view(8, 16).to(torch.bfloat16)
+    Wt = torch.zeros((16, 16), dtype=torch.bfloat16, device=cuda_device)
+    p = torch.ones(1, device=cuda_device)
+    mem = torch.zeros((4, 2, 16), dtype=torch.bfloat16, device=cuda_device)
+    gI = torch.empty_like(mem)
+    ws = torch.zeros(256, dtype=torch.uint8, device=cuda_device)
+    lib = snn.load_library()
+
+    def call(desc, K=16, spk=mem, ckpt=None, dI_up=dI):
+        return lib.snn_dense_leaky_bwd(ctypes.byref(desc), K, dI_up.data_ptr(), Wt.data_ptr(),
+                                       p.data_ptr(), p.data_ptr(), mem.data_ptr(),
+                                       None if spk is None else spk.data_ptr(),
+                                       None if ckpt is None else ckpt.data_ptr(),
+                                       gI.data_ptr(), ws.data_ptr(), 256, None)
+
+    assert call(snn.make_desc(w)) == 0
+    assert call(snn.make_desc(w), spk=None) == 1                        # no spike source
+    assert call(snn.make_desc(w.scaled(save="recompute"))) == 3
+    assert call(snn.make_desc(w.scaled(io_dtype=W.F32))) == 3
+    assert call(snn.make_desc(w.scaled(T=129))) == 3
+    assert call(snn.make_desc(w), K=12) == 3                            # K % 8
+    assert call(snn.make_desc(w.scaled(N=12))) == 3                     # N % 8
+    assert call(snn.make_desc(w.scaled(beta_mode="per_channel", C=4, HW=4))) == 3
+    assert call(snn.make_desc(w), dI_up=buf[1:].view(-1)[:128].view(8, 16)) == 2  # alignment
     torch.cuda.synchronize()
