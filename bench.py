@@ -623,7 +623,10 @@ def conv_op_bytes(net):
         out["fc_fwd"] = flat + nb(net.W[-1]) + nb(net.I_fc)
         out["scan_fwd_out"] = f * ns
     out["ce_loss"] = nb(o.spk) + nb(net.grad_out)
-    out["scan_bwd_out"] = b * ns
+    if net.fused_loss:   # the readout's BPTT in the loss launch: its trace in, dL/dI out
+        out["ce_loss"] += nb(o.mem) + nb(o.grad_I)
+    else:
+        out["scan_bwd_out"] = b * ns
     out["fc_bwd"] = flat + nb(net.W[-1]) + nb(o.grad_I) + nb(net.grad_pool[-1]) + nb(net.dW[-1])
     out["adamw"] = (4 * 2 * nb(net.W32_flat) + nb(net.W_flat)
                     + 4 * 2 * nb(net.beta_flat))

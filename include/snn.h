@@ -338,6 +338,31 @@ snn_status_t snn_rate_ce_loss(int64_t T, int64_t B, int64_t C, int64_t pop, int6
                               size_t ws_bytes, snn_stream_t stream);
 
 /*
+ * The rate-coded loss of snn_rate_ce_loss fused with the BPTT of the
+ * readout layer that produced spk (a Leaky layer, Eq. 4; reverse pass of
+ * Sec. III-B): the spike gradient of every output neuron is the loss
+ * gradient above, and the same launch runs the neuron's reverse scan on the
+ * stored trace and writes its dL/dI.
+ *   desc  the readout layer: T, B, N = ld neurons per sample, io_dtype (any),
+ *         save SNN_SAVE_MEM, any reset, detach and surrogate; beta_mode and
+ *         thr_mode scalar or per neuron (of ld)
+ *   C, pop, batch_total, labels, loss, ws   as for snn_rate_ce_loss
+ *   spk   [T, B, ld] the layer's spikes (io dtype); also the spike decisions
+ *         of the reverse scan unless ckpt is given
+ *   mem   [T, B, ld] the layer's stored membrane trace (io dtype)
+ *   ckpt  the spike bits its store-mode forward wrote, or NULL
+ *   grad_spk [T, B, ld] (out, nullable): the loss gradient, as written by
+ *         snn_rate_ce_loss
+ *   grad_I [T, B, ld] (out): the readout's dL/dI (io dtype)
+ * No parameter or initial-state gradients (snn_leaky_bwd gives those).
+ */
+snn_status_t snn_rate_ce_leaky_bwd(const snn_scan_desc* desc, int64_t C, int64_t pop,
+                                   int64_t batch_total, const void* spk, const int32_t* labels,
+                                   const float* beta, const float* thr, const void* mem,
+                                   const float* ckpt, float* loss, void* grad_spk, void* grad_I,
+                                   void* ws, size_t ws_bytes, snn_stream_t stream);
+
+/*
  * Dense layer fused with its Leaky scan (Fig. 3's synaptic operation w.x
  * feeding Eqs. 3-4): the currents of all T steps come out of one tcgen05
  * GEMM and are scanned in its epilogue, so they never reach HBM.

@@ -162,6 +162,7 @@ class ConvSNN:
                             thr=("const", w.thr), reset=w.reset, surrogate="fast_sigmoid",
                             sg_param=w.sg_param, save=scan_save, want_mem=scan_save == "mem")
         self.out_layer = snn.ScanLayer(fw, device=dev)
+        self.fused_loss = scan_save == "mem"
         self.ws_fwd = torch.zeros(256, dtype=torch.uint8, device=dev)
         self.ws_bwd.append(torch.zeros(snn.snn_dense_workspace_bytes(M, self.n_flat, self.n_out),
                                        dtype=torch.uint8, device=dev))
@@ -218,12 +219,19 @@ class ConvSNN:
                                                                    self.ws_fwd, stream)))
             out.append(("scan_fwd_out", lambda: self.out_layer.forward(
                 self.I_fc.view(T, B, -1), self.beta_fc, self.thr, stream=stream)))
-        out.append(("ce_loss", lambda: snn.snn_rate_ce_loss(
-            self.out_layer.spk, labels, self.w.n_classes, self.loss, self.grad_out,
-            self.ws_loss, stream, batch_total=self.batch_total)))
-        out.append(("scan_bwd_out", lambda: self.out_layer.backward(
-            None if self.I_fc is None else self.I_fc.view(T, B, -1), self.beta_fc, self.thr,
-            self.grad_out, want_param_grads=False, want_state_grads=False, stream=stream)))
+        o = self.out_layer
+        if self.fused_loss:  # the readout's trace is stored: its BPTT in the loss launch
+            out.append(("ce_loss", lambda: snn.snn_rate_ce_leaky_bwd(
+                o.desc, o.spk, labels, self.w.n_classes, self.beta_fc, self.thr, o.mem, None,
+                self.loss, self.grad_out, o.grad_I, self.ws_loss, stream,
+                batch_total=self.batch_total)))
+        else:
+            out.append(("ce_loss", lambda: snn.snn_rate_ce_loss(
+                o.spk, labels, self.w.n_classes, self.loss, self.grad_out, self.ws_loss, stream,
+                batch_total=self.batch_total)))
+            out.append(("scan_bwd_out", lambda: o.backward(
+                None if self.I_fc is None else self.I_fc.view(T, B, -1), self.beta_fc, self.thr,
+                self.grad_out, want_param_grads=False, want_state_grads=False, stream=stream)))
         out.append(("fc_bwd", lambda: snn.snn_dense_layer_bwd(
             flat, self.W[L], self.out_layer.grad_I.view(M, -1),
             self.grad_pool[-1].view(M, -1), self.dW[L], self.ws_bwd[L], stream)))

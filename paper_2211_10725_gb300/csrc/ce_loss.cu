@@ -22,6 +22,11 @@
 // published) adds the B loss terms in sample order: deterministic.  The
 // softmax runs in float (double arithmetic is slow on this part); the loss
 // terms and their sum are in double.
+//
+// With the readout's BPTT (snn_rate_ce_leaky_bwd), step 4 also runs the
+// output layer's reverse scan (Sec. III-B) for each of the sample's neurons
+// on its stored trace: the spike gradient is the constant of step 3, so
+// dL/dI of the readout comes out of the same launch.
 #include <cuda_bf16.h>
 #include <cuda_fp16.h>
 #include <cuda_runtime.h>
@@ -48,12 +53,27 @@ __device__ __forceinline__ float warp_sum(float v) {
   return v;
 }
 
+// The readout layer's stored state and parameters for the fused BPTT.
 template <typename T>
+struct ReadoutBptt {
+  ScanArgs sa;            // reset, detach and surrogate of bwd_step
+  const float* beta;      // scalar (beta_col 0) or one per neuron of ld
+  const float* thr;
+  int beta_col, thr_col;
+  const T* mem;           // [T, B, ld] stored trace
+  const unsigned char* bits;  // spike bits (store-mode layout), or null: z from spk
+  int64_t bits_row;
+  T* gI;                  // [T, B, ld] dL/dI
+};
+
+constexpr int kCeChunk = 8;  // steps of stored trace loaded ahead
+
+template <typename T, bool BPTT>
 __global__ void __launch_bounds__(kCeThreads) rate_ce_kernel(int64_t Tn, int64_t B, int C,
                                                              int pop, int64_t ld, int64_t Bn,
                                                              const T* spk, const int* labels,
                                                              float* loss, T* grad, double* terms,
-                                                             int* ticket) {
+                                                             int* ticket, const ReadoutBptt<T> r) {
   extern __shared__ __align__(16) float ce_smem[];
   const int CP = C * pop;
   float* ncnt = ce_smem;       // [CP] neuron counts
@@ -106,10 +126,42 @@ __global__ void __launch_bounds__(kCeThreads) rate_ce_kernel(int64_t Tn, int64_t
       ccnt[c] = (expf(ccnt[c] - m) / se - (c == y ? 1.0f : 0.0f)) * inv_b;
   }
   __syncthreads();
-  T* grow = grad + b * ld;
-  for (int64_t n = threadIdx.x; n < ld; n += kCeThreads) {
-    const float g = n < CP ? ccnt[n / pop] : 0.0f;
-    for (int64_t t = 0; t < Tn; ++t) Elem<T>::store1(grow + t * step + n, g);
+  if constexpr (BPTT) {
+    // neuron n of sample b is lane b*ld + n of every step
+    for (int64_t n = threadIdx.x; n < ld; n += kCeThreads) {
+      const float g = n < CP ? ccnt[n / pop] : 0.0f;
+      const int64_t lane = b * ld + n;
+      const float beta = __ldg(r.beta + (r.beta_col ? n : 0));
+      const float thr = __ldg(r.thr + (r.thr_col ? n : 0));
+      BwdLane st{0.0f, 0.0f, 0.0f, 0.0f, 0.0f};
+      for (int64_t tc = Tn - 1; tc >= 0; tc -= kCeChunk) {
+        float uu[kCeChunk];
+        uint32_t zz = 0;  // bit c: z at step tc - c
+#pragma unroll
+        for (int c = 0; c < kCeChunk; ++c) {
+          const int64_t ts = tc - c >= 0 ? tc - c : 0;  // steps before 0 reload step 0, unused
+          uu[c] = Elem<T>::load1(r.mem + ts * step + lane);
+          const uint32_t z = r.bits ? (__ldg(r.bits + ts * r.bits_row + (lane >> 3)) >> (lane & 7)) & 1u
+                                    : (Elem<T>::load1(spk + ts * step + lane) != 0.0f ? 1u : 0u);
+          zz |= z << c;
+        }
+#pragma unroll
+        for (int c = 0; c < kCeChunk; ++c) {
+          const int64_t ts = tc - c;
+          if (ts < 0) break;
+          const float du = bwd_step<false, -1, -1>(r.sa, beta, thr, 0.0f, ts + 1 < Tn, uu[c],
+                                                   ((zz >> c) & 1u) != 0, 0.0f, g, 0.0f, 0.0f, st);
+          Elem<T>::store1(r.gI + ts * step + lane, du);
+          if (grad) Elem<T>::store1(grad + ts * step + lane, g);
+        }
+      }
+    }
+  } else {
+    T* grow = grad + b * ld;
+    for (int64_t n = threadIdx.x; n < ld; n += kCeThreads) {
+      const float g = n < CP ? ccnt[n / pop] : 0.0f;
+      for (int64_t t = 0; t < Tn; ++t) Elem<T>::store1(grow + t * step + n, g);
+    }
   }
   // the last block to finish adds the loss terms in sample order
   __threadfence();
@@ -126,17 +178,46 @@ __global__ void __launch_bounds__(kCeThreads) rate_ce_kernel(int64_t Tn, int64_t
   }
 }
 
-template <typename T>
+template <typename T, bool BPTT = false>
 cudaError_t launch_ce(int64_t Tn, int64_t B, int C, int pop, int64_t ld, int64_t Bn,
                       const void* spk, const int* labels, float* loss, void* grad, double* terms,
-                      int* ticket, cudaStream_t st) {
+                      int* ticket, cudaStream_t st, const ReadoutBptt<T>& r = ReadoutBptt<T>{}) {
   const size_t smem = (size_t)(C * pop + C) * sizeof(float);
-  const void* k = (const void*)rate_ce_kernel<T>;
+  const void* k = (const void*)rate_ce_kernel<T, BPTT>;
   const cudaError_t e = ensure_smem(k, smem);
   if (e != cudaSuccess) return e;
-  return launch_pdl(rate_ce_kernel<T>, dim3((unsigned)B), dim3(kCeThreads), smem, st, Tn, B, C,
-                    pop, ld, Bn, static_cast<const T*>(spk), labels, loss, static_cast<T*>(grad),
-                    terms, ticket);
+  return launch_pdl(rate_ce_kernel<T, BPTT>, dim3((unsigned)B), dim3(kCeThreads), smem, st, Tn,
+                    B, C, pop, ld, Bn, static_cast<const T*>(spk), labels, loss,
+                    static_cast<T*>(grad), terms, ticket, r);
+}
+
+template <typename T>
+cudaError_t launch_ce_bptt(const snn_scan_desc* d, int C, int pop, int64_t Bn, const void* spk,
+                           const int* labels, const float* beta, const float* thr, int beta_col,
+                           int thr_col, const void* mem, const void* bits, float* loss,
+                           void* grad, void* gI, double* terms, int* ticket, cudaStream_t st) {
+  ReadoutBptt<T> r{};
+  r.sa.reset = d->reset;
+  r.sa.detach = d->detach_reset != 0;
+  r.sa.sg = d->surrogate;
+  r.sa.rec = 0;
+  if (d->surrogate == SNN_SG_FAST_SIGMOID) {
+    r.sa.sg_a = d->sg_param;
+    r.sa.sg_b = 0.0f;
+  } else {  // the constants the scan kernels take
+    r.sa.sg_a = (float)(0.5 * (double)d->sg_param);
+    r.sa.sg_b = (float)(3.14159265358979323846 * 0.5 * (double)d->sg_param);
+  }
+  r.beta = beta;
+  r.thr = thr;
+  r.beta_col = beta_col;
+  r.thr_col = thr_col;
+  r.mem = static_cast<const T*>(mem);
+  r.bits = static_cast<const unsigned char*>(bits);
+  r.bits_row = ((d->B * d->N + 7) / 8 + 15) / 16 * 16;
+  r.gI = static_cast<T*>(gI);
+  return launch_ce<T, true>(d->T, d->B, C, pop, d->N, Bn, spk, labels, loss, grad, terms, ticket,
+                            st, r);
 }
 
 }  // namespace
@@ -179,6 +260,65 @@ extern "C" snn_status_t snn_rate_ce_loss(int64_t T, int64_t B, int64_t C, int64_
     default:
       e = snn::launch_ce<__half>(T, B, (int)C, (int)pop, ld, Bn, spk, labels, loss, grad_spk,
                                  terms, ticket, st);
+  }
+  return e == cudaSuccess ? SNN_OK : SNN_ERR_CUDA;
+}
+
+extern "C" snn_status_t snn_rate_ce_leaky_bwd(const snn_scan_desc* d, int64_t C, int64_t pop,
+                                              int64_t batch_total, const void* spk,
+                                              const int32_t* labels, const float* beta,
+                                              const float* thr, const void* mem,
+                                              const float* ckpt, float* loss, void* grad_spk,
+                                              void* grad_I, void* ws, size_t ws_bytes,
+                                              snn_stream_t stream) {
+  if (!d || d->T < 0 || d->B < 0 || d->B > INT_MAX || d->N < 1 || d->reserved0 != 0 ||
+      d->reserved1 != 0)
+    return SNN_ERR_INVALID_ARG;
+  if (C < 1 || pop < 1 || C > snn::kMaxClasses || pop > snn::kCeMaxNeurons / C || d->N < C * pop)
+    return SNN_ERR_INVALID_ARG;
+  if (d->reset < SNN_RESET_SUBTRACT || d->reset > SNN_RESET_NONE) return SNN_ERR_INVALID_ARG;
+  if (d->surrogate != SNN_SG_FAST_SIGMOID && d->surrogate != SNN_SG_ATAN) return SNN_ERR_INVALID_ARG;
+  if (!(d->sg_param > 0.0f)) return SNN_ERR_INVALID_ARG;
+  if (d->io_dtype != SNN_F32 && d->io_dtype != SNN_BF16 && d->io_dtype != SNN_F16)
+    return SNN_ERR_INVALID_ARG;
+  if (d->save != SNN_SAVE_MEM) return SNN_ERR_UNSUPPORTED;
+  int beta_col = 0, thr_col = 0;
+  auto col_mode = [](int32_t mode, int* col) {
+    if (mode == SNN_P_SCALAR) { *col = 0; return true; }
+    if (mode == SNN_P_PER_NEURON) { *col = 1; return true; }
+    return false;
+  };
+  if (!col_mode(d->beta_mode, &beta_col) || !col_mode(d->thr_mode, &thr_col)) return SNN_ERR_UNSUPPORTED;
+  const int64_t Bn = batch_total > 0 ? batch_total : (d->B > 0 ? d->B : 1);
+  if (batch_total > 0 && batch_total < d->B) return SNN_ERR_INVALID_ARG;
+  const bool work = d->T > 0 && d->B > 0;
+  if (!loss || (work && (!spk || !labels || !beta || !thr || !mem || !grad_I)))
+    return SNN_ERR_INVALID_ARG;
+  auto al16 = [](const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; };
+  if (!al16(spk) || !al16(mem) || !al16(grad_I) || !al16(grad_spk) || !al16(ckpt) || !al16(ws))
+    return SNN_ERR_ALIGNMENT;
+  if (!ws || ws_bytes < snn_rate_ce_workspace_bytes(d->B)) return SNN_ERR_WORKSPACE;
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  if (d->B == 0)
+    return cudaMemsetAsync(loss, 0, sizeof(float), st) == cudaSuccess ? SNN_OK : SNN_ERR_CUDA;
+  unsigned char* w = static_cast<unsigned char*>(ws);
+  int* ticket = reinterpret_cast<int*>(w);
+  double* terms = reinterpret_cast<double*>(w + 256);
+  cudaError_t e;
+  switch (d->io_dtype) {
+    case SNN_F32:
+      e = snn::launch_ce_bptt<float>(d, (int)C, (int)pop, Bn, spk, labels, beta, thr, beta_col,
+                                     thr_col, mem, ckpt, loss, grad_spk, grad_I, terms, ticket, st);
+      break;
+    case SNN_BF16:
+      e = snn::launch_ce_bptt<__nv_bfloat16>(d, (int)C, (int)pop, Bn, spk, labels, beta, thr,
+                                             beta_col, thr_col, mem, ckpt, loss, grad_spk, grad_I,
+                                             terms, ticket, st);
+      break;
+    default:
+      e = snn::launch_ce_bptt<__half>(d, (int)C, (int)pop, Bn, spk, labels, beta, thr, beta_col,
+                                      thr_col, mem, ckpt, loss, grad_spk, grad_I, terms, ticket,
+                                      st);
   }
   return e == cudaSuccess ? SNN_OK : SNN_ERR_CUDA;
 }

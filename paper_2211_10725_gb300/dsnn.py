@@ -18,7 +18,8 @@ bf16 trace to be stored by the forward.  ``save="fused"`` stores the trace
 too, but runs each layer's forward as one kernel, the GEMM with the Leaky
 scan in its epilogue (the currents never reach HBM), and, for T > 1, each
 input-gradient product with the BPTT of the layer below in its epilogue (the
-spike gradients never reach HBM).
+spike gradients never reach HBM).  Whenever the readout's trace is stored, the
+loss launch also runs the readout's BPTT.
 """
 from __future__ import annotations
 
@@ -46,6 +47,8 @@ class DenseSNN:
         # has a time chain to hide the GEMM behind (T = 1: separate kernels)
         self.fused_bwd = self.fused and w.T > 1
         scan_save = "mem" if self.fused else save
+        # with the readout's trace stored, the loss launch also runs its BPTT
+        self.fused_loss = scan_save == "mem"
         self.lr, self.betas, self.eps, self.weight_decay = lr, betas, eps, weight_decay
         # batch the loss is averaged over (the global batch under data
         # parallelism; None: this replica's batch)
@@ -144,13 +147,20 @@ class DenseSNN:
                 self.layer_input(l, X), self.W[l], self.I[l], self.ws_fwd, stream)))
             out.append((f"scan_fwd{l}", lambda l=l, layer=layer: layer.forward(
                 self.I[l].view(T, B, -1), self.beta, self.thr, stream=stream)))
-        out.append(("ce_loss", lambda: snn.snn_rate_ce_loss(
-            self.layers[-1].spk, labels, self.w.n_classes, self.loss, self.grad_out,
-            self.ws_loss, stream, batch_total=self.batch_total, pop=self.w.pop)))
         top = len(self.layers) - 1
+        o = self.layers[top]
+        if self.fused_loss:
+            out.append(("ce_loss", lambda: snn.snn_rate_ce_leaky_bwd(
+                o.desc, o.spk, labels, self.w.n_classes, self.beta, self.thr, o.mem, None,
+                self.loss, self.grad_out, o.grad_I, self.ws_loss, stream,
+                batch_total=self.batch_total, pop=self.w.pop)))
+        else:
+            out.append(("ce_loss", lambda: snn.snn_rate_ce_loss(
+                o.spk, labels, self.w.n_classes, self.loss, self.grad_out, self.ws_loss, stream,
+                batch_total=self.batch_total, pop=self.w.pop)))
         for l in range(top, -1, -1):
             grad = self.grad_out if l == top else self.grad_in[l].view(T, B, -1)
-            if l == top or not self.fused_bwd:
+            if (l == top and not self.fused_loss) or (l < top and not self.fused_bwd):
                 out.append((f"scan_bwd{l}", lambda l=l, grad=grad: self.layers[l].backward(
                     None if self.I[l] is None else self.I[l].view(T, B, -1), self.beta,
                     self.thr, grad, want_param_grads=False, want_state_grads=False,

@@ -91,6 +91,8 @@ _SIGS = {
     "snn_maxpool2_bwd_nhwc": ([ctypes.c_int64] * 4 + [_P] * 4, ctypes.c_int),
     "snn_rate_ce_loss": ([ctypes.c_int64] * 6 + [ctypes.c_int32] + [_P] * 5 + [ctypes.c_size_t, _P],
                          ctypes.c_int),
+    "snn_rate_ce_leaky_bwd": ([ctypes.POINTER(ScanDesc)] + [ctypes.c_int64] * 3 + [_P] * 10
+                              + [ctypes.c_size_t, _P], ctypes.c_int),
     "snn_adamw_step": ([ctypes.c_int64] + [_P] * 5 + [ctypes.c_float] * 5 + [ctypes.c_int64] +
                        [_P, _P], ctypes.c_int),
 }
@@ -290,6 +292,19 @@ def snn_rate_ce_loss(spk, labels, C, loss, grad_spk, ws=None, stream=None, batch
                                            _ptr(labels), _ptr(loss), _ptr(grad_spk), _ptr(ws),
                                            ws.numel() * ws.element_size(), _stream(stream)),
            "snn_rate_ce_loss")
+
+
+def snn_rate_ce_leaky_bwd(desc, spk, labels, C, beta, thr, mem, ckpt, loss, grad_spk, grad_I,
+                          ws, stream=None, batch_total=None, pop=1):
+    """snn_rate_ce_loss with the readout layer's BPTT in the same launch:
+    writes loss, grad_I [T, B, ld] and (unless None) grad_spk.  ckpt: the
+    forward's spike bits, or None to take the spike decisions from spk."""
+    _check(load_library().snn_rate_ce_leaky_bwd(ctypes.byref(desc), C, pop, batch_total or 0,
+                                                _ptr(spk), _ptr(labels), _ptr(beta), _ptr(thr),
+                                                _ptr(mem), _ptr(ckpt), _ptr(loss), _ptr(grad_spk),
+                                                _ptr(grad_I), _ptr(ws),
+                                                ws.numel() * ws.element_size(), _stream(stream)),
+           "snn_rate_ce_leaky_bwd")
 
 
 def snn_adamw_step(w, w_bf16, grad, m, v, lr, beta1=0.9, beta2=0.999, eps=1e-8,

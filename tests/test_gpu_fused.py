@@ -2,7 +2,8 @@
 (snn_dense_leaky_fwd) against the oracle's GEMM followed by its Leaky
 forward; the input-gradient GEMM with the lower layer's BPTT in its
 epilogue (snn_dense_leaky_bwd) against the oracle's product followed by its
-Leaky backward.
+Leaky backward; the rate-coded loss with the readout's BPTT in the same
+launch (snn_rate_ce_leaky_bwd) against the oracle's loss and Leaky backward.
 
 Comparison protocol: the layer inputs are 0/1 spikes and the weights bf16
 values flushed to zero below 2^-7 in magnitude (and at most 0.25).  Every
@@ -220,4 +221,99 @@ def test_fused_backward_argument_checks(cuda_device):
     assert call(snn.make_desc(w.scaled(N=12))) == 3                     # N % 8
     assert call(snn.make_desc(w.scaled(beta_mode="per_channel", C=4, HW=4))) == 3
     assert call(snn.make_desc(w), dI_up=buf[1:].view(-1)[:128].view(8, 16)) == 2  # alignment
+    torch.cuda.synchronize()
+
+
+# The rate-coded loss with the readout's BPTT in the same launch
+# (snn_rate_ce_leaky_bwd) against the oracle's loss followed by its Leaky
+# backward on the same stored state.
+# T, B, C, pop, ld, reset, parameter mode, surrogate, detached reset, io dtype, spike source
+CE_CASES = [
+    (25, 128, 10, 1, 16, "subtract", "scalar", "fast_sigmoid", True, torch.bfloat16, "spk"),
+    (25, 128, 10, 1, 16, "subtract", "scalar", "fast_sigmoid", True, torch.bfloat16, "bits"),
+    (1, 128, 10, 50, 504, "subtract", "scalar", "fast_sigmoid", True, torch.bfloat16, "spk"),
+    (7, 37, 13, 7, 96, "zero", "per_neuron", "atan", False, torch.float32, "spk"),
+    (30, 5, 3, 1, 8, "none", "per_neuron", "fast_sigmoid", False, torch.bfloat16, "bits"),
+    (9, 300, 100, 1, 104, "subtract", "scalar", "atan", False, torch.float32, "bits"),
+]
+
+
+@pytest.mark.parametrize("T,B,C,pop,ld,reset,mode,sg,detach,dtype,src", CE_CASES)
+def test_rate_ce_with_readout_bptt(T, B, C, pop, ld, reset, mode, sg, detach, dtype, src,
+                                   cuda_device):
+    g = torch.Generator().manual_seed(T + 3 * B + C + ld)
+    L = B * ld
+    spk = (torch.rand((T, B, ld), generator=g) < 0.3).to(dtype)
+    spk[:, :, C * pop:] = 0
+    mem = (torch.randn((T, B, ld), generator=g) * 0.6 + 0.9).to(dtype)
+    labels = torch.randint(0, C, (B,), generator=g, dtype=torch.int32)
+    per = mode != "scalar"
+    beta = (0.8 + 0.19 * torch.rand(ld if per else 1, generator=g)).float()
+    thr = (0.7 + 0.6 * torch.rand(ld if per else 1, generator=g)).float()
+    w = W.ScanWorkload(name="readout", neuron="leaky", T=T, B=B, N=ld, C=ld, HW=1,
+                       in_dtype=W.F32, io_dtype=W.BF16 if dtype == torch.bfloat16 else W.F32,
+                       beta_mode=mode, thr_mode=mode, reset=reset, surrogate=sg,
+                       sg_param=25.0 if sg == "fast_sigmoid" else 2.0, detach_reset=detach,
+                       save="mem", want_mem=True)
+    z = _np(spk).reshape(T, L)
+    d = lambda t: t.to(cuda_device)
+    ckpt = d(_pack_bits(z, T, L)) if src == "bits" else None
+    loss = torch.zeros(1, dtype=torch.float32, device=cuda_device)
+    gs = torch.full((T, B, ld), float("nan"), dtype=dtype, device=cuda_device)
+    gI = torch.full((T, B, ld), float("nan"), dtype=dtype, device=cuda_device)
+    ws = torch.zeros(snn.snn_rate_ce_workspace_bytes(B), dtype=torch.uint8, device=cuda_device)
+    spk_in = d(spk)
+    if src == "bits":   # the spike decisions must come from the bits: spk keeps the counts only
+        assert np.array_equal(_np(spk_in.cpu()).reshape(T, L), z)
+    snn.snn_rate_ce_leaky_bwd(snn.make_desc(w), spk_in, d(labels), C, d(beta), d(thr), d(mem),
+                              ckpt, loss, gs, gI, ws, pop=pop)
+    torch.cuda.synchronize()
+    rl, rg = O.rate_ce_loss(_np(spk[:, :, :C * pop]), labels.numpy(), pop)
+    assert abs(loss.item() - rl) <= 1e-6 * max(1.0, abs(rl))
+    full = np.zeros((T, B, ld))
+    full[:, :, :C * pop] = rg
+    got_gs = _np(gs.cpu())
+    assert np.all(got_gs[:, :, C * pop:] == 0)
+    rtol = 1e-5 if dtype == torch.float32 else 2e-2
+    np.testing.assert_allclose(got_gs, full, rtol=rtol, atol=1e-7 * np.abs(rg).max())
+    lanes_b = O.lane_param(beta.numpy(), B, ld, mode, ld, 1)
+    lanes_t = O.lane_param(thr.numpy(), B, ld, mode, ld, 1)
+    kw = dict(reset=reset, detach=detach, sg=sg, sg_param=w.sg_param)
+    m = _np(mem).reshape(T, L)
+    ref = O.leaky_backward(m, z, full.reshape(T, L), lanes_b, lanes_t, **kw)["grad_I"]
+    scale = np.maximum(np.abs(ref), O.leaky_backward(m, z, np.abs(full.reshape(T, L)), lanes_b,
+                                                     lanes_t, **kw)["grad_I"])
+    got = _np(gI.cpu()).reshape(T, L)
+    assert np.isfinite(got).all()
+    floor = (1e-6 if dtype == torch.float32 else 1e-3) * np.abs(ref).max()
+    bad = np.abs(got - ref) > floor + rtol * scale
+    assert not bad.any(), f"{bad.sum()} of {bad.size} beyond tolerance"
+    assert np.abs(ref).max() > 0
+
+
+def test_rate_ce_with_readout_bptt_argument_checks(cuda_device):
+    T, B, C, ld = 4, 2, 3, 8
+    w = W.ScanWorkload(name="readout", neuron="leaky", T=T, B=B, N=ld, in_dtype=W.F32,
+                       io_dtype=W.BF16, save="mem", want_mem=True)
+    buf = torch.zeros(1 << 12, dtype=torch.float32, device=cuda_device)
+    p = torch.ones(1, device=cuda_device)
+    lab = torch.zeros(B, dtype=torch.int32, device=cuda_device)
+    out = torch.zeros(1, dtype=torch.float32, device=cuda_device)   # the loss
+    ws = torch.zeros(snn.snn_rate_ce_workspace_bytes(B), dtype=torch.uint8, device=cuda_device)
+    lib = snn.load_library()
+    x = buf.data_ptr()
+
+    def call(desc, C=C, pop=1, total=0, spk=x, nbytes=None):
+        return lib.snn_rate_ce_leaky_bwd(ctypes.byref(desc), C, pop, total, spk, lab.data_ptr(),
+                                         p.data_ptr(), p.data_ptr(), x + 1024, None, out.data_ptr(),
+                                         x + 2048, x + 3072, ws.data_ptr(),
+                                         ws.numel() if nbytes is None else nbytes, None)
+
+    assert call(snn.make_desc(w)) == 0
+    assert call(snn.make_desc(w), C=5, pop=2) == 1                      # C*pop > ld
+    assert call(snn.make_desc(w), total=1) == 1                        # batch_total < B
+    assert call(snn.make_desc(w.scaled(save="recompute"))) == 3        # needs the stored trace
+    assert call(snn.make_desc(w.scaled(beta_mode="per_channel", C=2, HW=4))) == 3
+    assert call(snn.make_desc(w), spk=x + 2) == 2                       # alignment
+    assert call(snn.make_desc(w), nbytes=64) == 4                       # workspace
     torch.cuda.synchronize()
