@@ -328,7 +328,7 @@ snn_status_t snn_rleaky_bwd(const snn_scan_desc* desc, const void* I, const floa
  *   ws    device workspace of snn_rate_ce_workspace_bytes(B) bytes, 16-byte
  *         aligned, zeroed once before the first call (every call leaves its
  *         completion ticket at zero; re-zero after an error)
- * One block per sample; the loss terms are added in sample order
+ * One block per sample; the loss terms are added in a fixed order
  * (deterministic).
  */
 size_t snn_rate_ce_workspace_bytes(int64_t B);

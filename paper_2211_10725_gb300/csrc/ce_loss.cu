@@ -19,7 +19,8 @@
 //      the class counts;
 //   4. the threads write the gradient of every neuron for every t.
 // The last block to finish (a ticket taken after its loss term is
-// published) adds the B loss terms in sample order: deterministic.  The
+// published) adds the B loss terms in a fixed order (strided per thread,
+// then by warps): deterministic.  The
 // softmax runs in float (double arithmetic is slow on this part); the loss
 // terms and their sum are in double.
 //
@@ -134,26 +135,37 @@ __global__ void __launch_bounds__(kCeThreads) rate_ce_kernel(int64_t Tn, int64_t
       const float beta = __ldg(r.beta + (r.beta_col ? n : 0));
       const float thr = __ldg(r.thr + (r.thr_col ? n : 0));
       BwdLane st{0.0f, 0.0f, 0.0f, 0.0f, 0.0f};
-      for (int64_t tc = Tn - 1; tc >= 0; tc -= kCeChunk) {
-        float uu[kCeChunk];
-        uint32_t zz = 0;  // bit c: z at step tc - c
+      // chunks of kCeChunk steps from the last; the next chunk's loads are
+      // issued before the current one is stepped (steps before 0 reload
+      // step 0 and are not stepped)
+      auto load_chunk = [&](int64_t tc, float (&u)[kCeChunk], uint32_t& zm) {
+        zm = 0;
 #pragma unroll
         for (int c = 0; c < kCeChunk; ++c) {
-          const int64_t ts = tc - c >= 0 ? tc - c : 0;  // steps before 0 reload step 0, unused
-          uu[c] = Elem<T>::load1(r.mem + ts * step + lane);
+          const int64_t ts = tc - c >= 0 ? tc - c : 0;
+          u[c] = Elem<T>::load1(r.mem + ts * step + lane);
           const uint32_t z = r.bits ? (__ldg(r.bits + ts * r.bits_row + (lane >> 3)) >> (lane & 7)) & 1u
                                     : (Elem<T>::load1(spk + ts * step + lane) != 0.0f ? 1u : 0u);
-          zz |= z << c;
+          zm |= z << c;
         }
+      };
+      float ucur[kCeChunk], unext[kCeChunk];
+      uint32_t zcur, znext = 0;
+      load_chunk(Tn - 1, ucur, zcur);
+      for (int64_t tc = Tn - 1; tc >= 0; tc -= kCeChunk) {
+        if (tc - kCeChunk >= 0) load_chunk(tc - kCeChunk, unext, znext);
 #pragma unroll
         for (int c = 0; c < kCeChunk; ++c) {
           const int64_t ts = tc - c;
           if (ts < 0) break;
-          const float du = bwd_step<false, -1, -1>(r.sa, beta, thr, 0.0f, ts + 1 < Tn, uu[c],
-                                                   ((zz >> c) & 1u) != 0, 0.0f, g, 0.0f, 0.0f, st);
+          const float du = bwd_step<false, -1, -1>(r.sa, beta, thr, 0.0f, ts + 1 < Tn, ucur[c],
+                                                   ((zcur >> c) & 1u) != 0, 0.0f, g, 0.0f, 0.0f, st);
           Elem<T>::store1(r.gI + ts * step + lane, du);
           if (grad) Elem<T>::store1(grad + ts * step + lane, g);
         }
+#pragma unroll
+        for (int c = 0; c < kCeChunk; ++c) ucur[c] = unext[c];
+        zcur = znext;
       }
     }
   } else {
@@ -163,16 +175,24 @@ __global__ void __launch_bounds__(kCeThreads) rate_ce_kernel(int64_t Tn, int64_t
       for (int64_t t = 0; t < Tn; ++t) Elem<T>::store1(grow + t * step + n, g);
     }
   }
-  // the last block to finish adds the loss terms in sample order
+  // the last block to finish adds the loss terms
   __threadfence();
   __syncthreads();
   if (threadIdx.x == 0) last = atomicAdd(ticket, 1) == (int)(B - 1);
   __syncthreads();
   if (!last) return;
   __threadfence();
+  // fixed order: thread i adds terms i, i + 256, ... in turn, each warp
+  // folds its lanes by halves, and thread 0 adds the warp sums in order
+  __shared__ double wsum[kCeThreads / 32];
+  double part = 0.0;
+  for (int64_t q = threadIdx.x; q < B; q += kCeThreads) part += __ldcg(terms + q);
+  for (int o = 16; o > 0; o >>= 1) part += __shfl_down_sync(0xffffffffu, part, o);
+  if ((threadIdx.x & 31) == 0) wsum[threadIdx.x >> 5] = part;
+  __syncthreads();
   if (threadIdx.x == 0) {
     double total = 0.0;
-    for (int64_t q = 0; q < B; ++q) total += terms[q];
+    for (int k = 0; k < kCeThreads / 32; ++k) total += wsum[k];
     loss[0] = (float)(total / (double)Bn);
     *ticket = 0;
   }

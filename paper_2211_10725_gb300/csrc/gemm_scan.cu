@@ -42,7 +42,7 @@ constexpr int kScanWarps = 10;  // warps 2..11 scan; 2..5 also drain the accumul
 constexpr int kScanThreads = 32 * kScanWarps;
 constexpr int kFusedThreads = 64 + kScanThreads;
 constexpr int kScanLanes = 2;  // lanes a scan thread steps together (independent chains)
-constexpr int kBwdChunk = 4;   // steps of stored trace a backward scan thread loads ahead (8 spills)
+constexpr int kBwdChunk = 8;   // steps of stored trace a backward scan thread loads ahead
 
 struct FusedArgs {
   int T, R, K, N;   // steps, rows per step, reduction, output columns (neurons / channels)
@@ -225,65 +225,54 @@ __global__ void __launch_bounds__(kFusedThreads, 2)
         break;
       }
       if constexpr (BWD) {
-      // the reverse scan: thread e steps lanes j = g0 + kScanThreads*v + e
-      // from t = T-1 down to 0; the staged value of (t, lane) is dL/dz_t.
-      // The stored trace of kBwdChunk steps is loaded before they are
-      // stepped, so the loads of a chunk overlap instead of each step
-      // waiting for its own.
+      // the reverse scan: thread e steps lanes j = g0 + e from t = T-1 down
+      // to 0; the staged value of (t, lane) is dL/dz_t.  The stored trace
+      // comes in chunks of kBwdChunk steps, the next chunk's loads issued
+      // before the current chunk is stepped, so a lane waits for memory
+      // about once rather than once per step.
       const int64_t RN = (int64_t)f.R * f.N;
-      for (int g0 = 0; g0 < lanes; g0 += kScanThreads * kScanLanes) {
-        const int nv = (lanes - g0 + kScanThreads - 1) / kScanThreads;  // block-uniform
-        float beta[kScanLanes], thr[kScanLanes];
-        bool ok[kScanLanes];
-        int srow_i[kScanLanes], col[kScanLanes];
-        int64_t o[kScanLanes];
-        BwdLane st[kScanLanes];
-#pragma unroll
-        for (int v = 0; v < kScanLanes; ++v) {
-          const int j = g0 + kScanThreads * v + e;
-          const int jj = j < lanes ? j : 0;  // lanes past the tile read row 0
-          const int sr = jj / BN, n = jj - (jj / BN) * BN;
-          srow_i[v] = sr;
-          col[v] = n;
-          ok[v] = j < lanes && r0 + sr < f.R && n0 + n < f.N;
-          const int nc = ok[v] ? n0 + n : 0;
-          beta[v] = __ldg(f.beta + (f.beta_col ? nc : 0));
-          thr[v] = __ldg(f.thr + (f.thr_col ? nc : 0));
-          o[v] = ok[v] ? (int64_t)(r0 + sr) * f.N + nc : 0;
-          st[v] = BwdLane{0.0f, 0.0f, 0.0f, 0.0f, 0.0f};
-        }
-        for (int tc = f.T - 1; tc >= 0; tc -= kBwdChunk) {
-          static_assert(kScanLanes == 2, "the trace of a step's two lanes is one bf16 pair");
-          __nv_bfloat162 uu[kBwdChunk];  // the bf16 trace as stored (x: lane 0, y: lane 1)
-          uint32_t zz[kScanLanes] = {};  // bit c: z at step tc - c
+      for (int g0 = 0; g0 < lanes; g0 += kScanThreads) {
+        const int j = g0 + e;
+        const int jj = j < lanes ? j : 0;  // lanes past the tile read row 0
+        const int sr = jj / BN, n = jj - (jj / BN) * BN;
+        const bool ok = j < lanes && r0 + sr < f.R && n0 + n < f.N;
+        const int nc = ok ? n0 + n : 0;
+        const float beta = __ldg(f.beta + (f.beta_col ? nc : 0));
+        const float thr = __ldg(f.thr + (f.thr_col ? nc : 0));
+        const int64_t o = ok ? (int64_t)(r0 + sr) * f.N + nc : 0;
+        const float* gsp = stg + sr * SP + n;
+        BwdLane st{0.0f, 0.0f, 0.0f, 0.0f, 0.0f};
+        // chunk at tc: steps tc, tc-1, ..., tc-kBwdChunk+1; steps before 0
+        // load step 0 (in bounds) and are not stepped
+        auto load_chunk = [&](int tc, __nv_bfloat16 (&u)[kBwdChunk], uint32_t& zm) {
+          zm = 0;
 #pragma unroll
           for (int c = 0; c < kBwdChunk; ++c) {
-#pragma unroll
-            for (int v = 0; v < kScanLanes; ++v) {
-              // steps before t = 0 and lanes past the tile load lane 0 of
-              // step 0 (in bounds) and are not stepped
-              const int ts = tc - c >= 0 && v < nv ? tc - c : 0;
-              const int64_t q = (int64_t)ts * RN + o[v];
-              if (v == 0) uu[c].x = f.mem_in[q];
-              else uu[c].y = f.mem_in[q];
-              const uint32_t z = f.bits_in ? (__ldg(f.bits_in + (int64_t)ts * f.bits_row + (o[v] >> 3)) >> (o[v] & 7)) & 1u
-                                           : (__bfloat162float(f.spk_in[q]) != 0.0f ? 1u : 0u);
-              zz[v] |= z << c;
-            }
+            const int ts = tc - c >= 0 ? tc - c : 0;
+            const int64_t q = (int64_t)ts * RN + o;
+            u[c] = f.mem_in[q];
+            const uint32_t z = f.bits_in ? (__ldg(f.bits_in + (int64_t)ts * f.bits_row + (o >> 3)) >> (o & 7)) & 1u
+                                         : (__bfloat162float(f.spk_in[q]) != 0.0f ? 1u : 0u);
+            zm |= z << c;
           }
+        };
+        __nv_bfloat16 ucur[kBwdChunk], unext[kBwdChunk];
+        uint32_t zcur, znext = 0;
+        load_chunk(f.T - 1, ucur, zcur);
+        for (int tc = f.T - 1; tc >= 0; tc -= kBwdChunk) {
+          if (tc - kBwdChunk >= 0) load_chunk(tc - kBwdChunk, unext, znext);
 #pragma unroll
           for (int c = 0; c < kBwdChunk; ++c) {
             const int ts = tc - c;
-            if (ts < 0) break;  // uniform
-#pragma unroll
-            for (int v = 0; v < kScanLanes; ++v) {
-              if (v >= nv) break;  // uniform: the whole group is past the tile
-              const float gs = stg[(ts * f.BS + srow_i[v]) * SP + col[v]];
-              const float du = bwd_step<false, RESET, SG>(f.sa, beta[v], thr[v], 0.0f, ts + 1 < f.T,
-                                                          __bfloat162float(v == 0 ? uu[c].x : uu[c].y), ((zz[v] >> c) & 1u) != 0, 0.0f, gs, 0.0f, 0.0f, st[v]);
-              if (ok[v]) f.gI[(int64_t)ts * RN + o[v]] = __float2bfloat16_rn(du);
-            }
+            if (ts < 0) break;
+            const float du = bwd_step<false, RESET, SG>(f.sa, beta, thr, 0.0f, ts + 1 < f.T,
+                                                        __bfloat162float(ucur[c]), ((zcur >> c) & 1u) != 0,
+                                                        0.0f, gsp[ts * f.BS * SP], 0.0f, 0.0f, st);
+            if (ok) f.gI[(int64_t)ts * RN + o] = __float2bfloat16_rn(du);
           }
+#pragma unroll
+          for (int c = 0; c < kBwdChunk; ++c) ucur[c] = unext[c];
+          zcur = znext;
         }
       }
       } else {
