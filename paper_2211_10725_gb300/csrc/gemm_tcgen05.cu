@@ -80,6 +80,8 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm)
   constexpr int B_BYTES = BN * BK * 2;
   constexpr uint32_t TCOLS = tmem_cols<BN>();
   constexpr int kEpiWarps = 4;
+  constexpr int kStages = gemm_stages<BN>();
+  static_assert(smem_bytes<BN, TMA_OUT>() <= 227 * 1024, "the ring and staging fit one CTA");
   extern __shared__ unsigned char smem_raw[];
   unsigned char* smem =
       reinterpret_cast<unsigned char*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -344,12 +346,13 @@ cudaError_t launch_out(const CUtensorMap& ta, const CUtensorMap& tb, const GemmA
 // rather than 128 when 128-wide tiles would leave most SMs idle.
 template <bool OUT_BF16, bool A_MN = false, bool B_MN = false>
 cudaError_t gemm_tn(const void* A, const void* B, void* D, int M, int N, int K, int* status,
-                    cudaStream_t st, int ksplit = 1) {
+                    cudaStream_t st, int ksplit = 1, int bn_force = 0) {
   // a 128 x 256 tile keeps the tensor core busier per instruction (about
   // 1.6x the rate of 128 x 128 at large K); below K = 512 the per-tile
   // fixed costs dominate and the narrower tile's parallelism wins
   int bn = (!B_MN && N > 128 && K >= 512) ? 256 : 128;
-  if (N <= 16 && !B_MN) bn = 16;
+  if (bn_force > 0) bn = bn_force;
+  else if (N <= 16 && !B_MN) bn = 16;
   else if (N <= 32 && !B_MN) bn = 32;
   else if (N <= 64) bn = 64;
   else {
@@ -366,6 +369,7 @@ cudaError_t gemm_tn(const void* A, const void* B, void* D, int M, int N, int K, 
   GemmArgs g{M, N, K, D, (int64_t)N, status, kDefaultWaitNs, ksplit, (int64_t)M * N};
   if constexpr (B_MN) {
     if (bn == 64) return launch_out<64, OUT_BF16, A_MN, B_MN>(ta, tb, g, st);
+    if (bn == 256) return launch_out<256, OUT_BF16, A_MN, B_MN>(ta, tb, g, st);
     return launch_out<128, OUT_BF16, A_MN, B_MN>(ta, tb, g, st);
   } else {
     switch (bn) {
@@ -385,15 +389,30 @@ size_t round256(size_t b) { return (b + 255) & ~size_t(255); }
 // the M rows), from the shapes alone so that a shape always sums in the same
 // order: enough (tile, split) items to give each of about one GPU's worth of
 // SMs (kSplitSlots) one, with at least kMinSplitKBlocks k-blocks per split.
+// A wide layer (N >= 256 neurons, K >= 512 inputs) with a long reduction
+// takes 128 x 256 tiles: its operands' L2 traffic is half that of the
+// 64-wide tiles, which re-read dI once per 64 columns; the splits then fill
+// the SMs.  Otherwise the GEMM's own tile choice, split to fill the SMs.
 constexpr int64_t kSplitSlots = 152;
 constexpr int64_t kMinSplitKBlocks = 8;
-int dw_splits(int64_t M, int64_t K, int64_t N) {
-  const int64_t tiles = ((N + BM - 1) / BM) * ((K + 63) / 64);
+struct DwPlan {
+  int bn;  // 0: the GEMM's own choice
+  int S;
+};
+DwPlan dw_plan(int64_t M, int64_t K, int64_t N) {
   const int64_t nk = (M + BK - 1) / BK;
-  int64_t s = kSplitSlots / (tiles > 0 ? tiles : 1);
-  if (s > nk / kMinSplitKBlocks) s = nk / kMinSplitKBlocks;
-  return s < 1 ? 1 : (int)s;
+  auto splits = [&](int64_t tiles) {
+    int64_t s = kSplitSlots / (tiles > 0 ? tiles : 1);
+    if (s > nk / kMinSplitKBlocks) s = nk / kMinSplitKBlocks;
+    return s < 1 ? 1 : (int)s;
+  };
+  if (N >= 256 && K >= 512) {
+    const int S = splits(((N + BM - 1) / BM) * ((K + 255) / 256));
+    if (S >= 2) return DwPlan{256, S};
+  }
+  return DwPlan{0, splits(((N + BM - 1) / BM) * ((K + 63) / 64))};
 }
+int dw_splits(int64_t M, int64_t K, int64_t N) { return dw_plan(M, K, N).S; }
 
 // out[i] = sum over s = 0 .. S-1 of part[s * n + i], in split order.
 __global__ void __launch_bounds__(256) sum_splits(const float4* __restrict__ part,
@@ -472,14 +491,15 @@ snn_status_t snn_dense_layer_bwd(int64_t M, int64_t K, int64_t N, const void* X,
   }
   if (dW && N > 0 && K > 0) {
     // dW[N, K] = dI[M, N]^T * X[M, K]: both operands MN-major (K = M here)
-    const int S = dw_splits(M, K, N);
+    const DwPlan plan = dw_plan(M, K, N);
+    const int S = plan.S;
     if (M == 0) {
       e = cudaMemsetAsync(dW, 0, (size_t)N * K * sizeof(float), st);
     } else if (S == 1) {
-      e = gemm_tn<false, true, true>(dI, X, dW, (int)N, (int)K, (int)M, status, st);
+      e = gemm_tn<false, true, true>(dI, X, dW, (int)N, (int)K, (int)M, status, st, 1, plan.bn);
     } else {
       float* part = reinterpret_cast<float*>(static_cast<unsigned char*>(ws) + 256);
-      e = gemm_tn<false, true, true>(dI, X, part, (int)N, (int)K, (int)M, status, st, S);
+      e = gemm_tn<false, true, true>(dI, X, part, (int)N, (int)K, (int)M, status, st, S, plan.bn);
       const int64_t n4 = N * K / 4;  // K is a multiple of 8
       if (e == cudaSuccess)
         e = snn::launch_pdl(sum_splits, dim3((unsigned)((n4 + 255) / 256)), dim3(256), 0, st,

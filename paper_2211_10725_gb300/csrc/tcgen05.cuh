@@ -18,9 +18,6 @@
 namespace snn {
 namespace gemm {
 
-#ifndef SNN_GEMM_STAGES
-#define SNN_GEMM_STAGES 4
-#endif
 #ifndef SNN_GEMM_CTAS_PER_SM
 #define SNN_GEMM_CTAS_PER_SM 1
 #endif
@@ -30,7 +27,12 @@ namespace gemm {
 
 constexpr int BM = 128;
 constexpr int BK = 64;  // 64 bf16 = 128 bytes: one swizzle atom row
-constexpr int kStages = SNN_GEMM_STAGES;
+// Ring depth of the plain GEMM: one CTA per SM streams its operands through
+// a TMA ring, and its feed rate is the bytes it has in flight, so each tile
+// width takes as many stages as fit beside the output staging in the 227 KB
+// a CTA may use (all three come to 225 KB with the staging).
+template <int BN>
+__host__ __device__ constexpr int gemm_stages() { return BN <= 64 ? 8 : (BN <= 128 ? 6 : 4); }
 constexpr int kCtasPerSm = SNN_GEMM_CTAS_PER_SM;  // resident CTAs the tile size aims for
 constexpr int kThreads = 192;
 constexpr uint64_t kDefaultWaitNs = 2000000000ull;
@@ -212,7 +214,7 @@ __host__ __device__ constexpr uint32_t tmem_cols() {
 
 template <int BN, bool TMA_OUT = false>
 __host__ __device__ constexpr size_t smem_bytes() {
-  return 1024 /* alignment slack */ + (size_t)kStages * (BM * BK * 2 + BN * BK * 2) +
+  return 1024 /* alignment slack */ + (size_t)gemm_stages<BN>() * (BM * BK * 2 + BN * BK * 2) +
          (TMA_OUT ? kOutStaging : 0) + 256;
 }
 
