@@ -225,111 +225,112 @@ __global__ void __launch_bounds__(kFusedThreads, 2)
         break;
       }
       if constexpr (BWD) {
-      // the reverse scan: thread e steps lanes j = g0 + e from t = T-1 down
-      // to 0; the staged value of (t, lane) is dL/dz_t.  The stored trace
-      // comes in chunks of kBwdChunk steps, the next chunk's loads issued
-      // before the current chunk is stepped, so a lane waits for memory
-      // about once rather than once per step.
-      const int64_t RN = (int64_t)f.R * f.N;
-      for (int g0 = 0; g0 < lanes; g0 += kScanThreads) {
-        const int j = g0 + e;
-        const int jj = j < lanes ? j : 0;  // lanes past the tile read row 0
-        const int sr = jj / BN, n = jj - (jj / BN) * BN;
-        const bool ok = j < lanes && r0 + sr < f.R && n0 + n < f.N;
-        const int nc = ok ? n0 + n : 0;
-        const float beta = __ldg(f.beta + (f.beta_col ? nc : 0));
-        const float thr = __ldg(f.thr + (f.thr_col ? nc : 0));
-        const int64_t o = ok ? (int64_t)(r0 + sr) * f.N + nc : 0;
-        const float* gsp = stg + sr * SP + n;
-        BwdLane st{0.0f, 0.0f, 0.0f, 0.0f, 0.0f};
-        // chunk at tc: steps tc, tc-1, ..., tc-kBwdChunk+1; steps before 0
-        // load step 0 (in bounds) and are not stepped
-        auto load_chunk = [&](int tc, __nv_bfloat16 (&u)[kBwdChunk], uint32_t& zm) {
-          zm = 0;
-#pragma unroll
-          for (int c = 0; c < kBwdChunk; ++c) {
-            const int ts = tc - c >= 0 ? tc - c : 0;
-            const int64_t q = (int64_t)ts * RN + o;
-            u[c] = f.mem_in[q];
-            const uint32_t z = f.bits_in ? (__ldg(f.bits_in + (int64_t)ts * f.bits_row + (o >> 3)) >> (o & 7)) & 1u
-                                         : (__bfloat162float(f.spk_in[q]) != 0.0f ? 1u : 0u);
-            zm |= z << c;
-          }
-        };
-        __nv_bfloat16 ucur[kBwdChunk], unext[kBwdChunk];
-        uint32_t zcur, znext = 0;
-        load_chunk(f.T - 1, ucur, zcur);
-        for (int tc = f.T - 1; tc >= 0; tc -= kBwdChunk) {
-          if (tc - kBwdChunk >= 0) load_chunk(tc - kBwdChunk, unext, znext);
-#pragma unroll
-          for (int c = 0; c < kBwdChunk; ++c) {
-            const int ts = tc - c;
-            if (ts < 0) break;
-            const float du = bwd_step<false, RESET, SG>(f.sa, beta, thr, 0.0f, ts + 1 < f.T,
-                                                        __bfloat162float(ucur[c]), ((zcur >> c) & 1u) != 0,
-                                                        0.0f, gsp[ts * f.BS * SP], 0.0f, 0.0f, st);
-            if (ok) f.gI[(int64_t)ts * RN + o] = __float2bfloat16_rn(du);
-          }
-#pragma unroll
-          for (int c = 0; c < kBwdChunk; ++c) ucur[c] = unext[c];
-          zcur = znext;
-        }
-      }
-      } else {
-      // the scan: thread e steps lanes j = g0 + kScanThreads*v + e together
-      // (independent chains); groups wholly past the tile are skipped
-      const int64_t RN = (int64_t)f.R * f.N;  // elements per step of spk / mem
-      for (int g0 = 0; g0 < lanes; g0 += kScanThreads * kScanLanes) {
-        const int nv = (lanes - g0 + kScanThreads - 1) / kScanThreads;  // block-uniform
-        float u[kScanLanes], beta[kScanLanes], thr[kScanLanes];
-        bool z[kScanLanes], ok[kScanLanes];
-        const float* xs[kScanLanes];
-        __nv_bfloat16* ps[kScanLanes];
-        __nv_bfloat16* pm[kScanLanes];
-        unsigned char* pb[kScanLanes];
-#pragma unroll
-        for (int v = 0; v < kScanLanes; ++v) {
-          const int j = g0 + kScanThreads * v + e;
+        // the reverse scan: thread e steps lanes j = g0 + e from t = T-1 down
+        // to 0; the staged value of (t, lane) is dL/dz_t.  The stored trace
+        // comes in chunks of kBwdChunk steps, the next chunk's loads issued
+        // before the current chunk is stepped, so a lane waits for memory
+        // about once rather than once per step.
+        const int64_t RN = (int64_t)f.R * f.N;
+        for (int g0 = 0; g0 < lanes; g0 += kScanThreads) {
+          const int j = g0 + e;
           const int jj = j < lanes ? j : 0;  // lanes past the tile read row 0
-          const int s = jj / BN, n = jj - (jj / BN) * BN;
-          ok[v] = j < lanes && r0 + s < f.R && n0 + n < f.N;
-          const int nc = ok[v] ? n0 + n : 0;
-          beta[v] = __ldg(f.beta + (f.beta_col ? nc : 0));
-          thr[v] = __ldg(f.thr + (f.thr_col ? nc : 0));
-          u[v] = 0.0f;
-          z[v] = false;
-          const int64_t o = ok[v] ? (int64_t)(r0 + s) * f.N + nc : 0;  // lane index within a step
-          xs[v] = stg + s * SP + n;
-          ps[v] = f.spk + o;
-          pm[v] = f.mem + o;
-          pb[v] = f.bits ? f.bits + (o >> 3) : nullptr;
+          const int sr = jj / BN, n = jj - (jj / BN) * BN;
+          const bool ok = j < lanes && r0 + sr < f.R && n0 + n < f.N;
+          const int nc = ok ? n0 + n : 0;
+          const float beta = __ldg(f.beta + (f.beta_col ? nc : 0));
+          const float thr = __ldg(f.thr + (f.thr_col ? nc : 0));
+          const int64_t o = ok ? (int64_t)(r0 + sr) * f.N + nc : 0;
+          const float* gsp = stg + sr * SP + n;
+          BwdLane st{0.0f, 0.0f, 0.0f, 0.0f, 0.0f};
+          // chunk at tc: steps tc, tc-1, ..., tc-kBwdChunk+1; steps before 0
+          // load step 0 (in bounds) and are not stepped
+          auto load_chunk = [&](int tc, __nv_bfloat16 (&u)[kBwdChunk], uint32_t& zm) {
+            zm = 0;
+#pragma unroll
+            for (int c = 0; c < kBwdChunk; ++c) {
+              const int ts = tc - c >= 0 ? tc - c : 0;
+              const int64_t q = (int64_t)ts * RN + o;
+              u[c] = f.mem_in[q];
+              const uint32_t z =
+                  f.bits_in ? (__ldg(f.bits_in + (int64_t)ts * f.bits_row + (o >> 3)) >> (o & 7)) & 1u
+                            : (__bfloat162float(f.spk_in[q]) != 0.0f ? 1u : 0u);
+              zm |= z << c;
+            }
+          };
+          __nv_bfloat16 ucur[kBwdChunk], unext[kBwdChunk];
+          uint32_t zcur, znext = 0;
+          load_chunk(f.T - 1, ucur, zcur);
+          for (int tc = f.T - 1; tc >= 0; tc -= kBwdChunk) {
+            if (tc - kBwdChunk >= 0) load_chunk(tc - kBwdChunk, unext, znext);
+#pragma unroll
+            for (int c = 0; c < kBwdChunk; ++c) {
+              const int ts = tc - c;
+              if (ts < 0) break;
+              const float du =
+                  bwd_step<false, RESET, SG>(f.sa, beta, thr, 0.0f, ts + 1 < f.T, __bfloat162float(ucur[c]),
+                                             ((zcur >> c) & 1u) != 0, 0.0f, gsp[ts * f.BS * SP], 0.0f, 0.0f, st);
+              if (ok) f.gI[(int64_t)ts * RN + o] = __float2bfloat16_rn(du);
+            }
+#pragma unroll
+            for (int c = 0; c < kBwdChunk; ++c) ucur[c] = unext[c];
+            zcur = znext;
+          }
         }
-        const int xstep = f.BS * SP;
-        for (int ts = 0; ts < f.T; ++ts) {
+      } else {
+        // the scan: thread e steps lanes j = g0 + kScanThreads*v + e together
+        // (independent chains); groups wholly past the tile are skipped
+        const int64_t RN = (int64_t)f.R * f.N;  // elements per step of spk / mem
+        for (int g0 = 0; g0 < lanes; g0 += kScanThreads * kScanLanes) {
+          const int nv = (lanes - g0 + kScanThreads - 1) / kScanThreads;  // block-uniform
+          float u[kScanLanes], beta[kScanLanes], thr[kScanLanes];
+          bool z[kScanLanes], ok[kScanLanes];
+          const float* xs[kScanLanes];
+          __nv_bfloat16* ps[kScanLanes];
+          __nv_bfloat16* pm[kScanLanes];
+          unsigned char* pb[kScanLanes];
 #pragma unroll
           for (int v = 0; v < kScanLanes; ++v) {
-            if (v >= nv) break;  // uniform: the whole group is past the tile
-            const float x = *xs[v];
-            xs[v] += xstep;
-            float idummy = 0.0f;
-            fwd_step<false, RESET, 0>(f.reset, beta[v], thr[v], 0.0f, x, u[v], z[v], idummy);
-            const bool zz = ok[v] && z[v];
-            if (ok[v]) {
-              *ps[v] = __float2bfloat16_rn(zz ? 1.0f : 0.0f);
-              *pm[v] = __float2bfloat16_rn(u[v]);
-            }
-            ps[v] += RN;
-            pm[v] += RN;
-            if (f.bits) {
-              // 8 consecutive threads hold 8 consecutive lanes of one row (BN
-              // and N are multiples of 8): one byte of the step's bit row
-              const uint32_t m = __ballot_sync(0xffffffffu, zz);
-              if ((lid & 7) == 0 && ok[v]) *pb[v] = (unsigned char)((m >> lid) & 0xFFu);
-              pb[v] += f.bits_row;
+            const int j = g0 + kScanThreads * v + e;
+            const int jj = j < lanes ? j : 0;  // lanes past the tile read row 0
+            const int s = jj / BN, n = jj - (jj / BN) * BN;
+            ok[v] = j < lanes && r0 + s < f.R && n0 + n < f.N;
+            const int nc = ok[v] ? n0 + n : 0;
+            beta[v] = __ldg(f.beta + (f.beta_col ? nc : 0));
+            thr[v] = __ldg(f.thr + (f.thr_col ? nc : 0));
+            u[v] = 0.0f;
+            z[v] = false;
+            const int64_t o = ok[v] ? (int64_t)(r0 + s) * f.N + nc : 0;  // lane index within a step
+            xs[v] = stg + s * SP + n;
+            ps[v] = f.spk + o;
+            pm[v] = f.mem + o;
+            pb[v] = f.bits ? f.bits + (o >> 3) : nullptr;
+          }
+          const int xstep = f.BS * SP;
+          for (int ts = 0; ts < f.T; ++ts) {
+#pragma unroll
+            for (int v = 0; v < kScanLanes; ++v) {
+              if (v >= nv) break;  // uniform: the whole group is past the tile
+              const float x = *xs[v];
+              xs[v] += xstep;
+              float idummy = 0.0f;
+              fwd_step<false, RESET, 0>(f.reset, beta[v], thr[v], 0.0f, x, u[v], z[v], idummy);
+              const bool zz = ok[v] && z[v];
+              if (ok[v]) {
+                *ps[v] = __float2bfloat16_rn(zz ? 1.0f : 0.0f);
+                *pm[v] = __float2bfloat16_rn(u[v]);
+              }
+              ps[v] += RN;
+              pm[v] += RN;
+              if (f.bits) {
+                // 8 consecutive threads hold 8 consecutive lanes of one row (BN
+                // and N are multiples of 8): one byte of the step's bit row
+                const uint32_t m = __ballot_sync(0xffffffffu, zz);
+                if ((lid & 7) == 0 && ok[v]) *pb[v] = (unsigned char)((m >> lid) & 0xFFu);
+                pb[v] += f.bits_row;
+              }
             }
           }
         }
-      }
       }
       epi_barrier();  // the staged rows are consumed before the next tile's copy
     }
