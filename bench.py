@@ -10,8 +10,10 @@ Other scan workloads (`--workload`, the names in workloads.SCAN_WORKLOADS)
 time the same step on their shapes.  The network workloads time a whole
 training step as one CUDA graph: the dense SNN (Tab. I DSNN) and its
 population-coded variant, and the convolutional SNN (Tab. I CSNN) --
-forward (by default each GEMM layer fused with its scan), loss, BPTT and
-AdamW -- in the same metric, with images/s and per-op times beside it.
+forward (by default each GEMM layer fused with its scan), loss (with the
+readout's BPTT in the same launch), BPTT (for T > 1 each dense input-gradient
+GEMM fused with the lower layer's reverse scan) and AdamW -- in the same
+metric, with images/s and per-op times beside it.
 
 Prints one JSON line (rank 0).  `--impl reference` times the CPU oracle (the
 only other implementation of this path) on a bounded sample of the same
