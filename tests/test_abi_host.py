@@ -122,3 +122,63 @@ def test_backward_argument_checks(lib):
     assert _bwd(lib, d5, **rec) == 1
     rec = dict(beta=16, thr=16, grad_spk=16, grad_I=16, ws=16, ckpt=16)
     assert _bwd(lib, d5, **rec) == 1
+
+
+# The fused entry points check their arguments before any CUDA call.  The
+# pointers below are never dereferenced: every call here is rejected first.
+def _fused_desc(**over):
+    w = W.ScanWorkload(name="fused", neuron="leaky", T=25, B=16, N=64, in_dtype=W.F32,
+                       io_dtype=W.BF16, save="mem", want_mem=True)
+    return snn.make_desc(w, **over)
+
+
+def test_dense_leaky_fwd_argument_checks(lib):
+    f = lambda d, P=1, K=64, X=16, ws_bytes=256: lib.snn_dense_leaky_fwd(
+        ctypes.byref(d), P, K, X, 16, 16, 16, 16, 16, None, 16, ws_bytes, None)
+    assert f(_fused_desc(T=129)) == 3                  # a tile holds every step
+    assert f(_fused_desc(io_dtype=0)) == 3             # bf16 storage only
+    assert f(_fused_desc(save=1, ckpt_every=8)) == 3   # the trace is stored
+    assert f(_fused_desc(), K=12) == 3                 # 16-byte rows
+    assert f(_fused_desc(N=12)) == 3
+    assert f(_fused_desc(), P=3) == 1                  # N % P
+    assert f(_fused_desc(reset=3)) == 1
+    assert f(_fused_desc(), X=None) == 1
+    assert f(_fused_desc(), X=24) == 2
+    assert f(_fused_desc(), ws_bytes=64) == 4
+
+
+def test_dense_leaky_bwd_argument_checks(lib):
+    def f(d, K=64, dI=16, Wp=16, spk=16, ckpt=None, ws_bytes=256):
+        return lib.snn_dense_leaky_bwd(ctypes.byref(d), K, dI, Wp, 16, 16, 16, spk, ckpt, 16,
+                                       16, ws_bytes, None)
+    assert f(_fused_desc(T=129)) == 3
+    assert f(_fused_desc(io_dtype=0)) == 3
+    assert f(_fused_desc(save=1, ckpt_every=8)) == 3
+    assert f(_fused_desc(), K=12) == 3
+    assert f(_fused_desc(N=12)) == 3
+    assert f(_fused_desc(beta_mode=2, C=64, HW=1)) == 3   # scalar or per neuron only
+    assert f(_fused_desc(surrogate=5)) == 1
+    assert f(_fused_desc(sg_param=0.0)) == 1
+    assert f(_fused_desc(), spk=None, ckpt=None) == 1     # no spike source
+    assert f(_fused_desc(), Wp=None) == 1
+    assert f(_fused_desc(), dI=24) == 2
+    assert f(_fused_desc(), ckpt=40) == 2
+    assert f(_fused_desc(), ws_bytes=64) == 4
+
+
+def test_rate_ce_leaky_bwd_argument_checks(lib):
+    need = snn.snn_rate_ce_workspace_bytes(16)
+
+    def f(d, C=10, pop=1, total=0, spk=16, mem=16, ws_bytes=need):
+        return lib.snn_rate_ce_leaky_bwd(ctypes.byref(d), C, pop, total, spk, 16, 16, 16, mem,
+                                         None, 16, None, 16, 16, ws_bytes, None)
+    assert f(_fused_desc(), C=10, pop=7) == 1             # C * pop > ld
+    assert f(_fused_desc(), total=8) == 1                 # batch_total < B
+    assert f(_fused_desc(), C=2000) == 1                  # at most 1024 classes
+    assert f(_fused_desc(save=1, ckpt_every=8)) == 3      # needs the stored trace
+    assert f(_fused_desc(thr_mode=2, C=64, HW=1)) == 3
+    assert f(_fused_desc(io_dtype=7)) == 1
+    assert f(_fused_desc(reset=3)) == 1
+    assert f(_fused_desc(), mem=None) == 1
+    assert f(_fused_desc(), spk=24) == 2
+    assert f(_fused_desc(), ws_bytes=64) == 4
