@@ -4,8 +4,9 @@
 // fp32 accumulation in tensor memory, fp32 or bf16 output.
 //
 // Persistent CTAs (one per SM) take 128 x BN tiles (BN up to 256) in turn.  Warp 0 (one
-// thread) streams 128x64 and BNx64 operand tiles into a 4-stage
-// shared-memory ring with TMA (128-byte swizzle); warp 1 allocates two TMEM
+// thread) streams 128x64 and BNx64 operand tiles into a shared-memory ring
+// with TMA (128-byte swizzle), 8, 6 or 4 stages deep for BN = 64, 128, 256
+// (as deep as fits beside the output staging); warp 1 allocates two TMEM
 // accumulators and one thread issues tcgen05.mma (M=128, N=BN, K=16 per
 // instruction) as stages land, freeing each stage through tcgen05.commit;
 // warps 2-5 read a finished accumulator back with tcgen05.ld (each warp its
@@ -32,7 +33,9 @@
 // gradient of a convolution sums over every patch row) runs as tiles x S
 // work items, item (tile, s) summing k-blocks [s*nk/S, (s+1)*nk/S) into
 // partial output s; a second kernel adds the S partials in split order, so
-// the result does not depend on which CTA ran which item.
+// the result does not depend on which CTA ran which item.  Weight gradients
+// of wide layers use 128 x 256 tiles (four 64-column MN-major B boxes) and
+// splits, which cuts the re-reads of dI across output columns.
 #include <cuda.h>
 #include <cudaTypedefs.h>
 #include <cuda_bf16.h>
