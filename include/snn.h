@@ -21,7 +21,10 @@
  *   l = b*N + n, element (t, l) at offset t*B*N + l.  Per-lane states and
  *   their gradients (mem0, syn0, mem_final, grad_mem0, ...) are fp32 [B, N].
  * - Every pointer argument is a DEVICE pointer unless stated, owned by the
- *   caller; the library allocates nothing and keeps no state between calls.
+ *   caller; the library allocates nothing.  Between calls it keeps only a
+ *   process-wide count of its kernel launches (snn_kernel_launches), per
+ *   device caches of launch plans and device attributes, and the fixed
+ *   device array of snn_leaky_bwd_noalloc.  Results never depend on them.
  *   Outputs are overwritten, never accumulated into.
  * - Calls are asynchronous on `stream` and never synchronise it (except
  *   snn_workspace_status).  Arguments are checked before anything is
@@ -501,14 +504,18 @@ snn_status_t snn_adamw_step(int64_t n, float* w, void* w_bf16, const float* grad
  * held by every GPU that loads the library until the process exits.
  *   status   device int (4-byte aligned) or NULL: receives SNN_OK or
  *            SNN_ERR_TIMEOUT from the kernels (asynchronously, on stream)
- * Returns SNN_ERR_WORKSPACE, launching nothing, when
- * snn_scan_workspace_bytes(desc) exceeds 16 MiB.  Allocates nothing.
+ * Argument checks and their order are those of snn_leaky_bwd; a request
+ * whose snn_scan_workspace_bytes(desc) exceeds 16 MiB fails them with
+ * SNN_ERR_WORKSPACE, launching nothing.  Allocates nothing.
  * The first call on each device looks up the array's device address (a
  * one-time set-up that is not a stream operation); make that first call
  * before any stream capture.  Every call shares the one array and it keeps
- * the last call's contents (the status word is cleared at the start of each
- * call); calls whose work overlaps on the GPU (other streams, other host
- * threads) race on it and must be serialised by the caller.
+ * the last call's contents.  Each call zeroes, on stream and before its
+ * kernels, the status word and every completion ticket its reductions take,
+ * so a call is correct whatever the previous call's shape or parameter
+ * layouts were and after a call that reported SNN_ERR_TIMEOUT.  Calls whose
+ * work overlaps on the GPU (other streams, other host threads) race on the
+ * array and must be serialised by the caller.
  */
 snn_status_t snn_leaky_bwd_noalloc(const snn_scan_desc* desc, const void* I, const float* ckpt,
                                    const void* mem, const void* spk, const float* beta,

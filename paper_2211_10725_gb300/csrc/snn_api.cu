@@ -206,7 +206,8 @@ snn_status_t scan_bwd(const snn_scan_desc* d, int neuron, const void* I, const f
                       const void* grad_spk, const void* grad_mem, const float* grad_mem_final,
                       const float* grad_syn_final, void* grad_I, float* grad_alpha,
                       float* grad_beta, float* grad_thr, float* grad_mem0, float* grad_syn0,
-                      void* ws, size_t ws_bytes, cudaStream_t stream) {
+                      void* ws, size_t ws_bytes, cudaStream_t stream,
+                      bool reset_control = false) {
   snn_status_t s = check_desc(d);
   if (s != SNN_OK) return s;
   const bool syn = neuron == kSynaptic, rec = neuron == kRecurrentLeaky;
@@ -229,6 +230,16 @@ snn_status_t scan_bwd(const snn_scan_desc* d, int neuron, const void* I, const f
                        grad_mem0, grad_syn0})) != SNN_OK)
     return s;
   if ((s = check_ws(d, ws, ws_bytes)) != SNN_OK) return s;
+  if (reset_control) {
+    // a workspace whose previous contents are unknown (another layout, or a
+    // call that gave up): zero the status word and every ticket this call's
+    // reductions take, on the stream, before any kernel reads them
+    const size_t tickets = kStatusBytes + 3 * lane_bytes(d) + 3 * (size_t)red_scratch(d) * sizeof(double);
+    if (cudaMemsetAsync(ws, 0, kStatusBytes, stream) != cudaSuccess) return SNN_ERR_CUDA;
+    if (cudaMemsetAsync(static_cast<unsigned char*>(ws) + tickets, 0, 3 * ticket_bytes(d), stream) !=
+        cudaSuccess)
+      return SNN_ERR_CUDA;
+  }
   const int64_t L = d->B * d->N;
   float* outs[3] = {grad_beta, grad_thr, (syn || rec) ? grad_alpha : nullptr};
   const int modes[3] = {d->beta_mode, d->thr_mode, d->alpha_mode};
@@ -288,6 +299,21 @@ snn_status_t scan_bwd(const snn_scan_desc* d, int neuron, const void* I, const f
 }  // namespace
 
 std::atomic<unsigned long long> g_kernel_launches{0};
+
+// snn_leaky_bwd on a workspace whose contents are left over from earlier
+// calls of any layout: after the argument checks, the status word and the
+// reductions' tickets are zeroed on the stream (snn_noalloc.cu).
+snn_status_t leaky_bwd_reset_workspace(const snn_scan_desc* d, const void* I, const float* ckpt,
+                                       const void* mem, const void* spk, const float* beta,
+                                       const float* thr, const float* mem0, const void* grad_spk,
+                                       const void* grad_mem, const float* grad_mem_final,
+                                       void* grad_I, float* grad_beta, float* grad_thr,
+                                       float* grad_mem0, void* ws, size_t ws_bytes,
+                                       cudaStream_t stream) {
+  return scan_bwd(d, kLeaky, I, ckpt, mem, spk, nullptr, nullptr, beta, thr, mem0, nullptr,
+                  grad_spk, grad_mem, grad_mem_final, nullptr, grad_I, nullptr, grad_beta,
+                  grad_thr, grad_mem0, nullptr, ws, ws_bytes, stream, true);
+}
 
 }  // namespace snn
 

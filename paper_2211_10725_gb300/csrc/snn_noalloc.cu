@@ -52,25 +52,37 @@ cudaError_t scratch_address(void** out) {
 
 }  // namespace
 
+namespace snn {
+// snn_leaky_bwd that first zeroes the workspace's status word and the
+// tickets of this call's reductions (snn_api.cu).
+snn_status_t leaky_bwd_reset_workspace(const snn_scan_desc* d, const void* I, const float* ckpt,
+                                       const void* mem, const void* spk, const float* beta,
+                                       const float* thr, const float* mem0, const void* grad_spk,
+                                       const void* grad_mem, const float* grad_mem_final,
+                                       void* grad_I, float* grad_beta, float* grad_thr,
+                                       float* grad_mem0, void* ws, size_t ws_bytes,
+                                       cudaStream_t stream);
+}  // namespace snn
+
 extern "C" snn_status_t snn_leaky_bwd_noalloc(
     const snn_scan_desc* desc, const void* I, const float* ckpt, const void* mem,
     const void* spk, const float* beta, const float* thr, const float* mem0,
     const void* grad_spk, const void* grad_mem, const float* grad_mem_final, void* grad_I,
     float* grad_beta, float* grad_thr, float* grad_mem0, int* status, snn_stream_t stream) {
-  const size_t need = snn_scan_workspace_bytes(desc);
-  if (need == 0) return SNN_ERR_INVALID_ARG;
-  if (need > kNoAllocScratchBytes) return SNN_ERR_WORKSPACE;  // beyond the fixed scratch
   if (status && (reinterpret_cast<uintptr_t>(status) & 3u) != 0) return SNN_ERR_ALIGNMENT;
   void* ws = nullptr;
   if (scratch_address(&ws) != cudaSuccess) return SNN_ERR_CUDA;
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
-  // The scratch keeps the previous call's contents.  Only the status word
-  // must start at zero; the partials and reduction scratch are fully
+  // The scratch keeps whatever the previous call left: another layout (its
+  // tickets sit at offsets that depend on B, N and C), or the leftovers of a
+  // call that timed out.  After the same argument checks as snn_leaky_bwd
+  // (a workspace beyond kNoAllocScratchBytes fails them with
+  // SNN_ERR_WORKSPACE), the status word and every reduction ticket this call
+  // takes are zeroed on the stream; the partials and the fp64 scratch are
   // written by this call before they are read.
-  if (cudaMemsetAsync(ws, 0, sizeof(int), st) != cudaSuccess) return SNN_ERR_CUDA;
-  const snn_status_t s =
-      snn_leaky_bwd(desc, I, ckpt, mem, spk, beta, thr, mem0, grad_spk, grad_mem, grad_mem_final,
-                    grad_I, grad_beta, grad_thr, grad_mem0, ws, kNoAllocScratchBytes, stream);
+  const snn_status_t s = snn::leaky_bwd_reset_workspace(
+      desc, I, ckpt, mem, spk, beta, thr, mem0, grad_spk, grad_mem, grad_mem_final, grad_I,
+      grad_beta, grad_thr, grad_mem0, ws, kNoAllocScratchBytes, st);
   if (s != SNN_OK) return s;
   if (status &&
       cudaMemcpyAsync(status, ws, sizeof(int), cudaMemcpyDeviceToDevice, st) != cudaSuccess)
