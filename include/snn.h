@@ -94,6 +94,9 @@ typedef enum {
                                       timeout path without any fault          */
 #define SNN_DEBUG_FORCE_PLAIN 2u   /* take the plain per-lane kernels even
                                       where the staged ones apply             */
+#define SNN_DEBUG_NO_SEGMENT 4u    /* recompute BPTT of the Leaky neuron: take
+                                      the shared-memory replay kernel even
+                                      where the register-segment one applies  */
 
 typedef struct snn_scan_desc {
   int64_t T, B, N;       /* time steps, batch, neurons per sample (C*H*W maps) */
@@ -208,6 +211,13 @@ snn_status_t snn_leaky_fwd(const snn_scan_desc* desc, const void* I, const float
  * d u_{t+1}/d z_t = -thr (subtract), -beta*u_t (zero), 0 (none).
  * Parameter sums are accumulated in fp32 per lane and reduced across lanes
  * in fp64 in a fixed order (deterministic).
+ * SNN_SAVE_RECOMPUTE replays Eq. (4) from each checkpoint bit for bit as the
+ * forward evaluated it.  With ckpt_every 8 (any dtype pair) or 16 (bf16 or
+ * fp16 input and io), no grad_mem, a reset other than SNN_RESET_NONE and B*N
+ * a multiple of 8, the replayed segment stays in registers and a segment's
+ * rows stream in whole (the fast path); otherwise the replay goes through
+ * shared memory.  Both give the same spikes and trace, and gradients within
+ * fp32 rounding of each other.
  */
 snn_status_t snn_leaky_bwd(const snn_scan_desc* desc, const void* I, const float* ckpt,
                            const void* mem, const void* spk, const float* beta,

@@ -20,7 +20,11 @@ template <bool SYN, typename TI, typename TO, int RESET, bool REC = false>
 cudaError_t fwd_staged(ScanArgs a, cudaStream_t st, bool* launched) {
   const void* k = (const void*)scan_fwd_staged<SYN, TI, TO, RESET, REC>;
   StagedPlan p;
-  if (!plan_staged(k, a.L, a.T, (int)sizeof(TI), 0, kLanes<SYN>, &p)) return cudaSuccess;
+  // a stage holds kFwdRows steps of the strip's input row; one CTA per SM
+  // where it fits (the longer rows stream faster)
+  if (!plan_staged(k, a.L, ceil_div(a.T, kFwdRows), kFwdRows * (int)sizeof(TI), 0, kLanes<SYN>, &p,
+                   0, 0, 1))
+    return cudaSuccess;
   a.lanes_per_cta = p.lanes_per_cta;
   a.stages = p.stages;
   a.stage_bytes = p.stage_bytes;

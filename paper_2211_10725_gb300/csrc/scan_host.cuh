@@ -76,16 +76,17 @@ struct StagedPlan {
 //   lanes_per_thread: lanes each consumer thread owns
 //   fixed_bytes_per_lane: other shared memory per lane of the strip
 //   force_stages: exact ring depth the kernel was compiled for (0 = any)
+//   max_cps: most CTAs per SM to try (larger strips first when 1)
 inline bool plan_staged(const void* kernel, int64_t L, int64_t items, int stage_bytes_per_lane,
                         int seg_bytes_per_thread, int lanes_per_thread, StagedPlan* plan,
-                        int fixed_bytes_per_lane = 0, int force_stages = 0) {
+                        int fixed_bytes_per_lane = 0, int force_stages = 0, int max_cps = 2) {
   static std::mutex mu;
   static std::map<std::tuple<int, const void*, int64_t, int64_t, int, int>, StagedPlan> cache;
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess) return false;
   const auto key = std::make_tuple(dev, kernel, L, items, stage_bytes_per_lane,
-                                   (seg_bytes_per_thread * 64 + fixed_bytes_per_lane) * 64 +
-                                       force_stages);
+                                   ((seg_bytes_per_thread * 64 + fixed_bytes_per_lane) * 64 +
+                                    force_stages) * 4 + max_cps);
   {
     std::lock_guard<std::mutex> g(mu);
     auto it = cache.find(key);
@@ -100,7 +101,7 @@ inline bool plan_staged(const void* kernel, int64_t L, int64_t items, int stage_
   if (cudaFuncGetAttributes(&fa, kernel) != cudaSuccess) return false;
   const int min_stages = (int)(items < 3 ? (items < 1 ? 1 : items) : 3);
   for (int waves = 1; waves <= 64; ++waves) {
-    for (int cps = 2; cps >= 1; --cps) {
+    for (int cps = max_cps; cps >= 1; --cps) {
       const int64_t ctas = (int64_t)d.sms * cps * waves;
       const int64_t lpc = round_up(ceil_div(L, ctas), 8);
       const int64_t cthreads = round_up(ceil_div(lpc, lanes_per_thread), 32);
@@ -153,6 +154,11 @@ cudaError_t launch_scan_bwd_leaky_recompute(ScanArgs a, int in_dt, int io_dt, bo
                                             cudaStream_t stream);
 cudaError_t launch_scan_bwd_synaptic_recompute(ScanArgs a, int in_dt, int io_dt, bool staged,
                                                cudaStream_t stream);
+// the recompute BPTT of the Leaky neuron with the replayed segment in
+// registers (scan_bwd_seg), for checkpoint intervals 8 and 16; sets
+// *launched, and launches nothing where it does not apply
+cudaError_t launch_scan_bwd_leaky_seg(ScanArgs a, int in_dt, int io_dt, bool staged,
+                                      cudaStream_t stream, bool* launched);
 // fp64 scratch the reduction of one parameter needs (elements)
 inline int64_t param_reduce_scratch(int64_t N, int64_t C) {
   const int64_t a = 1024, b = 8 * N, c = 64 * C;

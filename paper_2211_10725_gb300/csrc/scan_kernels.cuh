@@ -31,6 +31,7 @@ enum { RESET_SUBTRACT = 0, RESET_ZERO = 1, RESET_NONE = 2 };
 enum { SG_FAST_SIGMOID = 0, SG_ATAN = 1 };
 enum { PM_SCALAR = 0, PM_PER_NEURON = 1, PM_PER_CHANNEL = 2 };
 constexpr uint32_t DEBUG_PRODUCER_IDLE = 1u;
+constexpr uint32_t DEBUG_NO_SEGMENT = 4u;
 constexpr int VEC = 8;                 // lane granularity of a staged CTA strip
 constexpr int kBarrierBytes = 1024;    // full[60], empty[60], ck_full[2], ck_empty[2]
 constexpr int kMaxStages = 60;
@@ -230,19 +231,70 @@ __device__ __forceinline__ float2 add2(float2 a, float2 b) { return __fadd2_rn(a
 __device__ __forceinline__ float2 mul2(float2 a, float2 b) { return __fmul2_rn(a, b); }
 __device__ __forceinline__ float2 fma2(float2 a, float2 b, float2 c) { return __ffma2_rn(a, b, c); }
 
-// Forward step on a pair of lanes: fwd_step on each lane (scalar operations
-// with explicit rounding, which the compiler never fuses; packed fp32x2
-// multiply and add may be fused into a packed FMA, which would change the
-// result).  negthr = -thr; z[0..1] hold z_{t-1} on entry and z_t on exit.
+// Packed fp32x2 add and multiply, round to nearest: one instruction, two
+// correctly rounded lane results.  Measured on sm_103a: a packed multiply
+// whose product feeds a packed add is contracted into a packed fused
+// multiply-add (about half of all results then differ in the last bit), even
+// when both are written in PTX with explicit .rn modifiers, while a scalar
+// __fmul_rn product feeding a packed add is not.  So a product that is added
+// to something else is formed with scalar __fmul_rn (mul_rn_pair); the packed
+// multiply is used only where the product is exact (a spike 0/1 times a
+// value), where a fused rounding gives the same result.
+__device__ __forceinline__ float2 add2_rn(float2 a, float2 b) { return __fadd2_rn(a, b); }
+__device__ __forceinline__ float2 mul_rn_pair(float2 a, float2 b) {
+  return make_float2(__fmul_rn(a.x, b.x), __fmul_rn(a.y, b.y));
+}
+__device__ __forceinline__ float2 mul2_rn(float2 a, float2 b) { return __fmul2_rn(a, b); }
+
+// Eq. (3) as a float: 1.0f where u > thr, else 0.0f (NaN gives 0).
+__device__ __forceinline__ float fire(float u, float thr) {
+  float d;
+  asm("set.gt.f32.f32 %0, %1, %2;" : "=f"(d) : "f"(u), "f"(thr));
+  return d;
+}
+__device__ __forceinline__ float2 fire2(float2 u, float2 negthr) {
+  return make_float2(fire(u.x, -negthr.x), fire(u.y, -negthr.y));
+}
+
+// Forward step on a pair of lanes, the packed form of fwd_step: Eq. (4) /
+// Eqs. (5)-(6) left to right, one correctly rounded operation at a time, so
+// it is bit-identical to fwd_step (and to the float32 evaluation of the
+// equations).  z holds z_{t-1} on entry and z_t on exit as 0.0f / 1.0f.
+//   subtract   u = ((beta*u) + in) + z*(-thr)   z*(-thr) is exact: -thr or -0,
+//              and adding -0 leaves every value (signed zeros included) as is;
+//              one fused multiply-add, which rounds the same single sum
+//   zero       u = (beta*((1-z)*u)) + in        (1-z)*u is u or a zero of u's sign
+//   none       u = (beta*u) + in
+//   Eq. (7)    u = ((beta*u) + in) + z*vmt      vmt = v - thr, rounded once
+// For the Synaptic neuron in = i = (alpha*i) + x first.  `third` is alpha
+// (Synaptic) or vmt (recurrent Leaky).
 template <bool SYN, int RESET, int REC = 0>
-__device__ __forceinline__ void fwd_pair(int reset_rt, float2 beta, float2 negthr, float2 alpha,
-                                         float2 x, float2& u, bool* z, float2& i) {
-  fwd_step<SYN, RESET, REC>(reset_rt, beta.x, -negthr.x, alpha.x, x.x, u.x, z[0], i.x);
-  fwd_step<SYN, RESET, REC>(reset_rt, beta.y, -negthr.y, alpha.y, x.y, u.y, z[1], i.y);
+__device__ __forceinline__ void fwd_pair(int reset_rt, float2 beta, float2 negthr, float2 third,
+                                         float2 x, float2& u, float2& z, float2& i) {
+  const int reset = RESET >= 0 ? RESET : reset_rt;
+  float2 in = x;
+  if (SYN) {
+    i = add2_rn(mul_rn_pair(third, i), x);
+    in = i;
+  }
+  float2 un;
+  if (reset == RESET_ZERO) {
+    const float2 keep = mul2_rn(make_float2(1.0f - z.x, 1.0f - z.y), u);  // exact
+    un = add2_rn(mul_rn_pair(beta, keep), in);
+  } else {
+    un = add2_rn(mul_rn_pair(beta, u), in);
+    // z*(-thr) (or z*vmt) is exact, so the fused z*(-thr) + un rounds once,
+    // exactly as the separate add of the exact product
+    if (REC > 0) un = fma2(z, third, un);
+    else if (reset == RESET_SUBTRACT) un = fma2(z, negthr, un);
+  }
+  u = un;
+  z = fire2(un, negthr);
 }
 
 // Approximate reciprocal (one hardware instruction, relative error ~2^-23)
-// of a value >= 1: the surrogates' denominators, so no subnormals occur.
+// of a surrogate's denominator (>= 1, or >= 1/a for the arctan form with
+// a = alpha/2), so no subnormal occurs.
 __device__ __forceinline__ float rcp_ge1(float d) {
   float r;
   asm("rcp.approx.ftz.f32 %0, %1;" : "=f"(r) : "f"(d));
@@ -332,25 +384,21 @@ struct RingPos {
 
 // Warp-uniform bounded wait: every lane polls the barrier (so every lane
 // acquires the completed phase); the decision to give up is taken by lane 0's
-// clock and shared, so the warp never diverges around it.
+// clock (read every 64 polls) and shared, so the warp never diverges around it.
 __device__ __forceinline__ bool warp_wait(uint64_t* bar, uint32_t parity, uint64_t limit_ns) {
   bool done = mbar_try_wait(bar, parity);
   if (__all_sync(0xffffffffu, done)) return true;
   const uint64_t t0 = globaltimer_ns();
-  while (true) {
+  for (uint32_t i = 1;; ++i) {  // i is warp-uniform
     if (!done) done = mbar_try_wait(bar, parity);
     if (__all_sync(0xffffffffu, done)) return true;
-    uint64_t el = globaltimer_ns() - t0;
-    el = __shfl_sync(0xffffffffu, el, 0);
-    if (el > limit_ns) return false;
+    if ((i & 63u) == 0) {  // the clock every 64 polls
+      uint64_t el = globaltimer_ns() - t0;
+      el = __shfl_sync(0xffffffffu, el, 0);
+      if (el > limit_ns) return false;
+    }
   }
 }
-
-struct Tile {
-  const void* src;  // global address of the strip's row (16-byte aligned)
-  uint32_t bytes;   // multiple of 16
-  uint32_t dst;     // byte offset inside the stage (multiple of 16)
-};
 
 // The single producer thread: fills stage after stage once the consumers
 // have released it, and drains its copies before the CTA may exit.
@@ -365,19 +413,25 @@ struct Producer {
   int64_t issued = 0;
   bool ok = true;
 
-  __device__ __forceinline__ void issue(const Tile* tiles, int n, const ScanArgs& a) {
-    if (!ok) return;
-    // round r >= 1 of stage s waits for the consumers' release of round r-1
-    if (wrapped && !mbar_wait_bounded(&empty[pos.s], pos.ph ^ 1u, a.wait_ns)) {
+  // One item in three calls: begin() waits (bounded) for the consumers'
+  // release of the stage's previous round and announces the item's total
+  // bytes on its full barrier, copy() issues one bulk copy into the stage,
+  // end() moves to the next stage.  Items are built in place, with no
+  // array of copy descriptors in local memory.
+  __device__ __forceinline__ bool begin(uint32_t total, const ScanArgs& a) {
+    if (!ok) return false;
+    if (wrapped && !mbar_wait_spin(&empty[pos.s], pos.ph ^ 1u, a.wait_ns)) {
       record_status(a.status, kStatusTimeout);
       ok = false;
-      return;
+      return false;
     }
-    uint32_t total = 0;
-    for (int k = 0; k < n; ++k) total += tiles[k].bytes;
     mbar_arrive_expect_tx(&full[pos.s], total);
-    unsigned char* dst = ring + (size_t)pos.s * stage_bytes;
-    for (int k = 0; k < n; ++k) bulk_g2s(dst + tiles[k].dst, tiles[k].src, tiles[k].bytes, &full[pos.s]);
+    return true;
+  }
+  __device__ __forceinline__ void copy(uint32_t dst, const void* src, uint32_t bytes) {
+    bulk_g2s(ring + (size_t)pos.s * stage_bytes + dst, src, bytes, &full[pos.s]);
+  }
+  __device__ __forceinline__ void end() {
     ++issued;
     pos.next(S);
     if (pos.s == 0) wrapped = true;
@@ -493,9 +547,13 @@ __device__ __forceinline__ void initial_state(const ScanArgs& a, int64_t l, cons
 // Staged forward
 // ---------------------------------------------------------------------------
 
+// Rows (time steps) per ring stage of the staged forward: one wait and one
+// release per kFwdRows steps instead of per step.
+constexpr int kFwdRows = 8;
+
 template <bool SYN, typename TI, typename TO, int RESET, bool REC = false>
 __global__ void __launch_bounds__(kMaxStagedThreads) scan_fwd_staged(const ScanArgs a) {
-  constexpr int V = kLanes<SYN>, NP = V / 2;
+  constexpr int V = kLanes<SYN>, NP = V / 2, R = kFwdRows;
   extern __shared__ __align__(1024) unsigned char smem[];
   uint64_t* full = reinterpret_cast<uint64_t*>(smem);
   uint64_t* empty = full + kMaxStages;
@@ -505,16 +563,21 @@ __global__ void __launch_bounds__(kMaxStagedThreads) scan_fwd_staged(const ScanA
   const int warp = threadIdx.x >> 5, lid = threadIdx.x & 31;
   const int64_t lane0 = (int64_t)blockIdx.x * a.lanes_per_cta;
   const int cta_lanes = (int)min((int64_t)a.lanes_per_cta, a.L - lane0);
+  const int row_elems = a.lanes_per_cta;  // a stage holds R rows of the strip
   init_ring_barriers(full, empty, S, cwarps);
   grid_dep_wait();  // the previous kernel on the stream is complete
 
   if (warp == cwarps) {  // producer warp
     if (lid == 0 && !(a.debug & DEBUG_PRODUCER_IDLE)) {
       Producer p{ring, full, empty, S, a.stage_bytes};
-      Tile tile{static_cast<const TI*>(a.I) + lane0, (uint32_t)cta_lanes * (uint32_t)sizeof(TI), 0};
-      for (int64_t t = 0; t < a.T && p.ok; ++t) {
-        p.issue(&tile, 1, a);
-        tile.src = static_cast<const TI*>(tile.src) + a.L;
+      const uint32_t bytes = (uint32_t)cta_lanes * (uint32_t)sizeof(TI);
+      const uint32_t row_bytes = (uint32_t)row_elems * (uint32_t)sizeof(TI);
+      const TI* src = static_cast<const TI*>(a.I) + lane0;
+      for (int64_t t0 = 0; t0 < a.T; t0 += R) {
+        const int nr = (int)min((int64_t)R, a.T - t0);
+        if (!p.begin((uint32_t)nr * bytes, a)) break;
+        for (int r = 0; r < nr; ++r) p.copy((uint32_t)r * row_bytes, src + (t0 + r) * a.L, bytes);
+        p.end();
       }
       p.drain();
     }
@@ -524,11 +587,16 @@ __global__ void __launch_bounds__(kMaxStagedThreads) scan_fwd_staged(const ScanA
   const int c = threadIdx.x;
   const int64_t l = lane0 + (int64_t)c * V;
   const bool active = c * V < cta_lanes;
-  float2 beta[NP], negthr[NP], alpha[NP], u[NP], in[NP];
-  bool z[V];
+  float2 beta[NP], negthr[NP], third[NP], u[NP], z[NP], in[NP];
   if (active) {
-    load_params<SYN || REC, NP>(a, l, beta, negthr, alpha);
-    initial_state<SYN, NP>(a, l, negthr, u, z, in);
+    load_params<SYN || REC, NP>(a, l, beta, negthr, third);
+    bool zb[V];
+    initial_state<SYN, NP>(a, l, negthr, u, zb, in);
+#pragma unroll
+    for (int k = 0; k < NP; ++k) {
+      z[k] = make_float2(zb[2 * k] ? 1.0f : 0.0f, zb[2 * k + 1] ? 1.0f : 0.0f);
+      if (REC) third[k] = add2_rn(third[k], negthr[k]);  // v - thr, rounded once
+    }
   }
   TO* spk = static_cast<TO*>(a.spk) + l;
   TO* mem = a.mem ? static_cast<TO*>(a.mem) + l : nullptr;
@@ -542,50 +610,65 @@ __global__ void __launch_bounds__(kMaxStagedThreads) scan_fwd_staged(const ScanA
   const int stage_elems = a.stage_bytes / (int)sizeof(TI);
   RingPos pos;
   int kk = a.nseg > 0 ? seg_phase0(a) : 0;  // position inside the current checkpoint segment
-  for (int64_t t = 0; t < a.T; ++t) {
+  for (int64_t t0 = 0; t0 < a.T; t0 += R) {
     if (!warp_wait(&full[pos.s], pos.ph, a.wait_ns)) {
       if (lid == 0) record_status(a.status, kStatusTimeout);
       break;
     }
-    unsigned zbits = 0;
+    const int nr = (int)min((int64_t)R, a.T - t0);
+    unsigned zbits[R];
     if (active) {
-      float2 x[NP];
-      load_pairs<TI, NP>(my + pos.s * stage_elems, x);
-      float2 zf[NP];
+      const TI* st = my + pos.s * stage_elems;
 #pragma unroll
-      for (int k = 0; k < NP; ++k) {
-        fwd_pair<SYN, RESET, REC ? 1 : 0>(a.reset, beta[k], negthr[k], alpha[k], x[k], u[k],
-                                          &z[2 * k], in[k]);
-        zf[k] = make_float2(z[2 * k] ? 1.0f : 0.0f, z[2 * k + 1] ? 1.0f : 0.0f);
-      }
+      for (int r = 0; r < R; ++r) {
+        zbits[r] = 0;
+        if (r < nr) {
+          float2 x[NP];
+          load_pairs<TI, NP>(st + r * row_elems, x);
 #pragma unroll
-      for (int k = 0; k < V; ++k) zbits |= (z[k] ? 1u : 0u) << k;
-      store_pairs<TO, NP>(spk, zf);
-      if (mem) store_pairs<TO, NP>(mem, u);
-      if (SYN && syn) store_pairs<TO, NP>(syn, in);
-      if (++kk == a.K) {
-        kk = 0;
-        if (ck && t + 1 < a.T) {
-          store_pairs<float, NP>(ck, u);
-          if (SYN) store_pairs<float, NP>(ck + a.L, in);
-          ck += ck_stride;
+          for (int k = 0; k < NP; ++k)
+            fwd_pair<SYN, RESET, REC ? 1 : 0>(a.reset, beta[k], negthr[k], third[k], x[k], u[k],
+                                              z[k], in[k]);
+          if (bits) {
+#pragma unroll
+            for (int k = 0; k < NP; ++k) {
+              zbits[r] |= ((z[k].x != 0.0f) ? 1u : 0u) << (2 * k);
+              zbits[r] |= ((z[k].y != 0.0f) ? 1u : 0u) << (2 * k + 1);
+            }
+          }
+          store_pairs<TO, NP>(spk + r * a.L, z);
+          if (mem) store_pairs<TO, NP>(mem + r * a.L, u);
+          if (SYN && syn) store_pairs<TO, NP>(syn + r * a.L, in);
+          if (++kk == a.K) {
+            kk = 0;
+            if (ck && t0 + r + 1 < a.T) {
+              store_pairs<float, NP>(ck, u);
+              if (SYN) store_pairs<float, NP>(ck + a.L, in);
+              ck += ck_stride;
+            }
+          }
         }
       }
     }
     if (bits) {
-      if (SYN) {
-        const unsigned hi = __shfl_down_sync(0xffffffffu, zbits, 1);
-        if (active && !(c & 1)) *bits = (unsigned char)(zbits | (hi << 4));
-      } else if (active) {
-        *bits = (unsigned char)zbits;
+#pragma unroll
+      for (int r = 0; r < R; ++r) {
+        if (r < nr) {
+          if (SYN) {
+            const unsigned hi = __shfl_down_sync(0xffffffffu, zbits[r], 1);
+            if (active && !(c & 1)) bits[r * a.bits_row] = (unsigned char)(zbits[r] | (hi << 4));
+          } else if (active) {
+            bits[r * a.bits_row] = (unsigned char)zbits[r];
+          }
+        }
       }
-      bits += a.bits_row;
+      bits += R * a.bits_row;
     }
     release_stage(empty, pos.s, lid);
     pos.next(S);
-    spk += a.L;
-    if (mem) mem += a.L;
-    if (SYN && syn) syn += a.L;
+    spk += R * a.L;
+    if (mem) mem += R * a.L;
+    if (SYN && syn) syn += R * a.L;
   }
   if (active) {
     if (a.mem_final) store_pairs<float, NP>(a.mem_final + l, u);
@@ -658,23 +741,22 @@ __global__ void __launch_bounds__(kMaxStagedThreads) scan_bwd_staged(const ScanA
       const uint32_t bo = (uint32_t)cta_lanes * sizeof(TO);
       const uint32_t bi = (uint32_t)cta_lanes * sizeof(TI);
       const uint32_t bc = (uint32_t)cta_lanes * 4u;
-      (void)bi;
-      Tile tiles[5];
       if (!RECOMP) {
-        for (int64_t t = a.T - 1; t >= 0 && p.ok; --t) {
-          int n = 0;
-          tiles[n] = Tile{row<TO>(a.gs, t, a.L, lane0), bo, (uint32_t)(n * io_stride)}; ++n;
-          tiles[n] = Tile{row<TO>(a.mem_in, t, a.L, lane0), bo, (uint32_t)(n * io_stride)}; ++n;
-          if (use_bits) {
-            const unsigned char* src = a.bits + t * a.bits_row + lane0 / 8 - bits_skew;
-            const uint32_t nb = (uint32_t)(bits_skew + cta_lanes / 8 + 15) & ~15u;
-            tiles[n] = Tile{src, nb, (uint32_t)(n * io_stride)}; ++n;
-          } else if (half_store) {
-            tiles[n] = Tile{row<TO>(a.spk_in, t, a.L, lane0), bo, (uint32_t)(n * io_stride)}; ++n;
-          }
-          if (want_syn) { tiles[n] = Tile{row<TO>(a.syn_in, t, a.L, lane0), bo, (uint32_t)(n * io_stride)}; ++n; }
-          if (a.gm) { tiles[n] = Tile{row<TO>(a.gm, t, a.L, lane0), bo, (uint32_t)(n * io_stride)}; ++n; }
-          p.issue(tiles, n, a);
+        const uint32_t nb = (uint32_t)(bits_skew + cta_lanes / 8 + 15) & ~15u;  // bit row
+        const int n_io = 2 + ((half_store && !use_bits) ? 1 : 0) + (want_syn ? 1 : 0) + (a.gm ? 1 : 0);
+        const uint32_t total = (uint32_t)n_io * bo + (use_bits ? nb : 0u);
+        for (int64_t t = a.T - 1; t >= 0; --t) {
+          if (!p.begin(total, a)) break;
+          uint32_t n = 0;
+          p.copy(n++ * io_stride, row<TO>(a.gs, t, a.L, lane0), bo);
+          p.copy(n++ * io_stride, row<TO>(a.mem_in, t, a.L, lane0), bo);
+          if (use_bits)
+            p.copy(n++ * io_stride, a.bits + t * a.bits_row + lane0 / 8 - bits_skew, nb);
+          else if (half_store)
+            p.copy(n++ * io_stride, row<TO>(a.spk_in, t, a.L, lane0), bo);
+          if (want_syn) p.copy(n++ * io_stride, row<TO>(a.syn_in, t, a.L, lane0), bo);
+          if (a.gm) p.copy(n++ * io_stride, row<TO>(a.gm, t, a.L, lane0), bo);
+          p.end();
         }
       } else {
         int64_t ck_n = 0;  // checkpoint loads issued
@@ -685,7 +767,7 @@ __global__ void __launch_bounds__(kMaxStagedThreads) scan_bwd_staged(const ScanA
             // the segment's starting state: checkpoint rows fp32 [nseg-1][SYN?2:1][L]
             const int slot = (int)(ck_n & 1);
             if (ck_n >= 2 &&
-                !mbar_wait_bounded(&ck_empty[slot], (uint32_t)(((ck_n >> 1) - 1) & 1), a.wait_ns)) {
+                !mbar_wait_spin(&ck_empty[slot], (uint32_t)(((ck_n >> 1) - 1) & 1), a.wait_ns)) {
               record_status(a.status, kStatusTimeout);
               p.ok = false;
               break;
@@ -698,14 +780,15 @@ __global__ void __launch_bounds__(kMaxStagedThreads) scan_bwd_staged(const ScanA
             ++ck_n;
           }
           for (int64_t t = t0; t < t1 && p.ok; ++t) {
-            const Tile tile{row<TI>(a.I, t, a.L, lane0), bi, 0};
-            p.issue(&tile, 1, a);
+            if (!p.begin(bi, a)) break;
+            p.copy(0, row<TI>(a.I, t, a.L, lane0), bi);
+            p.end();
           }
           for (int64_t t = t1 - 1; t >= t0 && p.ok; --t) {
-            int n = 0;
-            tiles[n++] = Tile{row<TO>(a.gs, t, a.L, lane0), bo, 0};
-            if (a.gm) tiles[n++] = Tile{row<TO>(a.gm, t, a.L, lane0), bo, (uint32_t)io_stride};
-            p.issue(tiles, n, a);
+            if (!p.begin(bo * (a.gm ? 2u : 1u), a)) break;
+            p.copy(0, row<TO>(a.gs, t, a.L, lane0), bo);
+            if (a.gm) p.copy((uint32_t)io_stride, row<TO>(a.gm, t, a.L, lane0), bo);
+            p.end();
           }
         }
         for (int64_t j = ck_n > 2 ? ck_n - 2 : 0; j < ck_n; ++j)
@@ -816,8 +899,10 @@ __global__ void __launch_bounds__(kMaxStagedThreads) scan_bwd_staged(const ScanA
     }
   } else {
     int64_t ck_u = 0;  // checkpoints consumed
-    float2 u[NP], ii[NP];
-    bool z[V];
+    float2 u[NP], ii[NP], z[NP], third[NP];
+#pragma unroll
+    for (int q = 0; q < NP; ++q)  // alpha (Synaptic), or v - thr rounded once (Eq. 7)
+      third[q] = REC ? add2_rn(alpha[q], negthr[q]) : alpha[q];
     // Start of segment k: its starting state from the checkpoint slot (k > 0)
     // or the initial state (k = 0).
     auto seg_start = [&](int k) -> bool {
@@ -832,13 +917,14 @@ __global__ void __launch_bounds__(kMaxStagedThreads) scan_bwd_staged(const ScanA
           load_pairs<float, NP>(cb, u);
           if (SYN) load_pairs<float, NP>(cb + a.lanes_per_cta, ii);
 #pragma unroll
-          for (int q = 0; q < NP; ++q) {
-            z[2 * q] = u[q].x > -negthr[q].x;
-            z[2 * q + 1] = u[q].y > -negthr[q].y;
-          }
+          for (int q = 0; q < NP; ++q) z[q] = fire2(u[q], negthr[q]);
         }
       } else if (active) {
-        initial_state<SYN, NP>(a, l, negthr, u, z, ii);
+        bool zb[V];
+        initial_state<SYN, NP>(a, l, negthr, u, zb, ii);
+#pragma unroll
+        for (int q = 0; q < NP; ++q)
+          z[q] = make_float2(zb[2 * q] ? 1.0f : 0.0f, zb[2 * q + 1] ? 1.0f : 0.0f);
       }
       return true;
     };
@@ -857,8 +943,8 @@ __global__ void __launch_bounds__(kMaxStagedThreads) scan_bwd_staged(const ScanA
       load_pairs<TI, NP>(xin, x);
 #pragma unroll
       for (int q = 0; q < NP; ++q)
-        fwd_pair<SYN, RESET, REC ? 1 : 0>(a.reset, beta[q], negthr[q], alpha[q], x[q], u[q],
-                                          &z[2 * q], ii[q]);
+        fwd_pair<SYN, RESET, REC ? 1 : 0>(a.reset, beta[q], negthr[q], third[q], x[q], u[q],
+                                          z[q], ii[q]);
 #pragma unroll
       for (int q = 0; q < V / 4; ++q) {
         *reinterpret_cast<float4*>(su + q * nthr * 4) =

@@ -158,12 +158,7 @@ __device__ __forceinline__ bool mbar_wait_poll(uint64_t* bar, uint32_t parity, u
 #if SNN_GEMM_SLEEP_WAIT
   return mbar_wait_bounded(bar, parity, limit_ns);
 #else
-  if (mbar_try_wait(bar, parity)) return true;
-  const uint64_t t0 = globaltimer_ns();
-  for (uint32_t i = 1;; ++i) {
-    if (mbar_try_wait(bar, parity)) return true;
-    if ((i & 63u) == 0 && globaltimer_ns() - t0 > limit_ns) return false;
-  }
+  return mbar_wait_spin(bar, parity, limit_ns);
 #endif
 }
 

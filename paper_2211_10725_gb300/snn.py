@@ -32,6 +32,7 @@ PMODE_CODE = {"scalar": 0, "per_neuron": 1, "per_channel": 2}
 SAVE_CODE = {"mem": 0, "recompute": 1}
 DEBUG_PRODUCER_IDLE = 1
 DEBUG_FORCE_PLAIN = 2
+DEBUG_NO_SEGMENT = 4
 
 
 class SnnError(RuntimeError):
