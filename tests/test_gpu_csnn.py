@@ -475,3 +475,226 @@ def test_csnn_training_lowers_the_loss(cuda_device):
     # the padded channels' betas never move
     for l, (c, _) in enumerate(w.convs):
         assert torch.all(net.beta[l][c:] == w.beta)
+
+
+# ---------------------------------------------------------------------------
+# Stage by stage with He-uniform weights as drawn (no flushing), teacher-forced
+# ---------------------------------------------------------------------------
+
+BF16_HALF_ULP = 2.0 ** -8   # |bf16 rounding error| <= 2^-8 |value|
+ACC_RTOL = 1e-5             # fp32 accumulation, of the magnitude of the summed terms
+GEMM_RTOL = 1e-5
+
+
+def _close_bf16(name, got, ref, scale):
+    """One bf16 rounding of an fp32 result: |got - ref| <= 2^-8 |ref| +
+    1e-5 * scale (the magnitude of the summed terms); returns the count
+    needing the scale term."""
+    return H.assert_close(name, got, ref, BF16_HALF_ULP, ACC_RTOL * scale + 1e-30)
+
+
+def _col2im(dcols, Hh, Ww, k):
+    """Sum of the patch-row gradients [M, Ho, Wo, k, k, C] into the input
+    map [M, Hh, Ww, C] (float64)."""
+    M, Ho, Wo, _, _, C = dcols.shape
+    out = np.zeros((M, Hh, Ww, C))
+    for ky in range(k):
+        for kx in range(k):
+            out[:, ky:ky + Ho, kx:kx + Wo, :] += dcols[:, :, :, ky, kx, :]
+    return out
+
+
+def _scan_forced(w, l_name, I32, beta, zg, bound, counts, sizes, mem_gpu=None):
+    """The oracle's float32 Leaky scan (Eq. 4, reset to zero) with its reset
+    held at the GPU's spikes zg [T, L]; a GPU spike may differ from the
+    oracle's decision only within the currents' error bound of the
+    threshold.  Returns the trace the GPU's reverse pass reads (its stored
+    bf16 trace, checked against the oracle's, or the oracle's fp32 one)."""
+    T, L = zg.shape
+    z_reset = np.vstack([np.zeros((1, L)), zg[:-1]])
+    spk32, mem32 = O.leaky_forward(I32, beta.astype(np.float32), np.full(L, w.thr, np.float32),
+                                   w.reset, dtype=np.float32, z_reset=z_reset)
+    spk32, mem32 = spk32.astype(np.float64), mem32.astype(np.float64)
+    diff = spk32 != zg
+    allowed = np.maximum(H.AMBIGUITY, 2.0 * bound)
+    assert np.all(np.abs(mem32 - w.thr)[diff] < allowed[diff]), f"{l_name}: spike off threshold"
+    counts[f"{l_name}_spk_forced"], sizes[f"{l_name}_spk_forced"] = int(diff.sum()), T * L
+    if mem_gpu is None:
+        return mem32
+    # the GPU rounds its own fp32 membrane, within 2 * bound of the oracle's:
+    # rounding is monotone, so the stored value lies between the roundings
+    # of the interval's ends
+    exact = O.bf16_round(mem32)
+    lo = O.bf16_round(mem32 - 2.0 * bound - 1e-7)
+    hi = O.bf16_round(mem32 + 2.0 * bound + 1e-7)
+    bad = ~((mem_gpu == exact) | ((mem_gpu >= lo) & (mem_gpu <= hi)))
+    if bad.any():
+        i = np.argwhere(bad)[:5]
+        d = np.abs(mem_gpu - mem32)[bad]
+        raise AssertionError(
+            f"{l_name}: stored membrane: {bad.sum()} of {bad.size}; first {i.tolist()}; "
+            f"gpu {mem_gpu[bad][:5]} oracle {mem32[bad][:5]} bound {bound[bad][:5]}; "
+            f"max |diff| {d.max()}; forced here {diff[bad].sum()}")
+    counts[f"{l_name}_mem_midpoint"] = int((mem_gpu != exact).sum())
+    sizes[f"{l_name}_mem_midpoint"] = T * L
+    return mem_gpu
+
+
+def _bound(w, S, T, beta):
+    """Running bound on the membrane from currents within GEMM_RTOL of their
+    summed terms S [T, L] (Eq. 4 carries it with factor beta)."""
+    e, out = np.zeros(S.shape[1]), np.zeros_like(S)
+    for t in range(T):
+        e = beta * e + GEMM_RTOL * S[t] + 1e-6 + 4 * H.EPS32 * (1.0 + S[t])
+        out[t] = e
+    return out
+
+
+def check_csnn_stagewise(w, inp, net, widened_frac=1e-3):
+    """Each stage of the CSNN step against the oracle's, fed the GPU's own
+    inputs to that stage (teacher forcing at every element where several
+    results are correct; see check_dsnn_stagewise).  Layout stages (pooling,
+    its backward) must be exact functions of the GPU's inputs; every bf16
+    result is one rounding of an fp32 one (2^-8 of |ref| plus 1e-5 of the
+    summed terms); fp32 weight and beta gradients are within 1e-5 of their
+    summed terms."""
+    T, B, M = w.T, w.B, w.T * w.B
+    convs = [_np(c) for c in inp["convs"]]
+    Wfc = _np(inp["Wfc"])
+    X = _np(inp["X"]).reshape(M, w.H, w.W, w.Cin)
+    labels = _np(inp["labels"]).astype(np.int64)
+    nl = len(convs)
+    counts, sizes = {}, {}
+    stored = net.layers[0].mem is not None
+    ins, traces, spks = [], [], []
+    x = X
+    for l in range(nl):
+        cout, k = w.convs[l]
+        _, _, cin_p, cp, _, Ho, Wo, *_r = net.geo[l]
+        L = B * Ho * Wo * cout
+        I64 = O.conv2d_nhwc(x, convs[l])
+        S = O.conv2d_nhwc(np.abs(x), np.abs(convs[l]))
+        beta = np.tile(np.full(cout, w.beta), B * Ho * Wo)
+        zg = _np(net.layers[l].spk).reshape(M, Ho, Wo, cp)[..., :cout].reshape(T, L)
+        if net.I[l] is not None:
+            Ig = _np(net.I[l]).reshape(M, Ho, Wo, cp)
+            H.assert_close(f"I{l}", Ig[..., :cout], I64, GEMM_RTOL, 1e-6, S)
+            I32, bound = Ig[..., :cout].reshape(T, L).astype(np.float32), np.zeros((T, L))
+        else:
+            I32 = I64.reshape(T, L).astype(np.float32)
+            bound = _bound(w, S.reshape(T, L), T, w.beta)
+        mem_g = None
+        if stored:
+            mem_g = _np(net.layers[l].mem).reshape(M, Ho, Wo, cp)[..., :cout].reshape(T, L)
+        traces.append(_scan_forced(w, f"conv{l}", I32, beta, zg, bound, counts, sizes, mem_g))
+        spks.append(zg)
+        s = zg.reshape(M, Ho, Wo, cout)
+        p, idx = O.maxpool2_nhwc(s)
+        pg = _np(net.pool[l])
+        assert np.array_equal(pg[..., :cout], p) and not pg[..., cout:].any(), f"pool {l}"
+        assert np.array_equal(net.idx[l].cpu().numpy().astype(np.int64)[..., :cout], idx)
+        ins.append(x)
+        x = p
+    n = w.n_classes
+    flat = x.reshape(M, -1)
+    Lf = B * n
+    Ifc64 = O.dense_forward(flat, Wfc)
+    Sfc = np.abs(flat) @ np.abs(Wfc).T
+    zo = _np(net.out_layer.spk)[:, :, :n].reshape(T, Lf)
+    if net.I_fc is not None:
+        Ig = _np(net.I_fc)[:, :n]
+        H.assert_close("I_fc", Ig, Ifc64, GEMM_RTOL, 1e-6, Sfc)
+        I32, bound = Ig.reshape(T, Lf).astype(np.float32), np.zeros((T, Lf))
+    else:
+        I32, bound = Ifc64.reshape(T, Lf).astype(np.float32), _bound(w, Sfc.reshape(T, Lf), T,
+                                                                      w.beta_fc)
+    mem_o = _np(net.out_layer.mem)[:, :, :n].reshape(T, Lf) if stored else None
+    trace_o = _scan_forced(w, "out", I32, np.full(Lf, w.beta_fc), zo, bound, counts, sizes, mem_o)
+
+    # loss and readout
+    loss_o, g_o = O.rate_ce_loss(zo.reshape(T, B, n), labels)
+    assert abs(float(net.loss.item()) - loss_o) <= 1e-6 * max(1.0, abs(loss_o))
+    go = _np(net.grad_out)
+    H.assert_close("grad_out", go[:, :, :n], g_o, BF16_HALF_ULP, 1e-7)
+    gs = g_o.reshape(T, Lf) if net.fused_loss else go[:, :, :n].reshape(T, Lf)
+    kw = dict(reset=w.reset, detach=True, sg="fast_sigmoid", sg_param=w.sg_param)
+    thr_o = np.full(Lf, w.thr)
+    ref = O.leaky_backward(trace_o, zo, gs, np.full(Lf, w.beta_fc), thr_o, **kw)
+    mag = O.leaky_backward(trace_o, zo, np.abs(gs), np.full(Lf, w.beta_fc), thr_o, **kw)
+    gI = _np(net.out_layer.grad_I)[:, :, :n].reshape(T, Lf)
+    counts["grad_I_fc"] = _close_bf16("grad_I_fc", gI, ref["grad_I"],
+                                      np.maximum(mag["grad_I"], np.abs(ref["grad_I"])))
+    sizes["grad_I_fc"] = T * Lf
+    dI = gI.reshape(M, n)
+    H.assert_close("dW_fc", _np(net.fc_weight(net.dW_flat)), dI.T @ flat, ACC_RTOL, 1e-12,
+                   np.abs(dI).T @ np.abs(flat))
+    d_flat, d_mag = dI @ Wfc, np.abs(dI) @ np.abs(Wfc)
+    cl = w.convs[-1][0]
+    gp = _np(net.grad_pool[-1])
+    Hp, Wp, cpl = gp.shape[1], gp.shape[2], gp.shape[3]
+    counts["grad_pool_top"] = _close_bf16("grad_pool_top", gp[..., :cl].reshape(M, -1), d_flat,
+                                          d_mag)
+    sizes["grad_pool_top"] = d_flat.size
+    # the conv layers, top down
+    for l in range(nl - 1, -1, -1):
+        cout, k = w.convs[l]
+        _, _, cin_p, cp, _, Ho, Wo, *_r = net.geo[l]
+        L = B * Ho * Wo * cout
+        gpool = _np(net.grad_pool[l])[..., :cout]
+        _, idx = O.maxpool2_nhwc(spks[l].reshape(M, Ho, Wo, cout))
+        d_spk = O.maxpool2_nhwc_backward(gpool, idx, (M, Ho, Wo, cout))
+        gsp = _np(net.grad_spk[l]).reshape(M, Ho, Wo, cp)
+        assert np.array_equal(gsp[..., :cout], d_spk) and not gsp[..., cout:].any(), \
+            f"pool {l} backward"
+        g = d_spk.reshape(T, L)
+        beta = np.tile(np.full(cout, w.beta), B * Ho * Wo)
+        ref = O.leaky_backward(traces[l], spks[l], g, beta, np.full(L, w.thr), **kw)
+        mag = O.leaky_backward(traces[l], spks[l], np.abs(g), beta, np.full(L, w.thr), **kw)
+        gI = _np(net.layers[l].grad_I).reshape(M, Ho, Wo, cp)
+        counts[f"grad_I{l}"] = _close_bf16(f"grad_I{l}", gI[..., :cout].reshape(T, L),
+                                           ref["grad_I"],
+                                           np.maximum(mag["grad_I"], np.abs(ref["grad_I"])))
+        sizes[f"grad_I{l}"] = T * L
+        # per-channel beta: du_t * (1 - z_{t-1}) u_{t-1}, summed over t and the channel's lanes
+        prev = np.vstack([np.zeros((1, L)), np.abs(traces[l][:-1])])
+        db_mag = (mag["grad_I"] * prev).reshape(-1, cout).sum(axis=0)
+        db_ref = O.reduce_lane_grad(ref["grad_beta_lane"], B, Ho * Wo * cout, "per_channel",
+                                    C=cout, HW=1)
+        H.assert_close(f"dbeta{l}", _np(net.dbeta[l])[:cout], db_ref, ACC_RTOL, 1e-9, db_mag)
+        dIl = gI[..., :cout]
+        dX, dW = O.conv2d_nhwc_backward(ins[l], convs[l], dIl)
+        _, dW_mag = O.conv2d_nhwc_backward(np.abs(ins[l]), np.abs(convs[l]), np.abs(dIl))
+        H.assert_close(f"dW{l}", _np(net.conv_weight(l, net.dW_flat)), dW, ACC_RTOL, 1e-12, dW_mag)
+        if l > 0:
+            # patch-row gradients (one rounding each), then col2im of the GPU's
+            # patch rows (one rounding of their fp32 sum)
+            cin = w.convs[l - 1][0]
+            dc = _np(net.dcols[l])[:, : k * k * cin_p].reshape(M, Ho, Wo, k, k, cin_p)[..., :cin]
+            W2 = convs[l].reshape(cout, -1)
+            rows = dIl.reshape(-1, cout)
+            dc_ref = (rows @ W2).reshape(M, Ho, Wo, k, k, cin)
+            dc_mag = (np.abs(rows) @ np.abs(W2)).reshape(M, Ho, Wo, k, k, cin)
+            counts[f"dcols{l}"] = _close_bf16(f"dcols{l}", dc, dc_ref, dc_mag)
+            sizes[f"dcols{l}"] = dc.size
+            Hh, Ww = ins[l].shape[1], ins[l].shape[2]
+            gp = _np(net.grad_pool[l - 1])[..., :cin]
+            ci_ref, ci_mag = _col2im(dc, Hh, Ww, k), _col2im(np.abs(dc), Hh, Ww, k)
+            counts[f"col2im{l}"] = _close_bf16(f"col2im{l}", gp, ci_ref, ci_mag)
+            sizes[f"col2im{l}"] = gp.size
+    H.assert_widened(counts, sizes, widened_frac)
+    return counts
+
+
+@pytest.mark.parametrize("save", ["recompute", "fused"])
+@pytest.mark.parametrize("w", [SMALL, W.CSNN_C4], ids=lambda w: w.name)
+def test_csnn_step_real_weights_stagewise(w, save, cuda_device):
+    """The step with the He-uniform weights as drawn (every sum rounds in
+    fp32), at T = 4, B = 8 and at the benchmark's T = 25, B = 128: every
+    element of every stage, teacher-forced."""
+    inp = W.make_conv_inputs(w)
+    net, X, labels = _run(w, inp, cuda_device, save=save)
+    net.step(X, labels)
+    torch.cuda.synchronize()
+    for layer in net.layers + [net.out_layer]:
+        assert layer.status() == 0
+    print(w.name, save, check_csnn_stagewise(w, inp, net))
