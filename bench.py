@@ -67,6 +67,8 @@ def parse():
                    help="scan workloads: skip timing the other save variants")
     p.add_argument("--ckpt-every", type=int, default=None,
                    help="recompute variant: checkpoint interval K")
+    p.add_argument("--batch", type=int, default=None,
+                   help="scan workloads: another batch size B (a smaller case for profiling)")
     p.add_argument("--no-torch-eager", action="store_true",
                    help="skip the PyTorch-eager per-timestep context measurement")
     p.add_argument("--cpu-seconds", type=float, default=15.0)
@@ -80,6 +82,8 @@ def workload(args):
     w = W.SCAN_WORKLOADS[args.workload]
     save = args.save or DEFAULT_SAVE.get(w.name, ("mem", w.ckpt_every))[0]
     k = args.ckpt_every or DEFAULT_SAVE.get(w.name, ("mem", w.ckpt_every))[1]
+    if args.batch and args.batch != w.B:
+        w = w.scaled(B=args.batch, name=w.name.replace(f"_B{w.B}_", f"_B{args.batch}_"))
     return w.scaled(save=save, ckpt_every=k)
 
 

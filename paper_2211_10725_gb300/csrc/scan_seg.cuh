@@ -21,16 +21,18 @@
 //
 // Against the shared-memory replay buffer of scan_bwd_staged, the trace
 // costs no shared memory and no load or store instructions, so the ring
-// takes all of the shared memory and KC = 16 halves the checkpoint bytes of
-// KC = 8.
+// takes all of the shared memory.  KC = 16 would halve the checkpoint bytes
+// of KC = 8, but at 128 registers a thread it runs slower (0.32 against
+// 0.29 ms on the 524,288-lane, T = 500 workload); KC = 8 is the default.
 #pragma once
 
 #include "scan_kernels.cuh"
 
 namespace snn {
 
-// Lanes per consumer thread (8 lanes at KC = 8 measured slower: the trace
-// then spills past 128 registers).
+// Lanes per consumer thread: the trace is KC x kSegLanes fp32 registers.
+// Measured slower: 8 lanes at KC = 8 (the trace spills past 128 registers),
+// 2 lanes at KC = 16 or 32 (more steps' overhead per lane, and three waves).
 template <int KC>
 constexpr int kSegLanes = 4;
 
