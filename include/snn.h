@@ -210,10 +210,11 @@ snn_status_t snn_leaky_fwd(const snn_scan_desc* desc, const void* I, const float
  * where d u_{t+1}/d u_t = beta (subtract/none) or beta*(1-z_t) (zero) and
  * d u_{t+1}/d z_t = -thr (subtract), -beta*u_t (zero), 0 (none).
  * Parameter sums are accumulated in fp32 per lane and reduced across lanes
- * in fp64 in a fixed order (deterministic).
+ * in a fixed order (deterministic): runs of a few lanes in fp32, everything
+ * above them in fp64.
  * SNN_SAVE_RECOMPUTE replays Eq. (4) from each checkpoint bit for bit as the
- * forward evaluated it.  With ckpt_every 8 (any dtype pair) or 16 (bf16 or
- * fp16 input and io), no grad_mem, a reset other than SNN_RESET_NONE and B*N
+ * forward evaluated it.  With ckpt_every 8 (any dtype pair), 12 or 16 (bf16
+ * or fp16 input and io), no grad_mem, a reset other than SNN_RESET_NONE and B*N
  * a multiple of 8, the replayed segment stays in registers and a segment's
  * rows stream in whole (the fast path); otherwise the replay goes through
  * shared memory.  Both give the same spikes and trace, and gradients within

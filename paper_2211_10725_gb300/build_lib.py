@@ -21,6 +21,7 @@ BUILD_DIR = os.path.join(PKG, "_build")
 LIB_PATH = os.path.join(OUT_DIR, "libsnn.so")
 
 SOURCES = ["snn_api.cu", "scan_fwd.cu", "scan_bwd_leaky.cu", "scan_bwd_leaky_recompute.cu", "scan_bwd_leaky_seg.cu", "scan_bwd_leaky_seg8.cu",
+           "scan_bwd_leaky_seg12.cu",
            "scan_bwd_synaptic.cu", "scan_bwd_synaptic_recompute.cu", "reduce.cu", "snn_noalloc.cu",
            "gemm_tcgen05.cu", "gemm_scan.cu", "ce_loss.cu", "adamw.cu", "conv_pool.cu", "conv_small.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]

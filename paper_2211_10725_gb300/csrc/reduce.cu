@@ -9,11 +9,12 @@
 // 524,288-lane workload take 11.5 us.
 //
 // One launch reduces every parameter that shares a layout (blockIdx.z picks
-// the parameter).  Block (x, y) of a parameter sums split y of output group
-// x into fp64 scratch; the last of a group's splits to finish (a ticket
-// taken after its partial is published) adds the group's partials in split
-// order and writes the result, then resets the group's ticket to zero for
-// the next call.
+// the parameter).  Scalar and per-channel: block (x, y) of a parameter sums
+// split y of output group x into fp64 scratch; the last of a group's splits
+// to finish (a ticket taken after its partial is published) adds the
+// group's partials in split order and writes the result, then resets the
+// group's ticket to zero for the next call.  Per neuron, a neuron's B
+// partials fit one block, which sums them in a single pass.
 #include "scan_host.cuh"
 
 namespace snn {
@@ -83,28 +84,32 @@ __global__ void __launch_bounds__(kRedThreads) reduce_scalar(ReduceJobs js, int6
   }
 }
 
-// Per neuron: group x = neurons [256x, 256x + 256), split y = samples
-// [B*y/S, B*(y+1)/S); the last split adds the S partials of each neuron.
+// Per neuron, in one pass: block x covers neurons [32x, 32x + 32), warp y
+// sums split y of the samples, [B*y/S, B*(y+1)/S), in fp32 in order; warp 0
+// then adds the S split sums of each neuron in fp64 in split order.  The
+// whole sum over b of a neuron lives in one block, so no partial leaves it
+// and no ticket or second round trip through memory is needed.
 __global__ void __launch_bounds__(kRedThreads) reduce_per_neuron(ReduceJobs js, int64_t B,
                                                                   int64_t N) {
+  __shared__ double sh[kNeuronSplit][32];
   grid_dep_wait();
   const ReduceJob& j = js.job[blockIdx.z];
-  const int64_t n = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
-  const int64_t S = gridDim.y, s = blockIdx.y;
+  const int lid = threadIdx.x & 31, s = threadIdx.x >> 5;
+  const int S = blockDim.x >> 5;
+  const int64_t n = (int64_t)blockIdx.x * 32 + lid;
   if (n < N) {
     // the split's samples (8 at B = 64) in fp32, in order; the splits in fp64
     const int64_t b0 = B * s / S, b1 = B * (s + 1) / S;
     float acc = 0.0f;
     for (int64_t b = b0; b < b1; ++b) acc += j.part[b * N + n];
-    j.scratch[s * N + n] = (double)acc;
+    sh[s][lid] = (double)acc;
   }
-  if (!last_of_group(&j.tickets[blockIdx.x], (int)S)) return;
-  if (n < N) {
+  __syncthreads();
+  if (s == 0 && n < N) {
     double acc = 0.0;
-    for (int64_t q = 0; q < S; ++q) acc += j.scratch[q * N + n];
+    for (int q = 0; q < S; ++q) acc += sh[q][lid];
     j.out[n] = (float)acc;
   }
-  if (threadIdx.x == 0) j.tickets[blockIdx.x] = 0;
 }
 
 // Per channel: group x = channel c, split y sums the runs j = y, y + S, ...
@@ -210,13 +215,10 @@ cudaError_t launch_param_reduce(const ParamReduce* p, int n, int64_t B, int64_t 
     if (e != cudaSuccess) return e;
   } else if (mode == PM_PER_NEURON) {
     if (N > 0) {
-      int64_t S = B < kNeuronSplit ? B : kNeuronSplit;
-      if (S * N > scratch_len) S = scratch_len / N;
-      if (S < 1) return cudaErrorInvalidValue;  // the workspace is sized for S >= 1
+      const int64_t S = B < kNeuronSplit ? (B < 1 ? 1 : B) : kNeuronSplit;
       const cudaError_t e =
-          launch_pdl(reduce_per_neuron, dim3((unsigned)ceil_div(N, kRedThreads), (unsigned)S,
-                                             (unsigned)n),
-                     dim3(kRedThreads), 0, stream, js, B, N);
+          launch_pdl(reduce_per_neuron, dim3((unsigned)ceil_div(N, 32), 1, (unsigned)n),
+                     dim3((unsigned)(32 * S)), 0, stream, js, B, N);
       if (e != cudaSuccess) return e;
     }
   } else if (C > 0 && HW == 1 && kRedThreads % C == 0) {

@@ -155,7 +155,7 @@ cudaError_t launch_scan_bwd_leaky_recompute(ScanArgs a, int in_dt, int io_dt, bo
 cudaError_t launch_scan_bwd_synaptic_recompute(ScanArgs a, int in_dt, int io_dt, bool staged,
                                                cudaStream_t stream);
 // the recompute BPTT of the Leaky neuron with the replayed segment in
-// registers (scan_bwd_seg), for checkpoint intervals 8 and 16; sets
+// registers (scan_bwd_seg), for checkpoint intervals 8, 12 and 16; sets
 // *launched, and launches nothing where it does not apply
 cudaError_t launch_scan_bwd_leaky_seg(ScanArgs a, int in_dt, int io_dt, bool staged,
                                       cudaStream_t stream, bool* launched);
@@ -166,7 +166,8 @@ inline int64_t param_reduce_scratch(int64_t N, int64_t C) {
 }
 // One parameter's reduction: per-lane partials in, gradient out, fp64
 // scratch and zero-initialised tickets (one per output group: 1 for a
-// scalar, ceil(N/256) per neuron, C per channel) from the workspace.
+// scalar, C per channel; the per-neuron reduction needs neither, the
+// workspace keeps ceil(N/256) slots for it) from the workspace.
 struct ParamReduce {
   const float* part;
   float* out;

@@ -47,6 +47,8 @@ cudaError_t seg_modes(ScanArgs a, cudaStream_t st, bool* launched) {
 // One checkpoint interval's dtype dispatch (scan_bwd_leaky_seg*.cu).
 cudaError_t launch_scan_bwd_leaky_seg_k8(ScanArgs a, int in_dt, int io_dt, cudaStream_t stream,
                                          bool* launched);
+cudaError_t launch_scan_bwd_leaky_seg_k12(ScanArgs a, int in_dt, int io_dt, cudaStream_t stream,
+                                          bool* launched);
 cudaError_t launch_scan_bwd_leaky_seg_k16(ScanArgs a, int in_dt, int io_dt, cudaStream_t stream,
                                           bool* launched);
 

@@ -224,7 +224,8 @@ def check_every_lane_in_blocks(w, inp, layer, block=1024):
     return totals
 
 
-@pytest.mark.parametrize("save,k", [("recompute", 16), ("recompute", 8), ("mem", 8)])
+@pytest.mark.parametrize("save,k", [("recompute", 16), ("recompute", 12), ("recompute", 8),
+                                    ("mem", 8)])
 def test_full_size_large_bf16(save, k, cuda_device):
     """T=500, B=64, N=8192, bf16 storage (the benchmark's workload, in the
     launch configuration it times): every one of the 524,288 lanes against
@@ -318,7 +319,7 @@ def test_rleaky_full_size_large_bf16(save, k, cuda_device):
 
 
 # ---------------------------------------------------------------------------
-# Recompute BPTT with the replayed segment in registers (8- and 16-step
+# Recompute BPTT with the replayed segment in registers (8-, 12- and 16-step
 # checkpoint segments of the Leaky and recurrent Leaky neurons)
 # ---------------------------------------------------------------------------
 
@@ -326,8 +327,74 @@ SEG_CASES = [
     # T, B, N, K: a short first segment, one segment shorter than K, T = K,
     # several CTAs with a ragged last strip
     (37, 3, 1368, 16), (9, 4, 1000, 16), (16, 2, 2048, 16), (40, 5, 1000, 8),
-    (5, 7, 1000, 8), (64, 16, 8192, 16), (33, 9, 4096, 8),
+    (5, 7, 1000, 8), (64, 16, 8192, 16), (33, 9, 4096, 8), (29, 3, 1368, 12),
+    (12, 2, 2048, 12), (50, 6, 4096, 12),
 ]
+
+
+# The per-neuron parameter-gradient reduction, bit for bit against its
+# stated summation order: T, B, N, K, neuron.  One sample; B not a multiple
+# of the 8 splits; 64 samples; a width below one warp's 32 neurons and a
+# ragged last block; the recurrent neuron's v; the register-segment BPTT (K
+# 8, 12, 16) and the shared-memory replay (K = 5), store mode in between.
+REDUCE_CASES = [(24, 1, 2048, 8, "leaky"), (17, 3, 4096, 8, "leaky"), (40, 64, 1024, 12, "leaky"),
+                (9, 5, 20, 8, "rleaky"), (33, 11, 8192, 16, "rleaky"), (20, 9, 1000, 5, "leaky"),
+                (12, 10, 200, 0, "leaky")]
+
+
+def neuron_order_sum(part, B, N):
+    """The order the per-neuron sum takes on the GPU: split s of the samples,
+    [B*s/S, B*(s+1)/S) with S = min(B, 8), added in fp32 in sample order; the
+    S split sums added in fp64 in split order; rounded to fp32."""
+    S = min(B, 8)
+    total = np.zeros(N, np.float64)
+    for s in range(S):
+        acc = np.zeros(N, np.float32)
+        for b in range(B * s // S, B * (s + 1) // S):
+            acc = (acc + part[b]).astype(np.float32)
+        total = total + acc.astype(np.float64)
+    return total.astype(np.float32)
+
+
+@pytest.mark.parametrize("case", range(len(REDUCE_CASES)))
+def test_per_neuron_reduction_order(case, cuda_device):
+    T, B, N, K, neuron = REDUCE_CASES[case]
+    dt = W.BF16 if K in (12, 16) else [W.BF16, W.F32][case % 2]
+    w = W.ScanWorkload(
+        name=f"reduce_{case}", neuron=neuron, T=T, B=B, N=N, C=4, HW=max(1, N // 4), in_dtype=dt,
+        io_dtype=dt, i_mean=0.5, i_std=0.6, beta=("uniform", 0.5, 0.95),
+        thr=("uniform", 0.6, 1.4), v=("uniform", -0.6, 0.6), beta_mode="per_neuron",
+        thr_mode="per_neuron", v_mode="per_neuron", reset="subtract", detach_reset=True,
+        surrogate="atan", sg_param=2.0, save="recompute" if K else "mem", ckpt_every=K or 8,
+        want_mem=True, seed_index=700 + case)
+    inp = W.make_scan_inputs(w)
+    layer = H.run_gpu(w, inp)
+    assert layer.status() == 0
+    H.check_all(w, inp, layer, H.oracle_expect(w, inp))
+    # the reduction's order applied to the kernel's own per-lane partials
+    # (workspace: a 256-byte status block, then one 256-byte-aligned partial
+    # array per parameter)
+    pnames = ["beta", "thr"] + (["v"] if neuron == "rleaky" else [])
+    L = B * N
+    lb = (L * 4 + 255) // 256 * 256
+    ws = layer.ws.cpu().numpy()
+    got = {}
+    for k, pname in enumerate(pnames):
+        part = ws[256 + k * lb: 256 + k * lb + 4 * L].view(np.float32).reshape(B, N)
+        got[pname] = getattr(layer, f"grad_{pname}").cpu().numpy().copy()
+        assert np.array_equal(got[pname], neuron_order_sum(part, B, N), equal_nan=True), pname
+    # a second backward into cleared outputs writes the same bits
+    for pname in pnames:
+        getattr(layer, f"grad_{pname}").fill_(-1.0)
+    d = {k: v.to("cuda") for k, v in inp.items()}
+    layer.backward(d["I"], d["beta"], d["thr"], d["grad_spk"], alpha=d.get("alpha"),
+                   mem0=d.get("mem0"), grad_mem=d.get("grad_mem"),
+                   grad_mem_final=d.get("grad_mem_final"), v=d.get("v"))
+    torch.cuda.synchronize()
+    assert layer.status() == 0
+    for pname in pnames:
+        assert np.array_equal(getattr(layer, f"grad_{pname}").cpu().numpy(), got[pname],
+                              equal_nan=True), pname
 
 
 @pytest.mark.parametrize("neuron", ["leaky", "rleaky"])
