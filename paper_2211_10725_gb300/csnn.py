@@ -177,10 +177,15 @@ class ConvSNN:
         """[T*B, H, W, Cin_p] bf16 input map of conv layer l."""
         return X if l == 0 else self.pool[l - 1]
 
-    def ops(self, X, labels, stream=None):
+    def ops(self, X, labels, stream=None, side=None):
         """(name, call) in launch order: per conv layer im2col, GEMM, scan,
         max pool; the output layer's GEMM and scan; the loss; the reverse
-        pass from the top; AdamW on the weights and on the betas."""
+        pass from the top; AdamW on the weights and on the betas.  With a
+        snn.SideStream the output layer's weight gradient runs on it, beside
+        the reverse pass, and the first layer's backward joins it back before
+        the update.  The convolutions' weight gradients stay in line: beside
+        the second convolution's input-gradient GEMM and the first layer's
+        scan they took the SMs those need and the step got longer."""
         T, B, M = self.w.T, self.w.B, self.M
         out = []
         for l, (h, wd, cin, cout, k, ho, wo, hp, wp, kpad) in enumerate(self.geo):
@@ -232,9 +237,9 @@ class ConvSNN:
             out.append(("scan_bwd_out", lambda: o.backward(
                 None if self.I_fc is None else self.I_fc.view(T, B, -1), self.beta_fc, self.thr,
                 self.grad_out, want_param_grads=False, want_state_grads=False, stream=stream)))
-        out.append(("fc_bwd", lambda: snn.snn_dense_layer_bwd(
+        out.append(("fc_bwd", lambda: snn.dense_layer_bwd_split(
             flat, self.W[L], self.out_layer.grad_I.view(M, -1),
-            self.grad_pool[-1].view(M, -1), self.dW[L], self.ws_bwd[L], stream)))
+            self.grad_pool[-1].view(M, -1), self.dW[L], self.ws_bwd[L], stream, side)))
         for l in range(L - 1, -1, -1):
             h, wd, cin, cout, k, ho, wo, hp, wp, kpad = self.geo[l]
             layer = self.layers[l]
@@ -251,6 +256,9 @@ class ConvSNN:
                             snn.snn_dense_layer_bwd(self.cols[l], self.W[l],
                                                     layer.grad_I.view(rows, c), self.dcols[l],
                                                     self.dW[l], self.ws_bwd[l], stream)))
+            if l == 0 and side is not None:  # the reverse pass ends here
+                name, call = out[-1]
+                out[-1] = (name, lambda call=call: (call(), side.join(stream)))
             if l > 0:
                 out.append((f"col2im{l}", lambda l=l, k=k: snn.snn_col2im_nhwc(
                     self.dcols[l], self.grad_pool[l - 1], k, k, stream)))
@@ -297,8 +305,10 @@ class ConvSNN:
         self.forward(X, labels, stream)
         return self.backward(X, stream)
 
-    def train_step(self, X, labels, stream=None):
-        for _, call in self.ops(X, labels, stream):
+    def train_step(self, X, labels, stream=None, side=None):
+        """One full training step (weight gradients on `side`, a
+        snn.SideStream, if given)."""
+        for _, call in self.ops(X, labels, stream, side):
             call()
         return self.loss
 

@@ -131,10 +131,13 @@ class DenseSNN:
                            self.lr, self.betas[0], self.betas[1], self.eps, self.weight_decay,
                            step_counter=self.step_counter, stream=stream)
 
-    def ops(self, X, labels, stream=None):
+    def ops(self, X, labels, stream=None, side=None):
         """The training step as a list of (name, call) in launch order: per
         layer the forward GEMM and scan, the loss, per layer from the top the
-        scan BPTT and the dense backward, then the AdamW update."""
+        scan BPTT and the dense backward, then the AdamW update.  With a
+        snn.SideStream the weight gradients of the upper layers run on it,
+        beside the input-gradient products of the reverse pass, and the last
+        dense backward joins it back before the update."""
         T, B = self.w.T, self.w.B
         out = []
         for l, layer in enumerate(self.layers):
@@ -168,9 +171,8 @@ class DenseSNN:
             # fused: layer l's input gradient is the spike gradient of layer
             # l - 1, whose BPTT runs in the epilogue of that product
             dX = self.grad_in[l - 1] if (l > 0 and not self.fused_bwd) else None
-            out.append((f"dense_bwd{l}", lambda l=l, dX=dX: snn.snn_dense_layer_bwd(
-                self.layer_input(l, X), self.W[l], self.layers[l].grad_I.view(self.M, -1), dX,
-                self.dW[l], self.ws_bwd[l], stream)))
+            out.append((f"dense_bwd{l}", lambda l=l, dX=dX: self._dense_bwd(
+                l, X, dX, stream, side)))
             if l > 0 and self.fused_bwd:
                 lo = self.layers[l - 1]
                 out.append((f"dense_scan_bwd{l}", lambda l=l, lo=lo: snn.snn_dense_leaky_bwd(
@@ -179,14 +181,28 @@ class DenseSNN:
         out.append(("adamw", lambda: self.update(stream)))
         return out
 
+    def _dense_bwd(self, l, X, dX, stream, side):
+        dI = self.layers[l].grad_I.view(self.M, -1)
+        if side is not None and l == 0:
+            # the last product of the reverse pass: on the main stream, then
+            # wait for the weight gradients forked onto the side stream
+            snn.snn_dense_layer_bwd(self.layer_input(l, X), self.W[l], dI, dX, self.dW[l],
+                                    self.ws_bwd[l], stream)
+            side.join(stream)
+            return
+        snn.dense_layer_bwd_split(self.layer_input(l, X), self.W[l], dI, dX, self.dW[l],
+                                  self.ws_bwd[l], stream, side)
+
     def step(self, X, labels, stream=None):
         """Forward, loss and BPTT (weights unchanged); returns the dW list."""
         self.forward(X, labels, stream)
         return self.backward(X, stream)
 
-    def train_step(self, X, labels, stream=None):
-        """One full training step: forward, loss, BPTT and the AdamW update."""
-        for _, call in self.ops(X, labels, stream):
+    def train_step(self, X, labels, stream=None, side=None):
+        """One full training step: forward, loss, BPTT and the AdamW update
+        (the upper layers' weight gradients on `side`, a snn.SideStream, if
+        given)."""
+        for _, call in self.ops(X, labels, stream, side):
             call()
         return self.loss
 

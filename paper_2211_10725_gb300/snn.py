@@ -275,6 +275,48 @@ def snn_dense_layer_bwd(X, W, dI, dX, dW, ws, stream=None):
                                               _stream(stream)), "snn_dense_layer_bwd")
 
 
+class SideStream:
+    """A second stream for launches off a training step's critical path (the
+    weight-gradient products, which nothing waits on until the optimiser):
+    fork() queues a call on it behind the work already queued on the main
+    stream, join() makes the main stream wait for every call forked since the
+    last join.  Both are event records and waits, so a captured CUDA graph
+    holds them as fork and join edges."""
+
+    def __init__(self, device=None):
+        self.stream = torch.cuda.Stream(device)
+        self._done = []
+
+    def fork(self, main, call):
+        """call(stream) on the side stream, after main's queued work."""
+        main = torch.cuda.current_stream() if main is None else main
+        ready = torch.cuda.Event()
+        ready.record(main)
+        self.stream.wait_event(ready)
+        call(self.stream)
+        done = torch.cuda.Event()
+        done.record(self.stream)
+        self._done.append(done)
+
+    def join(self, main):
+        main = torch.cuda.current_stream() if main is None else main
+        for done in self._done:
+            main.wait_event(done)
+        self._done = []
+
+
+def dense_layer_bwd_split(X, W, dI, dX, dW, ws, stream=None, side: Optional[SideStream] = None):
+    """snn_dense_layer_bwd with, given a side stream, the weight gradient
+    forked onto it (issued first, so it runs beside the input gradient,
+    which the rest of the reverse pass waits on)."""
+    if side is None or dW is None:
+        snn_dense_layer_bwd(X, W, dI, dX, dW, ws, stream)
+        return
+    side.fork(stream, lambda st: snn_dense_layer_bwd(X, W, dI, None, dW, ws, st))
+    if dX is not None:
+        snn_dense_layer_bwd(X, W, dI, dX, None, ws, stream)
+
+
 def snn_rate_ce_workspace_bytes(B: int) -> int:
     return load_library().snn_rate_ce_workspace_bytes(B)
 

@@ -97,3 +97,56 @@ def test_dsnn_training_lowers_the_loss(cuda_device):
         assert layer.status() == 0
     assert np.all(np.isfinite(losses))
     assert min(losses[-5:]) < 0.8 * losses[0], losses
+
+
+def _net(kind, save, device):
+    if kind == "dsnn":
+        w = W.DSNN_C3
+        inp = W.make_dense_inputs(w)
+        net = DenseSNN(w, inp["W"], device=device, save=save, lr=2e-3)
+        X = inp["X"].reshape(w.T * w.B, -1).to(device)
+    else:
+        from paper_2211_10725_gb300.csnn import ConvSNN
+        w = W.CSNN_C4
+        inp = W.make_conv_inputs(w)
+        net = ConvSNN(w, inp["convs"], inp["Wfc"], device=device, save=save)
+        X = inp["X"].reshape(w.T * w.B, w.H, w.W, w.Cin).to(device)
+    return net, X, inp["labels"].to(device)
+
+
+def _state(net):
+    out = [net.loss, net.W32_flat, net.W_flat, net.m_flat, net.v_flat, net.dW_flat]
+    for name in ("beta_flat", "dbeta_flat"):
+        if getattr(net, name, None) is not None:
+            out.append(getattr(net, name))
+    return [t.detach().clone() for t in out]
+
+
+@pytest.mark.parametrize("kind,save", [("dsnn", "fused"), ("dsnn", "mem"), ("csnn", "fused")])
+def test_side_stream_step_is_bit_identical(kind, save, cuda_device):
+    """Three training steps with the weight gradients forked onto a second
+    stream (eagerly, then replayed from a captured CUDA graph) leave every
+    weight, moment, gradient and the loss bit for bit as the same steps with
+    every launch in line on one stream: the fork moves launches, not
+    arithmetic."""
+    ref, X, labels = _net(kind, save, cuda_device)
+    for _ in range(3):
+        ref.train_step(X, labels)
+    torch.cuda.synchronize()
+    want = _state(ref)
+
+    net, X, labels = _net(kind, save, cuda_device)
+    side = snn.SideStream(cuda_device)
+    net.train_step(X, labels, side=side)
+    stream = torch.cuda.Stream(cuda_device)
+    stream.wait_stream(torch.cuda.current_stream())
+    g = torch.cuda.CUDAGraph()
+    # the capture records the second step's launches; the step counter
+    # lives on the device, so each replay is the next step
+    with torch.cuda.graph(g, stream=stream):
+        net.train_step(X, labels, stream=None, side=side)
+    for _ in range(2):
+        g.replay()
+    torch.cuda.synchronize()
+    for a, b in zip(_state(net), want):
+        assert torch.equal(a, b)
