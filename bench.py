@@ -219,7 +219,7 @@ def hbm_peak():
 
 SCAN_SOURCES = ("scan_kernels.cuh", "scan_dispatch.cuh", "scan_host.cuh", "snn_device.cuh",
                 "scan_seg.cuh", "scan_seg_launch.cuh", "scan_bwd_leaky_seg.cu",
-                "scan_bwd_leaky_seg8.cu",
+                "scan_bwd_leaky_seg8.cu", "scan_bwd_leaky_seg12.cu",
                 "scan_fwd.cu", "scan_bwd_leaky.cu", "scan_bwd_leaky_recompute.cu",
                 "scan_bwd_synaptic.cu", "scan_bwd_synaptic_recompute.cu", "snn_api.cu")
 
