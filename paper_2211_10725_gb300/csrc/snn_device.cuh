@@ -217,14 +217,16 @@ struct Elem<__half> {
   static __device__ __forceinline__ void store1(__half* p, float v) { *p = __float2half_rn(v); }
 };
 
-// V consecutive elements (V = 4 or 8)
+// V consecutive elements (V = 4 or 8), aligned to V elements
 template <typename T, int V>
 __device__ __forceinline__ void loadv(const T* p, float* v) {
+  static_assert(V == 4 || V == 8, "vector accesses of 4 or 8 elements");
   if constexpr (V == 8) Elem<T>::load8(p, v);
   else Elem<T>::load4(p, v);
 }
 template <typename T, int V>
 __device__ __forceinline__ void storev(T* p, const float* v) {
+  static_assert(V == 4 || V == 8, "vector accesses of 4 or 8 elements");
   if constexpr (V == 8) Elem<T>::store8(p, v);
   else Elem<T>::store4(p, v);
 }
