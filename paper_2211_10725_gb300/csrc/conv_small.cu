@@ -389,6 +389,132 @@ __global__ void __launch_bounds__(kSlideMaxThreads) conv_slide_fwd_kernel(
   }
 }
 
+// ---- Weight gradient, single input channel, fixed KH x KW: sliding windows
+//
+// dW[o, k] = sum over (m, oy, ox) of dI[m, oy, ox, o] * X[m, oy+ky, ox+kx].
+// Thread t owns output row oy = t / CG and channel pair cg = t % CG (CG =
+// Cout/2) and keeps both channels' KH*KW tap sums in fp32 (a float2 per
+// tap).  For each of the block's images (m = b, b + G, ... in order) it
+// walks its row left to right with the KH x KW input window in registers
+// (KH new values a column, as in the forward) and reads one bf16 pair of
+// dL/dI a pixel straight from the staged raw rows: per pixel KH + 1
+// shared-memory loads for KH*KW paired FMAs.  Images are staged with
+// cp.async, double-buffered; the input map is expanded to fp32.  At the end
+// the Ho rows' sums are added in row order through shared memory into the
+// block partial part[b][o][k], so the result is the same on every call.
+constexpr int kSlideDwBlocks = 456;  // fixed block count (3 per SM of 152)
+
+// At most 96 registers a thread (92 for 5x5: 25 float2 sums, the 5x5 window,
+// no spills), so three blocks of the CSNN's first layer (24 rows x 8
+// channel pairs: 192 threads) fit on an SM and the 456 blocks run in one
+// wave (with 608, a third of them waited for a second wave: 12 images a
+// block's slot instead of 8).
+
+template <int KH_, int KW_>
+__global__ void __maxnreg__(96) conv_slide_dw_kernel(
+    const __nv_bfloat16* __restrict__ X, const __nv_bfloat16* __restrict__ dI,
+    float* __restrict__ part, int64_t M, int H, int W, int Cout, int vec) {
+  constexpr int KK = KH_ * KW_;
+  extern __shared__ __align__(16) unsigned char dsm[];
+  const int Ho = H - KH_ + 1, Wo = W - KW_ + 1, P = Ho * Wo;
+  const int img = H * W, pix = P * Cout;
+  const int rx = (img * 2 + 15) & ~15, rd = (pix * 2 + 15) & ~15;  // raw bytes
+  auto raw = [&](int b) { return dsm + b * (rx + rd); };             // two raw buffers
+  float* sx = reinterpret_cast<float*>(dsm + 2 * (rx + rd));         // [img] fp32
+  const int CG = Cout / 2;
+  const int t = threadIdx.x;
+  const bool active = t < Ho * CG;
+  const int oy = active ? t / CG : 0, cg = active ? t - (t / CG) * CG : 0;
+  const int64_t G = gridDim.x;
+  grid_dep_wait();
+  auto stage = [&](int64_t m, int b) {
+    if (vec) {
+      const unsigned char* gx = reinterpret_cast<const unsigned char*>(X + m * img);
+      const unsigned char* gd = reinterpret_cast<const unsigned char*>(dI + m * pix);
+      for (int c = t; c < img / 8; c += blockDim.x) cp_async16(raw(b) + 16 * c, gx + 16 * c);
+      for (int c = t; c < pix / 8; c += blockDim.x) cp_async16(raw(b) + rx + 16 * c, gd + 16 * c);
+    } else {
+      __nv_bfloat16* hx = reinterpret_cast<__nv_bfloat16*>(raw(b));
+      __nv_bfloat16* hd = reinterpret_cast<__nv_bfloat16*>(raw(b) + rx);
+      for (int e = t; e < img; e += blockDim.x) hx[e] = X[m * img + e];
+      for (int e = t; e < pix; e += blockDim.x) hd[e] = dI[m * pix + e];
+    }
+    cp_async_commit();
+  };
+  float2 acc[KK];
+#pragma unroll
+  for (int k = 0; k < KK; ++k) acc[k] = make_float2(0.0f, 0.0f);
+  // image i of this block is copy group i: two groups in flight before the
+  // loop, one more per image
+  if ((int64_t)blockIdx.x < M) stage(blockIdx.x, 0);
+  else cp_async_commit();
+  if ((int64_t)blockIdx.x + G < M) stage(blockIdx.x + G, 1);
+  else cp_async_commit();
+  int i = 0;
+  for (int64_t m = blockIdx.x; m < M; m += G, ++i) {
+    const int b = i & 1;
+    cp_async_wait_all_but_one();  // image m's copies have landed (m + G may be in flight)
+    __syncthreads();              // ... for every thread's copies
+    const __nv_bfloat16* hx = reinterpret_cast<const __nv_bfloat16*>(raw(b));
+    if (vec) {
+      for (int v = t; v < img / 8; v += blockDim.x)
+        unpack8(reinterpret_cast<const uint4*>(hx)[v], sx + 8 * v);
+    } else {
+      for (int e = t; e < img; e += blockDim.x) sx[e] = __bfloat162float(hx[e]);
+    }
+    __syncthreads();  // the fp32 map is complete
+    if (active) {
+      const float* row = sx + oy * W;
+      const __nv_bfloat162* g2 =
+          reinterpret_cast<const __nv_bfloat162*>(raw(b) + rx) + (int64_t)oy * Wo * CG + cg;
+      float win[KH_][KW_];
+#pragma unroll
+      for (int ky = 0; ky < KH_; ++ky)
+#pragma unroll
+        for (int kx = 1; kx < KW_; ++kx) win[ky][kx] = row[ky * W + kx - 1];
+#pragma unroll 2
+      for (int ox = 0; ox < Wo; ++ox) {
+#pragma unroll
+        for (int ky = 0; ky < KH_; ++ky) {
+#pragma unroll
+          for (int kx = 0; kx < KW_ - 1; ++kx) win[ky][kx] = win[ky][kx + 1];
+          win[ky][KW_ - 1] = row[ky * W + ox + KW_ - 1];
+        }
+        const float2 g = __bfloat1622float2(g2[ox * CG]);
+#pragma unroll
+        for (int ky = 0; ky < KH_; ++ky)
+#pragma unroll
+          for (int kx = 0; kx < KW_; ++kx)
+            acc[ky * KW_ + kx] =
+                __ffma2_rn(make_float2(win[ky][kx], win[ky][kx]), g, acc[ky * KW_ + kx]);
+      }
+    }
+    __syncthreads();  // raw buffer b and the fp32 map are no longer read
+    if (m + 2 * G < M) stage(m + 2 * G, b);
+    else cp_async_commit();  // an empty group keeps the wait count uniform
+  }
+  // every copy has landed (the last groups are empty) before the staging
+  // memory holds the row sums: red[(oy*CG + cg)*KK + k] = both channels
+  asm volatile("cp.async.wait_all;" ::: "memory");
+  __syncthreads();
+  float2* red = reinterpret_cast<float2*>(dsm);
+  if (active) {
+#pragma unroll
+    for (int k = 0; k < KK; ++k) red[(oy * CG + cg) * KK + k] = acc[k];
+  }
+  __syncthreads();
+  for (int e = t; e < Cout * KK; e += blockDim.x) {
+    const int o = e / KK, k = e - o * KK;
+    const int c2 = o >> 1;
+    float s = 0.0f;
+    for (int r = 0; r < Ho; ++r) {
+      const float2 v = red[(r * CG + c2) * KK + k];
+      s += (o & 1) ? v.y : v.x;
+    }
+    part[((int64_t)blockIdx.x * Cout + o) * KK + k] = s;
+  }
+}
+
 // dW[o, k] = sum of the G block partials, 0 for k >= K: one warp per
 // output, lane l adding partials l, l + 32, ... in order, then a fixed
 // shuffle tree over the lanes.
@@ -417,7 +543,31 @@ snn_status_t check_small(int64_t M, int64_t H, int64_t W, int64_t Cin, int64_t C
   return SNN_OK;
 }
 
-int64_t dw_blocks(int64_t M) { return M < kDwBlocks ? (M > 0 ? M : 1) : kDwBlocks; }
+// The sliding-window weight gradient applies: one input channel, a 5x5 or
+// 3x3 filter, a thread for each (output row, channel pair) of an image in
+// one block, and its staging (two raw image buffers and the fp32 map), and
+// later its row sums, within shared memory.  *smem: the bytes it takes.
+bool slide_dw_ok(int64_t H, int64_t W, int64_t Cin, int64_t Cout, int64_t KH, int64_t KW,
+                 size_t* smem) {
+  if (Cin != 1 || !((KH == 5 && KW == 5) || (KH == 3 && KW == 3))) return false;
+  const int64_t Ho = H - KH + 1, Wo = W - KW + 1;
+  if (Ho * (Cout / 2) > kSlideMaxThreads) return false;
+  const size_t rx = ((size_t)(H * W) * 2 + 15) / 16 * 16;
+  const size_t rd = ((size_t)(Ho * Wo * Cout) * 2 + 15) / 16 * 16;
+  const size_t staging = 2 * (rx + rd) + (size_t)(H * W) * sizeof(float);
+  const size_t sums = (size_t)(Ho * (Cout / 2) * KH * KW) * 2 * sizeof(float);
+  *smem = staging > sums ? staging : sums;
+  return *smem <= 200 * 1024;
+}
+
+// Blocks (= partials) of the weight gradient: a fixed count per kernel, so
+// that a shape always sums in the same order.
+int64_t dw_blocks(int64_t M, int64_t H, int64_t W, int64_t Cin, int64_t Cout, int64_t KH,
+                  int64_t KW) {
+  size_t smem = 0;
+  const int64_t cap = slide_dw_ok(H, W, Cin, Cout, KH, KW, &smem) ? kSlideDwBlocks : kDwBlocks;
+  return M < cap ? (M > 0 ? M : 1) : cap;
+}
 
 }  // namespace
 }  // namespace snn
@@ -490,7 +640,7 @@ extern "C" size_t snn_conv2d_small_dw_workspace_bytes(int64_t M, int64_t H, int6
                                                       int64_t Cin, int64_t Cout, int64_t KH,
                                                       int64_t KW) {
   if (check_small(M, H, W, Cin, Cout, KH, KW, KH * KW * Cin) != SNN_OK) return 0;
-  return (size_t)dw_blocks(M) * Cout * KH * KW * Cin * sizeof(float);
+  return (size_t)dw_blocks(M, H, W, Cin, Cout, KH, KW) * Cout * KH * KW * Cin * sizeof(float);
 }
 
 extern "C" snn_status_t snn_conv2d_small_dw_nhwc(int64_t M, int64_t H, int64_t W, int64_t Cin,
@@ -511,8 +661,33 @@ extern "C" snn_status_t snn_conv2d_small_dw_nhwc(int64_t M, int64_t H, int64_t W
     return SNN_ERR_ALIGNMENT;
   if ((reinterpret_cast<uintptr_t>(X) | reinterpret_cast<uintptr_t>(dI)) & 1u) return SNN_ERR_ALIGNMENT;
   const int K = (int)(KH * KW * Cin);
-  const int64_t G = dw_blocks(M);
+  const int64_t G = dw_blocks(M, H, W, Cin, Cout, KH, KW);
   float* part = static_cast<float*>(ws);
+  cudaError_t e = cudaSuccess;
+  size_t slide_smem = 0;
+  if (slide_dw_ok(H, W, Cin, Cout, KH, KW, &slide_smem)) {
+    const int thr = ((int)((H - KH + 1) * (Cout / 2)) + 31) / 32 * 32;
+    // raw 16-byte copies of whole images: both image sizes a multiple of 8
+    // elements, both bases 16-byte aligned (dI stays bf16 in shared memory)
+    const int vec1 = ((H * W) % 8 == 0 && ((H - KH + 1) * (W - KW + 1) * Cout) % 8 == 0 &&
+                      ((reinterpret_cast<uintptr_t>(X) | reinterpret_cast<uintptr_t>(dI)) & 15u) == 0)
+                         ? 1 : 0;
+    const void* ks = KH == 5 ? (const void*)conv_slide_dw_kernel<5, 5> : (const void*)conv_slide_dw_kernel<3, 3>;
+    if (slide_smem > 48 * 1024 &&
+        cudaFuncSetAttribute(ks, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)slide_smem) != cudaSuccess)
+      return SNN_ERR_CUDA;
+    const __nv_bfloat16* x1 = static_cast<const __nv_bfloat16*>(X);
+    const __nv_bfloat16* d1 = static_cast<const __nv_bfloat16*>(dI);
+    e = KH == 5 ? launch_pdl(conv_slide_dw_kernel<5, 5>, dim3((unsigned)G), dim3(thr), slide_smem, st, x1,
+                             d1, part, M, (int)H, (int)W, (int)Cout, vec1)
+                : launch_pdl(conv_slide_dw_kernel<3, 3>, dim3((unsigned)G), dim3(thr), slide_smem, st, x1,
+                             d1, part, M, (int)H, (int)W, (int)Cout, vec1);
+    if (e != cudaSuccess) return SNN_ERR_CUDA;
+    const int n = (int)(Cout * ldw);  // one warp each
+    e = launch_pdl(conv_small_dw_sum, dim3((unsigned)((n + 7) / 8)), dim3(256), 0, st,
+                   static_cast<const float*>(part), dW, (int)G, (int)Cout, K, (int)ldw);
+    return e == cudaSuccess ? SNN_OK : SNN_ERR_CUDA;
+  }
   const int P = (int)((H - KH + 1) * (W - KW + 1));
   const int img = (int)(H * W * Cin);
   const int64_t pix = (int64_t)P * Cout;
@@ -527,9 +702,8 @@ extern "C" snn_status_t snn_conv2d_small_dw_nhwc(int64_t M, int64_t H, int64_t W
   const void* k = (KH == 5 && KW == 5 && Cin == 1) ? (const void*)conv_small_dw_kernel<5, 5, 1, 25>
                   : (K <= 16) ? (const void*)conv_small_dw_kernel<0, 0, 0, 16>
                               : (const void*)conv_small_dw_kernel<0, 0, 0, 32>;
-  cudaError_t e = smem > 48 * 1024 ? cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                                          (int)smem)
-                                   : cudaSuccess;
+  e = smem > 48 * 1024 ? cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem)
+                       : cudaSuccess;
   if (e != cudaSuccess) return SNN_ERR_CUDA;
   if (KH == 5 && KW == 5 && Cin == 1)
     e = launch_pdl(conv_small_dw_kernel<5, 5, 1, 25>, dim3((unsigned)G), dim3(kDwThreads), smem, st,

@@ -176,12 +176,17 @@ def test_layout_argument_checks(cuda_device):
 
 @pytest.mark.parametrize("M,Hh,Ww,C,Cout,k,ldw", [(5, 28, 28, 1, 16, 5, 32), (3, 9, 11, 2, 8, 3, 24),
                                                   (2, 7, 7, 1, 4, 1, 8), (700, 28, 28, 1, 16, 5, 32),
-                                                  (4, 10, 13, 1, 8, 3, 16), (3, 70, 9, 1, 16, 5, 32)])
+                                                  (4, 10, 13, 1, 8, 3, 16), (3, 70, 9, 1, 16, 5, 32),
+                                                  (9, 28, 28, 1, 12, 5, 32), (1300, 28, 28, 1, 12, 5, 32),
+                                                  (6, 12, 12, 1, 8, 3, 16)])
 def test_small_conv_matches_oracle(M, Hh, Ww, C, Cout, k, ldw, cuda_device):
     """Forward currents and the weight gradient of the direct convolution
     against the oracle's convolution and its backward; the weight gradient
-    is the same bits on every call (more images than blocks in the last
-    case, so blocks sum several images)."""
+    is the same bits on every call.  One input channel with a 5x5 or 3x3
+    filter takes the sliding-window kernels (12 channels: the CSNN's first
+    layer; 700 and 1300 images: more images than blocks, so blocks sum
+    several); the others, and a 70-row map (more rows than one block's
+    threads), the general ones."""
     g = torch.Generator().manual_seed(M + 31 * Cout + k)
     X = (torch.rand((M, Hh, Ww, C), generator=g) < 0.3).to(torch.bfloat16)
     Wc = torch.randn((Cout, k, k, C), generator=g).to(torch.bfloat16)
