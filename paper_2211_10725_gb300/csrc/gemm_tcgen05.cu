@@ -345,8 +345,8 @@ cudaError_t launch_out(const CUtensorMap& ta, const CUtensorMap& tb, const GemmA
 
 // D[M, N] = A[M, K] * B[N, K]^T.  A is stored [M, K] row-major (K-major) or,
 // with A_MN, [K, M] row-major; B likewise [N, K] or, with B_MN, [K, N].
-// N tile: the widest the output needs (64 or 128 for an MN-major B), and 64
-// rather than 128 when 128-wide tiles would leave most SMs idle.
+// N tile: the widest the output needs (64, 128 or 192 for an MN-major B),
+// and 64 rather than 128 when 128-wide tiles would leave most SMs idle.
 template <bool OUT_BF16, bool A_MN = false, bool B_MN = false>
 cudaError_t gemm_tn(const void* A, const void* B, void* D, int M, int N, int K, int* status,
                     cudaStream_t st, int ksplit = 1, int bn_force = 0) {
@@ -358,6 +358,9 @@ cudaError_t gemm_tn(const void* A, const void* B, void* D, int M, int N, int K, 
   else if (N <= 16 && !B_MN) bn = 16;
   else if (N <= 32 && !B_MN) bn = 32;
   else if (N <= 64) bn = 64;
+  // an MN-major B wider than two 128-column tiles: 192-wide tiles when
+  // they need fewer tiles (each re-reads its A rows once)
+  else if (B_MN && N > 256 && (N + 191) / 192 < (N + 127) / 128) bn = 192;
   else {
     int dev = 0, sms = 152;
     if (cudaGetDevice(&dev) == cudaSuccess)
@@ -373,6 +376,7 @@ cudaError_t gemm_tn(const void* A, const void* B, void* D, int M, int N, int K, 
   if constexpr (B_MN) {
     if (bn == 64) return launch_out<64, OUT_BF16, A_MN, B_MN>(ta, tb, g, st);
     if (bn == 256) return launch_out<256, OUT_BF16, A_MN, B_MN>(ta, tb, g, st);
+    if (bn == 192) return launch_out<192, OUT_BF16, A_MN, B_MN>(ta, tb, g, st);
     return launch_out<128, OUT_BF16, A_MN, B_MN>(ta, tb, g, st);
   } else {
     switch (bn) {
@@ -392,10 +396,12 @@ size_t round256(size_t b) { return (b + 255) & ~size_t(255); }
 // the M rows), from the shapes alone so that a shape always sums in the same
 // order: enough (tile, split) items to give each of about one GPU's worth of
 // SMs (kSplitSlots) one, with at least kMinSplitKBlocks k-blocks per split.
-// A wide layer (N >= 256 neurons, K >= 512 inputs) with a long reduction
-// takes 128 x 256 tiles: its operands' L2 traffic is half that of the
-// 64-wide tiles, which re-read dI once per 64 columns; the splits then fill
-// the SMs.  Otherwise the GEMM's own tile choice, split to fill the SMs.
+// 128 x 256 tiles for K >= 256 inputs when the splits still give the SMs
+// work (always for a wide layer, N >= 256 neurons and K >= 512; for a
+// narrow one, such as a convolution's 64 channels over 304 patch columns,
+// when the reduction is long enough for at least 3/4 of kSplitSlots items):
+// dI is re-read once per 256 columns instead of once per 64.  Otherwise
+// the GEMM's own tile choice, split to fill the SMs.
 constexpr int64_t kSplitSlots = 152;
 constexpr int64_t kMinSplitKBlocks = 8;
 struct DwPlan {
@@ -409,9 +415,10 @@ DwPlan dw_plan(int64_t M, int64_t K, int64_t N) {
     if (s > nk / kMinSplitKBlocks) s = nk / kMinSplitKBlocks;
     return s < 1 ? 1 : (int)s;
   };
-  if (N >= 256 && K >= 512) {
-    const int S = splits(((N + BM - 1) / BM) * ((K + 255) / 256));
-    if (S >= 2) return DwPlan{256, S};
+  if (K >= 256) {
+    const int64_t tiles = ((N + BM - 1) / BM) * ((K + 255) / 256);
+    const int S = splits(tiles);
+    if (S >= 2 && ((N >= 256 && K >= 512) || tiles * S >= kSplitSlots * 3 / 4)) return DwPlan{256, S};
   }
   return DwPlan{0, splits(((N + BM - 1) / BM) * ((K + 63) / 64))};
 }
