@@ -70,7 +70,8 @@ cudaError_t bwd_staged(ScanArgs a, cudaStream_t st, bool* launched) {
     items = a.T;
   }
   StagedPlan p;
-  if (!plan_staged(k, a.L, items, per_lane, seg, kLanes<SYN>, &p, fixed, KC)) return cudaSuccess;
+  if (!plan_staged(k, a.L, items, per_lane, seg, kBwdLanes<SYN, RECOMP>, &p, fixed, KC))
+    return cudaSuccess;
   a.lanes_per_cta = p.lanes_per_cta;
   a.stages = p.stages;
   a.stage_bytes = p.stage_bytes;

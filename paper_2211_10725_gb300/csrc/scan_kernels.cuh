@@ -481,6 +481,10 @@ __device__ __forceinline__ void release_stage(uint64_t* empty, int s, int lid) {
 // Synaptic one (whose reverse pass carries five adjoints per lane).
 template <bool SYN>
 constexpr int kLanes = SYN ? 4 : 8;
+// Lanes per thread of the staged backward: 4 in store mode (half the
+// registers of 8, so twice the warps fit an SM), else kLanes.
+template <bool SYN, bool RECOMP>
+constexpr int kBwdLanes = (!SYN && !RECOMP) ? 4 : kLanes<SYN>;
 
 template <typename T, int NP>
 __device__ __forceinline__ void load_pairs(const T* p, float2 q[NP]) {
@@ -704,7 +708,7 @@ __device__ __forceinline__ void bwd_pairs(const ScanArgs& a, const float2 beta[N
 template <bool SYN, bool RECOMP, typename TI, typename TO, int RESET, int SG, int KC = 0,
           bool REC = false>
 __global__ void __launch_bounds__(kMaxStagedThreads) scan_bwd_staged(const ScanArgs a) {
-  constexpr int V = kLanes<SYN>, NP = V / 2;
+  constexpr int V = kBwdLanes<SYN, RECOMP>, NP = V / 2;
   extern __shared__ __align__(1024) unsigned char smem[];
   uint64_t* full = reinterpret_cast<uint64_t*>(smem);
   uint64_t* empty = full + kMaxStages;
@@ -864,8 +868,8 @@ __global__ void __launch_bounds__(kMaxStagedThreads) scan_bwd_staged(const ScanA
         load_pairs<TO, NP>(base + tile_io_elems, uu);
         if (use_bits) {
           const unsigned char* bb = reinterpret_cast<const unsigned char*>(base - c * V) +
-                                    t_spk * io_stride + bits_skew + (SYN ? c / 2 : c);
-          const unsigned zb = SYN ? (unsigned)(*bb >> ((c & 1) * 4)) : (unsigned)*bb;
+                                    t_spk * io_stride + bits_skew + (V == 4 ? c / 2 : c);
+          const unsigned zb = V == 4 ? (unsigned)(*bb >> ((c & 1) * 4)) : (unsigned)*bb;
 #pragma unroll
           for (int k = 0; k < V; ++k) zz[k] = (zb >> k) & 1u;
         } else if (half_store) {
