@@ -397,6 +397,48 @@ def test_per_neuron_reduction_order(case, cuda_device):
                               equal_nan=True), pname
 
 
+# Scalar and per-channel parameter gradients through their reduction
+# launches: T, B, N, C, HW, save, neuron.  Channel runs of one lane
+# (channel-last) and of many; a synaptic neuron (alpha); the shared-memory
+# recompute kernel; a shape small enough for the plain kernels.
+PARAM_CASES = [(25, 8, 6912, 12, 576, "mem", "leaky"), (25, 16, 4096, 64, 1, "mem", "leaky"),
+               (30, 4, 4096, 16, 256, "mem", "synaptic"), (33, 5, 1024, 8, 128, "recompute", "leaky"),
+               (3, 2, 8, 2, 4, "mem", "leaky")]
+
+
+@pytest.mark.parametrize("case", range(len(PARAM_CASES)))
+def test_scalar_and_channel_gradients(case, cuda_device):
+    """The oracle's parameter gradients, and the same bits from a second
+    backward into cleared outputs (every completion ticket back at zero)."""
+    T, B, N, C, HW, save, neuron = PARAM_CASES[case]
+    dt = [W.F32, W.BF16][case % 2]
+    w = W.ScanWorkload(
+        name=f"pfold_{case}", neuron=neuron, T=T, B=B, N=N, C=C, HW=HW, in_dtype=dt,
+        io_dtype=dt, i_mean=0.5, i_std=0.6, beta=("uniform", 0.5, 0.95),
+        thr=("uniform", 0.6, 1.4), alpha=("uniform", 0.5, 0.9),
+        beta_mode=["per_channel", "scalar"][case % 2], thr_mode=["scalar", "per_channel"][case % 2],
+        alpha_mode="per_channel", reset=["zero", "subtract"][case % 2], detach_reset=True,
+        surrogate="fast_sigmoid", sg_param=25.0, save=save, ckpt_every=3, want_mem=True,
+        seed_index=800 + case)
+    inp = W.make_scan_inputs(w)
+    layer = H.run_gpu(w, inp)
+    assert layer.status() == 0
+    H.check_all(w, inp, layer, H.oracle_expect(w, inp))
+    pnames = ["beta", "thr"] + (["alpha"] if neuron == "synaptic" else [])
+    got = {p: getattr(layer, f"grad_{p}").clone() for p in pnames}
+    for p in pnames:
+        getattr(layer, f"grad_{p}").fill_(-1.0)
+    d = {k: v.to("cuda") for k, v in inp.items()}
+    layer.backward(d["I"], d["beta"], d["thr"], d["grad_spk"], alpha=d.get("alpha"),
+                   mem0=d.get("mem0"), syn0=d.get("syn0"), grad_mem=d.get("grad_mem"),
+                   grad_mem_final=d.get("grad_mem_final"),
+                   grad_syn_final=d.get("grad_syn_final"))
+    torch.cuda.synchronize()
+    assert layer.status() == 0
+    for p in pnames:
+        assert torch.equal(getattr(layer, f"grad_{p}"), got[p]), p
+
+
 @pytest.mark.parametrize("neuron", ["leaky", "rleaky"])
 @pytest.mark.parametrize("case", range(len(SEG_CASES)))
 def test_register_segment_recompute(case, neuron, cuda_device):
