@@ -51,10 +51,10 @@ cudaError_t fwd_t(ScanArgs a, bool staged, cudaStream_t st) {
                     st, a);
 }
 
-template <bool SYN, bool RECOMP, typename TI, typename TO, int RESET, int SG, int KC = 0,
-          bool REC = false>
-cudaError_t bwd_staged(ScanArgs a, cudaStream_t st, bool* launched) {
-  const void* k = (const void*)scan_bwd_staged<SYN, RECOMP, TI, TO, RESET, SG, KC, REC>;
+template <bool SYN, bool RECOMP, typename TI, typename TO, int RESET, int SG, int KC, bool REC,
+          int VL>
+cudaError_t bwd_staged_vl(ScanArgs a, cudaStream_t st, bool* launched) {
+  const void* k = (const void*)scan_bwd_staged<SYN, RECOMP, TI, TO, RESET, SG, KC, REC, VL>;
   int per_lane, seg, fixed;
   int64_t items;
   if (RECOMP) {
@@ -72,14 +72,24 @@ cudaError_t bwd_staged(ScanArgs a, cudaStream_t st, bool* launched) {
     items = a.T;
   }
   StagedPlan p;
-  if (!plan_staged(k, a.L, items, per_lane, seg, kBwdLanes<SYN, RECOMP>, &p, fixed, KC))
-    return cudaSuccess;
+  if (!plan_staged(k, a.L, items, per_lane, seg, VL, &p, fixed, KC)) return cudaSuccess;
   a.lanes_per_cta = p.lanes_per_cta;
   a.stages = p.stages;
   a.stage_bytes = p.stage_bytes;
   *launched = true;
-  return launch_pdl(scan_bwd_staged<SYN, RECOMP, TI, TO, RESET, SG, KC, REC>,
+  return launch_pdl(scan_bwd_staged<SYN, RECOMP, TI, TO, RESET, SG, KC, REC, VL>,
                     dim3((unsigned)p.grid), dim3(p.threads), p.smem, st, a);
+}
+
+// The staged backward with its lanes per thread: 4 for the Leaky neuron's
+// store mode on sequences of at most 64 steps, else kLanes.
+template <bool SYN, bool RECOMP, typename TI, typename TO, int RESET, int SG, int KC = 0,
+          bool REC = false>
+cudaError_t bwd_staged(ScanArgs a, cudaStream_t st, bool* launched) {
+  if constexpr (!SYN && !RECOMP) {
+    if (a.T <= 64) return bwd_staged_vl<SYN, RECOMP, TI, TO, RESET, SG, KC, REC, 4>(a, st, launched);
+  }
+  return bwd_staged_vl<SYN, RECOMP, TI, TO, RESET, SG, KC, REC, kLanes<SYN>>(a, st, launched);
 }
 
 template <bool SYN, bool RECOMP, typename TI, typename TO>

@@ -481,10 +481,9 @@ __device__ __forceinline__ void release_stage(uint64_t* empty, int s, int lid) {
 // Synaptic one (whose reverse pass carries five adjoints per lane).
 template <bool SYN>
 constexpr int kLanes = SYN ? 4 : 8;
-// Lanes per thread of the staged backward: 4 in store mode (half the
-// registers of 8, so twice the warps fit an SM), else kLanes.
-template <bool SYN, bool RECOMP>
-constexpr int kBwdLanes = (!SYN && !RECOMP) ? 4 : kLanes<SYN>;
+// The staged backward takes its lanes per thread as VL: kLanes, or 4 for
+// the Leaky neuron's store mode on short sequences (half the registers of
+// 8, so twice the warps fit an SM: faster at T = 25, slower at T = 500).
 
 template <typename T, int NP>
 __device__ __forceinline__ void load_pairs(const T* p, float2 q[NP]) {
@@ -706,9 +705,10 @@ __device__ __forceinline__ void bwd_pairs(const ScanArgs& a, const float2 beta[N
 }
 
 template <bool SYN, bool RECOMP, typename TI, typename TO, int RESET, int SG, int KC = 0,
-          bool REC = false>
+          bool REC = false, int VL = kLanes<SYN>>
 __global__ void __launch_bounds__(kMaxStagedThreads) scan_bwd_staged(const ScanArgs a) {
-  constexpr int V = kBwdLanes<SYN, RECOMP>, NP = V / 2;
+  static_assert(VL == kLanes<SYN> || (VL == 4 && !SYN && !RECOMP), "lanes per thread");
+  constexpr int V = VL, NP = V / 2;
   extern __shared__ __align__(1024) unsigned char smem[];
   uint64_t* full = reinterpret_cast<uint64_t*>(smem);
   uint64_t* empty = full + kMaxStages;
