@@ -132,8 +132,8 @@ int snn_version(void);
 size_t snn_scan_desc_size(void);
 
 /* Bytes of device workspace every scan call of `desc` needs (a status word,
- * per-lane parameter-gradient partials, fp64 reduction scratch and the
- * reductions' completion tickets).  0 if desc is invalid.  The tickets must
+ * per-lane parameter-gradient partials, reduction scratch in 8-byte slots
+ * and the reductions' completion tickets).  0 if desc is invalid.  The tickets must
  * start at zero (snn_workspace_init) and each reduction leaves them at zero;
  * after a call that reported SNN_ERR_TIMEOUT, initialise the workspace
  * again. */
@@ -211,7 +211,8 @@ snn_status_t snn_leaky_fwd(const snn_scan_desc* desc, const void* I, const float
  * d u_{t+1}/d z_t = -thr (subtract), -beta*u_t (zero), 0 (none).
  * Parameter sums are accumulated in fp32 per lane and reduced across lanes
  * in a fixed order (deterministic): runs of a few lanes in fp32, everything
- * above them in fp64.
+ * above them in compensated fp32 (a sum and the rounding error of its
+ * additions, two-sum).
  * SNN_SAVE_RECOMPUTE replays Eq. (4) from each checkpoint bit for bit as the
  * forward evaluated it.  With ckpt_every 8 (any dtype pair), 12 or 16 (bf16
  * or fp16 input and io), no grad_mem, a reset other than SNN_RESET_NONE and B*N

@@ -342,18 +342,30 @@ REDUCE_CASES = [(24, 1, 2048, 8, "leaky"), (17, 3, 4096, 8, "leaky"), (40, 64, 1
                 (12, 10, 200, 0, "leaky")]
 
 
+def two_add(hi, lo, x):
+    """(hi, lo) += x in float32, the rounding error of hi + x kept in lo
+    (Knuth's two-sum, every operation rounded to nearest)."""
+    f = np.float32
+    s = (hi + x).astype(f)
+    z = (s - hi).astype(f)
+    e = ((hi - (s - z).astype(f)).astype(f) + (x - z).astype(f)).astype(f)
+    return s, (lo + e).astype(f)
+
+
 def neuron_order_sum(part, B, N):
     """The order the per-neuron sum takes on the GPU: split s of the samples,
     [B*s/S, B*(s+1)/S) with S = min(B, 8), added in fp32 in sample order; the
-    S split sums added in fp64 in split order; rounded to fp32."""
+    S split sums added in split order, compensated (two-sum); the sum plus
+    its error rounded to fp32."""
     S = min(B, 8)
-    total = np.zeros(N, np.float64)
+    hi = np.zeros(N, np.float32)
+    lo = np.zeros(N, np.float32)
     for s in range(S):
         acc = np.zeros(N, np.float32)
         for b in range(B * s // S, B * (s + 1) // S):
             acc = (acc + part[b]).astype(np.float32)
-        total = total + acc.astype(np.float64)
-    return total.astype(np.float32)
+        hi, lo = two_add(hi, lo, acc)
+    return (hi + lo).astype(np.float32)
 
 
 @pytest.mark.parametrize("case", range(len(REDUCE_CASES)))
