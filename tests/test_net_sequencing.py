@@ -81,3 +81,85 @@ def test_conv_network_launch_order(save):
     for l in range(len(net.geo)):
         i = names.index(f"pool_bwd{l}")
         assert names[i + 1] == f"scan_bwd{l}" and names[i + 2] == f"conv_bwd{l}"
+
+
+class _Recorder:
+    """Stands in for the library calls of the reverse pass and for a
+    snn.SideStream: records which product runs where, in call order."""
+
+    def __init__(self, monkeypatch):
+        self.log = []
+        self.stream = "side"
+        rec = self
+
+        def dense_bwd(X, Wt, dI, dX, dW, ws, stream=None):
+            rec.log.append(("dense_bwd", stream, dX is not None, dW is not None))
+
+        monkeypatch.setattr(snn, "snn_dense_layer_bwd", dense_bwd)
+        for name in ("snn_dense_leaky_bwd", "snn_rate_ce_leaky_bwd", "snn_rate_ce_loss",
+                     "snn_adamw_step", "snn_leaky_bwd", "snn_maxpool2_bwd_nhwc",
+                     "snn_col2im_nhwc", "snn_conv2d_small_dw_nhwc"):
+            monkeypatch.setattr(snn, name, lambda *a, _n=name, **k: rec.log.append((_n,)))
+
+    def fork(self, main, call):
+        self.log.append(("fork",))
+        call(self.stream)
+
+    def join(self, main):
+        self.log.append(("join",))
+
+
+def test_dense_network_weight_gradients_on_the_side_stream(monkeypatch):
+    """Fused mode: the upper layers' dW products are forked (queued on the
+    side stream before the main stream's next product), the first layer's
+    runs on the main stream and then joins the side stream, before AdamW."""
+    w = W.DSNN_C3
+    net = DenseSNN(w, W.make_dense_inputs(w)["W"], device="cpu", save="fused")
+    rec = _Recorder(monkeypatch)
+    ops = net.ops(None, None, None, rec)
+    start = [n for n, _ in ops].index("dense_bwd2")
+    for _, call in ops[start:-1]:   # the reverse pass, AdamW excluded
+        call()
+    log = rec.log
+    assert log[0] == ("fork",) and log[1] == ("dense_bwd", "side", False, True)
+    assert log[2] == ("snn_dense_leaky_bwd",)
+    assert log[3] == ("fork",) and log[4] == ("dense_bwd", "side", False, True)
+    assert log[5] == ("snn_dense_leaky_bwd",)
+    assert log[6] == ("dense_bwd", None, False, True) and log[7] == ("join",)
+    assert len(log) == 8
+
+
+def test_dense_network_split_products_in_stored_mode(monkeypatch):
+    """Stored-trace mode: each upper layer's dense backward forks its dW
+    before issuing its dX on the main stream (which the next scan needs)."""
+    w = W.DSNN_C3
+    net = DenseSNN(w, W.make_dense_inputs(w)["W"], device="cpu", save="mem")
+    rec = _Recorder(monkeypatch)
+    ops = net.ops(None, None, None, rec)
+    calls = dict(ops)
+    calls["dense_bwd2"]()
+    assert rec.log == [("fork",), ("dense_bwd", "side", False, True),
+                       ("dense_bwd", None, True, False)]
+    rec.log.clear()
+    calls["dense_bwd0"]()
+    assert rec.log == [("dense_bwd", None, False, True), ("join",)]
+
+
+def test_conv_network_side_stream_forks_only_the_readout(monkeypatch):
+    """CSNN: the readout's dW is forked; the second convolution's backward
+    stays in line; the first layer's weight gradient joins the side
+    stream."""
+    w = W.CSNN_C4
+    inp = W.make_conv_inputs(w)
+    net = ConvSNN(w, inp["convs"], inp["Wfc"], device="cpu", save="fused")
+    rec = _Recorder(monkeypatch)
+    calls = dict(net.ops(None, None, None, rec))
+    calls["fc_bwd"]()
+    assert rec.log == [("fork",), ("dense_bwd", "side", False, True),
+                       ("dense_bwd", None, True, False)]
+    rec.log.clear()
+    calls["conv_bwd1"]()
+    assert rec.log == [("dense_bwd", None, True, True)]
+    rec.log.clear()
+    calls["conv_bwd0"]()
+    assert rec.log == [("snn_conv2d_small_dw_nhwc",), ("join",)]
