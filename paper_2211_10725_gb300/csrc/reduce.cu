@@ -42,7 +42,11 @@ __device__ __forceinline__ float2 pair_add(float2 a, float2 b) {
   a.y = __fadd_rn(a.y, b.y);
   return a;
 }
-__device__ __forceinline__ float pair_value(float2 a) { return __fadd_rn(a.x, a.y); }
+// The pair's value; a non-finite sum is returned as it is (its error term
+// is NaN once an infinity entered the sum).
+__device__ __forceinline__ float pair_value(float2 a) {
+  return isfinite(a.x) ? __fadd_rn(a.x, a.y) : a.x;
+}
 
 // The block's values added in a fixed tree.
 __device__ __forceinline__ float2 block_sum(float2 v, float2* sh) {

@@ -356,7 +356,7 @@ def neuron_order_sum(part, B, N):
     """The order the per-neuron sum takes on the GPU: split s of the samples,
     [B*s/S, B*(s+1)/S) with S = min(B, 8), added in fp32 in sample order; the
     S split sums added in split order, compensated (two-sum); the sum plus
-    its error rounded to fp32."""
+    its error rounded to fp32 (a non-finite sum as it is)."""
     S = min(B, 8)
     hi = np.zeros(N, np.float32)
     lo = np.zeros(N, np.float32)
@@ -365,7 +365,8 @@ def neuron_order_sum(part, B, N):
         for b in range(B * s // S, B * (s + 1) // S):
             acc = (acc + part[b]).astype(np.float32)
         hi, lo = two_add(hi, lo, acc)
-    return (hi + lo).astype(np.float32)
+    with np.errstate(invalid="ignore"):
+        return np.where(np.isfinite(hi), (hi + lo).astype(np.float32), hi)
 
 
 @pytest.mark.parametrize("case", range(len(REDUCE_CASES)))
